@@ -1,0 +1,221 @@
+"""CPU oracle of one PRISM draft round (fp64 C, see ``oracle.c``).
+
+TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the
+benchmark's CPU-baseline leg use it.  The CUDA path never imports it and
+shares no code with it.
+
+Pins: every function here is checked against something other than itself in
+``tests/test_oracle_pins.py`` (library routines, closed forms, invariants,
+brute force on tiny inputs and an independent library-based reference block).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+STEP_TENSORS = ("w_fuse", "g_attn", "w_qkv", "w_o", "g_mlp", "w_gate_up", "w_down", "g_final")
+
+
+class _Config(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "hidden", "n_q_heads", "n_kv_heads", "head_dim", "ffn", "vocab", "n_steps",
+        "bf16", "round_acts", "final_norm", "topk", "max_ctx")] + [
+        ("rope_theta", ctypes.c_double), ("rms_eps", ctypes.c_double)]
+
+
+class _Module(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in STEP_TENSORS]
+
+
+def build(force: bool = False) -> str:
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        compile_source(_SRC, _LIB)
+    return _LIB
+
+
+def compile_source(src: str, out: str) -> str:
+    """Compile an oracle source file into a shared library at ``out``."""
+    tmp = out + f".tmp{os.getpid()}"
+    subprocess.check_call(["gcc", "-O2", "-fopenmp", "-ffp-contract=off", "-fPIC", "-shared",
+                           src, "-o", tmp, "-lm"])
+    os.replace(tmp, out)
+    return out
+
+
+def _bind(path: str):
+    lib = ctypes.CDLL(path)
+    vp, i32, i64, dbl = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_double
+    lib.orc_round_bf16.argtypes = [dbl]
+    lib.orc_round_bf16.restype = dbl
+    lib.orc_matvec.argtypes = [vp, ctypes.c_int, i64, i64, vp, vp]
+    lib.orc_rmsnorm.argtypes = [vp, vp, i64, dbl, vp]
+    lib.orc_rope.argtypes = [vp, i32, i64, dbl]
+    lib.orc_attend.argtypes = [vp, vp, vp, ctypes.c_int, i64, i64, i32, vp]
+    lib.orc_draft_round.argtypes = [ctypes.POINTER(_Config), vp, vp, ctypes.POINTER(_Module),
+                                    i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
+    lib.orc_draft_round.restype = ctypes.c_int
+    lib.orc_accept_greedy.argtypes = [i32, i32, vp, vp, vp, vp, vp, vp]
+    for f in (lib.orc_matvec, lib.orc_rmsnorm, lib.orc_rope, lib.orc_attend, lib.orc_accept_greedy):
+        f.restype = None
+    return lib
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            _lib = _bind(build())
+    return _lib
+
+
+class variant:
+    """Use another compiled copy of the oracle (e.g. one with a planted
+    mistake, built by a pin-strength test) inside a ``with`` block."""
+
+    def __init__(self, path: str):
+        self.path = path
+
+    def __enter__(self):
+        global _lib
+        _load()
+        with _lock:
+            self._saved, _lib = _lib, _bind(self.path)
+        return self
+
+    def __exit__(self, *exc):
+        global _lib
+        with _lock:
+            _lib = self._saved
+        return False
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+# ------------------------------------------------------------------ single ops
+
+def round_bf16(x: float) -> float:
+    return float(_load().orc_round_bf16(float(x)))
+
+
+def matvec(W: np.ndarray, x: np.ndarray) -> np.ndarray:
+    """y = W x in fp64; W float32 [rows, cols] or bf16 bit patterns (uint16)."""
+    bf = W.dtype == np.uint16
+    W = _c(W, np.uint16 if bf else np.float32)
+    x = _c(x, np.float64)
+    y = np.empty(W.shape[0], dtype=np.float64)
+    _load().orc_matvec(W.ctypes.data, int(bf), W.shape[0], W.shape[1], x.ctypes.data, y.ctypes.data)
+    return y
+
+
+def rmsnorm(x: np.ndarray, g: np.ndarray, eps: float) -> np.ndarray:
+    x = _c(x, np.float64)
+    g = _c(g, np.float64)
+    out = np.empty_like(x)
+    _load().orc_rmsnorm(x.ctypes.data, g.ctypes.data, x.size, eps, out.ctypes.data)
+    return out
+
+
+def rope(v: np.ndarray, pos: int, theta: float) -> np.ndarray:
+    v = _c(v, np.float64).copy()
+    _load().orc_rope(v.ctypes.data, v.size, pos, theta)
+    return v
+
+
+def attend(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
+    """Softmax attention of one query over rows of k, v ([n, D], float32)."""
+    q = _c(q, np.float64)
+    k = _c(k, np.float32)
+    v = _c(v, np.float32)
+    o = np.empty(q.size, dtype=np.float64)
+    _load().orc_attend(q.ctypes.data, k.ctypes.data, v.ctypes.data, 0, k.shape[1], k.shape[0],
+                       q.size, o.ctypes.data)
+    return o
+
+
+# ------------------------------------------------------------------ round
+
+def config_of(shape, *, topk: int, max_ctx: int, round_acts: bool | None = None,
+              final_norm: bool = True) -> _Config:
+    bf = shape.dtype == "bf16"
+    return _Config(shape.hidden, shape.n_q_heads, shape.n_kv_heads, shape.head_dim, shape.ffn,
+                   shape.vocab, shape.n_steps, int(bf), int(bf if round_acts is None else round_acts),
+                   int(final_norm), topk, max_ctx, float(shape.rope_theta), float(shape.rms_eps))
+
+
+def draft_round(shape, weights: dict, inputs: dict, *, topk: int = 1, round_acts: bool | None = None,
+                final_norm: bool = True, want_logits: bool = False, want_hidden: bool = True,
+                seqs=None) -> dict:
+    """Run one draft round on the host.
+
+    ``weights``: {"embed", "lm_head", "modules": {m: {...}}, "f_map"} as made
+    by the synthetic generator (bf16 arrays are uint16 bit patterns).
+    ``inputs``: {"tokens", "hidden", "n_new", "kv_len", "k_cache", "v_cache", "max_ctx"}.
+    ``seqs``: optional list of sequence indices to compute (sequences are
+    independent); outputs then cover only those sequences, in that order.
+    The caches in ``inputs`` are not modified; updated copies are returned."""
+    lib = _load()
+    bf = shape.dtype == "bf16"
+    wdt = np.uint16 if bf else np.float32
+    K = shape.n_steps
+    sel = list(range(inputs["tokens"].shape[0])) if seqs is None else list(seqs)
+    B = len(sel)
+    tokens = _c(inputs["tokens"][sel], np.int32)
+    max_new = tokens.shape[1]
+    hidden = _c(inputs["hidden"][sel], wdt)
+    n_new = _c(inputs["n_new"][sel], np.int32)
+    kv_len = _c(inputs["kv_len"][sel], np.int32)
+    k_cache = _c(inputs["k_cache"][sel], wdt).copy()
+    v_cache = _c(inputs["v_cache"][sel], wdt).copy()
+    cfg = config_of(shape, topk=topk, max_ctx=int(inputs["max_ctx"]), round_acts=round_acts,
+                    final_norm=final_norm)
+    keep = []
+    mods = (_Module * K)()
+    for k in range(K):
+        mod = weights["modules"][weights["f_map"][k]]
+        arrs = [_c(mod[n], wdt) for n in STEP_TENSORS]
+        keep.extend(arrs)
+        mods[k] = _Module(*[a.ctypes.data for a in arrs])
+    embed = _c(weights["embed"], wdt)
+    lm = _c(weights["lm_head"], wdt)
+    draft = np.empty((B, K), dtype=np.int32)
+    tids = np.empty((B, K, topk), dtype=np.int32)
+    tvals = np.empty((B, K, topk), dtype=np.float64)
+    logits = np.empty((B, K, shape.vocab), dtype=np.float64) if want_logits else None
+    hout = np.empty((B, K, shape.hidden), dtype=np.float64) if want_hidden else None
+    rc = lib.orc_draft_round(ctypes.byref(cfg), embed.ctypes.data, lm.ctypes.data, mods, B, max_new,
+                             tokens.ctypes.data, hidden.ctypes.data, n_new.ctypes.data,
+                             kv_len.ctypes.data, k_cache.ctypes.data, v_cache.ctypes.data,
+                             draft.ctypes.data, tids.ctypes.data, tvals.ctypes.data,
+                             _ptr(logits), _ptr(hout))
+    if rc != 0:
+        raise ValueError(f"oracle draft round rejected its input (code {rc})")
+    return {"draft_ids": draft, "topk_ids": tids, "topk_logits": tvals, "logits": logits,
+            "hidden_out": hout, "k_cache": k_cache, "v_cache": v_cache}
+
+
+def accept_greedy(draft: np.ndarray, target: np.ndarray, n_new: np.ndarray, kv_len: np.ndarray) -> dict:
+    draft = _c(draft, np.int32)
+    target = _c(target, np.int32)
+    B, K = draft.shape
+    kv = _c(kv_len, np.int32).copy()
+    acc = np.empty(B, dtype=np.int32)
+    out = np.empty((B, K + 1), dtype=np.int32)
+    _load().orc_accept_greedy(B, K, draft.ctypes.data, target.ctypes.data, _c(n_new, np.int32).ctypes.data,
+                              kv.ctypes.data, acc.ctypes.data, out.ctypes.data)
+    return {"accept_len": acc, "out_tokens": out, "kv_len": kv}

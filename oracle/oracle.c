@@ -1,0 +1,362 @@
+/*
+ * CPU oracle of one PRISM draft round.
+ *
+ * TEST INFRASTRUCTURE ONLY.  The tests, the smoke check and the benchmark's
+ * CPU-baseline leg may call it; the CUDA path never does, and the two share
+ * no code.  Arithmetic is IEEE double throughout (fp64), with no blocking,
+ * fusion or reordering: every dot product is one left-to-right loop.
+ *
+ * What it computes (PRISM, Sec. 3.2 "Draft with PRISM", notation of Table 2):
+ *   step 1 (prefill): for each accepted token x_i with its target hidden
+ *     state, the fused input F_{f_map(1)}(E(x_i), h) passes through the
+ *     transformer layer L_{f_map(1)} with causal attention over the draft KV
+ *     cache; the last output row is h^_0 and x^_1 = argmax LM_head(h^_0).
+ *   steps k = 2..K (decode): H_in = F_{f_map(k)}(E(x^_{k-1}), h^_{k-2});
+ *     h^_{k-1} = L_{f_map(k)}(H_in) with the shared KV cache;
+ *     x^_k = argmax LM_head(h^_{k-1}).
+ *   greedy acceptance (Sec. 2 "Speculative Decoding", the rejection rule at
+ *     temperature 0): the longest prefix on which draft and target agree,
+ *     followed by the target's token at the first disagreement.
+ *
+ * Readings where the paper is silent (each is a reading, not a quote):
+ *   fusion F = one bias-free linear map W_fuse [d, 2d] applied to the
+ *     concatenation [E(x); h] in that order;
+ *   transformer layer = Llama pre-norm block (RMSNorm, grouped-query attention
+ *     with rotate-half RoPE, SwiGLU MLP, no biases), matching the Llama targets
+ *     of Sec. 4;
+ *   an RMSNorm with gain g_final precedes the frozen LM head (switchable);
+ *     the un-normed h^ is what feeds the next step;
+ *   argmax ties go to the lowest token id; top-k lists are sorted by logit
+ *     descending, then id ascending;
+ *   bf16 numeric contract (round_acts = 1): each projection's activation
+ *     operand is rounded to bf16 (nearest even) right before the product, and
+ *     K/V are rounded to the cache's storage type when stored; the residual
+ *     stream, q, scores, softmax and logits are not rounded.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+typedef struct {
+    int32_t hidden, n_q_heads, n_kv_heads, head_dim, ffn, vocab, n_steps;
+    int32_t bf16;        /* 1: weights, E, LM head, hidden inputs and KV cache hold bf16
+                            bit patterns (uint16); 0: they hold float32 */
+    int32_t round_acts;  /* 1: apply the bf16 rounding of projection operands */
+    int32_t final_norm;  /* 1: RMSNorm(h^) * g_final before the LM head */
+    int32_t topk;        /* candidates reported per step (>= 1) */
+    int32_t max_ctx;     /* cache capacity in positions */
+    double rope_theta, rms_eps;
+} orc_config;
+
+typedef struct {
+    const void *w_fuse;    /* [d, 2d] */
+    const void *g_attn;    /* [d] */
+    const void *w_qkv;     /* [(Hq + 2 Hkv) D, d]: q rows, then k rows, then v rows */
+    const void *w_o;       /* [d, Hq D] */
+    const void *g_mlp;     /* [d] */
+    const void *w_gate_up; /* [2F, d]: gate rows [0, F), up rows [F, 2F) */
+    const void *w_down;    /* [d, F] */
+    const void *g_final;   /* [d] */
+} orc_module;
+
+/* ---------------------------------------------------------------- scalars */
+
+static double bf16_bits_to_double(uint16_t h) {
+    uint32_t u = (uint32_t)h << 16;
+    float f;
+    memcpy(&f, &u, 4);
+    return (double)f;
+}
+
+/* Round a double to the nearest bf16 value (ties to even), for values in the
+ * normal float range.  bf16 keeps 7 explicit mantissa bits of the 52. */
+double orc_round_bf16(double x) {
+    uint64_t u;
+    memcpy(&u, &x, 8);
+    uint64_t keep_lsb = (u >> 45) & 1u;
+    u += 0x00000FFFFFFFFFFFULL + keep_lsb;
+    u &= ~0x00001FFFFFFFFFFFULL;
+    memcpy(&x, &u, 8);
+    return x;
+}
+
+static uint16_t double_to_bf16_bits(double x) {
+    float f = (float)orc_round_bf16(x); /* exact: the value already has 8 significant bits */
+    uint32_t u;
+    memcpy(&u, &f, 4);
+    return (uint16_t)(u >> 16);
+}
+
+static double load_el(const void *p, int64_t i, int bf16) {
+    return bf16 ? bf16_bits_to_double(((const uint16_t *)p)[i]) : (double)((const float *)p)[i];
+}
+
+static void store_el(void *p, int64_t i, int bf16, double v) {
+    if (bf16)
+        ((uint16_t *)p)[i] = double_to_bf16_bits(v);
+    else
+        ((float *)p)[i] = (float)v;
+}
+
+static void round_vec(double *v, int64_t n, int on) {
+    if (!on) return;
+    for (int64_t i = 0; i < n; ++i) v[i] = orc_round_bf16(v[i]);
+}
+
+/* ---------------------------------------------------------------- ops */
+
+/* y[r] = sum_c W[r, c] x[c], W row-major [rows, cols]. */
+void orc_matvec(const void *W, int bf16, int64_t rows, int64_t cols, const double *x, double *y) {
+#pragma omp parallel for schedule(static) if (rows * cols > (1 << 16))
+    for (int64_t r = 0; r < rows; ++r) {
+        double acc = 0.0;
+        const int64_t base = r * cols;
+        for (int64_t c = 0; c < cols; ++c) acc += load_el(W, base + c, bf16) * x[c];
+        y[r] = acc;
+    }
+}
+
+/* RMSNorm: out = x / sqrt(mean(x^2) + eps) * g. */
+void orc_rmsnorm(const double *x, const double *g, int64_t n, double eps, double *out) {
+    double ss = 0.0;
+    for (int64_t i = 0; i < n; ++i) ss += x[i] * x[i];
+    double inv = 1.0 / sqrt(ss / (double)n + eps);
+    for (int64_t i = 0; i < n; ++i) out[i] = x[i] * inv * g[i];
+}
+
+/* Rotary position embedding of one head vector at position pos, rotate-half
+ * pairing (j, j + D/2) with angle pos * theta^(-2j/D). */
+void orc_rope(double *v, int32_t D, int64_t pos, double theta) {
+    int32_t half = D / 2;
+    for (int32_t j = 0; j < half; ++j) {
+        double ang = (double)pos * pow(theta, -2.0 * (double)j / (double)D);
+        double c = cos(ang), s = sin(ang);
+        double a = v[j], b = v[j + half];
+        v[j] = a * c - b * s;
+        v[j + half] = b * c + a * s;
+    }
+}
+
+/* Softmax attention of one query head over positions [0, n_pos) of one KV
+ * head: scores (q . k_j) / sqrt(D), softmax over j, weighted sum of v_j.
+ * kv rows are row_stride elements apart in storage of the given type. */
+void orc_attend(const double *q, const void *kc, const void *vc, int bf16, int64_t row_stride,
+                int64_t n_pos, int32_t D, double *o) {
+    double *s = (double *)malloc(sizeof(double) * (size_t)(n_pos > 0 ? n_pos : 1));
+    double scale = 1.0 / sqrt((double)D);
+    double mx = -INFINITY;
+    for (int64_t j = 0; j < n_pos; ++j) {
+        double dot = 0.0;
+        for (int32_t t = 0; t < D; ++t) dot += q[t] * load_el(kc, j * row_stride + t, bf16);
+        s[j] = dot * scale;
+        if (s[j] > mx) mx = s[j];
+    }
+    double den = 0.0;
+    for (int64_t j = 0; j < n_pos; ++j) {
+        s[j] = exp(s[j] - mx);
+        den += s[j];
+    }
+    for (int32_t t = 0; t < D; ++t) o[t] = 0.0;
+    for (int64_t j = 0; j < n_pos; ++j)
+        for (int32_t t = 0; t < D; ++t) o[t] += s[j] * load_el(vc, j * row_stride + t, bf16);
+    for (int32_t t = 0; t < D; ++t) o[t] /= den;
+    free(s);
+}
+
+static double silu(double t) { return t / (1.0 + exp(-t)); }
+
+/* ---------------------------------------------------------------- layer */
+
+typedef struct {
+    double *x0, *n1, *qkv, *o, *a, *n2, *gu, *mm, *y;
+    double *g_attn, *g_mlp, *g_final;
+} scratch;
+
+static void widen(const void *p, int bf16, int64_t n, double *out) {
+    for (int64_t i = 0; i < n; ++i) out[i] = load_el(p, i, bf16);
+}
+
+/* One row through fusion + transformer layer of module m at cache position
+ * pos.  u = [E(x); h] (already rounded per the contract).  Writes this row's
+ * K/V at pos of sequence b's cache and the layer output to y. */
+static void layer_row(const orc_config *c, const orc_module *m, const double *u, int64_t pos,
+                      void *kc_b, void *vc_b, scratch *w) {
+    const int64_t d = c->hidden, Hq = c->n_q_heads, Hkv = c->n_kv_heads, D = c->head_dim, F = c->ffn;
+    const int bf = c->bf16, ra = c->round_acts;
+    const int64_t group = Hq / Hkv;
+
+    /* fusion F_i(E(x), h) */
+    orc_matvec(m->w_fuse, bf, d, 2 * d, u, w->x0);
+
+    /* attention sub-block */
+    widen(m->g_attn, bf, d, w->g_attn);
+    orc_rmsnorm(w->x0, w->g_attn, d, c->rms_eps, w->n1);
+    round_vec(w->n1, d, ra);
+    orc_matvec(m->w_qkv, bf, (Hq + 2 * Hkv) * D, d, w->n1, w->qkv);
+    double *q = w->qkv, *k = w->qkv + Hq * D, *v = w->qkv + (Hq + Hkv) * D;
+    for (int64_t h = 0; h < Hq; ++h) orc_rope(q + h * D, (int32_t)D, pos, c->rope_theta);
+    for (int64_t g = 0; g < Hkv; ++g) orc_rope(k + g * D, (int32_t)D, pos, c->rope_theta);
+    for (int64_t g = 0; g < Hkv; ++g)
+        for (int64_t t = 0; t < D; ++t) {
+            int64_t idx = (g * c->max_ctx + pos) * D + t;
+            store_el(kc_b, idx, bf, k[g * D + t]);
+            store_el(vc_b, idx, bf, v[g * D + t]);
+        }
+#pragma omp parallel for schedule(static) if (pos > 256)
+    for (int64_t h = 0; h < Hq; ++h) {
+        int64_t g = h / group;
+        const char *kb = (const char *)kc_b + (size_t)(g * c->max_ctx * D) * (bf ? 2 : 4);
+        const char *vb = (const char *)vc_b + (size_t)(g * c->max_ctx * D) * (bf ? 2 : 4);
+        orc_attend(q + h * D, kb, vb, bf, D, pos + 1, (int32_t)D, w->o + h * D);
+    }
+    round_vec(w->o, Hq * D, ra);
+    orc_matvec(m->w_o, bf, d, Hq * D, w->o, w->a);
+    for (int64_t i = 0; i < d; ++i) w->a[i] += w->x0[i];
+
+    /* MLP sub-block */
+    widen(m->g_mlp, bf, d, w->g_mlp);
+    orc_rmsnorm(w->a, w->g_mlp, d, c->rms_eps, w->n2);
+    round_vec(w->n2, d, ra);
+    orc_matvec(m->w_gate_up, bf, 2 * F, d, w->n2, w->gu);
+    for (int64_t j = 0; j < F; ++j) w->mm[j] = silu(w->gu[j]) * w->gu[F + j];
+    round_vec(w->mm, F, ra);
+    orc_matvec(m->w_down, bf, d, F, w->mm, w->y);
+    for (int64_t i = 0; i < d; ++i) w->y[i] += w->a[i];
+}
+
+/* ---------------------------------------------------------------- selection */
+
+static const double *g_sort_keys;
+static int cmp_desc(const void *pa, const void *pb) {
+    int32_t a = *(const int32_t *)pa, b = *(const int32_t *)pb;
+    double va = g_sort_keys[a], vb = g_sort_keys[b];
+    if (va > vb) return -1;
+    if (va < vb) return 1;
+    return (a > b) - (a < b);
+}
+
+/* LM head on h^ (after the optional final RMSNorm) and top-k selection. */
+static void select_tokens(const orc_config *c, const void *lm_head, const orc_module *m,
+                          const double *h, double *z, int32_t *order, scratch *w,
+                          int32_t *top_ids, double *top_vals) {
+    const int64_t d = c->hidden, V = c->vocab;
+    double *nf = w->n1; /* reuse */
+    if (c->final_norm) {
+        widen(m->g_final, c->bf16, d, w->g_final);
+        orc_rmsnorm(h, w->g_final, d, c->rms_eps, nf);
+    } else {
+        memcpy(nf, h, sizeof(double) * (size_t)d);
+    }
+    round_vec(nf, d, c->round_acts);
+    orc_matvec(lm_head, c->bf16, V, d, nf, z);
+    for (int32_t i = 0; i < V; ++i) order[i] = i;
+    g_sort_keys = z;
+    qsort(order, (size_t)V, sizeof(int32_t), cmp_desc);
+    for (int32_t r = 0; r < c->topk; ++r) {
+        top_ids[r] = order[r];
+        top_vals[r] = z[order[r]];
+    }
+}
+
+/* ---------------------------------------------------------------- round */
+
+/* Returns 0 on success; 1 bad argument; 2 token id out of range; 3 cache
+ * capacity exceeded (kv_len + n_new + K - 1 > max_ctx).
+ * steps[k] is the module of draft step k+1 (the surjection f_map applied).
+ * Outputs: draft_ids [B, K]; topk_ids/topk_logits [B, K, topk];
+ * logits [B, K, V] and hidden_out [B, K, d] when non-NULL. */
+int orc_draft_round(const orc_config *c, const void *embed, const void *lm_head,
+                    const orc_module *steps, int32_t B, int32_t max_new,
+                    const int32_t *tokens, const void *hidden, const int32_t *n_new,
+                    const int32_t *kv_len, void *k_cache, void *v_cache,
+                    int32_t *draft_ids, int32_t *topk_ids, double *topk_logits,
+                    double *logits, double *hidden_out) {
+    const int64_t d = c->hidden, V = c->vocab, K = c->n_steps, F = c->ffn;
+    const int64_t Hq = c->n_q_heads, Hkv = c->n_kv_heads, D = c->head_dim;
+    const int bf = c->bf16;
+    if (K < 1 || c->topk < 1 || c->topk > V || Hq % Hkv != 0 || D % 2 != 0) return 1;
+    for (int32_t b = 0; b < B; ++b) {
+        if (n_new[b] < 1 || n_new[b] > max_new || kv_len[b] < 0) return 1;
+        if ((int64_t)kv_len[b] + n_new[b] + K - 1 > c->max_ctx) return 3;
+        for (int32_t i = 0; i < n_new[b]; ++i)
+            if (tokens[b * max_new + i] < 0 || tokens[b * max_new + i] >= V) return 2;
+    }
+    scratch w;
+    w.x0 = calloc((size_t)d, 8); w.n1 = calloc((size_t)d, 8);
+    w.qkv = calloc((size_t)((Hq + 2 * Hkv) * D), 8); w.o = calloc((size_t)(Hq * D), 8);
+    w.a = calloc((size_t)d, 8); w.n2 = calloc((size_t)d, 8);
+    w.gu = calloc((size_t)(2 * F), 8); w.mm = calloc((size_t)F, 8); w.y = calloc((size_t)d, 8);
+    w.g_attn = calloc((size_t)d, 8); w.g_mlp = calloc((size_t)d, 8); w.g_final = calloc((size_t)d, 8);
+    double *u = calloc((size_t)(2 * d), 8), *hhat = calloc((size_t)d, 8);
+    double *z = calloc((size_t)V, 8);
+    int32_t *order = calloc((size_t)V, 4);
+    int32_t *tid = calloc((size_t)c->topk, 4);
+    double *tval = calloc((size_t)c->topk, 8);
+    const size_t el = bf ? 2 : 4;
+    const int64_t cache_seq = Hkv * (int64_t)c->max_ctx * D;
+
+    for (int32_t b = 0; b < B; ++b) {
+        void *kc_b = (char *)k_cache + (size_t)(b * cache_seq) * el;
+        void *vc_b = (char *)v_cache + (size_t)(b * cache_seq) * el;
+        const int64_t L = kv_len[b], n = n_new[b];
+        int32_t prev = -1;
+        for (int64_t k = 1; k <= K; ++k) {
+            const orc_module *m = &steps[k - 1];
+            if (k == 1) {
+                /* prefill: rows x_1..x_n with their hidden states, positions L..L+n-1 */
+                for (int64_t i = 0; i < n; ++i) {
+                    int32_t x = tokens[b * max_new + i];
+                    for (int64_t t = 0; t < d; ++t) {
+                        u[t] = load_el(embed, (int64_t)x * d + t, bf);
+                        u[d + t] = load_el(hidden, ((int64_t)b * max_new + i) * d + t, bf);
+                    }
+                    round_vec(u, 2 * d, c->round_acts);
+                    layer_row(c, m, u, L + i, kc_b, vc_b, &w);
+                }
+            } else {
+                for (int64_t t = 0; t < d; ++t) {
+                    u[t] = load_el(embed, (int64_t)prev * d + t, bf);
+                    u[d + t] = hhat[t];
+                }
+                round_vec(u, 2 * d, c->round_acts);
+                layer_row(c, m, u, L + n + k - 2, kc_b, vc_b, &w);
+            }
+            memcpy(hhat, w.y, sizeof(double) * (size_t)d);
+            select_tokens(c, lm_head, m, hhat, z, order, &w, tid, tval);
+            prev = tid[0];
+            draft_ids[b * K + (k - 1)] = prev;
+            for (int32_t r = 0; r < c->topk; ++r) {
+                if (topk_ids) topk_ids[(b * K + (k - 1)) * c->topk + r] = tid[r];
+                if (topk_logits) topk_logits[(b * K + (k - 1)) * c->topk + r] = tval[r];
+            }
+            if (logits) memcpy(logits + (b * K + (k - 1)) * V, z, sizeof(double) * (size_t)V);
+            if (hidden_out) memcpy(hidden_out + (b * K + (k - 1)) * d, hhat, sizeof(double) * (size_t)d);
+        }
+    }
+    free(w.x0); free(w.n1); free(w.qkv); free(w.o); free(w.a); free(w.n2); free(w.gu);
+    free(w.mm); free(w.y); free(w.g_attn); free(w.g_mlp); free(w.g_final);
+    free(u); free(hhat); free(z); free(order); free(tid); free(tval);
+    return 0;
+}
+
+/* Greedy acceptance (temperature 0).  accept_len[b] = largest a in [0, K]
+ * with draft[b, j] == target[b, j] for all j < a; out_tokens[b] =
+ * draft[b, 0:a] followed by target[b, a], the rest -1; kv_len[b] += n_new[b]
+ * (only the step-1 rows are committed; draft-step rows are scratch). */
+void orc_accept_greedy(int32_t B, int32_t K, const int32_t *draft, const int32_t *target,
+                       const int32_t *n_new, int32_t *kv_len, int32_t *accept_len,
+                       int32_t *out_tokens) {
+    for (int32_t b = 0; b < B; ++b) {
+        int32_t a = 0;
+        while (a < K && draft[b * K + a] == target[b * (K + 1) + a]) ++a;
+        accept_len[b] = a;
+        for (int32_t j = 0; j <= K; ++j) {
+            int32_t v = -1;
+            if (j < a) v = draft[b * K + j];
+            else if (j == a) v = target[b * (K + 1) + a];
+            out_tokens[b * (K + 1) + j] = v;
+        }
+        kv_len[b] += n_new[b];
+    }
+}
