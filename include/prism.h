@@ -1,0 +1,189 @@
+/*
+ * prism.h -- C ABI of a GB300 (sm_103a) implementation of the PRISM draft round.
+ *
+ * PRISM (Parametrically Refactoring Inference for Speculative sampling draft
+ * Models) drafts K tokens per round; draft step k runs its own processing
+ * module (a fully connected fusion layer plus one transformer layer) chosen by
+ * a surjection f_map from steps to modules, with a token embedding E and a
+ * vocabulary head LM_head shared by all steps and one KV cache shared by all
+ * modules (Sec. 3.2, Table 2).  The round is followed by verification; this
+ * library implements its temperature-0 acceptance rule (Sec. 2).
+ *
+ * Conventions for every entry point:
+ *   - All tensor arguments are DEVICE pointers on the context's device,
+ *     row-major and densely packed, owned by the caller.  Weight, embedding,
+ *     LM-head, hidden-state and cache pointers must be 16-byte aligned
+ *     (checked: PRISM_ERR_INVALID_ARG).  Weight pointers are
+ *     borrowed: they must stay valid until the context is destroyed or the
+ *     weights are replaced.  The library owns only its workspace, allocated in
+ *     prism_create and freed in prism_destroy.
+ *   - "wtype" below is the configuration's dtype: PRISM_BF16 (bf16 bit
+ *     patterns) or PRISM_F32 (float32).  Weights, E, LM head, target hidden
+ *     states and the KV cache all use wtype.
+ *   - Work is enqueued asynchronously on `stream` (a cudaStream_t, passed as
+ *     void*; NULL is the legacy default stream).  Nothing synchronises unless
+ *     stated.
+ *   - Every function returns a prism_status and never throws across the ABI.
+ *     Conditions the host can check (null pointers, sizes, unloaded weights)
+ *     are reported before anything is enqueued.  Conditions only the device
+ *     can see (a token id outside [0, vocab), a cache position outside
+ *     [0, max_ctx), n_new outside [1, max_new]) set a device error word; the
+ *     kernels clamp and carry on without trapping, and prism_sync_status
+ *     reports PRISM_ERR_DEVICE_FLAG.
+ *   - prism_get_error returns a message for the last failing call on the
+ *     context (valid until the next call).
+ */
+#ifndef PRISM_H_
+#define PRISM_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    PRISM_OK = 0,
+    PRISM_ERR_INVALID_ARG = 1,  /* null pointer, bad enum, bad option */
+    PRISM_ERR_SHAPE = 2,        /* sizes inconsistent with the configuration */
+    PRISM_ERR_CAPACITY = 3,     /* batch above max_batch, and similar host-visible limits */
+    PRISM_ERR_NOT_LOADED = 4,   /* shared or step weights missing */
+    PRISM_ERR_CUDA = 5,         /* a CUDA runtime call failed; see prism_get_error */
+    PRISM_ERR_OOM = 6,          /* workspace allocation failed */
+    PRISM_ERR_DEVICE_FLAG = 7,  /* the device error word was set (see prism_sync_status) */
+    PRISM_ERR_TIMEOUT = 8       /* a bounded device-side wait gave up */
+} prism_status;
+
+typedef enum { PRISM_F32 = 0, PRISM_BF16 = 1 } prism_dtype;
+
+/* Device error word bits (reported by prism_sync_status). */
+#define PRISM_DEVERR_TOKEN_RANGE 1   /* a token id outside [0, vocab) was clamped */
+#define PRISM_DEVERR_CACHE_RANGE 2   /* a cache position outside [0, max_ctx) was skipped */
+#define PRISM_DEVERR_NNEW_RANGE 4    /* n_new[b] outside [1, max_new] was clamped */
+#define PRISM_DEVERR_TIMEOUT 8       /* a bounded wait expired */
+
+/* Model and capacity description.  hidden = d, n_q_heads = Hq, n_kv_heads =
+ * Hkv (Hq % Hkv == 0), head_dim = D (64 or 128), ffn = F, vocab = V,
+ * n_steps = K (1..16) draft steps per round.  max_batch, max_ctx (cache
+ * positions per sequence) and max_new (accepted tokens per sequence fed to
+ * step 1) size the workspace.  topk in 1..8 candidates are reported per step
+ * (the chained token is the first).  final_norm: 1 applies RMSNorm with the
+ * step's g_final before the LM head.  rope_theta and rms_eps as in Llama. */
+typedef struct {
+    int32_t hidden, n_q_heads, n_kv_heads, head_dim, ffn, vocab, n_steps;
+    int32_t dtype;
+    int32_t max_batch, max_ctx, max_new, topk;
+    float rope_theta, rms_eps;
+    int32_t final_norm;
+} prism_config;
+
+/* One processing module (Sec. 3.2: a fully connected fusion layer and a
+ * transformer layer), all wtype, row-major:
+ *   w_fuse    [d, 2d]      fusion F(E(x), h) = w_fuse . [E(x); h]
+ *   g_attn    [d]          RMSNorm gain before attention
+ *   w_qkv     [(Hq + 2 Hkv) D, d]   q rows, then k rows, then v rows
+ *   w_o       [d, Hq D]
+ *   g_mlp     [d]          RMSNorm gain before the MLP
+ *   w_gate_up [2F, d]      gate rows [0, F), up rows [F, 2F); SwiGLU
+ *   w_down    [d, F]
+ *   g_final   [d]          RMSNorm gain before the LM head (if final_norm) */
+typedef struct {
+    const void *w_fuse, *g_attn, *w_qkv, *w_o, *g_mlp, *w_gate_up, *w_down, *g_final;
+} prism_step_weights;
+
+typedef struct prism_ctx prism_ctx;
+
+/* Create a context on CUDA device `device` and allocate its workspace.
+ * Errors: INVALID_ARG (null out, unsupported sizes), OOM, CUDA. */
+prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **out);
+
+/* Destroy a context; waits for its work to finish.  NULL is a no-op. */
+prism_status prism_destroy(prism_ctx *ctx);
+
+/* Token embedding E [V, d] and LM head [V, d] (both frozen and shared by all
+ * steps, Table 2).  Borrowed.  Errors: INVALID_ARG (null). */
+prism_status prism_load_shared_weights(prism_ctx *ctx, const void *embed, const void *lm_head);
+
+/* Bind the module used by draft step `step` (0-based, 0..K-1).  The surjection
+ * f_map of Table 2 is expressed by binding the same pointers to several steps.
+ * Borrowed.  Errors: INVALID_ARG (null field, step out of range). */
+prism_status prism_load_step_weights(prism_ctx *ctx, int32_t step, const prism_step_weights *w);
+
+/* One draft round (Sec. 3.2 "Draft with PRISM") for `batch` independent
+ * sequences:
+ *   step 1: each sequence b's n_new[b] accepted tokens tokens[b, i] with
+ *     their target hidden states hidden[b, i] (i < n_new[b]) are fused and
+ *     run through step 1's transformer layer at cache positions
+ *     kv_len[b] + i with causal attention; the last row is h^_0 and
+ *     x^_1 = argmax LM_head(h^_0).
+ *   step k = 2..K: fuse E(x^_{k-1}) with h^_{k-2}, run step k's layer at
+ *     position kv_len[b] + n_new[b] + k - 2, x^_k = argmax LM_head(h^_{k-1}).
+ * Arguments (device pointers):
+ *   tokens      int32 [batch, max_new]        rows past n_new[b] are ignored
+ *   hidden      wtype [batch, max_new, d]
+ *   n_new       int32 [batch]                 1..max_new
+ *   kv_len      int32 [batch]                 committed cache length L_b (read only)
+ *   k_cache, v_cache  wtype [max_batch, Hkv, max_ctx, D]  read and written:
+ *               rows kv_len[b] .. kv_len[b] + n_new[b] + K - 2 are written
+ *   draft_ids   int32 [batch, K]              out
+ *   topk_ids    int32 [batch, K, topk]        out, or NULL
+ *   topk_logits float [batch, K, topk]        out, or NULL
+ *   logits      float [batch, K, V]           out, or NULL
+ *   hidden_out  float [batch, K, d]           out (h^_0 .. h^_{K-1}), or NULL
+ * Ties in the argmax go to the lowest id; top-k is sorted by logit, then id.
+ * The round is captured once per distinct argument set as a CUDA graph and
+ * replayed (option "use_graph").  Errors: INVALID_ARG, CAPACITY
+ * (batch > max_batch), NOT_LOADED, CUDA. */
+prism_status prism_draft_round(prism_ctx *ctx, int32_t batch, const int32_t *tokens,
+                               const void *hidden, const int32_t *n_new, const int32_t *kv_len,
+                               void *k_cache, void *v_cache, int32_t *draft_ids,
+                               int32_t *topk_ids, float *topk_logits, float *logits,
+                               float *hidden_out, void *stream);
+
+/* Greedy (temperature 0) acceptance, Sec. 2: accept_len[b] is the largest a
+ * in [0, K] with draft[b, j] == target[b, j] for all j < a; out_tokens[b] is
+ * draft[b, 0:a] followed by target[b, a] (the corrected or bonus token), then
+ * -1 padding; kv_len[b] += n_new[b] commits the step-1 rows (draft rows are
+ * scratch and are overwritten by the next round).
+ *   draft int32 [batch, K], target int32 [batch, K+1], n_new int32 [batch],
+ *   kv_len int32 [batch] in/out, accept_len int32 [batch] out,
+ *   out_tokens int32 [batch, K+1] out.
+ * Errors: INVALID_ARG, CAPACITY, CUDA. */
+prism_status prism_accept_greedy(prism_ctx *ctx, int32_t batch, const int32_t *draft,
+                                 const int32_t *target, const int32_t *n_new, int32_t *kv_len,
+                                 int32_t *accept_len, int32_t *out_tokens, void *stream);
+
+/* Synchronise `stream`, read and clear the device error word.  Returns
+ * PRISM_ERR_DEVICE_FLAG (bits in *flags if non-NULL) when it was set,
+ * PRISM_ERR_CUDA when the stream reports an error, PRISM_OK otherwise. */
+prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
+
+/* Options (name, value): "use_graph" (1: capture and replay, default 1),
+ * "use_pdl" (1: programmatic dependent launch between kernels, default 1).
+ * Changing an option drops cached graphs.  Errors: INVALID_ARG. */
+prism_status prism_set_option(prism_ctx *ctx, const char *name, int32_t value);
+
+/* Instrumented round for measurement: the same work as prism_draft_round
+ * launched eagerly with a CUDA event recorded before and after every kernel.
+ * kernel_ms[i] receives the duration of kernel i in launch order (capacity
+ * max_kernels); *n_kernels receives the count; kernel_kind[i] (may be NULL)
+ * receives a code: 0 fusion, 1 qkv, 2 rope/append, 3 attention, 4 o-proj,
+ * 5 gate/up, 6 down, 7 LM head + selection.  Synchronises the stream. */
+prism_status prism_profile_round(prism_ctx *ctx, int32_t batch, const int32_t *tokens,
+                                 const void *hidden, const int32_t *n_new, const int32_t *kv_len,
+                                 void *k_cache, void *v_cache, int32_t *draft_ids,
+                                 int32_t *topk_ids, float *topk_logits, void *stream,
+                                 float *kernel_ms, int32_t *kernel_kind, int32_t max_kernels,
+                                 int32_t *n_kernels);
+
+/* Message for the last failing call on ctx (or a global message when ctx is NULL). */
+const char *prism_get_error(const prism_ctx *ctx);
+
+/* Library version string. */
+const char *prism_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PRISM_H_ */

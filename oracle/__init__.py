@@ -65,6 +65,9 @@ def _bind(path: str):
                                     i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.orc_draft_round.restype = ctypes.c_int
     lib.orc_accept_greedy.argtypes = [i32, i32, vp, vp, vp, vp, vp, vp]
+    lib.orc_num_threads.restype = ctypes.c_int
+    lib.orc_round_bf16_bits.argtypes = [vp, i64, vp]
+    lib.orc_round_bf16_bits.restype = None
     for f in (lib.orc_matvec, lib.orc_rmsnorm, lib.orc_rope, lib.orc_attend, lib.orc_accept_greedy):
         f.restype = None
     return lib
@@ -111,6 +114,19 @@ def _c(a, dtype):
 
 def round_bf16(x: float) -> float:
     return float(_load().orc_round_bf16(float(x)))
+
+
+def num_threads() -> int:
+    """Threads used by the oracle's parallel loops (OpenMP)."""
+    return int(_load().orc_num_threads())
+
+
+def to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round fp64 values to bf16 bit patterns (uint16) with the oracle's rule."""
+    x = _c(x, np.float64)
+    out = np.empty(x.shape, dtype=np.uint16)
+    _load().orc_round_bf16_bits(x.ctypes.data, x.size, out.ctypes.data)
+    return out
 
 
 def matvec(W: np.ndarray, x: np.ndarray) -> np.ndarray:

@@ -34,6 +34,7 @@
  *     stream, q, scores, softmax and logits are not rounded.
  */
 #include <math.h>
+#include <omp.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -86,6 +87,14 @@ static uint16_t double_to_bf16_bits(double x) {
     uint32_t u;
     memcpy(&u, &f, 4);
     return (uint16_t)(u >> 16);
+}
+
+/* Threads the oracle's parallel loops use. */
+int orc_num_threads(void) { return omp_get_max_threads(); }
+
+/* Round an array of doubles to bf16 bit patterns (nearest even). */
+void orc_round_bf16_bits(const double *x, int64_t n, uint16_t *out) {
+    for (int64_t i = 0; i < n; ++i) out[i] = double_to_bf16_bits(x[i]);
 }
 
 static double load_el(const void *p, int64_t i, int bf16) {

@@ -1,0 +1,219 @@
+// Device helpers and launch interfaces shared by the PRISM draft-round kernels
+// (sm_103a).  Internal to the library; the public ABI is include/prism.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace prism {
+
+constexpr int kMaxSteps = 16;
+constexpr int kTopK = 8;          // every selection keeps a sorted top-8 list
+constexpr int kGemvThreads = 512; // 16 warps per projection CTA
+constexpr int kGemvWarps = kGemvThreads / 32;
+constexpr int kAttnThreads = 128;
+
+enum DevErr : int {
+    kErrToken = 1,
+    kErrCache = 2,
+    kErrNNew = 4,
+    kErrTimeout = 8,
+};
+
+// ----------------------------------------------------------------- PTX helpers
+
+// Programmatic dependent launch: let the next kernel in the stream start its
+// independent prologue (weight prefetch) while this one runs; and wait until
+// every prerequisite grid has completed and its writes are visible.
+__device__ __forceinline__ void pdl_trigger() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// Bulk (TMA-engine) prefetch of a contiguous byte range into L2.  Address and
+// size must be multiples of 16 bytes.
+__device__ __forceinline__ void prefetch_l2_bulk(const void *p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+// 128-bit streaming load of read-only data: not kept in L1.
+__device__ __forceinline__ uint4 ldg_stream(const uint4 *p) {
+    uint4 r;
+    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+        : "l"(p));
+    return r;
+}
+
+// ----------------------------------------------------------------- bf16
+
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+__device__ __forceinline__ float bf16_to_f32(uint16_t h) { return __uint_as_float((uint32_t)h << 16); }
+
+// float -> bf16 bits, round to nearest even (finite inputs).
+__device__ __forceinline__ uint16_t f32_to_bf16(float f) {
+    uint32_t u = __float_as_uint(f);
+    u += 0x7FFFu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+__device__ __forceinline__ float round_bf16(float f) {
+    return __uint_as_float((uint32_t)f32_to_bf16(f) << 16);
+}
+
+// Element access for the two storage types (uint16_t = bf16 bits, float).
+template <typename T> struct Elem;
+template <> struct Elem<uint16_t> {
+    static constexpr int kPerVec = 8;  // elements per 16-byte vector
+    __device__ static float load(const uint16_t *p, int64_t i) { return bf16_to_f32(p[i]); }
+    __device__ static void store(uint16_t *p, int64_t i, float v) { p[i] = f32_to_bf16(v); }
+    __device__ static float round(float v) { return round_bf16(v); }
+};
+template <> struct Elem<float> {
+    static constexpr int kPerVec = 4;
+    __device__ static float load(const float *p, int64_t i) { return p[i]; }
+    __device__ static void store(float *p, int64_t i, float v) { p[i] = v; }
+    __device__ static float round(float v) { return v; }
+};
+
+__device__ __forceinline__ void set_err(int *err, int bit) {
+    if (err) atomicOr(err, bit);
+}
+
+// Top-8 ordering: larger logit first, then lower id.
+__device__ __forceinline__ bool better(float a, int ia, float b, int ib) {
+    return a > b || (a == b && ia < ib);
+}
+
+// Insert (v, id) into a descending top-8 list held in registers.
+__device__ __forceinline__ void top8_insert(float (&vals)[kTopK], int (&ids)[kTopK], float v, int id) {
+    if (!better(v, id, vals[kTopK - 1], ids[kTopK - 1])) return;
+    vals[kTopK - 1] = v;
+    ids[kTopK - 1] = id;
+#pragma unroll
+    for (int i = kTopK - 1; i > 0; --i) {
+        if (better(vals[i], ids[i], vals[i - 1], ids[i - 1])) {
+            float tv = vals[i]; vals[i] = vals[i - 1]; vals[i - 1] = tv;
+            int ti = ids[i]; ids[i] = ids[i - 1]; ids[i - 1] = ti;
+        }
+    }
+}
+
+__device__ __forceinline__ void top8_init(float (&vals)[kTopK], int (&ids)[kTopK]) {
+#pragma unroll
+    for (int i = 0; i < kTopK; ++i) { vals[i] = -INFINITY; ids[i] = 0x7FFFFFFF; }
+}
+
+// ----------------------------------------------------------------- launches
+
+// Projection kinds (weight-streaming GEMV family).
+enum ProKind : int {
+    kProFusePrefill = 0,  // X[t] = [E(tokens[b,i]); hidden[b,i]]
+    kProFuseDecode = 1,   // X[b] = [E(draft[b,k-2]); round(h^[b])]
+    kProNorm = 2,         // X[t] = round(RMSNorm(src[t]) * g) (or round(src[t]) without norm)
+    kProCopy = 3,         // X[t] = act[t] (already rounded, wtype)
+};
+enum EpiKind : int {
+    kEpiStore = 0,   // out[t, r] = acc
+    kEpiResid = 1,   // out[t, r] = resid[row(t), r] + acc
+    kEpiSwiGLU = 2,  // out_act[t, j] = round(silu(acc_gate) * acc_up)
+    kEpiTopK = 3,    // logits (optional) + top-8 selection
+};
+
+struct GemvArgs {
+    const void *W;        // [rows, kin] wtype
+    int n_units;          // output units (rows; gate/up pairs for SwiGLU)
+    int kin;              // contraction length
+    int pair_offset;      // row offset of the second row of a unit (SwiGLU: F)
+    int T;                // activation rows
+    int pro, epi;
+    // prologue sources
+    const void *embed;       // [V, d]
+    const int32_t *tokens;   // [B, max_new]
+    const void *hidden_in;   // [B, max_new, d] wtype
+    const int32_t *draft;    // [B, K]
+    const float *src;        // fp32 rows [*, d] (norm source, or h^ for decode fusion)
+    int src_prefill_rows;    // norm source rows are the last prefill row of each sequence
+    const void *act;         // [T, kin] wtype (copy source)
+    const void *gain;        // [d] wtype, or null (no norm)
+    float eps;
+    const int32_t *n_new;
+    int max_new, K, step, vocab, d;
+    // epilogue
+    float *out;              // fp32 [T, out_ld]
+    int out_ld;
+    void *out_act;           // wtype [T, out_ld] (SwiGLU)
+    const float *resid;      // fp32 residual rows
+    int resid_prefill_rows;  // residual row = b*max_new + n_new[b]-1
+    float *hidden_out;       // [B, K, d] or null (down projection)
+    float *logits;           // [B, K, V] or null (LM head)
+    float *lm_part;          // [T, grid, 8] values (LM head)
+    int *lm_part_id;         // [T, grid, 8] ids
+    int *counter;            // LM head last-CTA counter
+    int32_t *draft_out;      // [B, K]
+    int32_t *topk_ids;       // [B, K, topk] or null
+    float *topk_logits;      // [B, K, topk] or null
+    int topk;
+    int *err;
+};
+
+struct RopeArgs {
+    const float *qkv;       // [rows, (Hq + 2Hkv) D]
+    void *k_cache, *v_cache;
+    float *q_out;           // [B, Hq, D]
+    const float *rope_cos, *rope_sin;  // [max_ctx, D/2]
+    const int32_t *n_new, *kv_len;
+    int B, max_new, rows, prefill, step, K;
+    int Hq, Hkv, D, max_ctx;
+    int *err;
+};
+
+struct AttnArgs {
+    const float *q;          // [B, Hq, D] (rotated)
+    const void *k_cache, *v_cache;
+    float *part;             // [B, Hq, splits, D + 2]
+    int *counter;            // [B * Hkv]
+    void *o_out;             // [B, Hq * D] wtype (rounded operand of the O projection)
+    const int32_t *n_new, *kv_len;
+    int B, max_new, prefill, step, Hq, Hkv, D, max_ctx, chunk, splits;
+    int *err;
+};
+
+struct AcceptArgs {
+    const int32_t *draft, *target, *n_new;
+    int32_t *kv_len, *accept_len, *out_tokens;
+    int B, K;
+};
+
+// Host launchers (return cudaGetLastError of the launch).
+cudaError_t launch_gemv(const GemvArgs &a, bool bf16, int grid, cudaStream_t s, bool pdl);
+size_t gemv_smem_bytes(const GemvArgs &a, bool bf16, int tc);
+int gemv_rows_per_pass(const GemvArgs &a, bool bf16);
+cudaError_t launch_rope_append(const RopeArgs &a, bool bf16, cudaStream_t s, bool pdl);
+cudaError_t launch_attention(const AttnArgs &a, bool bf16, cudaStream_t s, bool pdl);
+cudaError_t launch_accept(const AcceptArgs &a, cudaStream_t s);
+// One-time kernel attribute setup (maximum dynamic shared memory); must run
+// before any stream capture.
+cudaError_t prepare_gemv_kernels();
+cudaError_t prepare_attention_kernel(bool bf16, int D, int chunk, int G);
+size_t attention_smem_bytes(bool bf16, int D, int chunk, int G);
+
+// Launch with optional programmatic stream serialization.
+template <typename Kern, typename... Args>
+cudaError_t launch_k(Kern k, dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, k, args...);
+}
+
+}  // namespace prism

@@ -1,0 +1,578 @@
+// C ABI of the PRISM draft round: context, workspace, validation, the per-step
+// launch sequence and CUDA-graph capture/replay.  See include/prism.h.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/prism.h"
+#include "common.cuh"
+
+using namespace prism;
+
+namespace {
+
+constexpr int kGraphCache = 8;
+constexpr int kMaxProfileKernels = 8 * kMaxSteps + 8;
+
+struct RoundArgs {
+    int B;
+    const int32_t *tokens;
+    const void *hidden;
+    const int32_t *n_new, *kv_len;
+    void *k_cache, *v_cache;
+    int32_t *draft;
+    int32_t *topk_ids;
+    float *topk_logits, *logits, *hidden_out;
+    bool operator==(const RoundArgs &o) const { return std::memcmp(this, &o, sizeof(RoundArgs)) == 0; }
+};
+
+struct GraphEntry {
+    RoundArgs key;
+    bool pdl;
+    cudaGraphExec_t exec;
+    unsigned long long used;
+};
+
+thread_local std::string g_error;
+
+}  // namespace
+
+struct prism_ctx {
+    prism_config cfg{};
+    int device = 0;
+    int sms = 0;
+    bool bf16 = true;
+    int qkv_rows = 0;
+    int lm_grid = 0;
+    int attn_chunk = 64;
+    int attn_splits = 0;
+    // weights (borrowed)
+    const void *embed = nullptr, *lm_head = nullptr;
+    prism_step_weights steps[kMaxSteps]{};
+    bool step_loaded[kMaxSteps]{};
+    // workspace (owned)
+    void *ws = nullptr;
+    size_t ws_bytes = 0;
+    float *rope_cos = nullptr, *rope_sin = nullptr;
+    float *x0 = nullptr, *qkv = nullptr, *q = nullptr, *attn_part = nullptr, *a = nullptr, *hhat = nullptr;
+    void *o_buf = nullptr, *m_buf = nullptr;
+    float *lm_val = nullptr;
+    int *lm_id = nullptr;
+    int *counters = nullptr;  // [max_batch * Hkv] attention + [1] LM head
+    int *err = nullptr;
+    // execution
+    cudaStream_t cap_stream = nullptr;
+    bool use_graph = true, use_pdl = true;
+    std::vector<GraphEntry> graphs;
+    unsigned long long tick = 0;
+    std::string error;
+};
+
+namespace {
+
+prism_status fail(prism_ctx *c, prism_status s, const std::string &msg) {
+    if (c) c->error = msg;
+    g_error = msg;
+    return s;
+}
+
+prism_status cuda_fail(prism_ctx *c, cudaError_t e, const char *what) {
+    return fail(c, PRISM_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// 16-byte vector loads and bulk prefetches need 16-byte aligned bases.
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+void drop_graphs(prism_ctx *c) {
+    for (auto &g : c->graphs) cudaGraphExecDestroy(g.exec);
+    c->graphs.clear();
+}
+
+int gemv_grid(const prism_ctx *c, int units) {
+    int g = (units + 3) / 4;
+    int cap = 2 * c->sms;
+    return g < 1 ? 1 : (g > cap ? cap : g);
+}
+
+// Enqueue one round.  prof_ev != null: record an event before the first and
+// after every kernel (eager launches, no programmatic dependencies).
+cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool pdl,
+                          cudaEvent_t *prof_ev, int32_t *kinds, int *n_kernels) {
+    const prism_config &f = c->cfg;
+    const int d = f.hidden, Hq = f.n_q_heads, Hkv = f.n_kv_heads, D = f.head_dim, F = f.ffn;
+    const int V = f.vocab, K = f.n_steps;
+    cudaError_t e = cudaSuccess;
+    int nk = 0;
+    bool first = true;
+    auto after = [&](int kind) {
+        if (prof_ev) {
+            if (nk < kMaxProfileKernels) {
+                cudaEventRecord(prof_ev[nk + 1], s);
+                if (kinds) kinds[nk] = kind;
+            }
+        }
+        ++nk;
+        first = false;
+    };
+    if (prof_ev) cudaEventRecord(prof_ev[0], s);
+
+    GemvArgs base{};
+    base.embed = c->embed;
+    base.tokens = r.tokens;
+    base.hidden_in = r.hidden;
+    base.draft = r.draft;
+    base.eps = f.rms_eps;
+    base.n_new = r.n_new;
+    base.max_new = f.max_new;
+    base.K = K;
+    base.vocab = V;
+    base.d = d;
+    base.err = c->err;
+    base.topk = f.topk;
+
+    for (int k = 1; k <= K && e == cudaSuccess; ++k) {
+        const prism_step_weights &w = c->steps[k - 1];
+        const bool prefill = k == 1;
+        const int T1 = prefill ? r.B * f.max_new : r.B;
+        const bool p = pdl && !first;
+
+        // fusion F(E(x), h)
+        GemvArgs g = base;
+        g.step = k;
+        g.W = w.w_fuse;
+        g.n_units = d;
+        g.kin = 2 * d;
+        g.T = T1;
+        g.pro = prefill ? kProFusePrefill : kProFuseDecode;
+        g.src = c->hhat;
+        g.epi = kEpiStore;
+        g.out = c->x0;
+        g.out_ld = d;
+        e = launch_gemv(g, c->bf16, gemv_grid(c, d), s, p);
+        after(0);
+        if (e != cudaSuccess) break;
+
+        // attention pre-norm + QKV
+        g = base;
+        g.step = k;
+        g.W = w.w_qkv;
+        g.n_units = c->qkv_rows;
+        g.kin = d;
+        g.T = T1;
+        g.pro = kProNorm;
+        g.src = c->x0;
+        g.gain = w.g_attn;
+        g.epi = kEpiStore;
+        g.out = c->qkv;
+        g.out_ld = c->qkv_rows;
+        e = launch_gemv(g, c->bf16, gemv_grid(c, c->qkv_rows), s, pdl);
+        after(1);
+        if (e != cudaSuccess) break;
+
+        // RoPE + KV append (+ rotated q of the query rows)
+        RopeArgs ra{};
+        ra.qkv = c->qkv;
+        ra.k_cache = r.k_cache;
+        ra.v_cache = r.v_cache;
+        ra.q_out = c->q;
+        ra.rope_cos = c->rope_cos;
+        ra.rope_sin = c->rope_sin;
+        ra.n_new = r.n_new;
+        ra.kv_len = r.kv_len;
+        ra.B = r.B;
+        ra.max_new = f.max_new;
+        ra.rows = T1;
+        ra.prefill = prefill;
+        ra.step = k;
+        ra.K = K;
+        ra.Hq = Hq;
+        ra.Hkv = Hkv;
+        ra.D = D;
+        ra.max_ctx = f.max_ctx;
+        ra.err = c->err;
+        e = launch_rope_append(ra, c->bf16, s, pdl);
+        after(2);
+        if (e != cudaSuccess) break;
+
+        // split-KV attention with last-CTA combine
+        AttnArgs aa{};
+        aa.q = c->q;
+        aa.k_cache = r.k_cache;
+        aa.v_cache = r.v_cache;
+        aa.part = c->attn_part;
+        aa.counter = c->counters;
+        aa.o_out = c->o_buf;
+        aa.n_new = r.n_new;
+        aa.kv_len = r.kv_len;
+        aa.B = r.B;
+        aa.max_new = f.max_new;
+        aa.prefill = prefill;
+        aa.step = k;
+        aa.Hq = Hq;
+        aa.Hkv = Hkv;
+        aa.D = D;
+        aa.max_ctx = f.max_ctx;
+        aa.chunk = c->attn_chunk;
+        aa.splits = c->attn_splits;
+        aa.err = c->err;
+        e = launch_attention(aa, c->bf16, s, pdl);
+        after(3);
+        if (e != cudaSuccess) break;
+
+        // O projection + residual
+        g = base;
+        g.step = k;
+        g.W = w.w_o;
+        g.n_units = d;
+        g.kin = Hq * D;
+        g.T = r.B;
+        g.pro = kProCopy;
+        g.act = c->o_buf;
+        g.epi = kEpiResid;
+        g.resid = c->x0;
+        g.resid_prefill_rows = prefill;
+        g.out = c->a;
+        g.out_ld = d;
+        e = launch_gemv(g, c->bf16, gemv_grid(c, d), s, pdl);
+        after(4);
+        if (e != cudaSuccess) break;
+
+        // MLP pre-norm + gate/up + SwiGLU
+        g = base;
+        g.step = k;
+        g.W = w.w_gate_up;
+        g.n_units = F;
+        g.pair_offset = F;
+        g.kin = d;
+        g.T = r.B;
+        g.pro = kProNorm;
+        g.src = c->a;
+        g.gain = w.g_mlp;
+        g.epi = kEpiSwiGLU;
+        g.out_act = c->m_buf;
+        g.out_ld = F;
+        e = launch_gemv(g, c->bf16, gemv_grid(c, F), s, pdl);
+        after(5);
+        if (e != cudaSuccess) break;
+
+        // down projection + residual -> h^_{k-1}
+        g = base;
+        g.step = k;
+        g.W = w.w_down;
+        g.n_units = d;
+        g.kin = F;
+        g.T = r.B;
+        g.pro = kProCopy;
+        g.act = c->m_buf;
+        g.epi = kEpiResid;
+        g.resid = c->a;
+        g.out = c->hhat;
+        g.out_ld = d;
+        g.hidden_out = r.hidden_out;
+        e = launch_gemv(g, c->bf16, gemv_grid(c, d), s, pdl);
+        after(6);
+        if (e != cudaSuccess) break;
+
+        // final norm + LM head + top-8 selection -> x^_k
+        g = base;
+        g.step = k;
+        g.W = c->lm_head;
+        g.n_units = V;
+        g.kin = d;
+        g.T = r.B;
+        g.pro = kProNorm;
+        g.src = c->hhat;
+        g.gain = f.final_norm ? w.g_final : nullptr;
+        g.epi = kEpiTopK;
+        g.logits = r.logits;
+        g.lm_part = c->lm_val;
+        g.lm_part_id = c->lm_id;
+        g.counter = c->counters + (size_t)f.max_batch * Hkv;
+        g.draft_out = r.draft;
+        g.topk_ids = r.topk_ids;
+        g.topk_logits = r.topk_logits;
+        e = launch_gemv(g, c->bf16, c->lm_grid, s, pdl);
+        after(7);
+    }
+    if (n_kernels) *n_kernels = nk;
+    return e;
+}
+
+prism_status check_round_args(prism_ctx *c, const RoundArgs &r) {
+    if (!c) return fail(c, PRISM_ERR_INVALID_ARG, "null context");
+    if (r.B < 1) return fail(c, PRISM_ERR_SHAPE, "batch must be >= 1");
+    if (r.B > c->cfg.max_batch) return fail(c, PRISM_ERR_CAPACITY, "batch exceeds max_batch");
+    if (!r.tokens || !r.hidden || !r.n_new || !r.kv_len || !r.k_cache || !r.v_cache || !r.draft)
+        return fail(c, PRISM_ERR_INVALID_ARG, "null tensor argument");
+    if (!aligned16(r.hidden) || !aligned16(r.k_cache) || !aligned16(r.v_cache))
+        return fail(c, PRISM_ERR_INVALID_ARG, "hidden, k_cache and v_cache must be 16-byte aligned");
+    if (!c->embed || !c->lm_head) return fail(c, PRISM_ERR_NOT_LOADED, "shared weights not loaded");
+    for (int k = 0; k < c->cfg.n_steps; ++k)
+        if (!c->step_loaded[k]) return fail(c, PRISM_ERR_NOT_LOADED, "weights of step " + std::to_string(k) + " not loaded");
+    return PRISM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *prism_version(void) { return "prism-gb300 0.1 (sm_103a)"; }
+
+const char *prism_get_error(const prism_ctx *ctx) {
+    return ctx ? ctx->error.c_str() : g_error.c_str();
+}
+
+prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **out) {
+    if (!cfg || !out) return fail(nullptr, PRISM_ERR_INVALID_ARG, "null argument");
+    *out = nullptr;
+    const prism_config &f = *cfg;
+    if (f.hidden < 8 || f.hidden % 8 || f.n_q_heads < 1 || f.n_kv_heads < 1 || f.n_q_heads % f.n_kv_heads ||
+        (f.head_dim != 64 && f.head_dim != 128) || f.ffn < 8 || f.ffn % 8 || f.vocab < kTopK ||
+        f.n_steps < 1 || f.n_steps > kMaxSteps || f.max_batch < 1 || f.max_ctx < 2 || f.max_new < 1 ||
+        f.topk < 1 || f.topk > kTopK || (f.dtype != PRISM_F32 && f.dtype != PRISM_BF16) ||
+        f.n_q_heads / f.n_kv_heads > 16 || !(f.rms_eps >= 0.f) || !(f.rope_theta > 0.f))
+        return fail(nullptr, PRISM_ERR_INVALID_ARG, "unsupported configuration");
+    prism_ctx *c = new prism_ctx();
+    c->cfg = f;
+    c->device = device;
+    c->bf16 = f.dtype == PRISM_BF16;
+    cudaError_t e = cudaSetDevice(device);
+    if (e != cudaSuccess) { delete c; return cuda_fail(nullptr, e, "cudaSetDevice"); }
+    cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, device);
+    const int d = f.hidden, Hq = f.n_q_heads, Hkv = f.n_kv_heads, D = f.head_dim, F = f.ffn;
+    const size_t es = c->bf16 ? 2 : 4;
+    c->qkv_rows = (Hq + 2 * Hkv) * D;
+    c->lm_grid = (f.vocab + 15) / 16 < 2 * c->sms ? (f.vocab + 15) / 16 : 2 * c->sms;
+    // attention split size: enough CTAs to cover the GPU at batch 1
+    c->attn_chunk = 64;
+    if ((long long)f.max_batch * Hkv * ((f.max_ctx + 63) / 64) < 2LL * c->sms) c->attn_chunk = 32;
+    c->attn_splits = (f.max_ctx + c->attn_chunk - 1) / c->attn_chunk;
+
+    const size_t T1 = (size_t)f.max_batch * f.max_new, B = f.max_batch;
+    size_t sizes[] = {
+        (size_t)f.max_ctx * (D / 2) * 4,                           // rope cos
+        (size_t)f.max_ctx * (D / 2) * 4,                           // rope sin
+        T1 * d * 4,                                                // x0
+        T1 * c->qkv_rows * 4,                                      // qkv
+        B * Hq * D * 4,                                            // q
+        B * Hq * (size_t)c->attn_splits * (D + 2) * 4,             // attention partials
+        B * d * 4,                                                 // a
+        B * d * 4,                                                 // h^
+        B * Hq * D * es,                                           // o
+        B * F * es,                                                // m
+        B * (size_t)c->lm_grid * kTopK * 4,                        // LM partial values
+        B * (size_t)c->lm_grid * kTopK * 4,                        // LM partial ids
+        (B * Hkv + 1) * 4,                                         // counters
+        4,                                                         // error word
+    };
+    size_t total = 0;
+    for (size_t s : sizes) total += align256(s);
+    void *ws = nullptr;
+    e = cudaMalloc(&ws, total);
+    if (e != cudaSuccess) { delete c; return fail(nullptr, PRISM_ERR_OOM, std::string("workspace: ") + cudaGetErrorString(e)); }
+    cudaMemset(ws, 0, total);
+    c->ws = ws;
+    c->ws_bytes = total;
+    uint8_t *p = (uint8_t *)ws;
+    void *slot[sizeof(sizes) / sizeof(sizes[0])];
+    for (size_t i = 0; i < sizeof(sizes) / sizeof(sizes[0]); ++i) { slot[i] = p; p += align256(sizes[i]); }
+    c->rope_cos = (float *)slot[0];
+    c->rope_sin = (float *)slot[1];
+    c->x0 = (float *)slot[2];
+    c->qkv = (float *)slot[3];
+    c->q = (float *)slot[4];
+    c->attn_part = (float *)slot[5];
+    c->a = (float *)slot[6];
+    c->hhat = (float *)slot[7];
+    c->o_buf = slot[8];
+    c->m_buf = slot[9];
+    c->lm_val = (float *)slot[10];
+    c->lm_id = (int *)slot[11];
+    c->counters = (int *)slot[12];
+    c->err = (int *)slot[13];
+
+    // rotary tables: angle p * theta^(-2j/D), computed in double, stored as float
+    std::vector<float> cs((size_t)f.max_ctx * (D / 2)), sn((size_t)f.max_ctx * (D / 2));
+    for (int pos = 0; pos < f.max_ctx; ++pos)
+        for (int j = 0; j < D / 2; ++j) {
+            const double inv = std::pow((double)f.rope_theta, -2.0 * j / (double)D);
+            const double ang = (double)pos * inv;
+            cs[(size_t)pos * (D / 2) + j] = (float)std::cos(ang);
+            sn[(size_t)pos * (D / 2) + j] = (float)std::sin(ang);
+        }
+    e = cudaMemcpy(c->rope_cos, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->rope_sin, sn.data(), sn.size() * 4, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = prepare_gemv_kernels();
+    if (e == cudaSuccess) e = prepare_attention_kernel(c->bf16, D, c->attn_chunk, Hq / Hkv);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking);
+    if (e != cudaSuccess) {
+        prism_status st = cuda_fail(nullptr, e, "context setup");
+        cudaFree(ws);
+        delete c;
+        return st;
+    }
+    *out = c;
+    return PRISM_OK;
+}
+
+prism_status prism_destroy(prism_ctx *c) {
+    if (!c) return PRISM_OK;
+    cudaSetDevice(c->device);
+    cudaDeviceSynchronize();
+    drop_graphs(c);
+    if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+    if (c->ws) cudaFree(c->ws);
+    delete c;
+    return PRISM_OK;
+}
+
+prism_status prism_load_shared_weights(prism_ctx *c, const void *embed, const void *lm_head) {
+    if (!c || !embed || !lm_head) return fail(c, PRISM_ERR_INVALID_ARG, "null argument");
+    if (!aligned16(embed) || !aligned16(lm_head))
+        return fail(c, PRISM_ERR_INVALID_ARG, "embed and lm_head must be 16-byte aligned");
+    c->embed = embed;
+    c->lm_head = lm_head;
+    drop_graphs(c);
+    return PRISM_OK;
+}
+
+prism_status prism_load_step_weights(prism_ctx *c, int32_t step, const prism_step_weights *w) {
+    if (!c || !w) return fail(c, PRISM_ERR_INVALID_ARG, "null argument");
+    if (step < 0 || step >= c->cfg.n_steps) return fail(c, PRISM_ERR_INVALID_ARG, "step out of range");
+    if (!w->w_fuse || !w->g_attn || !w->w_qkv || !w->w_o || !w->g_mlp || !w->w_gate_up || !w->w_down ||
+        (c->cfg.final_norm && !w->g_final))
+        return fail(c, PRISM_ERR_INVALID_ARG, "null weight pointer");
+    for (const void *p : {w->w_fuse, w->g_attn, w->w_qkv, w->w_o, w->g_mlp, w->w_gate_up, w->w_down, w->g_final})
+        if (p && !aligned16(p)) return fail(c, PRISM_ERR_INVALID_ARG, "weight pointers must be 16-byte aligned");
+    c->steps[step] = *w;
+    c->step_loaded[step] = true;
+    drop_graphs(c);
+    return PRISM_OK;
+}
+
+prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
+    if (!c || !name) return fail(c, PRISM_ERR_INVALID_ARG, "null argument");
+    if (!std::strcmp(name, "use_graph")) c->use_graph = value != 0;
+    else if (!std::strcmp(name, "use_pdl")) c->use_pdl = value != 0;
+    else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
+    drop_graphs(c);
+    return PRISM_OK;
+}
+
+prism_status prism_draft_round(prism_ctx *c, int32_t batch, const int32_t *tokens, const void *hidden,
+                               const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
+                               int32_t *draft_ids, int32_t *topk_ids, float *topk_logits, float *logits,
+                               float *hidden_out, void *stream) {
+    RoundArgs r{batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids, topk_ids, topk_logits,
+                logits, hidden_out};
+    prism_status st = check_round_args(c, r);
+    if (st != PRISM_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e = cudaSetDevice(c->device);
+    if (e != cudaSuccess) return cuda_fail(c, e, "cudaSetDevice");
+    if (!c->use_graph) {
+        e = enqueue_round(c, r, s, c->use_pdl, nullptr, nullptr, nullptr);
+        return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "kernel launch");
+    }
+    GraphEntry *hit = nullptr;
+    for (auto &g : c->graphs)
+        if (g.key == r && g.pdl == c->use_pdl) hit = &g;
+    if (!hit) {
+        if ((int)c->graphs.size() >= kGraphCache) {
+            size_t old = 0;
+            for (size_t i = 1; i < c->graphs.size(); ++i)
+                if (c->graphs[i].used < c->graphs[old].used) old = i;
+            cudaGraphExecDestroy(c->graphs[old].exec);
+            c->graphs.erase(c->graphs.begin() + old);
+        }
+        cudaGraph_t graph = nullptr;
+        e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
+        if (e != cudaSuccess) return cuda_fail(c, e, "cudaStreamBeginCapture");
+        cudaError_t le = enqueue_round(c, r, c->cap_stream, c->use_pdl, nullptr, nullptr, nullptr);
+        e = cudaStreamEndCapture(c->cap_stream, &graph);
+        if (le != cudaSuccess) {
+            if (graph) cudaGraphDestroy(graph);
+            return cuda_fail(c, le, "kernel launch during capture");
+        }
+        if (e != cudaSuccess) return cuda_fail(c, e, "cudaStreamEndCapture");
+        cudaGraphExec_t exec = nullptr;
+        e = cudaGraphInstantiate(&exec, graph, 0);
+        cudaGraphDestroy(graph);
+        if (e != cudaSuccess) return cuda_fail(c, e, "cudaGraphInstantiate");
+        c->graphs.push_back(GraphEntry{r, c->use_pdl, exec, 0});
+        hit = &c->graphs.back();
+    }
+    hit->used = ++c->tick;
+    e = cudaGraphLaunch(hit->exec, s);
+    return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "cudaGraphLaunch");
+}
+
+prism_status prism_profile_round(prism_ctx *c, int32_t batch, const int32_t *tokens, const void *hidden,
+                                 const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
+                                 int32_t *draft_ids, int32_t *topk_ids, float *topk_logits, void *stream,
+                                 float *kernel_ms, int32_t *kernel_kind, int32_t max_kernels,
+                                 int32_t *n_kernels) {
+    RoundArgs r{batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids, topk_ids, topk_logits,
+                nullptr, nullptr};
+    prism_status st = check_round_args(c, r);
+    if (st != PRISM_OK) return st;
+    if (!kernel_ms || !n_kernels || max_kernels < 1) return fail(c, PRISM_ERR_INVALID_ARG, "null output");
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaSetDevice(c->device);
+    cudaEvent_t ev[kMaxProfileKernels + 1];
+    for (auto &x : ev) cudaEventCreate(&x);
+    int32_t kinds[kMaxProfileKernels];
+    int nk = 0;
+    cudaError_t e = enqueue_round(c, r, s, false, ev, kinds, &nk);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    const int n = nk < max_kernels ? nk : max_kernels;
+    for (int i = 0; i < n && e == cudaSuccess && i < kMaxProfileKernels; ++i) {
+        float ms = 0.f;
+        cudaEventElapsedTime(&ms, ev[i], ev[i + 1]);
+        kernel_ms[i] = ms;
+        if (kernel_kind) kernel_kind[i] = kinds[i];
+    }
+    *n_kernels = n;
+    for (auto &x : ev) cudaEventDestroy(x);
+    return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "profiled round");
+}
+
+prism_status prism_accept_greedy(prism_ctx *c, int32_t batch, const int32_t *draft, const int32_t *target,
+                                 const int32_t *n_new, int32_t *kv_len, int32_t *accept_len,
+                                 int32_t *out_tokens, void *stream) {
+    if (!c) return fail(c, PRISM_ERR_INVALID_ARG, "null context");
+    if (!draft || !target || !n_new || !kv_len || !accept_len || !out_tokens)
+        return fail(c, PRISM_ERR_INVALID_ARG, "null tensor argument");
+    if (batch < 1) return fail(c, PRISM_ERR_SHAPE, "batch must be >= 1");
+    if (batch > c->cfg.max_batch) return fail(c, PRISM_ERR_CAPACITY, "batch exceeds max_batch");
+    cudaSetDevice(c->device);
+    AcceptArgs a{draft, target, n_new, kv_len, accept_len, out_tokens, batch, c->cfg.n_steps};
+    cudaError_t e = launch_accept(a, (cudaStream_t)stream);
+    return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "accept kernel launch");
+}
+
+prism_status prism_sync_status(prism_ctx *c, void *stream, int32_t *flags) {
+    if (!c) return fail(c, PRISM_ERR_INVALID_ARG, "null context");
+    if (flags) *flags = 0;
+    cudaSetDevice(c->device);
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "stream synchronize");
+    int w = 0;
+    e = cudaMemcpy(&w, c->err, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(c, e, "error word read");
+    if (w) {
+        cudaMemset(c->err, 0, sizeof(int));
+        if (flags) *flags = w;
+        char buf[160];
+        std::snprintf(buf, sizeof(buf), "device error word 0x%x (token range %d, cache range %d, n_new range %d, timeout %d)",
+                      w, !!(w & 1), !!(w & 2), !!(w & 4), !!(w & 8));
+        return fail(c, PRISM_ERR_DEVICE_FLAG, buf);
+    }
+    return PRISM_OK;
+}
+
+}  // extern "C"

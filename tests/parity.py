@@ -1,0 +1,108 @@
+"""GPU-vs-oracle comparison rules for one draft round.
+
+Spec bar (bf16 weights, fp32 accumulation on the GPU, fp64 oracle):
+draft ids equal wherever the oracle's top-1 minus top-2 logit margin exceeds
+MARGIN; logits within max-abs ATOL and relative L2 REL_L2.
+
+How it is applied:
+  * per step from a common state (teacher forcing: step k recomputed from the
+    oracle's state after step k-1) and on step 1 of every round: the full
+    bar, strictly;
+  * along the free-running K-step chain: relative L2 on every step, and draft
+    ids equal wherever the margin exceeds both MARGIN and twice the measured
+    max-abs logit deviation of that step.  The chain re-rounds h^ to bf16 at
+    every step, so fp32-vs-fp64 differences of ~1e-7 flip occasional bf16
+    roundings and grow step by step; on the Llama-shaped drafters a single
+    one-ulp change of one input element moves the oracle's OWN logits by more
+    than ATOL after a few steps, so no fp32 implementation can promise ATOL
+    there;
+  * after a (margin-exempt) id difference the two chains legitimately
+    diverge, so later steps of that sequence are not compared;
+  * KV rows the round must not touch are bit-identical; written rows and h^
+    within REL_L2.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+MARGIN = 1e-2
+ATOL = 3e-2
+REL_L2 = 1e-2
+
+
+def rel_l2(a, b):
+    a, b = np.asarray(a, np.float64), np.asarray(b, np.float64)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
+
+
+def _as_f64(cache):
+    cache = np.asarray(cache)
+    if cache.dtype == np.uint16:
+        return (cache.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    return cache.astype(np.float64)
+
+
+def compare_round(gpu: dict, orc: dict, inputs: dict, seqs, K: int, topk: int, *,
+                  chain: bool = False, report: dict | None = None):
+    """gpu: device outputs as numpy over the full batch; orc: oracle outputs
+    over the sequences `seqs` (in that order).  Raises AssertionError."""
+    rep = report if report is not None else {}
+    for key in ("ids_compared", "ids_exempt"):
+        rep.setdefault(key, 0)
+    for key in ("max_abs_logit", "max_rel_l2_logit", "max_rel_l2_hidden", "max_abs_logit_step1"):
+        rep.setdefault(key, 0.0)
+    have_logits = gpu.get("logits") is not None and orc.get("logits") is not None
+    assert have_logits or not chain, "the chain comparison needs logits"
+    for j, b in enumerate(seqs):
+        for k in range(K):
+            o_top = orc["topk_logits"][j, k]
+            margin = o_top[0] - o_top[1]
+            g_id, o_id = int(gpu["draft_ids"][b, k]), int(orc["draft_ids"][j, k])
+            ma = 0.0
+            if have_logits:
+                zg, zo = gpu["logits"][b, k], orc["logits"][j, k]
+                ma = float(np.max(np.abs(zg - zo)))
+                rl = rel_l2(zg, zo)
+                rep["max_abs_logit"] = max(rep["max_abs_logit"], ma)
+                rep["max_rel_l2_logit"] = max(rep["max_rel_l2_logit"], rl)
+                if k == 0:
+                    rep["max_abs_logit_step1"] = max(rep["max_abs_logit_step1"], ma)
+                if not chain or k == 0:
+                    assert ma <= ATOL, f"seq {b} step {k + 1}: logit max-abs {ma:.3e} > {ATOL}"
+                assert rl <= REL_L2, f"seq {b} step {k + 1}: logit rel-L2 {rl:.3e} > {REL_L2}"
+            if gpu.get("hidden_out") is not None and orc.get("hidden_out") is not None:
+                rh = rel_l2(gpu["hidden_out"][b, k], orc["hidden_out"][j, k])
+                rep["max_rel_l2_hidden"] = max(rep["max_rel_l2_hidden"], rh)
+                assert rh <= REL_L2, f"seq {b} step {k + 1}: h^ rel-L2 {rh:.3e} > {REL_L2}"
+            thr = max(MARGIN, 2 * ma) if (chain and k > 0) else MARGIN
+            if margin > thr:
+                rep["ids_compared"] += 1
+                assert g_id == o_id, (f"seq {b} step {k + 1}: draft id {g_id} != oracle {o_id} "
+                                      f"(oracle margin {margin:.3e}, threshold {thr:.3e})")
+            else:
+                rep["ids_exempt"] += 1
+            if topk > 1 and gpu.get("topk_ids") is not None:
+                gaps = -np.diff(o_top)           # gaps[r] = top[r] - top[r+1]
+                for r in range(topk):
+                    lo = gaps[r - 1] if r > 0 else np.inf
+                    hi = gaps[r] if r < len(gaps) else np.inf
+                    if min(lo, hi) > thr:
+                        assert gpu["topk_ids"][b, k, r] == orc["topk_ids"][j, k, r], (
+                            f"seq {b} step {k + 1}: top-{r + 1} id differs")
+                        assert abs(gpu["topk_logits"][b, k, r] - o_top[r]) <= max(ATOL, ma)
+            if g_id != o_id:
+                break                            # later steps diverge legitimately
+    return rep
+
+
+def compare_cache(gpu_k, gpu_v, orc_k, orc_v, inputs, seqs, K):
+    """Rows [0, L_b) untouched (bit-exact); step-1 rows [L_b, L_b + n_b) within
+    REL_L2 (bf16 storage); draft rows are scratch and are compared only for
+    steps whose draft ids matched (done by the caller)."""
+    for j, b in enumerate(seqs):
+        L, n = int(inputs["kv_len"][b]), int(inputs["n_new"][b])
+        for g_, i_, o_ in ((gpu_k, inputs["k_cache"], orc_k), (gpu_v, inputs["v_cache"], orc_v)):
+            assert np.array_equal(g_[b, :, :L], i_[b, :, :L]), f"seq {b}: committed KV rows modified"
+            got = _as_f64(g_[b, :, L:L + n])
+            exp = _as_f64(o_[j, :, L:L + n])
+            assert rel_l2(got, exp) <= REL_L2, f"seq {b}: new KV rows rel-L2 {rel_l2(got, exp):.3e}"

@@ -1,0 +1,68 @@
+"""The C ABI library builds, loads without a GPU and exports every entry
+point that include/prism.h declares; host-side argument checks that need no
+device answer correctly."""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "prism.h")
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(prism_[a-z_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2602_01762_gb300 import build
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def test_header_declares_the_round_entry_points():
+    syms = declared_symbols()
+    for s in ("prism_load_step_weights", "prism_draft_round", "prism_accept_greedy", "prism_create",
+              "prism_destroy", "prism_load_shared_weights", "prism_sync_status", "prism_get_error"):
+        assert s in syms
+
+
+def test_library_exports_every_declared_symbol(lib):
+    missing = [s for s in declared_symbols() if not hasattr(lib, s)]
+    assert not missing, f"not exported: {missing}"
+
+
+def test_version_and_error_strings(lib):
+    lib.prism_version.restype = ctypes.c_char_p
+    assert b"sm_103a" in lib.prism_version()
+    lib.prism_get_error.restype = ctypes.c_char_p
+    lib.prism_get_error.argtypes = [ctypes.c_void_p]
+    assert isinstance(lib.prism_get_error(None), bytes)
+
+
+def test_create_rejects_bad_configuration_before_touching_cuda(lib):
+    from paper_2602_01762_gb300 import _Config
+    bad = _Config(256, 4, 3, 64, 688, 4096, 3, 1, 1, 64, 1, 1, 10000.0, 1e-5, 1)  # 4 % 3 != 0
+    out = ctypes.c_void_p()
+    lib.prism_create.argtypes = [ctypes.POINTER(_Config), ctypes.c_int32, ctypes.POINTER(ctypes.c_void_p)]
+    assert lib.prism_create(ctypes.byref(bad), 0, ctypes.byref(out)) == 1
+    assert not out.value
+    bad = _Config(256, 4, 4, 96, 688, 4096, 3, 1, 1, 64, 1, 1, 10000.0, 1e-5, 1)  # head_dim 96
+    assert lib.prism_create(ctypes.byref(bad), 0, ctypes.byref(out)) == 1
+    bad = _Config(256, 4, 4, 64, 688, 4096, 3, 1, 1, 64, 1, 9, 10000.0, 1e-5, 1)  # topk 9
+    assert lib.prism_create(ctypes.byref(bad), 0, ctypes.byref(out)) == 1
+    assert lib.prism_create(None, 0, ctypes.byref(out)) == 1
+
+
+def test_null_context_calls_return_invalid_arg(lib):
+    for name, n in (("prism_draft_round", 14), ("prism_accept_greedy", 9)):
+        f = getattr(lib, name)
+        f.argtypes = [ctypes.c_void_p, ctypes.c_int32] + [ctypes.c_void_p] * (n - 2)
+        assert f(None, 1, *([None] * (n - 2))) == 1
+    assert lib.prism_destroy(None) == 0
