@@ -159,8 +159,14 @@ prism_status prism_accept_greedy(prism_ctx *ctx, int32_t batch, const int32_t *d
 prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
 
 /* Options (name, value): "use_graph" (1: capture and replay, default 1),
- * "use_pdl" (1: programmatic dependent launch between kernels, default 1).
- * Changing an option drops cached graphs.  Errors: INVALID_ARG. */
+ * "use_pdl" (1: programmatic dependent launch between kernels, default 1),
+ * "gemv_chunk_kb" (target TMA stage size of the projection kernels, 0..128,
+ * 0 = default), "gemv_smem_kb" (shared-memory budget of the projection
+ * ring, 0..200, 0 = default), "gemv_groups" (consumer warp groups of the
+ * projection kernels: 1, 2, 4, 8 or 16; 0 = default), "gemv_cuda_core"
+ * (1, the default: bf16 projections run on the CUDA-core kernel; 0: on the
+ * warp-level tensor-core kernel).  Changing an option drops cached
+ * graphs.  Errors: INVALID_ARG (unknown name or value out of range). */
 prism_status prism_set_option(prism_ctx *ctx, const char *name, int32_t value);
 
 /* Instrumented round for measurement: the same work as prism_draft_round

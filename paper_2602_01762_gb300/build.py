@@ -17,6 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 ROOT = os.path.dirname(HERE)
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(HERE, "libprism.so")
+LIB_CHECKED = os.path.join(HERE, "libprism_checked.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -44,8 +45,11 @@ def up_to_date() -> bool:
     return all(os.path.getmtime(p) <= t for p in _deps())
 
 
-def build(force: bool = False, ptxas_info: bool = False, verbose: bool = False) -> str:
-    if not force and up_to_date():
+def build(force: bool = False, ptxas_info: bool = False, verbose: bool = False, checked: bool = False) -> str:
+    """checked=True builds libprism_checked.so with device bounds checks and
+    per-kernel synchronisation (diagnostics only)."""
+    lib = LIB_CHECKED if checked else LIB
+    if not force and not checked and up_to_date():
         return LIB
     os.makedirs(BUILD, exist_ok=True)
     nvcc = _nvcc()
@@ -53,9 +57,11 @@ def build(force: bool = False, ptxas_info: bool = False, verbose: bool = False) 
                     "-I", os.path.join(ROOT, "include")]
     if ptxas_info:
         flags += ["-Xptxas", "-v"]
+    if checked:
+        flags += ["-DPRISM_CHECKED"]
 
     def compile_one(src):
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + (".chk.o" if checked else ".o"))
         cmd = [nvcc] + flags + ["-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -68,18 +74,19 @@ def build(force: bool = False, ptxas_info: bool = False, verbose: bool = False) 
         for _, err in results:
             if err.strip():
                 print(err, file=sys.stderr)
-    tmp = LIB + f".tmp{os.getpid()}"
+    tmp = lib + f".tmp{os.getpid()}"
     cmd = [nvcc] + ARCH + ["-shared", "-o", tmp] + [o for o, _ in results]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":
     ap = argparse.ArgumentParser()
     ap.add_argument("--force", action="store_true")
     ap.add_argument("--ptxas-info", action="store_true")
+    ap.add_argument("--checked", action="store_true")
     a = ap.parse_args()
-    print(build(force=a.force, ptxas_info=a.ptxas_info, verbose=True))
+    print(build(force=a.force, ptxas_info=a.ptxas_info, verbose=True, checked=a.checked))

@@ -33,6 +33,22 @@ __device__ __forceinline__ int query_pos(int prefill, int L, int n, int step) {
     return prefill ? L + n - 1 : L + n + step - 2;
 }
 
+// Asynchronous 16-byte global -> shared copy (no register staging) and the
+// wait for all of this thread's outstanding copies.
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
+    const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+}
+
+// Partial record of one (sequence, head, split): D output sums, running max,
+// running sum, two pad words (16-byte aligned records).
+template <int D> struct Part {
+    static constexpr int kStride = D + 4;
+};
+
 // acc += q[0..VEC) . k-vector (16 bytes of keys)
 template <typename WT>
 __device__ __forceinline__ void dot_qk(float &acc, const float *q, const uint4 &k);
@@ -135,6 +151,8 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const AttnArgs 
     WT *Vs = Ks + (size_t)C * RS;
     float *qs = (float *)(Vs + (size_t)C * RS);   // [G][D]
     float *ps = qs + (size_t)G * D;               // [G][C]
+    float *ws = ps + (size_t)G * C;               // [G][splits] combine weights
+    constexpr int PS = Part<D>::kStride;
 
     const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
@@ -149,6 +167,9 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const AttnArgs 
     if (P < 1) P = 1;
     const int j0 = s * C;
     const int nk = P - j0 < C ? P - j0 : C;
+    if (PRISM_CHECK(a.err, (((uintptr_t)a.k_cache | (uintptr_t)a.v_cache) & 15) == 0, 201, 0, 0) ||
+        PRISM_CHECK(a.err, j0 + (nk > 0 ? nk : 0) <= a.max_ctx, 202, j0, nk))
+        return;
     const float scale = 1.0f / sqrtf((float)D);
 
     if (nk > 0) {
@@ -157,11 +178,12 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const AttnArgs 
         constexpr int VPR = D / VEC;   // vectors per row
         for (int e = threadIdx.x; e < nk * VPR; e += blockDim.x) {
             const int r = e / VPR, c = e % VPR;
-            *(uint4 *)(Ks + (size_t)r * RS + c * VEC) = kg[e];
-            *(uint4 *)(Vs + (size_t)r * RS + c * VEC) = vg[e];
+            cp_async16(Ks + (size_t)r * RS + c * VEC, kg + e);
+            cp_async16(Vs + (size_t)r * RS + c * VEC, vg + e);
         }
         for (int e = threadIdx.x; e < G * D; e += blockDim.x)
             qs[e] = a.q[((size_t)b * a.Hq + (size_t)g * G) * D + e];
+        cp_async_wait_all();
         __syncthreads();
 
         for (int hl = warp; hl < G; hl += nwarp) {
@@ -198,7 +220,7 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const AttnArgs 
                 for (int u = 0; u < DPL; ++u) acc[u] = fmaf(p, vv[u], acc[u]);
             }
             const int h = g * G + hl;
-            float *part = a.part + (((size_t)b * a.Hq + h) * a.splits + s) * (D + 2);
+            float *part = a.part + (((size_t)b * a.Hq + h) * a.splits + s) * PS;
 #pragma unroll
             for (int u = 0; u < DPL; ++u) part[lane * DPL + u] = acc[u];
             if (lane == 0) { part[D] = mloc; part[D + 1] = lsum; }
@@ -206,7 +228,7 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const AttnArgs 
     } else {
         for (int hl = warp; hl < G; hl += nwarp) {
             const int h = g * G + hl;
-            float *part = a.part + (((size_t)b * a.Hq + h) * a.splits + s) * (D + 2);
+            float *part = a.part + (((size_t)b * a.Hq + h) * a.splits + s) * PS;
 #pragma unroll
             for (int u = 0; u < DPL; ++u) part[lane * DPL + u] = 0.f;
             if (lane == 0) { part[D] = -INFINITY; part[D + 1] = 0.f; }
@@ -223,20 +245,41 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const AttnArgs 
     __threadfence();
     for (int hl = warp; hl < G; hl += nwarp) {
         const int h = g * G + hl;
-        const float *part = a.part + ((size_t)b * a.Hq + h) * a.splits * (D + 2);
+        const float *part = a.part + ((size_t)b * a.Hq + h) * a.splits * PS;
+        float *wh = ws + (size_t)hl * a.splits;
+        // lanes over splits: global max, split weights exp(m_s - M), denominator
         float M = -INFINITY;
-        for (int sp = 0; sp < a.splits; ++sp) M = fmaxf(M, __ldcg(part + (size_t)sp * (D + 2) + D));
-        float acc[DPL], den = 0.f;
+        for (int sp = lane; sp < a.splits; sp += 32) M = fmaxf(M, __ldcg(part + (size_t)sp * PS + D));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xFFFFFFFFu, M, o));
+        float den = 0.f;
+        for (int sp = lane; sp < a.splits; sp += 32) {
+            const float l = __ldcg(part + (size_t)sp * PS + D + 1);
+            const float w = l > 0.f ? expf(__ldcg(part + (size_t)sp * PS + D) - M) : 0.f;
+            wh[sp] = w;
+            den = fmaf(w, l, den);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) den += __shfl_xor_sync(0xFFFFFFFFu, den, o);
+        __syncwarp();
+        // lanes over output dims: weighted sum of the split outputs in split order
+        float acc[DPL];
 #pragma unroll
         for (int u = 0; u < DPL; ++u) acc[u] = 0.f;
+#pragma unroll 8
         for (int sp = 0; sp < a.splits; ++sp) {
-            const float *ps_ = part + (size_t)sp * (D + 2);
-            const float l = __ldcg(ps_ + D + 1);
-            if (l == 0.f) continue;
-            const float w = expf(__ldcg(ps_ + D) - M);
-            den = fmaf(w, l, den);
+            const float w = wh[sp];
+            float v[DPL];
+            const float *src = part + (size_t)sp * PS + lane * DPL;
+            if constexpr (DPL == 4) {
+                const float4 t = __ldcg((const float4 *)src);
+                v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+            } else {
+                const float2 t = __ldcg((const float2 *)src);
+                v[0] = t.x; v[1] = t.y;
+            }
 #pragma unroll
-            for (int u = 0; u < DPL; ++u) acc[u] = fmaf(w, __ldcg(ps_ + lane * DPL + u), acc[u]);
+            for (int u = 0; u < DPL; ++u) acc[u] = fmaf(w, v[u], acc[u]);
         }
         WT *o = (WT *)a.o_out + (size_t)b * a.Hq * D + (size_t)h * D;
         const float inv = 1.0f / den;
@@ -263,21 +306,24 @@ __global__ void accept_kernel(const AcceptArgs a) {
 }
 
 template <typename WT, int D>
-size_t attn_smem(int chunk, int G) {
+size_t attn_smem(int chunk, int G, int splits) {
     constexpr int RS = D + Elem<WT>::kPerVec;
-    return (size_t)2 * chunk * RS * sizeof(WT) + (size_t)G * D * 4 + (size_t)G * chunk * 4;
+    return (size_t)2 * chunk * RS * sizeof(WT) + (size_t)G * D * 4 + (size_t)G * chunk * 4 + (size_t)G * splits * 4;
 }
 
 template <typename WT, int D>
 cudaError_t launch_attn_t(const AttnArgs &a, cudaStream_t s, bool pdl) {
-    const size_t smem = attn_smem<WT, D>(a.chunk, a.Hq / a.Hkv);
+    const size_t smem = attn_smem<WT, D>(a.chunk, a.Hq / a.Hkv, a.splits);
     return launch_k(attention_kernel<WT, D>, dim3(a.splits, a.Hkv, a.B), dim3(kAttnThreads), smem, s, pdl, a);
 }
 
+// The attribute is a per-function ceiling shared by every context, so it is
+// set to the cap that prism_create validates against, never lowered.
+constexpr int kAttnSmemCap = 200 * 1024;
 template <typename WT, int D>
-cudaError_t prepare_attn_t(int chunk, int G) {
-    return cudaFuncSetAttribute(attention_kernel<WT, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)attn_smem<WT, D>(chunk, G));
+cudaError_t prepare_attn_t(int chunk, int G, int splits) {
+    if (attn_smem<WT, D>(chunk, G, splits) > (size_t)kAttnSmemCap) return cudaErrorInvalidValue;
+    return cudaFuncSetAttribute(attention_kernel<WT, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmemCap);
 }
 
 }  // namespace
@@ -294,14 +340,14 @@ cudaError_t launch_attention(const AttnArgs &a, bool bf16, cudaStream_t s, bool 
     return a.D == 64 ? launch_attn_t<float, 64>(a, s, pdl) : launch_attn_t<float, 128>(a, s, pdl);
 }
 
-cudaError_t prepare_attention_kernel(bool bf16, int D, int chunk, int G) {
-    if (bf16) return D == 64 ? prepare_attn_t<uint16_t, 64>(chunk, G) : prepare_attn_t<uint16_t, 128>(chunk, G);
-    return D == 64 ? prepare_attn_t<float, 64>(chunk, G) : prepare_attn_t<float, 128>(chunk, G);
+cudaError_t prepare_attention_kernel(bool bf16, int D, int chunk, int G, int splits) {
+    if (bf16) return D == 64 ? prepare_attn_t<uint16_t, 64>(chunk, G, splits) : prepare_attn_t<uint16_t, 128>(chunk, G, splits);
+    return D == 64 ? prepare_attn_t<float, 64>(chunk, G, splits) : prepare_attn_t<float, 128>(chunk, G, splits);
 }
 
-size_t attention_smem_bytes(bool bf16, int D, int chunk, int G) {
-    if (bf16) return D == 64 ? attn_smem<uint16_t, 64>(chunk, G) : attn_smem<uint16_t, 128>(chunk, G);
-    return D == 64 ? attn_smem<float, 64>(chunk, G) : attn_smem<float, 128>(chunk, G);
+size_t attention_smem_bytes(bool bf16, int D, int chunk, int G, int splits) {
+    if (bf16) return D == 64 ? attn_smem<uint16_t, 64>(chunk, G, splits) : attn_smem<uint16_t, 128>(chunk, G, splits);
+    return D == 64 ? attn_smem<float, 64>(chunk, G, splits) : attn_smem<float, 128>(chunk, G, splits);
 }
 
 cudaError_t launch_accept(const AcceptArgs &a, cudaStream_t s) {

@@ -82,6 +82,23 @@ __device__ __forceinline__ void set_err(int *err, int bit) {
     if (err) atomicOr(err, bit);
 }
 
+// Checked builds (-DPRISM_CHECKED): record the first failed bounds or
+// alignment check (code, block, two values) in the four words after the
+// device error word, and skip the access.  Compiled out otherwise.
+#ifdef PRISM_CHECKED
+__device__ __forceinline__ bool dbg_fail(int *err, int code, long v1, long v2) {
+    if (err && atomicCAS(err + 1, 0, code) == 0) {
+        err[2] = (int)blockIdx.x;
+        err[3] = (int)v1;
+        err[4] = (int)v2;
+    }
+    return true;
+}
+#define PRISM_CHECK(err, cond, code, v1, v2) (!(cond) && dbg_fail((err), (code), (long)(v1), (long)(v2)))
+#else
+#define PRISM_CHECK(err, cond, code, v1, v2) false
+#endif
+
 // Top-8 ordering: larger logit first, then lower id.
 __device__ __forceinline__ bool better(float a, int ia, float b, int ib) {
     return a > b || (a == b && ia < ib);
@@ -157,6 +174,9 @@ struct GemvArgs {
     float *topk_logits;      // [B, K, topk] or null
     int topk;
     int *err;
+    // ring plan knobs: target stage bytes, smem budget bytes, consumer groups;
+    // force_cuda_core selects the CUDA-core kernel for bf16 too
+    int chunk_target, smem_budget, groups, force_cuda_core;
 };
 
 struct RopeArgs {
@@ -173,7 +193,7 @@ struct RopeArgs {
 struct AttnArgs {
     const float *q;          // [B, Hq, D] (rotated)
     const void *k_cache, *v_cache;
-    float *part;             // [B, Hq, splits, D + 2]
+    float *part;             // [B, Hq, splits, D + 4]
     int *counter;            // [B * Hkv]
     void *o_out;             // [B, Hq * D] wtype (rounded operand of the O projection)
     const int32_t *n_new, *kv_len;
@@ -197,8 +217,12 @@ cudaError_t launch_accept(const AcceptArgs &a, cudaStream_t s);
 // One-time kernel attribute setup (maximum dynamic shared memory); must run
 // before any stream capture.
 cudaError_t prepare_gemv_kernels();
-cudaError_t prepare_attention_kernel(bool bf16, int D, int chunk, int G);
-size_t attention_smem_bytes(bool bf16, int D, int chunk, int G);
+bool gemv_supported(const GemvArgs &a, bool bf16);
+bool gemv_mma_supported(const GemvArgs &a);
+cudaError_t prepare_gemv_mma_kernels();
+cudaError_t launch_gemv_mma(const GemvArgs &a, int grid, cudaStream_t s, bool pdl);
+cudaError_t prepare_attention_kernel(bool bf16, int D, int chunk, int G, int splits);
+size_t attention_smem_bytes(bool bf16, int D, int chunk, int G, int splits);
 
 // Launch with optional programmatic stream serialization.
 template <typename Kern, typename... Args>

@@ -3,51 +3,109 @@
 // Every projection of a draft step (fusion F, QKV, O, gate/up, down, LM head;
 // Sec. 3.2 and the Llama block) is y[t] = W x[t] for a handful of activation
 // rows t, so the kernel is bound by reading W once from HBM.  Design:
-//   * persistent grid (2 CTAs of 16 warps per SM); CTA c owns a contiguous,
-//     balanced range of output units; its warps take units round-robin;
-//   * one warp computes whole rows: each lane streams 16-byte vectors of the
-//     weight row (ld.global.nc, no L1 allocation, U vectors in flight) and
-//     multiplies them with the activation rows staged in shared memory; a
-//     butterfly shuffle finishes each dot product (no atomics: deterministic);
-//   * the activation rows are built in the prologue (embedding gather +
+//   * persistent grid, one CTA per SM; CTA c owns a contiguous, balanced range
+//     of output rows, i.e. one contiguous byte range of W;
+//   * a producer lane streams that range through a ring of shared-memory
+//     stages with TMA bulk copies (cp.async.bulk, mbarrier complete_tx), each
+//     stage holding R whole rows.  It starts before griddepcontrol.wait, so
+//     under programmatic dependent launch the ring fills while the previous
+//     kernel finishes;
+//   * sixteen consumer warps form G groups; group g owns the stages s with
+//     s % G == g (the stage count is a multiple of G) and takes them in
+//     order, so every stage has exactly one consumer group and no waiter can
+//     run two ring phases ahead of a barrier (parity waits stay
+//     unambiguous); G groups work on G stages at once.  Warps compute whole
+//     rows, or with fewer rows than warps per group, column segments whose
+//     partial sums are added in fixed segment order after a group barrier:
+//     no atomics, deterministic;
+//   * the prologue builds the activation rows (embedding gather +
 //     concatenation, RMSNorm with its gain, bf16 rounding) from the previous
-//     kernel's fp32 output, so no separate norm/concat kernels run;
-//   * the epilogue fuses the residual add, SwiGLU, or (LM head) the logits
-//     write and a top-8 selection whose per-CTA partials are merged by the
-//     last CTA to finish (a two-pass vocabulary argmax without a second launch);
-//   * programmatic dependent launch: before griddepcontrol.wait each CTA asks
-//     the TMA engine to prefetch the start of its weight range into L2, so the
-//     weight stream overlaps the previous kernel's tail.
+//     kernel's fp32 output; the epilogue fuses the residual add, SwiGLU, or
+//     (LM head) the logits write and a top-8 selection whose per-CTA partials
+//     are merged by the last CTA to finish (two-pass vocabulary argmax without
+//     a second launch);
+//   * every mbarrier wait is bounded; on expiry the kernel sets the timeout bit
+//     of the device error word, skips the rest of its work (still reaching
+//     every named barrier), drains its copies in flight and returns.
 #include "common.cuh"
 
 namespace prism {
 
 namespace {
 
-constexpr int kPrefetchBytes = 64 * 1024;
-constexpr int kPrefetchPiece = 16 * 1024;
+constexpr int kConsumers = 16;
+constexpr int kThreads = (kConsumers + 1) * 32;
+constexpr int kMaxStages = 16;
+constexpr long kWaitLimit = 1L << 22;
+constexpr size_t kChunkTarget = 32 * 1024;
+constexpr size_t kSmemAlone = 200 * 1024;
 
-template <typename WT>
-__device__ __forceinline__ void fma_vec(float &acc, const uint4 &w, const uint4 &x);
+__device__ __forceinline__ uint32_t saddr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
-template <>
-__device__ __forceinline__ void fma_vec<uint16_t>(float &acc, const uint4 &w, const uint4 &x) {
-    acc = fmaf(bf16lo(w.x), bf16lo(x.x), acc);
-    acc = fmaf(bf16hi(w.x), bf16hi(x.x), acc);
-    acc = fmaf(bf16lo(w.y), bf16lo(x.y), acc);
-    acc = fmaf(bf16hi(w.y), bf16hi(x.y), acc);
-    acc = fmaf(bf16lo(w.z), bf16lo(x.z), acc);
-    acc = fmaf(bf16hi(w.z), bf16hi(x.z), acc);
-    acc = fmaf(bf16lo(w.w), bf16lo(x.w), acc);
-    acc = fmaf(bf16hi(w.w), bf16hi(x.w), acc);
+__device__ __forceinline__ void mbar_init(uint64_t *b, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(saddr(b)), "r"(count));
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t *b) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(saddr(b)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint64_t *b, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(saddr(b)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+                 : "=r"(ok) : "r"(saddr(b)), "r"(parity) : "memory");
+    return ok != 0;
+}
+// Bounded wait for the completion of the phase with the given parity.
+__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity) {
+    for (long i = 0; i < kWaitLimit; ++i)
+        if (mbar_try(b, parity)) return true;
+    return false;
+}
+// 1-D TMA bulk copy global -> shared, completing on mbarrier b.
+__device__ __forceinline__ void tma_load(void *dst, const void *src, uint32_t bytes, uint64_t *b) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(saddr(dst)), "l"(src), "r"(bytes), "r"(saddr(b)) : "memory");
+}
+// Barrier among the consumer warps only (the producer warp never joins).
+__device__ __forceinline__ void consumers_sync() {
+    asm volatile("bar.sync 1, %0;" ::"r"(kConsumers * 32) : "memory");
 }
 
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+// Packed pair of fp32 lanes: acc += a * b on both halves (one FFMA2).
+__device__ __forceinline__ void ffma2(unsigned long long &acc, unsigned long long a, unsigned long long b) {
+    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(acc) : "l"(a), "l"(b));
+}
+__device__ __forceinline__ unsigned long long pack2(uint32_t lo, uint32_t hi) {
+    return ((unsigned long long)hi << 32) | lo;
+}
+__device__ __forceinline__ float sum2(unsigned long long v) {
+    return __uint_as_float((uint32_t)v) + __uint_as_float((uint32_t)(v >> 32));
+}
+// Two packed accumulators += 8 weights times 8 activations, both given as
+// one 16-byte vector of the storage type (bf16 pairs are widened exactly).
+template <typename WT>
+__device__ __forceinline__ void dot16B(unsigned long long &a0, unsigned long long &a1, const uint4 &w,
+                                       const uint4 &x);
 template <>
-__device__ __forceinline__ void fma_vec<float>(float &acc, const uint4 &w, const uint4 &x) {
-    acc = fmaf(__uint_as_float(w.x), __uint_as_float(x.x), acc);
-    acc = fmaf(__uint_as_float(w.y), __uint_as_float(x.y), acc);
-    acc = fmaf(__uint_as_float(w.z), __uint_as_float(x.z), acc);
-    acc = fmaf(__uint_as_float(w.w), __uint_as_float(x.w), acc);
+__device__ __forceinline__ void dot16B<uint16_t>(unsigned long long &a0, unsigned long long &a1, const uint4 &w,
+                                                 const uint4 &x) {
+    ffma2(a0, pack2(w.x << 16, w.x & 0xFFFF0000u), pack2(x.x << 16, x.x & 0xFFFF0000u));
+    ffma2(a1, pack2(w.y << 16, w.y & 0xFFFF0000u), pack2(x.y << 16, x.y & 0xFFFF0000u));
+    ffma2(a0, pack2(w.z << 16, w.z & 0xFFFF0000u), pack2(x.z << 16, x.z & 0xFFFF0000u));
+    ffma2(a1, pack2(w.w << 16, w.w & 0xFFFF0000u), pack2(x.w << 16, x.w & 0xFFFF0000u));
+}
+template <>
+__device__ __forceinline__ void dot16B<float>(unsigned long long &a0, unsigned long long &a1, const uint4 &w,
+                                              const uint4 &x) {
+    ffma2(a0, pack2(w.x, w.y), pack2(x.x, x.y));
+    ffma2(a1, pack2(w.z, w.w), pack2(x.z, x.w));
 }
 
 __device__ __forceinline__ float warp_sum(float v) {
@@ -56,20 +114,17 @@ __device__ __forceinline__ float warp_sum(float v) {
     return v;
 }
 
-// Deterministic block-wide sum (same tree in every CTA).
-__device__ float block_sum(float v, float *red) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+// Deterministic sum over the consumer threads (same tree in every CTA).
+__device__ float consumers_sum(float v, float *red) {
+    const int lane = threadIdx.x & 31, w = (threadIdx.x >> 5) - 1;
     v = warp_sum(v);
-    __syncthreads();
-    if (lane == 0) red[warp] = v;
-    __syncthreads();
+    consumers_sync();
+    if (lane == 0) red[w] = v;
+    consumers_sync();
     float s = 0.f;
-    if (threadIdx.x == 0) {
-        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += red[w];
-        red[32] = s;
-    }
-    __syncthreads();
-    return red[32];
+#pragma unroll
+    for (int i = 0; i < kConsumers; ++i) s += red[i];
+    return s;
 }
 
 __device__ __forceinline__ int clamp_nnew(const GemvArgs &a, int b) {
@@ -89,11 +144,17 @@ __device__ __forceinline__ int checked_token(const GemvArgs &a, int tok) {
     return tok;
 }
 
-// Build activation rows [t0, t0 + tc) in shared memory X ([TC][kin] WT);
-// rows tc..TC-1 are zeroed.
+template <typename WT>
+__device__ __forceinline__ void put(WT *x, int i, float v) {
+    if constexpr (sizeof(WT) == 2) x[i] = f32_to_bf16(v); else x[i] = v;
+}
+
+// Build activation rows [t0, t0 + tc) in shared memory X ([TC][kin] in the
+// weight type, rounded per the numeric contract), rows tc..TC-1 zeroed.
+// Consumer threads only.
 template <typename WT, int TC>
 __device__ void stage_x(const GemvArgs &a, int t0, int tc, WT *X, float *red) {
-    const int NT = blockDim.x, tid = threadIdx.x;
+    const int NT = kConsumers * 32, tid = threadIdx.x - 32;
     const int kin = a.kin, d = a.d;
     const WT *E = (const WT *)a.embed;
     for (int t = 0; t < TC; ++t) {
@@ -121,8 +182,7 @@ __device__ void stage_x(const GemvArgs &a, int t0, int tc, WT *X, float *red) {
             const float *h = a.src + (size_t)b * d;
             for (int c = tid; c < d; c += NT) {
                 xr[c] = er[c];
-                float v = Elem<WT>::round(h[c]);
-                if constexpr (sizeof(WT) == 2) xr[d + c] = f32_to_bf16(v); else xr[d + c] = v;
+                put<WT>(xr, d + c, Elem<WT>::round(h[c]));
             }
         } else if (a.pro == kProNorm) {
             const int sr = a.src_prefill_rows ? (row * a.max_new + clamp_nnew(a, row) - 1) : row;
@@ -131,14 +191,13 @@ __device__ void stage_x(const GemvArgs &a, int t0, int tc, WT *X, float *red) {
             if (a.gain) {
                 float ss = 0.f;
                 for (int c = tid; c < d; c += NT) ss = fmaf(s[c], s[c], ss);
-                ss = block_sum(ss, red);
+                ss = consumers_sum(ss, red);
                 inv = 1.0f / sqrtf(ss / (float)d + a.eps);
             }
             const WT *g = (const WT *)a.gain;
             for (int c = tid; c < d; c += NT) {
                 float v = a.gain ? s[c] * inv * Elem<WT>::load(g, c) : s[c];
-                v = Elem<WT>::round(v);
-                if constexpr (sizeof(WT) == 2) xr[c] = f32_to_bf16(v); else xr[c] = v;
+                put<WT>(xr, c, Elem<WT>::round(v));
             }
         } else {  // kProCopy
             const WT *src = (const WT *)a.act + (size_t)row * kin;
@@ -165,143 +224,239 @@ __device__ void warp_merge_top8(float (&v)[kTopK], int (&id)[kTopK]) {
     }
 }
 
+struct RingPlan {
+    int R;          // rows (units) per stage
+    int stages;     // a multiple of G
+    int G;          // consumer warp groups
+    size_t stage_bytes, x_bytes;
+};
+
 template <typename WT, int TC, int RPW, bool TOPK>
-__global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const GemvArgs a) {
-    extern __shared__ __align__(16) uint8_t smem_raw[];
-    __shared__ float red[33];
-    __shared__ float s_val[TOPK ? kGemvWarps : 1][TOPK ? TC : 1][kTopK];
-    __shared__ int s_id[TOPK ? kGemvWarps : 1][TOPK ? TC : 1][kTopK];
+__global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, const RingPlan plan) {
+    extern __shared__ __align__(128) uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full[kMaxStages], empty[kMaxStages];
+    __shared__ float red[kConsumers];
+    __shared__ float s_val[TOPK ? kConsumers : 1][TOPK ? TC : 1][kTopK];
+    __shared__ int s_id[TOPK ? kConsumers : 1][TOPK ? TC : 1][kTopK];
     __shared__ int s_last;
+    // per-chunk partial sums of the column segments, double-buffered by chunk
+    __shared__ float s_part[2][kConsumers][RPW][TC];   // column-segment partials
 
     constexpr int VEC = Elem<WT>::kPerVec;
-    constexpr int U0 = TC == 1 ? 8 : (TC == 4 ? 4 : 2);
-    constexpr int U = U0 / RPW > 0 ? U0 / RPW : 1;
-    WT *X = (WT *)smem_raw;
+    constexpr int U = TC <= 2 ? 4 : (TC == 4 ? 2 : 1);
+    static_assert(sizeof(WT) == 2 || sizeof(WT) == 4, "weight type");
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int u_begin = (int)((long long)blockIdx.x * a.n_units / gridDim.x);
-    const int u_end = (int)((long long)(blockIdx.x + 1) * a.n_units / gridDim.x);
+    const int R = plan.R, S = plan.stages;
     const size_t row_bytes = (size_t)a.kin * sizeof(WT);
+    const int u0 = (int)((long long)blockIdx.x * a.n_units / gridDim.x);
+    const int u1 = (int)((long long)(blockIdx.x + 1) * a.n_units / gridDim.x);
+    const int n_chunks = (u1 - u0 + R - 1) / R;
+    const int n_pass = (a.T + TC - 1) / TC;
+    uint8_t *ring = smem_raw;
+    WT *X = (WT *)(smem_raw + (size_t)S * plan.stage_bytes);
 
     pdl_trigger();
-    if (threadIdx.x == 0 && u_end > u_begin) {
-        // prefetch the start of this CTA's weight range (RPW ranges)
-        for (int r = 0; r < RPW; ++r) {
-            const uint8_t *base = (const uint8_t *)a.W + ((size_t)u_begin + (size_t)r * a.pair_offset) * row_bytes;
-            size_t total = (size_t)(u_end - u_begin) * row_bytes;
-            size_t lim = total < (size_t)(kPrefetchBytes / RPW) ? total : (size_t)(kPrefetchBytes / RPW);
-            for (size_t off = 0; off < lim; off += kPrefetchPiece) {
-                size_t n = lim - off < (size_t)kPrefetchPiece ? lim - off : (size_t)kPrefetchPiece;
-                prefetch_l2_bulk(base + off, (uint32_t)(n & ~(size_t)15));
-            }
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], kConsumers / plan.G);
         }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
+    __syncthreads();
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane != 0) return;
+        const long total = (long)n_pass * n_chunks;
+        long issued = 0;
+        for (long i = 0; i < total; ++i) {
+            const int s = (int)(i % S);
+            const uint32_t it = (uint32_t)(i / S);
+            if (!mbar_wait(&empty[s], (it & 1) ^ 1)) {
+                set_err(a.err, kErrTimeout);
+                break;
+            }
+            const int c = (int)(i % n_chunks);
+            const int first = u0 + c * R;
+            const int rows = u1 - first < R ? u1 - first : R;
+            const uint32_t bytes = (uint32_t)(rows * row_bytes);
+            if (PRISM_CHECK(a.err, (size_t)s * plan.stage_bytes + (size_t)(RPW - 1) * R * row_bytes + bytes <=
+                                       (size_t)S * plan.stage_bytes, 101, s, bytes) ||
+                PRISM_CHECK(a.err, first + rows <= a.n_units && first >= 0, 102, first, rows) ||
+                PRISM_CHECK(a.err, (((uintptr_t)a.W) & 15) == 0 && (row_bytes & 15) == 0, 103, 0, row_bytes))
+                break;
+            mbar_arrive_tx(&full[s], bytes * RPW);
+            uint8_t *st = ring + (size_t)s * plan.stage_bytes;
+#pragma unroll
+            for (int r = 0; r < RPW; ++r)
+                tma_load(st + (size_t)r * R * row_bytes,
+                         (const uint8_t *)a.W + ((size_t)first + (size_t)r * a.pair_offset) * row_bytes, bytes,
+                         &full[s]);
+            issued = i + 1;
+        }
+        // drain: the last stages' copies land before this CTA may exit
+        for (long i = issued > S ? issued - S : 0; i < issued; ++i)
+            if (!mbar_wait(&full[i % S], (uint32_t)((i / S) & 1))) set_err(a.err, kErrTimeout);
+        return;
+    }
+
+    // ---------------------------------------------------------------- consumers
+    const int cw = warp - 1;
+    const int G = plan.G, Wg = kConsumers / G;                // groups, warps per group
+    const int grp = cw / Wg, gw = cw % Wg;
+    const int SEG = R >= Wg ? 1 : Wg / R;                     // column segments per row
+    const int seg = gw % SEG;
+    const int nvec = a.kin / VEC;
+    const int v_lo = (int)((long)seg * nvec / SEG), v_hi = (int)((long)(seg + 1) * nvec / SEG);
+    const int rr0 = SEG == 1 ? gw : gw / SEG, rstep = SEG == 1 ? Wg : R;
+    const uint32_t x_base = saddr(X);
+    const uint32_t ring_base = saddr(ring);
+    bool dead = false;
+    int lc = 0;                                               // chunks this group has taken
     pdl_wait();
 
-    const int nvec = a.kin / VEC;
-    const uint4 *X4 = (const uint4 *)X;
-
-    for (int t0 = 0; t0 < a.T; t0 += TC) {
+    for (int p = 0; p < n_pass; ++p) {
+        const int t0 = p * TC;
         const int tc = a.T - t0 < TC ? a.T - t0 : TC;
         stage_x<WT, TC>(a, t0, tc, X, red);
-        __syncthreads();
-
-        // LM head: lane t keeps the top-8 list of activation row t0 + t in
-        // shared memory (s_val/s_id[warp][t]) and only its current 8th-best
-        // entry in registers; a logit that beats it is inserted (rare).
-        float thr_v = -INFINITY;
-        int thr_i = 0x7FFFFFFF;
         if constexpr (TOPK) {
             if (lane < TC) {
 #pragma unroll
-                for (int i = 0; i < kTopK; ++i) { s_val[warp][lane][i] = -INFINITY; s_id[warp][lane][i] = 0x7FFFFFFF; }
+                for (int i = 0; i < kTopK; ++i) { s_val[cw][lane][i] = -INFINITY; s_id[cw][lane][i] = 0x7FFFFFFF; }
             }
         }
+        consumers_sync();
+        float thr_v = -INFINITY;
+        int thr_i = 0x7FFFFFFF;
 
-        for (int u = u_begin + warp; u < u_end; u += kGemvWarps) {
-            const uint4 *wr[RPW];
+        for (int c = grp; c < n_chunks; c += G, ++lc) {
+            const long i = (long)p * n_chunks + c;
+            const int s = (int)(i % S);
+            if (!dead && !mbar_wait(&full[s], (uint32_t)((i / S) & 1))) {
+                set_err(a.err, kErrTimeout);
+                dead = true;
+            }
+            const int first = u0 + c * R;
+            const int rows = u1 - first < R ? u1 - first : R;
+            for (int rr = rr0; rr < R; rr += rstep) {
+                bool live = !dead && rr < rows;
+                if (live && (PRISM_CHECK(a.err, ((size_t)(RPW - 1) * R + rr + 1) * nvec * 16 <= plan.stage_bytes, 104, rr, nvec) ||
+                             PRISM_CHECK(a.err, (size_t)TC * a.kin * sizeof(WT) <= plan.x_bytes, 105, TC, a.kin)))
+                    live = false;   // skip the access, keep the barrier sequence
+                unsigned long long p0[RPW][TC], p1[RPW][TC];
 #pragma unroll
-            for (int r = 0; r < RPW; ++r)
-                wr[r] = (const uint4 *)((const uint8_t *)a.W + ((size_t)u + (size_t)r * a.pair_offset) * row_bytes);
-            float acc[RPW][TC];
+                for (int r = 0; r < RPW; ++r)
 #pragma unroll
-            for (int r = 0; r < RPW; ++r)
-#pragma unroll
-                for (int t = 0; t < TC; ++t) acc[r][t] = 0.f;
-
-            for (int v0 = lane; v0 < nvec; v0 += 32 * U) {
-                uint4 wv[RPW][U];
-#pragma unroll
-                for (int j = 0; j < U; ++j) {
-                    const int v = v0 + 32 * j;
+                    for (int t = 0; t < TC; ++t) p0[r][t] = p1[r][t] = 0ull;
+                if (live) {
+                    uint32_t wa[RPW];
 #pragma unroll
                     for (int r = 0; r < RPW; ++r)
-                        wv[r][j] = v < nvec ? ldg_stream(wr[r] + v) : make_uint4(0u, 0u, 0u, 0u);
-                }
+                        wa[r] = ring_base + (uint32_t)(s * plan.stage_bytes) + (uint32_t)(((r * R + rr) * nvec) * 16);
+                    const int vb = SEG == 1 ? 0 : v_lo, ve = SEG == 1 ? nvec : v_hi;
+                    int v = vb + lane;
+                    for (; v + 32 * (U - 1) < ve; v += 32 * U) {
+                        uint4 wv[RPW][U];
 #pragma unroll
-                for (int j = 0; j < U; ++j) {
-                    const int v = v0 + 32 * j;
-                    if (v < nvec) {
+                        for (int j = 0; j < U; ++j)
+#pragma unroll
+                            for (int r = 0; r < RPW; ++r) wv[r][j] = lds128(wa[r] + (uint32_t)(v + 32 * j) * 16u);
+#pragma unroll
+                        for (int j = 0; j < U; ++j) {
+#pragma unroll
+                            for (int t = 0; t < TC; ++t) {
+                                const uint4 xv = lds128(x_base + (uint32_t)(t * nvec + v + 32 * j) * 16u);
+#pragma unroll
+                                for (int r = 0; r < RPW; ++r) dot16B<WT>(p0[r][t], p1[r][t], wv[r][j], xv);
+                            }
+                        }
+                    }
+                    for (; v < ve; v += 32) {
 #pragma unroll
                         for (int t = 0; t < TC; ++t) {
-                            const uint4 xv = X4[(size_t)t * nvec + v];
+                            const uint4 xv = lds128(x_base + (uint32_t)(t * nvec + v) * 16u);
 #pragma unroll
-                            for (int r = 0; r < RPW; ++r) fma_vec<WT>(acc[r][t], wv[r][j], xv);
+                            for (int r = 0; r < RPW; ++r)
+                                dot16B<WT>(p0[r][t], p1[r][t], lds128(wa[r] + (uint32_t)v * 16u), xv);
                         }
                     }
                 }
-            }
+                float acc[RPW][TC];
 #pragma unroll
-            for (int r = 0; r < RPW; ++r)
+                for (int r = 0; r < RPW; ++r)
 #pragma unroll
-                for (int t = 0; t < TC; ++t) acc[r][t] = warp_sum(acc[r][t]);
-
-            // epilogue: lane t handles activation row t0 + t
+                    for (int t = 0; t < TC; ++t) acc[r][t] = warp_sum(sum2(p0[r][t]) + sum2(p1[r][t]));
+                if (SEG > 1) {
+                    // add the row's column segments in segment order (group barrier)
+                    const int buf = lc & 1;
+                    if (lane == 0) {
 #pragma unroll
-            for (int t = 0; t < TC; ++t) {
-                if (lane != t || t >= tc) continue;
-                const int row = t0 + t;
-                if constexpr (TOPK) {
-                    const float z = acc[0][t];
-                    if (a.logits) a.logits[((size_t)row * a.K + a.step - 1) * a.vocab + u] = z;
-                    if (better(z, u, thr_v, thr_i)) {
-                        float *lv = s_val[warp][t];
-                        int *li = s_id[warp][t];
-                        int pos = kTopK - 1;
-                        while (pos > 0 && better(z, u, lv[pos - 1], li[pos - 1])) {
-                            lv[pos] = lv[pos - 1];
-                            li[pos] = li[pos - 1];
-                            --pos;
+                        for (int r = 0; r < RPW; ++r)
+#pragma unroll
+                            for (int t = 0; t < TC; ++t) s_part[buf][cw][r][t] = acc[r][t];
+                    }
+                    asm volatile("bar.sync %0, %1;" ::"r"(2 + grp), "r"(Wg * 32) : "memory");
+                    if (seg != 0) continue;
+#pragma unroll
+                    for (int r = 0; r < RPW; ++r)
+#pragma unroll
+                        for (int t = 0; t < TC; ++t) {
+                            float v2 = 0.f;
+                            for (int q = 0; q < SEG; ++q) v2 += s_part[buf][cw + q][r][t];
+                            acc[r][t] = v2;
                         }
-                        lv[pos] = z;
-                        li[pos] = u;
-                        thr_v = lv[kTopK - 1];
-                        thr_i = li[kTopK - 1];
+                }
+                if (!live) continue;
+                const int u = first + rr;
+#pragma unroll
+                for (int t = 0; t < TC; ++t) {
+                    if (lane != t || t >= tc) continue;
+                    const int row = t0 + t;
+                    if constexpr (TOPK) {
+                        const float z = acc[0][t];
+                        if (a.logits) a.logits[((size_t)row * a.K + a.step - 1) * a.vocab + u] = z;
+                        if (better(z, u, thr_v, thr_i)) {
+                            float *lv = s_val[cw][t];
+                            int *li = s_id[cw][t];
+                            int pos = kTopK - 1;
+                            while (pos > 0 && better(z, u, lv[pos - 1], li[pos - 1])) {
+                                lv[pos] = lv[pos - 1];
+                                li[pos] = li[pos - 1];
+                                --pos;
+                            }
+                            lv[pos] = z;
+                            li[pos] = u;
+                            thr_v = lv[kTopK - 1];
+                            thr_i = li[kTopK - 1];
+                        }
+                    } else if constexpr (RPW == 2) {
+                        const float g = acc[0][t], up = acc[1][t];
+                        Elem<WT>::store((WT *)a.out_act, (size_t)row * a.out_ld + u, g / (1.0f + expf(-g)) * up);
+                    } else {
+                        float val = acc[0][t];
+                        if (a.epi == kEpiResid) {
+                            const int rrow = a.resid_prefill_rows ? (row * a.max_new + clamp_nnew(a, row) - 1) : row;
+                            val += a.resid[(size_t)rrow * a.out_ld + u];
+                            if (a.hidden_out) a.hidden_out[((size_t)row * a.K + a.step - 1) * a.d + u] = val;
+                        }
+                        a.out[(size_t)row * a.out_ld + u] = val;
                     }
-                } else if constexpr (RPW == 2) {
-                    const float g = acc[0][t], up = acc[1][t];
-                    const float m = g / (1.0f + expf(-g)) * up;
-                    Elem<WT>::store((WT *)a.out_act, (size_t)row * a.out_ld + u, m);
-                } else {
-                    float val = acc[0][t];
-                    if (a.epi == kEpiResid) {
-                        const int rr = a.resid_prefill_rows ? (row * a.max_new + clamp_nnew(a, row) - 1) : row;
-                        val += a.resid[(size_t)rr * a.out_ld + u];
-                        if (a.hidden_out) a.hidden_out[((size_t)row * a.K + a.step - 1) * a.d + u] = val;
-                    }
-                    a.out[(size_t)row * a.out_ld + u] = val;
                 }
             }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[s]);
         }
 
         if constexpr (TOPK) {
-            // per-CTA merge of the warps' lists, one warp per activation row
-            __syncthreads();
-            for (int t = warp; t < tc; t += kGemvWarps) {
+            // per-CTA merge of the consumer warps' lists, one warp per activation row
+            consumers_sync();
+            for (int t = cw; t < tc; t += kConsumers) {
                 float v[kTopK];
                 int id[kTopK];
                 top8_init(v, id);
-                for (int c = lane; c < kGemvWarps * kTopK; c += 32)
-                    top8_insert(v, id, s_val[c / kTopK][t][c % kTopK], s_id[c / kTopK][t][c % kTopK]);
+                for (int c2 = lane; c2 < kConsumers * kTopK; c2 += 32)
+                    top8_insert(v, id, s_val[c2 / kTopK][t][c2 % kTopK], s_id[c2 / kTopK][t][c2 % kTopK]);
                 warp_merge_top8(v, id);
                 if (lane == 0) {
                     const size_t base = (((size_t)(t0 + t)) * gridDim.x + blockIdx.x) * kTopK;
@@ -310,25 +465,25 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const GemvArgs a)
                 }
             }
         }
-        __syncthreads();
+        consumers_sync();
     }
 
     if constexpr (TOPK) {
         // the last CTA to finish merges every CTA's partial lists
         __threadfence();
-        __syncthreads();
-        if (threadIdx.x == 0) s_last = (atomicAdd(a.counter, 1) == (int)gridDim.x - 1);
-        __syncthreads();
+        consumers_sync();
+        if (threadIdx.x == 32) s_last = (atomicAdd(a.counter, 1) == (int)gridDim.x - 1);
+        consumers_sync();
         if (!s_last) return;
         __threadfence();
-        const int G = gridDim.x;
-        for (int t = warp; t < a.T; t += kGemvWarps) {
+        const int Gd = gridDim.x;
+        for (int t = cw; t < a.T; t += kConsumers) {
             float v[kTopK];
             int id[kTopK];
             top8_init(v, id);
-            const size_t base = (size_t)t * G * kTopK;
-            for (int c = lane; c < G * kTopK; c += 32)
-                top8_insert(v, id, __ldcg(a.lm_part + base + c), __ldcg(a.lm_part_id + base + c));
+            const size_t base = (size_t)t * Gd * kTopK;
+            for (int c2 = lane; c2 < Gd * kTopK; c2 += 32)
+                top8_insert(v, id, __ldcg(a.lm_part + base + c2), __ldcg(a.lm_part_id + base + c2));
             warp_merge_top8(v, id);
             if (lane == 0) {
                 const size_t o = (size_t)t * a.K + a.step - 1;
@@ -342,17 +497,18 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const GemvArgs a)
                 }
             }
         }
-        if (threadIdx.x == 0) *a.counter = 0;
+        if (threadIdx.x == 32) *a.counter = 0;
     }
 }
 
 template <typename WT, int TC>
-cudaError_t dispatch_kind(const GemvArgs &a, int grid, size_t smem, cudaStream_t s, bool pdl) {
+cudaError_t dispatch_kind(const GemvArgs &a, const RingPlan &pl, int grid, size_t smem, cudaStream_t s,
+                          bool pdl) {
     if (a.epi == kEpiTopK)
-        return launch_k(gemv_kernel<WT, TC, 1, true>, dim3(grid), dim3(kGemvThreads), smem, s, pdl, a);
+        return launch_k(gemv_kernel<WT, TC, 1, true>, dim3(grid), dim3(kThreads), smem, s, pdl, a, pl);
     if (a.epi == kEpiSwiGLU)
-        return launch_k(gemv_kernel<WT, TC, 2, false>, dim3(grid), dim3(kGemvThreads), smem, s, pdl, a);
-    return launch_k(gemv_kernel<WT, TC, 1, false>, dim3(grid), dim3(kGemvThreads), smem, s, pdl, a);
+        return launch_k(gemv_kernel<WT, TC, 2, false>, dim3(grid), dim3(kThreads), smem, s, pdl, a, pl);
+    return launch_k(gemv_kernel<WT, TC, 1, false>, dim3(grid), dim3(kThreads), smem, s, pdl, a, pl);
 }
 
 template <typename WT>
@@ -363,45 +519,94 @@ cudaError_t set_smem_attrs(int bytes) {
         e = cudaFuncSetAttribute(gemv_kernel<WT, TC, RPW, TK>,                                   \
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     PRISM_SET(1, 1, true) PRISM_SET(1, 2, false) PRISM_SET(1, 1, false)
+    PRISM_SET(2, 1, true) PRISM_SET(2, 2, false) PRISM_SET(2, 1, false)
     PRISM_SET(4, 1, true) PRISM_SET(4, 2, false) PRISM_SET(4, 1, false)
     PRISM_SET(8, 1, true) PRISM_SET(8, 2, false) PRISM_SET(8, 1, false)
 #undef PRISM_SET
     return e;
 }
 
+int rows_per_pass(int T) { return T <= 1 ? 1 : (T <= 2 ? 2 : (T <= 4 ? 4 : 8)); }
+
+// Ring plan: stage = R whole rows (R a power of two), G consumer groups, S
+// stages (a multiple of G).  Chosen for the fewest passes over W (largest
+// activation block), then the most bytes in flight within the budget, then
+// the preferred group count.
+bool make_plan(const GemvArgs &a, bool bf16, int &tc, RingPlan &pl, size_t &smem) {
+    const size_t es = bf16 ? 2 : 4;
+    const int RPW = a.epi == kEpiSwiGLU ? 2 : 1;
+    const size_t row = (size_t)a.kin * es;
+    const size_t target = a.chunk_target > 0 ? (size_t)a.chunk_target : kChunkTarget;
+    const size_t budget = a.smem_budget > 0 ? (size_t)a.smem_budget : kSmemAlone;
+    const int g_pref = a.groups > 0 ? a.groups : 4;
+    int R0 = 1;
+    while ((size_t)(R0 * 2) * row * RPW <= target && R0 < 64) R0 *= 2;
+    for (tc = rows_per_pass(a.T); tc >= 1; tc = tc == 1 ? 0 : tc / 2) {
+        const size_t x = (size_t)tc * row;
+        bool found = false;
+        size_t best_inflight = 0;
+        RingPlan best{};
+        for (int G : {g_pref, 4, 2, 8, 1, 16}) {
+            for (int R = R0; R >= 1; R /= 2) {
+                const size_t stage = (size_t)R * row * RPW;
+                if (x + (size_t)G * stage > budget) continue;
+                int S = (int)((budget - x) / stage);
+                if (S > kMaxStages) S = kMaxStages;
+                S = S / G * G;
+                if (S < 2) continue;
+                const size_t inflight = (size_t)S * stage;
+                if (!found || inflight > best_inflight + 16 * 1024) {
+                    found = true;
+                    best_inflight = inflight;
+                    best = RingPlan{R, S, G, stage, x};
+                }
+                break;   // largest R that fits for this G
+            }
+        }
+        if (found) {
+            pl = best;
+            smem = (size_t)pl.stages * pl.stage_bytes + pl.x_bytes;
+            return true;
+        }
+    }
+    return false;
+}
+
 }  // namespace
 
-// Shared-memory budget of the activation rows per CTA (two CTAs per SM).
-constexpr size_t kXBudget = 100 * 1024;
-
-int gemv_rows_per_pass(const GemvArgs &a, bool bf16) {
-    const size_t row = (size_t)a.kin * (bf16 ? 2 : 4);
-    int tc = a.T <= 1 ? 1 : (a.T <= 4 ? 4 : 8);
-    while (tc > 1 && (size_t)tc * row > kXBudget) tc = tc == 8 ? 4 : 1;
-    return tc;
-}
-
-size_t gemv_smem_bytes(const GemvArgs &a, bool bf16, int tc) {
-    return (size_t)tc * a.kin * (bf16 ? 2 : 4);
-}
-
 cudaError_t prepare_gemv_kernels() {
-    cudaError_t e = set_smem_attrs<uint16_t>((int)kXBudget);
-    if (e == cudaSuccess) e = set_smem_attrs<float>((int)kXBudget);
+    cudaError_t e = set_smem_attrs<uint16_t>((int)kSmemAlone);
+    if (e == cudaSuccess) e = set_smem_attrs<float>((int)kSmemAlone);
+    if (e == cudaSuccess) e = prepare_gemv_mma_kernels();
     return e;
 }
 
+bool gemv_supported(const GemvArgs &a, bool bf16) {
+    if (bf16 && gemv_mma_supported(a)) return true;
+    int tc;
+    RingPlan pl;
+    size_t smem;
+    return make_plan(a, bf16, tc, pl, smem);
+}
+
+// bf16 projections whose contraction length is a multiple of 32 run on the
+// tensor-core kernel (gemv_mma.cu); the rest on the CUDA-core ring kernel.
 cudaError_t launch_gemv(const GemvArgs &a, bool bf16, int grid, cudaStream_t s, bool pdl) {
-    const int tc = gemv_rows_per_pass(a, bf16);
-    const size_t smem = gemv_smem_bytes(a, bf16, tc);
+    if (bf16 && !a.force_cuda_core && gemv_mma_supported(a)) return launch_gemv_mma(a, grid, s, pdl);
+    int tc;
+    RingPlan pl;
+    size_t smem;
+    if (!make_plan(a, bf16, tc, pl, smem)) return cudaErrorInvalidValue;
     if (bf16) {
-        if (tc == 1) return dispatch_kind<uint16_t, 1>(a, grid, smem, s, pdl);
-        if (tc == 4) return dispatch_kind<uint16_t, 4>(a, grid, smem, s, pdl);
-        return dispatch_kind<uint16_t, 8>(a, grid, smem, s, pdl);
+        if (tc == 1) return dispatch_kind<uint16_t, 1>(a, pl, grid, smem, s, pdl);
+        if (tc == 2) return dispatch_kind<uint16_t, 2>(a, pl, grid, smem, s, pdl);
+        if (tc == 4) return dispatch_kind<uint16_t, 4>(a, pl, grid, smem, s, pdl);
+        return dispatch_kind<uint16_t, 8>(a, pl, grid, smem, s, pdl);
     }
-    if (tc == 1) return dispatch_kind<float, 1>(a, grid, smem, s, pdl);
-    if (tc == 4) return dispatch_kind<float, 4>(a, grid, smem, s, pdl);
-    return dispatch_kind<float, 8>(a, grid, smem, s, pdl);
+    if (tc == 1) return dispatch_kind<float, 1>(a, pl, grid, smem, s, pdl);
+    if (tc == 2) return dispatch_kind<float, 2>(a, pl, grid, smem, s, pdl);
+    if (tc == 4) return dispatch_kind<float, 4>(a, pl, grid, smem, s, pdl);
+    return dispatch_kind<float, 8>(a, pl, grid, smem, s, pdl);
 }
 
 }  // namespace prism

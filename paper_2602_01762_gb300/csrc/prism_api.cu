@@ -65,6 +65,8 @@ struct prism_ctx {
     // execution
     cudaStream_t cap_stream = nullptr;
     bool use_graph = true, use_pdl = true;
+    int gemv_chunk = 0, gemv_smem = 0, gemv_groups = 0;   // projection ring knobs (0 = built-in default)
+    int gemv_cuda_core = 1;                               // 1: bf16 projections on CUDA cores
     std::vector<GraphEntry> graphs;
     unsigned long long tick = 0;
     std::string error;
@@ -92,10 +94,9 @@ void drop_graphs(prism_ctx *c) {
     c->graphs.clear();
 }
 
+// Persistent projection grid: one CTA per SM (never more CTAs than units).
 int gemv_grid(const prism_ctx *c, int units) {
-    int g = (units + 3) / 4;
-    int cap = 2 * c->sms;
-    return g < 1 ? 1 : (g > cap ? cap : g);
+    return units < c->sms ? (units < 1 ? 1 : units) : c->sms;
 }
 
 // Enqueue one round.  prof_ev != null: record an event before the first and
@@ -109,6 +110,22 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
     int nk = 0;
     bool first = true;
     auto after = [&](int kind) {
+#ifdef PRISM_CHECKED
+        // checked builds run eagerly: localise a failing kernel
+        cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+        cudaStreamIsCapturing(s, &cap);
+        if (e == cudaSuccess && cap == cudaStreamCaptureStatusNone) {
+            cudaError_t se = cudaStreamSynchronize(s);
+            if (se != cudaSuccess) {
+                std::fprintf(stderr, "prism checked: kernel #%d (kind %d) failed: %s\n", nk, kind, cudaGetErrorString(se));
+                e = se;
+            }
+            int w[5] = {0};
+            if (cudaMemcpy(w, c->err, sizeof(w), cudaMemcpyDeviceToHost) == cudaSuccess && (w[0] || w[1]))
+                std::fprintf(stderr, "prism checked: after kernel #%d (kind %d): err 0x%x check %d block %d values %d %d\n",
+                             nk, kind, w[0], w[1], w[2], w[3], w[4]);
+        }
+#endif
         if (prof_ev) {
             if (nk < kMaxProfileKernels) {
                 cudaEventRecord(prof_ev[nk + 1], s);
@@ -133,6 +150,10 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
     base.d = d;
     base.err = c->err;
     base.topk = f.topk;
+    base.chunk_target = c->gemv_chunk;
+    base.smem_budget = c->gemv_smem;
+    base.groups = c->gemv_groups;
+    base.force_cuda_core = c->gemv_cuda_core;
 
     for (int k = 1; k <= K && e == cudaSuccess; ++k) {
         const prism_step_weights &w = c->steps[k - 1];
@@ -346,7 +367,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     const int d = f.hidden, Hq = f.n_q_heads, Hkv = f.n_kv_heads, D = f.head_dim, F = f.ffn;
     const size_t es = c->bf16 ? 2 : 4;
     c->qkv_rows = (Hq + 2 * Hkv) * D;
-    c->lm_grid = (f.vocab + 15) / 16 < 2 * c->sms ? (f.vocab + 15) / 16 : 2 * c->sms;
+    c->lm_grid = f.vocab < c->sms ? f.vocab : c->sms;
     // attention split size: enough CTAs to cover the GPU at batch 1
     c->attn_chunk = 64;
     if ((long long)f.max_batch * Hkv * ((f.max_ctx + 63) / 64) < 2LL * c->sms) c->attn_chunk = 32;
@@ -359,7 +380,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         T1 * d * 4,                                                // x0
         T1 * c->qkv_rows * 4,                                      // qkv
         B * Hq * D * 4,                                            // q
-        B * Hq * (size_t)c->attn_splits * (D + 2) * 4,             // attention partials
+        B * Hq * (size_t)c->attn_splits * (D + 4) * 4,             // attention partials
         B * d * 4,                                                 // a
         B * d * 4,                                                 // h^
         B * Hq * D * es,                                           // o
@@ -367,7 +388,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         B * (size_t)c->lm_grid * kTopK * 4,                        // LM partial values
         B * (size_t)c->lm_grid * kTopK * 4,                        // LM partial ids
         (B * Hkv + 1) * 4,                                         // counters
-        4,                                                         // error word
+        32,                                                        // error word (+ checked-build record)
     };
     size_t total = 0;
     for (size_t s : sizes) total += align256(s);
@@ -407,7 +428,29 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     e = cudaMemcpy(c->rope_cos, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(c->rope_sin, sn.data(), sn.size() * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = prepare_gemv_kernels();
-    if (e == cudaSuccess) e = prepare_attention_kernel(c->bf16, D, c->attn_chunk, Hq / Hkv);
+    if (e == cudaSuccess) {
+        // every projection shape must fit the shared-memory ring
+        const int T1 = f.max_batch * f.max_new;
+        const int kins[] = {2 * d, d, Hq * D, d, F, d};
+        const int epis[] = {kEpiStore, kEpiStore, kEpiResid, kEpiSwiGLU, kEpiResid, kEpiTopK};
+        for (int i = 0; i < 6; ++i) {
+            GemvArgs g{};
+            g.kin = kins[i];
+            g.epi = epis[i];
+            g.T = i < 2 ? T1 : f.max_batch;
+            if (!gemv_supported(g, c->bf16)) {
+                cudaFree(ws);
+                delete c;
+                return fail(nullptr, PRISM_ERR_INVALID_ARG, "a projection row does not fit shared memory");
+            }
+        }
+    }
+    if (e == cudaSuccess && attention_smem_bytes(c->bf16, D, c->attn_chunk, Hq / Hkv, c->attn_splits) > 200 * 1024) {
+        cudaFree(ws);
+        delete c;
+        return fail(nullptr, PRISM_ERR_INVALID_ARG, "max_ctx too large for the attention combine");
+    }
+    if (e == cudaSuccess) e = prepare_attention_kernel(c->bf16, D, c->attn_chunk, Hq / Hkv, c->attn_splits);
     if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking);
     if (e != cudaSuccess) {
         prism_status st = cuda_fail(nullptr, e, "context setup");
@@ -458,6 +501,11 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     if (!c || !name) return fail(c, PRISM_ERR_INVALID_ARG, "null argument");
     if (!std::strcmp(name, "use_graph")) c->use_graph = value != 0;
     else if (!std::strcmp(name, "use_pdl")) c->use_pdl = value != 0;
+    else if (!std::strcmp(name, "gemv_chunk_kb") && value >= 0 && value <= 128) c->gemv_chunk = value * 1024;
+    else if (!std::strcmp(name, "gemv_smem_kb") && value >= 0 && value <= 200) c->gemv_smem = value * 1024;
+    else if (!std::strcmp(name, "gemv_groups") && (value == 0 || value == 1 || value == 2 || value == 4 ||
+                                                   value == 8 || value == 16)) c->gemv_groups = value;
+    else if (!std::strcmp(name, "gemv_cuda_core")) c->gemv_cuda_core = value != 0;
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);
     return PRISM_OK;

@@ -99,6 +99,17 @@ def test_modes_are_bit_identical():
             assert np.array_equal(r[key], runs[0][key]), key
 
 
+def test_tensor_core_projection_path_matches_oracle():
+    """The warp-level tensor-core projection kernel (option gemv_cuda_core=0)
+    meets the same bar as the default CUDA-core kernel."""
+    W, I = mid_case()
+    g = gpu_round(MID_W, W, I, topk=8, options={"gemv_cuda_core": 0})
+    assert g["flags"] == 0
+    o = oracle.draft_round(MID_W.shape, W, I, topk=8, want_logits=True, seqs=[0, 1, 2])
+    compare_round(g, o, I, [0, 1, 2], MID_W.shape.n_steps, 8, chain=True)
+    compare_cache(g["k_cache"], g["v_cache"], o["k_cache"], o["v_cache"], I, [0, 1, 2], MID_W.shape.n_steps)
+
+
 def test_graph_replay_is_repeatable():
     import torch
     W, I = mid_case()
