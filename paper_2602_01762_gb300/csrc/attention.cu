@@ -248,16 +248,28 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const AttnArgs 
         const float *part = a.part + ((size_t)b * a.Hq + h) * a.splits * PS;
         float *wh = ws + (size_t)hl * a.splits;
         // lanes over splits: global max, split weights exp(m_s - M), denominator
+        // (each lane issues all its loads before using any of them)
+        constexpr int kMaxPerLane = 8;                 // splits <= 256
+        float mv[kMaxPerLane], lv[kMaxPerLane];
+#pragma unroll
+        for (int k = 0; k < kMaxPerLane; ++k) {
+            const int sp = lane + 32 * k;
+            const bool in = sp < a.splits;
+            mv[k] = in ? __ldcg(part + (size_t)sp * PS + D) : -INFINITY;
+            lv[k] = in ? __ldcg(part + (size_t)sp * PS + D + 1) : 0.f;
+        }
         float M = -INFINITY;
-        for (int sp = lane; sp < a.splits; sp += 32) M = fmaxf(M, __ldcg(part + (size_t)sp * PS + D));
+#pragma unroll
+        for (int k = 0; k < kMaxPerLane; ++k) M = fmaxf(M, mv[k]);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xFFFFFFFFu, M, o));
         float den = 0.f;
-        for (int sp = lane; sp < a.splits; sp += 32) {
-            const float l = __ldcg(part + (size_t)sp * PS + D + 1);
-            const float w = l > 0.f ? expf(__ldcg(part + (size_t)sp * PS + D) - M) : 0.f;
-            wh[sp] = w;
-            den = fmaf(w, l, den);
+#pragma unroll
+        for (int k = 0; k < kMaxPerLane; ++k) {
+            const int sp = lane + 32 * k;
+            const float w = lv[k] > 0.f ? expf(mv[k] - M) : 0.f;
+            if (sp < a.splits) wh[sp] = w;
+            den = fmaf(w, lv[k], den);
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) den += __shfl_xor_sync(0xFFFFFFFFu, den, o);
@@ -266,7 +278,7 @@ __global__ void __launch_bounds__(kAttnThreads) attention_kernel(const AttnArgs 
         float acc[DPL];
 #pragma unroll
         for (int u = 0; u < DPL; ++u) acc[u] = 0.f;
-#pragma unroll 8
+#pragma unroll 16
         for (int sp = 0; sp < a.splits; ++sp) {
             const float w = wh[sp];
             float v[DPL];

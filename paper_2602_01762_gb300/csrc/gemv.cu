@@ -268,16 +268,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane != 0) return;
-        const long total = (long)n_pass * n_chunks;
-        long issued = 0;
-        for (long i = 0; i < total; ++i) {
-            const int s = (int)(i % S);
-            const uint32_t it = (uint32_t)(i / S);
-            if (!mbar_wait(&empty[s], (it & 1) ^ 1)) {
+        const int total = n_pass * n_chunks;
+        int issued = 0;
+        int s = 0, c = 0;
+        uint32_t ph = 0;                                      // phase parity of stage s
+        for (int i = 0; i < total; ++i) {
+            if (!mbar_wait(&empty[s], ph ^ 1)) {
                 set_err(a.err, kErrTimeout);
                 break;
             }
-            const int c = (int)(i % n_chunks);
             const int first = u0 + c * R;
             const int rows = u1 - first < R ? u1 - first : R;
             const uint32_t bytes = (uint32_t)(rows * row_bytes);
@@ -294,9 +293,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
                          (const uint8_t *)a.W + ((size_t)first + (size_t)r * a.pair_offset) * row_bytes, bytes,
                          &full[s]);
             issued = i + 1;
+            if (++c == n_chunks) c = 0;
+            if (++s == S) { s = 0; ph ^= 1; }
         }
         // drain: the last stages' copies land before this CTA may exit
-        for (long i = issued > S ? issued - S : 0; i < issued; ++i)
+        for (int i = issued > S ? issued - S : 0; i < issued; ++i)
             if (!mbar_wait(&full[i % S], (uint32_t)((i / S) & 1))) set_err(a.err, kErrTimeout);
         return;
     }
@@ -314,6 +315,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
     const uint32_t ring_base = saddr(ring);
     bool dead = false;
     int lc = 0;                                               // chunks this group has taken
+    // Ring items are numbered i = pass * n_chunks + chunk in issue order; group
+    // g takes the items i = g, g + G, ... across all passes, so with G dividing
+    // S it only ever waits on stages s = g (mod G), each in fill order.
+    int item = grp, s = grp;
+    uint32_t ph = 0;                                          // phase parity of stage s
     pdl_wait();
 
     for (int p = 0; p < n_pass; ++p) {
@@ -330,10 +336,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
         float thr_v = -INFINITY;
         int thr_i = 0x7FFFFFFF;
 
-        for (int c = grp; c < n_chunks; c += G, ++lc) {
-            const long i = (long)p * n_chunks + c;
-            const int s = (int)(i % S);
-            if (!dead && !mbar_wait(&full[s], (uint32_t)((i / S) & 1))) {
+        for (; item < (p + 1) * n_chunks; item += G, ++lc) {
+            const int c = item - p * n_chunks;
+            if (!dead && !mbar_wait(&full[s], ph)) {
                 set_err(a.err, kErrTimeout);
                 dead = true;
             }
@@ -446,6 +451,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&empty[s]);
+            s += G;
+            if (s >= S) { s -= S; ph ^= 1; }
         }
 
         if constexpr (TOPK) {

@@ -368,9 +368,10 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     const size_t es = c->bf16 ? 2 : 4;
     c->qkv_rows = (Hq + 2 * Hkv) * D;
     c->lm_grid = f.vocab < c->sms ? f.vocab : c->sms;
-    // attention split size: enough CTAs to cover the GPU at batch 1
+    // attention split size: 64 keys, larger when the split count would exceed
+    // what the last-CTA combine reads per lane (256 splits)
     c->attn_chunk = 64;
-    if ((long long)f.max_batch * Hkv * ((f.max_ctx + 63) / 64) < 2LL * c->sms) c->attn_chunk = 32;
+    while ((f.max_ctx + c->attn_chunk - 1) / c->attn_chunk > 256) c->attn_chunk *= 2;
     c->attn_splits = (f.max_ctx + c->attn_chunk - 1) / c->attn_chunk;
 
     const size_t T1 = (size_t)f.max_batch * f.max_new, B = f.max_batch;
