@@ -153,6 +153,42 @@ prism_status prism_accept_greedy(prism_ctx *ctx, int32_t batch, const int32_t *d
                                  const int32_t *target, const int32_t *n_new, int32_t *kv_len,
                                  int32_t *accept_len, int32_t *out_tokens, void *stream);
 
+/* LM-head selection that allocates nothing.  The paper has no counterpart to
+ * this entry point; it serves callers that cannot call cudaMalloc, so cannot
+ * own a prism_ctx workspace: an inference server whose caching allocator has
+ * already reserved the device memory it may use, a plugin whose host
+ * framework forbids allocation outside its own pool, or code enqueued while a
+ * stream capture in a mode that treats allocation as an error is under way.
+ * It computes what the last stage of a draft step computes (final RMSNorm with
+ * gain g_final, logits = lm_head . norm(h), top-1 and top-k), using the same
+ * kernel, and keeps that kernel's scratch (the per-CTA partial top-8 lists,
+ * the last-CTA ticket and the device error word) in a static device array of
+ * 1 MiB + 256 bytes inside the library, which every process that loads the
+ * library holds on each device it uses until exit.
+ *   dtype PRISM_F32 or PRISM_BF16 (the type of lm_head and g_final);
+ *   h fp32 [batch, hidden] hidden rows before the final norm;
+ *   g_final [hidden] or NULL (no final norm); lm_head [vocab, hidden];
+ *   draft int32 [batch] out; topk_ids int32 [batch, topk], topk_logits fp32
+ *   [batch, topk], logits fp32 [batch, vocab]: outputs, each may be NULL;
+ *   dev_flags int32 [1] or NULL: receives the device error word of this call.
+ * All pointers are device pointers; h, lm_head and g_final 16-byte aligned.
+ * Limits: batch <= 64 rows; larger batches return PRISM_ERR_CAPACITY with a
+ * message from prism_get_error(NULL): split them into several calls.
+ * The first call on a device (the current one) does that device's set-up:
+ * it resolves the array's device address with cudaGetSymbolAddress and sets
+ * the kernel's shared-memory attribute; make that first call before any
+ * stream capture.  Each call clears the ticket and the error word with a
+ * stream-ordered memset, then launches the kernel on `stream`.  Every call
+ * shares the one array, so calls that can overlap on the GPU (different
+ * streams, or several host threads) race and corrupt each other's results:
+ * keep them on one stream.  Calls no cudaMalloc, cudaFree or allocating
+ * library routine.  Errors: INVALID_ARG, SHAPE, CAPACITY, CUDA. */
+prism_status prism_lm_head_topk_static(int32_t dtype, int32_t hidden, int32_t vocab, int32_t batch,
+                                       int32_t topk, float rms_eps, const float *h,
+                                       const void *g_final, const void *lm_head, int32_t *draft,
+                                       int32_t *topk_ids, float *topk_logits, float *logits,
+                                       int32_t *dev_flags, void *stream);
+
 /* Synchronise `stream`, read and clear the device error word.  Returns
  * PRISM_ERR_DEVICE_FLAG (bits in *flags if non-NULL) when it was set,
  * PRISM_ERR_CUDA when the stream reports an error, PRISM_OK otherwise. */

@@ -13,7 +13,7 @@ import os
 
 import torch
 
-__all__ = ["Drafter", "PrismError", "library", "STEP_TENSORS", "KERNEL_KINDS"]
+__all__ = ["Drafter", "PrismError", "library", "lm_head_topk_static", "STEP_TENSORS", "KERNEL_KINDS"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.environ.get("PRISM_LIB") or os.path.join(_HERE, "libprism.so")
@@ -62,12 +62,13 @@ def library() -> ctypes.CDLL:
         lib.prism_sync_status.argtypes = [vp, vp, P(i32)]
         lib.prism_set_option.argtypes = [vp, ctypes.c_char_p, i32]
         lib.prism_profile_round.argtypes = [vp, i32] + [vp] * 10 + [P(ctypes.c_float), P(i32), i32, P(i32)]
+        lib.prism_lm_head_topk_static.argtypes = [i32] * 5 + [ctypes.c_float] + [vp] * 9
         lib.prism_get_error.argtypes = [vp]
         lib.prism_get_error.restype = ctypes.c_char_p
         lib.prism_version.restype = ctypes.c_char_p
         for f in ("prism_create", "prism_destroy", "prism_load_shared_weights", "prism_load_step_weights",
                   "prism_draft_round", "prism_accept_greedy", "prism_sync_status", "prism_set_option",
-                  "prism_profile_round"):
+                  "prism_profile_round", "prism_lm_head_topk_static"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -240,3 +241,40 @@ class Drafter:
             self.close()
         except Exception:
             pass
+
+
+def lm_head_topk_static(h, g_final, lm_head, draft, topk_ids=None, topk_logits=None, logits=None,
+                        dev_flags=None, rms_eps=1e-5, stream=None):
+    """Final norm + LM head + top-k of the rows of ``h`` through
+    ``prism_lm_head_topk_static``, the entry point that allocates no device
+    memory (its scratch is a static array inside the library; for callers
+    that cannot call cudaMalloc).  ``h`` fp32 [B, d]; ``g_final`` [d] or None;
+    ``lm_head`` [V, d] (bf16 or fp32); ``draft`` int32 [B]; ``topk_ids`` int32
+    [B, k], ``topk_logits`` fp32 [B, k], ``logits`` fp32 [B, V] and
+    ``dev_flags`` int32 [1] optional outputs.  B <= 64; calls that may overlap
+    on the GPU race on the shared scratch."""
+    lib = library()
+    V, d = lm_head.shape
+    B = h.shape[0]
+    dt = {torch.bfloat16: 1, torch.float32: 0}.get(lm_head.dtype)
+    if dt is None:
+        raise TypeError("lm_head must be bfloat16 or float32")
+    topk = 1 if topk_ids is None and topk_logits is None else (topk_ids if topk_ids is not None else topk_logits).shape[1]
+    want = [(h, (B, d), torch.float32, "h"), (lm_head, (V, d), lm_head.dtype, "lm_head"),
+            (draft, (B,), torch.int32, "draft")]
+    if g_final is not None:
+        want.append((g_final, (d,), lm_head.dtype, "g_final"))
+    for t, shape, dtype, name in ((topk_ids, (B, topk), torch.int32, "topk_ids"),
+                                  (topk_logits, (B, topk), torch.float32, "topk_logits"),
+                                  (logits, (B, V), torch.float32, "logits"),
+                                  (dev_flags, (1,), torch.int32, "dev_flags")):
+        if t is not None:
+            want.append((t, shape, dtype, name))
+    for t, shape, dtype, name in want:
+        if tuple(t.shape) != shape or t.dtype != dtype or not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name}: expected contiguous CUDA {dtype} {shape}, got {t.dtype} {tuple(t.shape)}")
+    st = lib.prism_lm_head_topk_static(dt, d, V, B, topk, float(rms_eps), _ptr(h), _ptr(g_final),
+                                       _ptr(lm_head), _ptr(draft), _ptr(topk_ids), _ptr(topk_logits),
+                                       _ptr(logits), _ptr(dev_flags), _stream(stream))
+    if st != 0:
+        raise PrismError(st, (lib.prism_get_error(None) or b"").decode())

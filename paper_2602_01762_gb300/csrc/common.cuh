@@ -217,6 +217,8 @@ cudaError_t launch_accept(const AcceptArgs &a, cudaStream_t s);
 // One-time kernel attribute setup (maximum dynamic shared memory); must run
 // before any stream capture.
 cudaError_t prepare_gemv_kernels();
+// Message returned by prism_get_error(NULL) (host, thread-local).
+void set_global_error(const char *msg);
 bool gemv_supported(const GemvArgs &a, bool bf16);
 bool gemv_mma_supported(const GemvArgs &a);
 cudaError_t prepare_gemv_mma_kernels();

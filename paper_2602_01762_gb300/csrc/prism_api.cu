@@ -39,6 +39,8 @@ thread_local std::string g_error;
 
 }  // namespace
 
+void prism::set_global_error(const char *msg) { g_error = msg; }
+
 struct prism_ctx {
     prism_config cfg{};
     int device = 0;
