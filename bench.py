@@ -202,6 +202,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--opt", action="append", default=[], metavar="NAME=VALUE",
+                    help="drafter option (prism_set_option), repeatable")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -275,6 +277,11 @@ def run_ours(args, w, world, rank, local):
     dr = Drafter.from_shape(s, max_batch=B, max_ctx=int(I["max_ctx"]), max_new=max_new, topk=w.topk,
                             device=local)
     weights_dev = bind_weights(dr, W, device=dev)
+    options = {}
+    for kv in args.opt:
+        name, value = kv.split("=", 1)
+        options[name] = int(value)
+        dr.set_option(name, int(value))
     t = {n: to_device(I[n], dev) for n in ("tokens", "hidden", "n_new", "kv_len", "k_cache", "v_cache")}
     ids = torch.empty((B, K), dtype=torch.int32, device=dev)
     tk_ids = torch.empty((B, K, w.topk), dtype=torch.int32, device=dev)
@@ -324,7 +331,7 @@ def run_ours(args, w, world, rank, local):
     peak, peak_src = hbm_peak()
     lm_b = lm_head_bytes(w)
     achieved = lm_b / (lm_ms / 1e3) / 1e9
-    kernel_src = os.path.join(ROOT, "paper_2602_01762_gb300", "csrc", "gemv.cu")
+    kernel_src = os.path.join(ROOT, "paper_2602_01762_gb300", "csrc", "gemv_tc.cu")
 
     # ---- end to end through the public API with host buffers --------------------
     pin = {n: torch.from_numpy(np.ascontiguousarray(
@@ -369,7 +376,7 @@ def run_ours(args, w, world, rank, local):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": per_round_ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if s.dtype == "bf16" else "f32",
-            "data": "synthetic", "config": config_of(w),
+            "data": "synthetic", "config": dict(config_of(w), options=options),
             "round_latency_us": per_round_ms * 1e3,
             "hbm": {"bytes_per_round": total_bytes,
                     "achieved_gbs": total_bytes / (per_round_ms / 1e3) / 1e9,

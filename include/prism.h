@@ -199,9 +199,12 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * "gemv_chunk_kb" (target TMA stage size of the projection kernels, 0..128,
  * 0 = default), "gemv_smem_kb" (shared-memory budget of the projection
  * ring, 0..200, 0 = default), "gemv_groups" (consumer warp groups of the
- * projection kernels: 1, 2, 4, 8 or 16; 0 = default), "gemv_cuda_core"
- * (1, the default: bf16 projections run on the CUDA-core kernel; 0: on the
- * warp-level tensor-core kernel).  Changing an option drops cached
+ * projection kernels: 1, 2, 4, 8 or 16; 0 = default), "gemv_tcgen05"
+ * (1, the default: bf16 projections with at most 16 activation rows run on
+ * the tcgen05 kernel, TMA tensor loads into tensor-memory accumulators; 0:
+ * every projection on the kernels below), "gemv_cuda_core" (for projections
+ * not on the tcgen05 kernel: 1, the default, the CUDA-core TMA-ring kernel;
+ * 0: the warp-level mma.sync kernel).  Changing an option drops cached
  * graphs.  Errors: INVALID_ARG (unknown name or value out of range). */
 prism_status prism_set_option(prism_ctx *ctx, const char *name, int32_t value);
 

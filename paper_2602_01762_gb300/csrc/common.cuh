@@ -2,6 +2,7 @@
 // (sm_103a).  Internal to the library; the public ABI is include/prism.h.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -223,6 +224,16 @@ bool gemv_supported(const GemvArgs &a, bool bf16);
 bool gemv_mma_supported(const GemvArgs &a);
 cudaError_t prepare_gemv_mma_kernels();
 cudaError_t launch_gemv_mma(const GemvArgs &a, int grid, cudaStream_t s, bool pdl);
+// Tensor-core projections (gemv_tc.cu): tensor-map encoder and kernel
+// attributes (before any capture); a weight matrix [rows, kin] bf16 as a TMA
+// tensor map of 128 x 64 boxes; plan check, split-K workspace need, launch.
+cudaError_t prepare_gemv_tc_kernels();
+cudaError_t make_weight_map(CUtensorMap *m, const void *W, int rows, int kin);
+bool gemv_tc_supported(const GemvArgs &a, int sms);
+size_t gemv_tc_workspace_floats(const GemvArgs &a, int sms);
+int gemv_tc_tiles(const GemvArgs &a);
+cudaError_t launch_gemv_tc(const GemvArgs &a, const CUtensorMap &m, int sms, float *part, int *tile_ctr,
+                           cudaStream_t s, bool pdl);
 cudaError_t prepare_attention_kernel(bool bf16, int D, int chunk, int G, int splits);
 size_t attention_smem_bytes(bool bf16, int D, int chunk, int G, int splits);
 

@@ -1,0 +1,813 @@
+// Tensor-core (tcgen05) weight-streaming projections of the PRISM draft step.
+//
+// Each projection of a draft step (fusion F, QKV, O, gate/up, down, LM head;
+// Sec. 3.2 and the Llama block) is D = W X^T with W [rows, kin] in bf16 and a
+// handful of activation rows X [T, kin].  W is the A operand (M = 128 rows of
+// W per tile, K-major), X the B operand (N = 16, K-major), D accumulates in
+// fp32 in tensor memory.  Nothing on the SM touches individual weights:
+//   * warp 0, one lane: TMA tensor loads of 128-row x 64-column boxes of W
+//     (128-byte swizzle, the canonical K-major operand layout) into a ring of
+//     shared-memory stages; it starts before griddepcontrol.wait, so the ring
+//     fills while the previous kernel drains;
+//   * warps 1-5 build X once per CTA in shared memory (embedding gather,
+//     RMSNorm with its gain, bf16 rounding), already in the swizzled operand
+//     layout; with T <= 8 only 8 rows are stored and the descriptor's 8-row
+//     stride is 0, so the MMA's rows 8-15 re-read rows 0-7;
+//   * warp 1, one lane: tcgen05.mma (kind::f16, M=128, N=16, K=16) per
+//     32-byte K slice; tcgen05.commit releases a stage when its MMAs have
+//     read it and signals a finished accumulator;
+//   * warps 2-5: the epilogue reads the accumulator (tcgen05.ld, one TMEM
+//     lane = one output row per thread) into registers while the MMA fills
+//     the other of two accumulator buffers, and fuses the residual add,
+//     SwiGLU, or the logits write and top-8 selection;
+//   * split-K: with few 128-row tiles the contraction is split over CTAs
+//     (CTA c takes K slice c % S); the partial sums go to a workspace and the
+//     last CTA to finish a tile adds them in slice order, so results do not
+//     depend on timing;
+//   * every wait is bounded; on expiry the kernel sets the timeout bit of the
+//     device error word, stops waiting, drains its copies and MMAs, frees its
+//     tensor memory and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+
+namespace prism {
+
+namespace {
+
+constexpr int kTcThreads = 192;             // producer, MMA, 4 epilogue warps
+constexpr int kStageThreads = kTcThreads - 32;
+constexpr int kTileM = 128;
+constexpr int kBoxK = 64;                   // bf16 elements per 128-byte swizzle row
+constexpr uint32_t kBoxBytes = kTileM * 128;  // 16 KB
+constexpr int kMmaN = 16;
+constexpr int kTcMaxStages = 8;
+constexpr int kMaxSplits = 8;
+constexpr size_t kTcSmem = 212 * 1024;      // dynamic shared memory budget
+constexpr size_t kXBudget = 128 * 1024;     // largest X slice
+constexpr long kTcWaitLimit = 1L << 22;
+
+__device__ __forceinline__ uint32_t saddr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t *b, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(saddr(b)), "r"(count));
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t *b) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(saddr(b)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint64_t *b, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(saddr(b)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+                 : "=r"(ok) : "r"(saddr(b)), "r"(parity) : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity) {
+    for (long i = 0; i < kTcWaitLimit; ++i)
+        if (mbar_try(b, parity)) return true;
+    return false;
+}
+
+// Whole-warp wait: lane 0 polls with a short back-off (a warp of spinning
+// lanes would compete with the TMA and MMA traffic on shared memory), then
+// every lane observes the completed phase.  Warp-uniform result.
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t *b, uint32_t parity) {
+    bool ok = true;
+    if ((threadIdx.x & 31) == 0) {
+        ok = false;
+        for (long i = 0; i < kTcWaitLimit; ++i) {
+            if (mbar_try(b, parity)) { ok = true; break; }
+            __nanosleep(64);
+        }
+    }
+    ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+    if (ok) mbar_try(b, parity);
+    return ok;
+}
+
+// 2-D TMA tensor load (box at column x, row y) into shared memory.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        ::"r"(dst), "l"((uint64_t)map), "r"(x), "r"(y), "r"(saddr(bar)) : "memory");
+}
+
+// tcgen05 shared-memory matrix descriptor: K-major operand in the 128-byte
+// swizzle layout (8-row x 128-byte atoms, `sbo` bytes between 8-row groups).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr, uint32_t sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((addr & 0x3FFFFu) >> 4);    // start address
+    d |= (uint64_t)1 << 16;                     // leading-dimension offset (unused here)
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;  // stride-dimension offset
+    d |= (uint64_t)1 << 46;                     // descriptor version
+    d |= (uint64_t)2 << 61;                     // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor: bf16 A and B, fp32 D, both K-major, M = 128, N = 16.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kMmaN >> 3) << 17) |
+                            ((uint32_t)(kTileM >> 4) << 24);
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(a), "l"(b), "r"(kIdesc), "r"(accumulate));
+}
+// Arrive once on `bar` when every MMA this thread issued so far has completed.
+__device__ __forceinline__ void mma_commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(saddr(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// 16 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void stage_sync() {   // warps 1-5
+    asm volatile("bar.sync 1, %0;" ::"r"(kStageThreads) : "memory");
+}
+__device__ __forceinline__ void epi_sync() {     // warps 2-5
+    asm volatile("bar.sync 2, 128;" ::: "memory");
+}
+
+__device__ __forceinline__ int clamp_n(const GemvArgs &a, int b) {
+    int n = a.n_new[b];
+    if (n < 1 || n > a.max_new) {
+        set_err(a.err, kErrNNew);
+        n = n < 1 ? 1 : a.max_new;
+    }
+    return n;
+}
+__device__ __forceinline__ int token_ok(const GemvArgs &a, int tok) {
+    if (tok < 0 || tok >= a.vocab) {
+        set_err(a.err, kErrToken);
+        return 0;
+    }
+    return tok;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    return (uint32_t)f32_to_bf16(lo) | ((uint32_t)f32_to_bf16(hi) << 16);
+}
+struct TcPlan {
+    int n_tiles;        // 128-row tiles of output units
+    int nkb;            // 64-wide K blocks of the whole contraction
+    int splits;         // K slices (CTA c works on slice c % splits)
+    int stages;         // ring stages
+    int kb_per_stage;   // K blocks per stage (each RPW boxes)
+    uint32_t stage_bytes, x_bytes;
+    float *part;        // split-K partial sums [splits][RPW][T][n_units]
+    int *tile_ctr;      // per-tile arrival tickets (left at zero)
+};
+
+// X rows (bf16, swizzled K-major operand layout) for the K blocks [kb0, kb1).
+// Threads of warps 1-5.  This runs once per CTA while the weight ring waits,
+// so it is kept short in both senses: little code (it executes cold, one
+// instruction-cache miss per line) and few dependent memory round trips
+// (each costs microseconds behind a saturated HBM): a thread issues the loads
+// of all its chunks of a row (up to kStageGroup) before using any.
+constexpr int kStageGroup = 4;
+
+__device__ __forceinline__ void ld32(const void *p, uint4 &lo, uint4 &hi) {
+    lo = __ldcg((const uint4 *)p);
+    hi = __ldcg((const uint4 *)p + 1);
+}
+__device__ __forceinline__ float sumsq8(const uint4 &lo, const uint4 &hi) {
+    const float f[8] = {__uint_as_float(lo.x), __uint_as_float(lo.y), __uint_as_float(lo.z), __uint_as_float(lo.w),
+                        __uint_as_float(hi.x), __uint_as_float(hi.y), __uint_as_float(hi.z), __uint_as_float(hi.w)};
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s = fmaf(f[i], f[i], s);
+    return s;
+}
+// 8 fp32 values (lo, hi), times scale and the bf16 gains g when use_g, rounded to bf16.
+__device__ __forceinline__ uint4 round8r(const uint4 &lo, const uint4 &hi, float scale, bool use_g, const uint4 &g) {
+    float v[8] = {__uint_as_float(lo.x), __uint_as_float(lo.y), __uint_as_float(lo.z), __uint_as_float(lo.w),
+                  __uint_as_float(hi.x), __uint_as_float(hi.y), __uint_as_float(hi.z), __uint_as_float(hi.w)};
+    if (use_g) {
+        const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            v[2 * i] = v[2 * i] * scale * bf16lo(gw[i]);
+            v[2 * i + 1] = v[2 * i + 1] * scale * bf16hi(gw[i]);
+        }
+    }
+    return make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]), pack_bf16(v[6], v[7]));
+}
+
+// Deterministic sum over the staging threads (fixed shuffle tree, fixed warp order).
+__device__ __forceinline__ float stage_sum(float v, float *red) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    if ((threadIdx.x & 31) == 0) red[(threadIdx.x >> 5) - 1] = v;
+    stage_sync();
+    float tot = 0.f;
+#pragma unroll
+    for (int i = 0; i < kStageThreads / 32; ++i) tot += red[i];
+    stage_sync();
+    return tot;
+}
+
+template <int NB, int PRO>
+__device__ void stage_x_tc(const GemvArgs &a, int kb0, int kb1, uint8_t *X, float *red) {
+    const int tid = threadIdx.x - 32;
+    const int d = a.d, kin = a.kin, T = a.T;
+    // padding rows T..NB-1: zero (16-byte slot i of a K block holds row (i / 8) % NB)
+    const int nslots = (kb1 - kb0) * NB * 8;
+#pragma unroll 1
+    for (int i = tid; i < nslots; i += kStageThreads)
+        if (((i >> 3) & (NB - 1)) >= T) ((uint4 *)X)[i] = make_uint4(0, 0, 0, 0);
+
+    const int c0 = kb0 * 8, c1 = kb1 * 8;     // 8-element chunks of this CTA's K range
+#pragma unroll 1
+    for (int t = 0; t < T; ++t) {
+        // per-row sources
+        const uint16_t *e_row = nullptr, *h_row = nullptr;
+        const float *f_row = nullptr;
+        bool valid = true;
+        float inv = 1.f;
+        if constexpr (PRO == kProFusePrefill) {
+            const int b = t / a.max_new, r = t % a.max_new;
+            valid = r < clamp_n(a, b);
+            const int tok = valid ? token_ok(a, a.tokens[b * a.max_new + r]) : 0;
+            e_row = (const uint16_t *)a.embed + (size_t)tok * d;
+            h_row = (const uint16_t *)a.hidden_in + ((size_t)b * a.max_new + r) * d;
+        } else if constexpr (PRO == kProFuseDecode) {
+            e_row = (const uint16_t *)a.embed + (size_t)token_ok(a, a.draft[t * a.K + a.step - 2]) * d;
+            f_row = a.src + (size_t)t * d;
+        } else if constexpr (PRO == kProNorm) {
+            const int sr = a.src_prefill_rows ? (t * a.max_new + clamp_n(a, t) - 1) : t;
+            f_row = a.src + (size_t)sr * d;
+            if (a.gain) {
+                float ss = 0.f;
+#pragma unroll 1
+                for (int c = tid; c < d / 8; c += kStageGroup * kStageThreads) {
+                    uint4 lo[kStageGroup], hi[kStageGroup];
+#pragma unroll
+                    for (int g = 0; g < kStageGroup; ++g)
+                        if (c + g * kStageThreads < d / 8) ld32(f_row + (size_t)(c + g * kStageThreads) * 8, lo[g], hi[g]);
+#pragma unroll
+                    for (int g = 0; g < kStageGroup; ++g)
+                        if (c + g * kStageThreads < d / 8) ss += sumsq8(lo[g], hi[g]);
+                }
+                inv = 1.0f / sqrtf(stage_sum(ss, red) / (float)d + a.eps);
+            }
+        } else {
+            h_row = (const uint16_t *)a.act + (size_t)t * kin;
+        }
+        // this thread's chunks of the row: loads first, then convert and store
+#pragma unroll 1
+        for (int c = c0 + tid; c < c1; c += kStageGroup * kStageThreads) {
+            uint4 lo[kStageGroup], hi[kStageGroup], gv[kStageGroup];
+#pragma unroll
+            for (int g = 0; g < kStageGroup; ++g) {
+                const int k = (c + g * kStageThreads) * 8;
+                lo[g] = hi[g] = gv[g] = make_uint4(0, 0, 0, 0);
+                if (c + g * kStageThreads >= c1 || k >= kin || !valid) continue;
+                if constexpr (PRO == kProFusePrefill) {
+                    lo[g] = k < d ? __ldg((const uint4 *)(e_row + k)) : __ldcg((const uint4 *)(h_row + (k - d)));
+                } else if constexpr (PRO == kProFuseDecode) {
+                    if (k < d) lo[g] = __ldg((const uint4 *)(e_row + k));
+                    else ld32(f_row + (k - d), lo[g], hi[g]);
+                } else if constexpr (PRO == kProNorm) {
+                    ld32(f_row + k, lo[g], hi[g]);
+                    if (a.gain) gv[g] = __ldg((const uint4 *)((const uint16_t *)a.gain + k));
+                } else {
+                    lo[g] = __ldcg((const uint4 *)(h_row + k));
+                }
+            }
+#pragma unroll
+            for (int g = 0; g < kStageGroup; ++g) {
+                const int cc = c + g * kStageThreads;
+                if (cc >= c1) continue;
+                uint4 v = lo[g];
+                const int k = cc * 8;
+                if (k < kin && valid) {
+                    if constexpr (PRO == kProFuseDecode) {
+                        if (k >= d) v = round8r(lo[g], hi[g], 1.f, false, gv[g]);
+                    } else if constexpr (PRO == kProNorm) {
+                        v = round8r(lo[g], hi[g], inv, a.gain != nullptr, gv[g]);
+                    }
+                }
+                const int kb = cc >> 3, ci = cc & 7;
+                *(uint4 *)(X + (size_t)(kb - kb0) * (NB * 128) + t * 128 + ((ci ^ (t & 7)) << 4)) = v;
+            }
+        }
+    }
+}
+
+// Top 8 under `better` of candidates spread over a warp: kRounds rounds of a
+// warp-wide argmax over the lanes' best remaining candidate; the winning lane
+// retires it.  Each lane holds C candidates (cv, ci); ties between equal
+// entries break by lane, so the winner is warp-uniform.  The result goes to
+// out_v/out_i (written by lane 0).  Compact code on purpose: it runs cold.
+template <int C>
+__device__ void warp_top8(float (&cv)[C], int (&ci)[C], float *out_v, int *out_i) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll 1
+    for (int r = 0; r < kTopK; ++r) {
+        float bv = cv[0];
+        int bi = ci[0], bs = 0;
+#pragma unroll
+        for (int u = 1; u < C; ++u)
+            if (better(cv[u], ci[u], bv, bi)) { bv = cv[u]; bi = ci[u]; bs = u; }
+        float wv = bv;
+        int wi = bi, wl = lane;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float xv = __shfl_xor_sync(0xFFFFFFFFu, wv, o);
+            const int xi = __shfl_xor_sync(0xFFFFFFFFu, wi, o);
+            const int xl = __shfl_xor_sync(0xFFFFFFFFu, wl, o);
+            if (better(xv, xi, wv, wi) || (xv == wv && xi == wi && xl < wl)) { wv = xv; wi = xi; wl = xl; }
+        }
+        if (lane == wl) {
+#pragma unroll
+            for (int u = 0; u < C; ++u)
+                if (u == bs) { cv[u] = -INFINITY; ci[u] = 0x7FFFFFFF; }
+        }
+        if (lane == 0) { out_v[r] = wv; out_i[r] = wi; }
+    }
+}
+
+// Final epilogue of one output unit u for activation row t, given its
+// accumulators (RPW = 2: gate, up).
+template <int RPW>
+__device__ __forceinline__ void finish_unit(const GemvArgs &a, int t, int u, float acc0, float acc1) {
+    if constexpr (RPW == 2) {
+        Elem<uint16_t>::store((uint16_t *)a.out_act, (size_t)t * a.out_ld + u, acc0 / (1.0f + expf(-acc0)) * acc1);
+    } else {
+        float val = acc0;
+        if (a.epi == kEpiResid) {
+            const int rrow = a.resid_prefill_rows ? (t * a.max_new + clamp_n(a, t) - 1) : t;
+            val += a.resid[(size_t)rrow * a.out_ld + u];
+            if (a.hidden_out) a.hidden_out[((size_t)t * a.K + a.step - 1) * a.d + u] = val;
+        }
+        a.out[(size_t)t * a.out_ld + u] = val;
+    }
+}
+
+template <int NB, int RPW, bool TOPK, int PRO>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    gemv_tc_kernel(const GemvArgs a, const TcPlan p, const __grid_constant__ CUtensorMap tmW) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full[kTcMaxStages], empty[kTcMaxStages], acc_full[2], acc_empty[2], mma_done;
+    __shared__ uint32_t s_tmem;
+    __shared__ float red[kStageThreads / 32];
+    __shared__ float s_fin_v[TOPK ? kTopK : 1];
+    __shared__ int s_fin_i[TOPK ? kTopK : 1];
+    __shared__ float s_val[TOPK ? 4 : 1][TOPK ? NB : 1][kTopK];
+    __shared__ int s_id[TOPK ? 4 : 1][TOPK ? NB : 1][kTopK];
+    __shared__ int s_last;
+    constexpr uint32_t kCols = RPW == 1 ? 32 : 64;   // two accumulator buffers x RPW x 16 columns
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint8_t *base = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t *ring = base;
+    uint8_t *X = base + (size_t)p.stages * p.stage_bytes;
+    const int S = p.stages;
+    const int ks = blockIdx.x % p.splits;
+    const int tiles_step = gridDim.x / p.splits;
+    const int kb0 = (int)((long)ks * p.nkb / p.splits), kb1 = (int)((long)(ks + 1) * p.nkb / p.splits);
+    const int n_kst = (kb1 - kb0 + p.kb_per_stage - 1) / p.kb_per_stage;
+    int my_tiles = 0;
+    for (int tile = blockIdx.x / p.splits; tile < p.n_tiles; tile += tiles_step) ++my_tiles;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&acc_full[i], 1);
+            mbar_init(&acc_empty[i], 4);
+        }
+        mbar_init(&mma_done, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmW) : "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(&s_tmem)),
+                     "r"(kCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+    pdl_trigger();
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            int s = 0, issued = 0;
+            uint32_t ph = 0;
+            bool dead = false;
+            for (int i = 0; i < my_tiles && !dead; ++i) {
+                const int tile = blockIdx.x / p.splits + i * tiles_step;
+                for (int q = 0; q < n_kst; ++q) {
+                    if (!mbar_wait(&empty[s], ph ^ 1)) {
+                        set_err(a.err, kErrTimeout);
+                        dead = true;
+                        break;
+                    }
+                    const int kbs = kb0 + q * p.kb_per_stage;
+                    const int nkb = kb1 - kbs < p.kb_per_stage ? kb1 - kbs : p.kb_per_stage;
+                    mbar_arrive_tx(&full[s], (uint32_t)nkb * RPW * kBoxBytes);
+                    const uint32_t st = saddr(ring) + (uint32_t)s * p.stage_bytes;
+                    for (int j = 0; j < nkb; ++j)
+#pragma unroll
+                        for (int r = 0; r < RPW; ++r)
+                            tma_load_2d(st + (uint32_t)(j * RPW + r) * kBoxBytes, &tmW, (kbs + j) * kBoxK,
+                                        tile * kTileM + r * a.pair_offset, &full[s]);
+                    ++issued;
+                    if (++s == S) { s = 0; ph ^= 1; }
+                }
+            }
+            // drain: the copies in flight land before this CTA may exit
+            const int first = issued > S ? issued - S : 0;
+            for (int i = first; i < issued; ++i)
+                if (!mbar_wait(&full[i % S], (uint32_t)((i / S) & 1))) set_err(a.err, kErrTimeout);
+        }
+    } else {
+        pdl_wait();
+        stage_x_tc<NB, PRO>(a, kb0, kb1, X, red);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        stage_sync();
+
+        if (warp == 1) {
+            // ------------------------------------------------------------ MMA
+            if (lane == 0) {
+                int s = 0;
+                uint32_t ph = 0;
+                bool dead = false;
+                const uint32_t xb = saddr(X);
+                const uint32_t sbo_b = NB == 16 ? 1024u : 0u;
+                for (int i = 0; i < my_tiles && !dead; ++i) {
+                    const int ab = i & 1;
+                    if (!mbar_wait(&acc_empty[ab], ((i >> 1) & 1) ^ 1)) {
+                        set_err(a.err, kErrTimeout);
+                        dead = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    for (int q = 0; q < n_kst; ++q) {
+                        if (!mbar_wait(&full[s], ph)) {
+                            set_err(a.err, kErrTimeout);
+                            dead = true;
+                            break;
+                        }
+                        tc_fence_after();
+                        const int kbs = kb0 + q * p.kb_per_stage;
+                        const int nkb = kb1 - kbs < p.kb_per_stage ? kb1 - kbs : p.kb_per_stage;
+                        const uint32_t st = saddr(ring) + (uint32_t)s * p.stage_bytes;
+                        for (int j = 0; j < nkb; ++j) {
+                            const uint32_t xa = xb + (uint32_t)(kbs + j - kb0) * (NB * 128);
+#pragma unroll
+                            for (int kk = 0; kk < kBoxK / 16; ++kk) {
+                                const uint64_t bd = sw128_desc(xa + kk * 32, sbo_b);
+#pragma unroll
+                                for (int r = 0; r < RPW; ++r) {
+                                    const uint64_t ad =
+                                        sw128_desc(st + (uint32_t)(j * RPW + r) * kBoxBytes + kk * 32, 1024);
+                                    mma_bf16(tmem + (uint32_t)((ab * RPW + r) * kMmaN), ad, bd,
+                                             (q | j | kk) != 0 ? 1u : 0u);
+                                }
+                            }
+                        }
+                        mma_commit(&empty[s]);
+                        if (++s == S) { s = 0; ph ^= 1; }
+                    }
+                    if (!dead) mma_commit(&acc_full[ab]);
+                }
+                mma_commit(&mma_done);
+                if (!mbar_wait(&mma_done, 0)) set_err(a.err, kErrTimeout);
+            }
+            __syncwarp();
+        } else {
+            // ------------------------------------------------------------ epilogue
+            const int ew = warp - 2;                   // 0..3
+            const int quarter = warp & 3;              // TMEM lanes 32*quarter .. +31
+            const int row = quarter * 32 + lane;
+            const int T = a.T;
+            float thr_v[NB];
+            int thr_i[NB];
+            if constexpr (TOPK) {
+#pragma unroll
+                for (int t = 0; t < NB; ++t) { thr_v[t] = -INFINITY; thr_i[t] = 0x7FFFFFFF; }
+                if (lane < NB) {
+#pragma unroll
+                    for (int i = 0; i < kTopK; ++i) { s_val[ew][lane][i] = -INFINITY; s_id[ew][lane][i] = 0x7FFFFFFF; }
+                }
+                __syncwarp();
+            }
+            bool dead = false;
+            for (int i = 0; i < my_tiles; ++i) {
+                const int tile = blockIdx.x / p.splits + i * tiles_step;
+                const int ab = i & 1;
+                if (!dead && !mbar_wait_warp(&acc_full[ab], (i >> 1) & 1)) {
+                    if (lane == 0) set_err(a.err, kErrTimeout);
+                    dead = true;
+                }
+                float acc[RPW][16];
+                if (!dead) {
+                    tc_fence_after();
+#pragma unroll
+                    for (int r = 0; r < RPW; ++r)
+                        tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((ab * RPW + r) * kMmaN),
+                                  acc[r]);
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&acc_empty[ab]);
+                } else {
+#pragma unroll
+                    for (int r = 0; r < RPW; ++r)
+#pragma unroll
+                        for (int t = 0; t < 16; ++t) acc[r][t] = 0.f;
+                }
+
+                const int u = tile * kTileM + row;
+                const bool valid = !dead && u < a.n_units;
+                if constexpr (TOPK) {
+#pragma unroll
+                    for (int t = 0; t < NB; ++t) {
+                        if (t >= T) break;
+                        const float z = acc[0][t];
+                        if (valid && a.logits) a.logits[((size_t)t * a.K + a.step - 1) * a.vocab + u] = z;
+                        unsigned m = __ballot_sync(0xFFFFFFFFu, valid && better(z, u, thr_v[t], thr_i[t]));
+                        while (m) {
+                            const int src = __ffs(m) - 1;
+                            m &= m - 1;
+                            const float zv = __shfl_sync(0xFFFFFFFFu, z, src);
+                            const int uv = __shfl_sync(0xFFFFFFFFu, u, src);
+                            if (!better(zv, uv, thr_v[t], thr_i[t])) continue;
+                            if (lane == 0) {
+                                float *lv = s_val[ew][t];
+                                int *li = s_id[ew][t];
+                                int pos = kTopK - 1;
+                                while (pos > 0 && better(zv, uv, lv[pos - 1], li[pos - 1])) {
+                                    lv[pos] = lv[pos - 1];
+                                    li[pos] = li[pos - 1];
+                                    --pos;
+                                }
+                                lv[pos] = zv;
+                                li[pos] = uv;
+                            }
+                            __syncwarp();
+                            thr_v[t] = s_val[ew][t][kTopK - 1];
+                            thr_i[t] = s_id[ew][t][kTopK - 1];
+                            __syncwarp();
+                        }
+                    }
+                } else if (p.splits == 1) {
+                    if (valid) {
+#pragma unroll
+                        for (int t = 0; t < NB; ++t) {
+                            if (t >= T) break;
+                            finish_unit<RPW>(a, t, u, acc[0][t], acc[RPW - 1][t]);
+                        }
+                    }
+                } else {
+                    // split-K: publish this slice, the tile's last CTA adds all slices in order
+                    if (valid) {
+#pragma unroll
+                        for (int r = 0; r < RPW; ++r)
+#pragma unroll
+                            for (int t = 0; t < NB; ++t) {
+                                if (t >= T) break;
+                                p.part[(((size_t)ks * RPW + r) * T + t) * a.n_units + u] = acc[r][t];
+                            }
+                    }
+                    __threadfence();
+                    epi_sync();
+                    if (threadIdx.x == 64) s_last = atomicAdd(&p.tile_ctr[tile], 1) == p.splits - 1;
+                    epi_sync();
+                    if (s_last) {
+                        __threadfence();
+                        if (valid) {
+                            for (int t = 0; t < T; ++t) {
+                                float v0 = 0.f, v1 = 0.f;
+                                for (int k2 = 0; k2 < p.splits; ++k2) {
+                                    v0 += __ldcg(&p.part[(((size_t)k2 * RPW + 0) * T + t) * a.n_units + u]);
+                                    if (RPW == 2) v1 += __ldcg(&p.part[(((size_t)k2 * RPW + 1) * T + t) * a.n_units + u]);
+                                }
+                                finish_unit<RPW>(a, t, u, v0, v1);
+                            }
+                        }
+                        if (threadIdx.x == 64) p.tile_ctr[tile] = 0;
+                    }
+                    epi_sync();
+                }
+            }
+            if constexpr (TOPK) {
+                // per-CTA merge of the four epilogue warps' lists, then the last CTA merges all CTAs
+                epi_sync();
+                for (int t = ew; t < T; t += 4) {
+                    float cv[1] = {s_val[lane / kTopK][t][lane % kTopK]};
+                    int ci[1] = {s_id[lane / kTopK][t][lane % kTopK]};
+                    const size_t o = ((size_t)t * gridDim.x + blockIdx.x) * kTopK;
+                    warp_top8<1>(cv, ci, a.lm_part + o, a.lm_part_id + o);
+                }
+                __threadfence();
+                epi_sync();
+                if (threadIdx.x == 64) s_last = atomicAdd(a.counter, 1) == (int)gridDim.x - 1;
+                epi_sync();
+                if (s_last) {
+                    __threadfence();
+                    // each warp takes a quarter of every row's candidates (all
+                    // loads of a lane issued together), then one warp merges
+                    // the four partial lists
+                    constexpr int kC = 12;                         // grids up to 192 CTAs
+                    const int ncand = (int)gridDim.x * kTopK;
+                    const int lo = ew * ncand / 4, hi = (ew + 1) * ncand / 4;
+#pragma unroll 1
+                    for (int t = 0; t < T; ++t) {
+                        float cv[kC];
+                        int ci[kC];
+                        const size_t b0 = (size_t)t * ncand;
+#pragma unroll
+                        for (int u = 0; u < kC; ++u) {
+                            const int c = lo + lane + 32 * u;
+                            cv[u] = c < hi ? __ldcg(a.lm_part + b0 + c) : -INFINITY;
+                            ci[u] = c < hi ? __ldcg(a.lm_part_id + b0 + c) : 0x7FFFFFFF;
+                        }
+                        warp_top8<kC>(cv, ci, s_val[ew][0], s_id[ew][0]);
+                        epi_sync();
+                        if (ew == 0) {
+                            float fv[1] = {s_val[lane / kTopK][0][lane % kTopK]};
+                            int fi[1] = {s_id[lane / kTopK][0][lane % kTopK]};
+                            warp_top8<1>(fv, fi, s_fin_v, s_fin_i);
+                            __syncwarp();
+                            if (lane < a.topk) {
+                                const size_t o = (size_t)t * a.K + a.step - 1;
+                                if (lane == 0) a.draft_out[o] = s_fin_i[0];
+                                if (a.topk_ids) a.topk_ids[o * a.topk + lane] = s_fin_i[lane];
+                                if (a.topk_logits) a.topk_logits[o * a.topk + lane] = s_fin_v[lane];
+                            }
+                        }
+                        epi_sync();
+                    }
+                    if (threadIdx.x == 64) *a.counter = 0;
+                }
+            }
+        }
+    }
+
+    if (warp == 0) return;   // the producer takes no part in tensor memory
+    // teardown: every tcgen05 operation of this CTA is complete before the free
+    tc_fence_before();
+    stage_sync();
+    tc_fence_after();
+    if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols));
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+template <int NB>
+cudaError_t dispatch_tc(const GemvArgs &a, const TcPlan &p, const CUtensorMap &m, int grid, size_t smem,
+                        cudaStream_t s, bool pdl) {
+    const dim3 g(grid), b(kTcThreads);
+    if (a.epi == kEpiTopK && a.pro == kProNorm)
+        return launch_k(gemv_tc_kernel<NB, 1, true, kProNorm>, g, b, smem, s, pdl, a, p, m);
+    if (a.epi == kEpiSwiGLU && a.pro == kProNorm)
+        return launch_k(gemv_tc_kernel<NB, 2, false, kProNorm>, g, b, smem, s, pdl, a, p, m);
+    if (a.epi == kEpiStore || a.epi == kEpiResid) {
+        switch (a.pro) {
+            case kProFusePrefill: return launch_k(gemv_tc_kernel<NB, 1, false, kProFusePrefill>, g, b, smem, s, pdl, a, p, m);
+            case kProFuseDecode: return launch_k(gemv_tc_kernel<NB, 1, false, kProFuseDecode>, g, b, smem, s, pdl, a, p, m);
+            case kProNorm: return launch_k(gemv_tc_kernel<NB, 1, false, kProNorm>, g, b, smem, s, pdl, a, p, m);
+            case kProCopy: return launch_k(gemv_tc_kernel<NB, 1, false, kProCopy>, g, b, smem, s, pdl, a, p, m);
+        }
+    }
+    return cudaErrorInvalidValue;
+}
+
+template <int NB>
+cudaError_t set_tc_attrs(int bytes) {
+    cudaError_t e = cudaSuccess;
+#define PRISM_TC_ATTR(RPW, TK, PRO)                                                                      \
+    if (e == cudaSuccess)                                                                                \
+        e = cudaFuncSetAttribute(gemv_tc_kernel<NB, RPW, TK, PRO>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    PRISM_TC_ATTR(1, true, kProNorm)
+    PRISM_TC_ATTR(2, false, kProNorm)
+    PRISM_TC_ATTR(1, false, kProFusePrefill)
+    PRISM_TC_ATTR(1, false, kProFuseDecode)
+    PRISM_TC_ATTR(1, false, kProNorm)
+    PRISM_TC_ATTR(1, false, kProCopy)
+#undef PRISM_TC_ATTR
+    return e;
+}
+
+// Split count and ring for one projection: the fewest K blocks on the
+// busiest CTA, then the fewest splits.
+bool tc_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem) {
+    if (a.T < 1 || a.T > kMmaN || a.kin % 8 || a.n_units < 1) return false;
+    if ((a.epi == kEpiTopK || a.epi == kEpiSwiGLU) && a.pro != kProNorm) return false;
+    const int RPW = a.epi == kEpiSwiGLU ? 2 : 1;
+    const int NB = a.T <= 8 ? 8 : 16;
+    const int nkb = (a.kin + kBoxK - 1) / kBoxK;
+    const int n_tiles = (a.n_units + kTileM - 1) / kTileM;
+    const int max_s = a.epi == kEpiTopK ? 1 : kMaxSplits;
+    long best = -1;
+    int best_s = 0, best_ctas = 0;
+    for (int sp = 1; sp <= max_s && sp <= nkb; ++sp) {
+        const int per = (nkb + sp - 1) / sp;
+        if ((size_t)NB * 128 * per > kXBudget) continue;
+        int ctas = sms / sp;
+        if (ctas > n_tiles) ctas = n_tiles;
+        if (a.epi == kEpiTopK && ctas > 192) ctas = 192;   // candidates the final merge holds
+        if (ctas < 1) break;
+        const long cost = (long)((n_tiles + ctas - 1) / ctas) * per;
+        if (best < 0 || cost < best) { best = cost; best_s = sp; best_ctas = ctas; }
+    }
+    if (best < 0) return false;
+    p.n_tiles = n_tiles;
+    p.nkb = nkb;
+    p.splits = best_s;
+    p.x_bytes = (uint32_t)(NB * 128 * ((nkb + best_s - 1) / best_s));
+    const size_t room = kTcSmem - 1024 - p.x_bytes;
+    // 32 KB stages, or 16 KB ones when fewer than four 32 KB stages fit
+    p.kb_per_stage = (RPW == 1 && room >= 4 * 2 * (size_t)kBoxBytes) ? 2 : 1;
+    p.stage_bytes = (uint32_t)p.kb_per_stage * RPW * kBoxBytes;
+    p.stages = (int)(room / p.stage_bytes);
+    if (p.stages > kTcMaxStages) p.stages = kTcMaxStages;
+    if (p.stages < 2) return false;
+    grid = best_ctas * best_s;
+    smem = 1024 + (size_t)p.stages * p.stage_bytes + p.x_bytes;
+    return true;
+}
+
+}  // namespace
+
+cudaError_t prepare_gemv_tc_kernels() {
+    if (!g_encode) {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e != cudaSuccess) return e;
+        if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+        g_encode = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+    }
+    cudaError_t e = set_tc_attrs<8>((int)kTcSmem);
+    if (e == cudaSuccess) e = set_tc_attrs<16>((int)kTcSmem);
+    return e;
+}
+
+cudaError_t make_weight_map(CUtensorMap *m, const void *W, int rows, int kin) {
+    if (!g_encode) return cudaErrorNotSupported;
+    if (((uintptr_t)W & 15) || (kin % 8) || rows < 1) return cudaErrorInvalidValue;
+    cuuint64_t dims[2] = {(cuuint64_t)kin, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)kin * 2};
+    cuuint32_t box[2] = {(cuuint32_t)kBoxK, (cuuint32_t)kTileM};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(W), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+bool gemv_tc_supported(const GemvArgs &a, int sms) {
+    TcPlan p{};
+    int grid;
+    size_t smem;
+    return tc_plan(a, sms, p, grid, smem);
+}
+
+int gemv_tc_tiles(const GemvArgs &a) { return (a.n_units + kTileM - 1) / kTileM; }
+
+size_t gemv_tc_workspace_floats(const GemvArgs &a, int sms) {
+    TcPlan p{};
+    int grid;
+    size_t smem;
+    if (!tc_plan(a, sms, p, grid, smem) || p.splits == 1) return 0;
+    return (size_t)p.splits * (a.epi == kEpiSwiGLU ? 2 : 1) * a.T * a.n_units;
+}
+
+cudaError_t launch_gemv_tc(const GemvArgs &a, const CUtensorMap &m, int sms, float *part, int *tile_ctr,
+                           cudaStream_t s, bool pdl) {
+    TcPlan p{};
+    int grid;
+    size_t smem;
+    if (!tc_plan(a, sms, p, grid, smem)) return cudaErrorInvalidValue;
+    p.part = part;
+    p.tile_ctr = tile_ctr;
+    if (p.splits > 1 && (!part || !tile_ctr)) return cudaErrorInvalidValue;
+    return a.T <= 8 ? dispatch_tc<8>(a, p, m, grid, smem, s, pdl) : dispatch_tc<16>(a, p, m, grid, smem, s, pdl);
+}
+
+}  // namespace prism

@@ -69,6 +69,17 @@ struct prism_ctx {
     bool use_graph = true, use_pdl = true;
     int gemv_chunk = 0, gemv_smem = 0, gemv_groups = 0;   // projection ring knobs (0 = built-in default)
     int gemv_cuda_core = 1;                               // 1: bf16 projections on CUDA cores
+    int gemv_tcgen05 = 1;                                 // 1: bf16 projections on tcgen05 where they fit
+    // tensor-core path: TMA tensor maps of the weights, split-K workspace
+    bool tc_ready = false;
+    CUtensorMap tm_lm;
+    CUtensorMap tm_step[kMaxSteps][5];                    // fusion, QKV, O, gate/up, down
+    bool tm_lm_ok = false;
+    bool tm_step_ok[kMaxSteps]{};
+    float *tc_part = nullptr;
+    size_t tc_part_floats = 0;
+    int *tc_ctr = nullptr;
+    int tc_ctr_n = 0;
     std::vector<GraphEntry> graphs;
     unsigned long long tick = 0;
     std::string error;
@@ -157,8 +168,21 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
     base.groups = c->gemv_groups;
     base.force_cuda_core = c->gemv_cuda_core;
 
+    // a projection on the tensor-core kernel when enabled and it fits, else on
+    // the CUDA-core ring kernel
+    auto proj = [&](const GemvArgs &g, const CUtensorMap *tm, int grid, bool pdl_here) -> cudaError_t {
+        if (tm && c->gemv_tcgen05 && c->tc_ready && c->bf16 && gemv_tc_supported(g, c->sms)) {
+            // split-K launches need the partial-sum workspace and one ticket per tile
+            const size_t ws = gemv_tc_workspace_floats(g, c->sms);
+            if (ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n))
+                return launch_gemv_tc(g, *tm, c->sms, c->tc_part, c->tc_ctr, s, pdl_here);
+        }
+        return launch_gemv(g, c->bf16, grid, s, pdl_here);
+    };
+
     for (int k = 1; k <= K && e == cudaSuccess; ++k) {
         const prism_step_weights &w = c->steps[k - 1];
+        const CUtensorMap *tms = c->tm_step_ok[k - 1] ? c->tm_step[k - 1] : nullptr;
         const bool prefill = k == 1;
         const int T1 = prefill ? r.B * f.max_new : r.B;
         const bool p = pdl && !first;
@@ -175,7 +199,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.epi = kEpiStore;
         g.out = c->x0;
         g.out_ld = d;
-        e = launch_gemv(g, c->bf16, gemv_grid(c, d), s, p);
+        e = proj(g, tms ? &tms[0] : nullptr, gemv_grid(c, d), p);
         after(0);
         if (e != cudaSuccess) break;
 
@@ -192,7 +216,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.epi = kEpiStore;
         g.out = c->qkv;
         g.out_ld = c->qkv_rows;
-        e = launch_gemv(g, c->bf16, gemv_grid(c, c->qkv_rows), s, pdl);
+        e = proj(g, tms ? &tms[1] : nullptr, gemv_grid(c, c->qkv_rows), pdl);
         after(1);
         if (e != cudaSuccess) break;
 
@@ -260,7 +284,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.resid_prefill_rows = prefill;
         g.out = c->a;
         g.out_ld = d;
-        e = launch_gemv(g, c->bf16, gemv_grid(c, d), s, pdl);
+        e = proj(g, tms ? &tms[2] : nullptr, gemv_grid(c, d), pdl);
         after(4);
         if (e != cudaSuccess) break;
 
@@ -278,7 +302,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.epi = kEpiSwiGLU;
         g.out_act = c->m_buf;
         g.out_ld = F;
-        e = launch_gemv(g, c->bf16, gemv_grid(c, F), s, pdl);
+        e = proj(g, tms ? &tms[3] : nullptr, gemv_grid(c, F), pdl);
         after(5);
         if (e != cudaSuccess) break;
 
@@ -296,7 +320,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.out = c->hhat;
         g.out_ld = d;
         g.hidden_out = r.hidden_out;
-        e = launch_gemv(g, c->bf16, gemv_grid(c, d), s, pdl);
+        e = proj(g, tms ? &tms[4] : nullptr, gemv_grid(c, d), pdl);
         after(6);
         if (e != cudaSuccess) break;
 
@@ -318,7 +342,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.draft_out = r.draft;
         g.topk_ids = r.topk_ids;
         g.topk_logits = r.topk_logits;
-        e = launch_gemv(g, c->bf16, c->lm_grid, s, pdl);
+        e = proj(g, c->tm_lm_ok ? &c->tm_lm : nullptr, c->lm_grid, pdl);
         after(7);
     }
     if (n_kernels) *n_kernels = nk;
@@ -377,6 +401,26 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     c->attn_splits = (f.max_ctx + c->attn_chunk - 1) / c->attn_chunk;
 
     const size_t T1 = (size_t)f.max_batch * f.max_new, B = f.max_batch;
+    // split-K workspace of the tensor-core projections: the largest need of
+    // any projection of this shape
+    size_t tc_floats = 0;
+    int tc_tiles = 0;
+    if (c->bf16) {
+        const int units[] = {d, c->qkv_rows, d, F, d};
+        const int kins[] = {2 * d, d, Hq * D, d, F};
+        const int epis[] = {kEpiStore, kEpiStore, kEpiResid, kEpiSwiGLU, kEpiResid};
+        for (int i = 0; i < 5; ++i)
+            for (int T : {(int)T1, (int)B}) {
+                GemvArgs g{};
+                g.n_units = units[i];
+                g.kin = kins[i];
+                g.epi = epis[i];
+                g.T = T;
+                const size_t need = gemv_tc_workspace_floats(g, c->sms);
+                if (need > tc_floats) tc_floats = need;
+                if (gemv_tc_tiles(g) > tc_tiles) tc_tiles = gemv_tc_tiles(g);
+            }
+    }
     size_t sizes[] = {
         (size_t)f.max_ctx * (D / 2) * 4,                           // rope cos
         (size_t)f.max_ctx * (D / 2) * 4,                           // rope sin
@@ -392,6 +436,8 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         B * (size_t)c->lm_grid * kTopK * 4,                        // LM partial ids
         (B * Hkv + 1) * 4,                                         // counters
         32,                                                        // error word (+ checked-build record)
+        tc_floats * 4,                                             // tensor-core split-K partials
+        (size_t)tc_tiles * 4,                                      // tensor-core tile tickets
     };
     size_t total = 0;
     for (size_t s : sizes) total += align256(s);
@@ -418,6 +464,10 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     c->lm_id = (int *)slot[11];
     c->counters = (int *)slot[12];
     c->err = (int *)slot[13];
+    c->tc_part = (float *)slot[14];
+    c->tc_part_floats = tc_floats;
+    c->tc_ctr = (int *)slot[15];
+    c->tc_ctr_n = tc_tiles;
 
     // rotary tables: angle p * theta^(-2j/D), computed in double, stored as float
     std::vector<float> cs((size_t)f.max_ctx * (D / 2)), sn((size_t)f.max_ctx * (D / 2));
@@ -431,6 +481,12 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     e = cudaMemcpy(c->rope_cos, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(c->rope_sin, sn.data(), sn.size() * 4, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = prepare_gemv_kernels();
+    if (e == cudaSuccess && c->bf16) {
+        // the tensor-core path is optional: without a tensor-map encoder the
+        // CUDA-core kernels run everything
+        c->tc_ready = prepare_gemv_tc_kernels() == cudaSuccess;
+        cudaGetLastError();
+    }
     if (e == cudaSuccess) {
         // every projection shape must fit the shared-memory ring
         const int T1 = f.max_batch * f.max_new;
@@ -482,6 +538,7 @@ prism_status prism_load_shared_weights(prism_ctx *c, const void *embed, const vo
         return fail(c, PRISM_ERR_INVALID_ARG, "embed and lm_head must be 16-byte aligned");
     c->embed = embed;
     c->lm_head = lm_head;
+    c->tm_lm_ok = c->tc_ready && make_weight_map(&c->tm_lm, lm_head, c->cfg.vocab, c->cfg.hidden) == cudaSuccess;
     drop_graphs(c);
     return PRISM_OK;
 }
@@ -496,6 +553,16 @@ prism_status prism_load_step_weights(prism_ctx *c, int32_t step, const prism_ste
         if (p && !aligned16(p)) return fail(c, PRISM_ERR_INVALID_ARG, "weight pointers must be 16-byte aligned");
     c->steps[step] = *w;
     c->step_loaded[step] = true;
+    if (c->tc_ready) {
+        const prism_config &f = c->cfg;
+        const int d = f.hidden, F = f.ffn;
+        CUtensorMap *m = c->tm_step[step];
+        c->tm_step_ok[step] = make_weight_map(&m[0], w->w_fuse, d, 2 * d) == cudaSuccess &&
+                              make_weight_map(&m[1], w->w_qkv, c->qkv_rows, d) == cudaSuccess &&
+                              make_weight_map(&m[2], w->w_o, d, f.n_q_heads * f.head_dim) == cudaSuccess &&
+                              make_weight_map(&m[3], w->w_gate_up, 2 * F, d) == cudaSuccess &&
+                              make_weight_map(&m[4], w->w_down, d, F) == cudaSuccess;
+    }
     drop_graphs(c);
     return PRISM_OK;
 }
@@ -509,6 +576,7 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "gemv_groups") && (value == 0 || value == 1 || value == 2 || value == 4 ||
                                                    value == 8 || value == 16)) c->gemv_groups = value;
     else if (!std::strcmp(name, "gemv_cuda_core")) c->gemv_cuda_core = value != 0;
+    else if (!std::strcmp(name, "gemv_tcgen05")) c->gemv_tcgen05 = value != 0;
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);
     return PRISM_OK;

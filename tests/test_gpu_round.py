@@ -34,13 +34,13 @@ def mid_case():
     return W, I
 
 
-def _check(w, W, I, seqs, *, topk):
+def _check(w, W, I, seqs, *, topk, options=None):
     """Free-running round on the full batch, then every later step recomputed
     from the oracle's state (teacher forcing) in the same batch shape."""
     K = w.shape.n_steps
     model = GpuModel(W)
     try:
-        g = gpu_round(w, W, I, topk=topk, model=model)
+        g = gpu_round(w, W, I, topk=topk, model=model, options=options)
         assert g["flags"] == 0, f"device error word {g['flags']}"
         o = oracle.draft_round(w.shape, W, I, topk=max(2, topk), want_logits=True, seqs=seqs)
         rep = compare_round(g, o, I, seqs, K, topk, chain=True)
@@ -50,7 +50,7 @@ def _check(w, W, I, seqs, *, topk):
             Ik = forced_step_inputs(I, o, seqs, k)
             dr = model.drafter(w.shape, [W["f_map"][k - 1]], max_batch=w.batch, max_ctx=int(I["max_ctx"]),
                                max_new=1, topk=topk)
-            gk = run_round(dr, Ik, n_steps=1, topk=topk)
+            gk = run_round(dr, Ik, n_steps=1, topk=topk, options=options)
             dr.close()
             assert gk["flags"] == 0
             compare_round(gk, oracle_step(o, k), Ik, seqs, 1, topk, report=forced)
@@ -99,15 +99,72 @@ def test_modes_are_bit_identical():
             assert np.array_equal(r[key], runs[0][key]), key
 
 
-def test_tensor_core_projection_path_matches_oracle():
-    """The warp-level tensor-core projection kernel (option gemv_cuda_core=0)
-    meets the same bar as the default CUDA-core kernel."""
+@pytest.mark.parametrize("options", [{"gemv_tcgen05": 0}, {"gemv_tcgen05": 0, "gemv_cuda_core": 0}],
+                         ids=["cuda-core-ring", "mma-sync"])
+def test_fallback_projection_kernels_match_oracle(options):
+    """The kernels that carry projections the tcgen05 kernel does not take
+    (more than 16 activation rows, fp32 weights): the CUDA-core TMA-ring
+    kernel and the warp-level mma.sync kernel, forced for every projection."""
     W, I = mid_case()
-    g = gpu_round(MID_W, W, I, topk=8, options={"gemv_cuda_core": 0})
+    g = gpu_round(MID_W, W, I, topk=8, options=options)
     assert g["flags"] == 0
     o = oracle.draft_round(MID_W.shape, W, I, topk=8, want_logits=True, seqs=[0, 1, 2])
     compare_round(g, o, I, [0, 1, 2], MID_W.shape.n_steps, 8, chain=True)
     compare_cache(g["k_cache"], g["v_cache"], o["k_cache"], o["v_cache"], I, [0, 1, 2], MID_W.shape.n_steps)
+
+
+TCGEN05 = {"gemv_tcgen05": 1}
+
+
+@pytest.mark.parametrize("case", ["tiny-bf16", "mid"])
+def test_tcgen05_projection_path_matches_oracle(case):
+    """Projections on the tcgen05 kernel (TMA tensor loads, MMA into tensor
+    memory, split-K for short outputs); prefill rows beyond 16 stay on the
+    CUDA-core kernel, so the tiny case mixes both."""
+    if case == "mid":
+        w = MID_W
+        W, I = mid_case()
+        seqs = [0, 1, 2]
+    else:
+        w = synth.WORKLOADS[case]
+        W, I = synth.make_weights(w), synth.make_round_inputs(w)
+        seqs = [0]
+    _, _, rep = _check(w, W, I, seqs, topk=8, options=TCGEN05)
+    print(case, rep)
+    assert rep["ids_compared"] >= 1
+
+
+def test_tcgen05_modes_bit_identical():
+    """Graph replay, eager launches, with and without programmatic dependent
+    launch: identical outputs on the tcgen05 path (split-K sums in fixed order)."""
+    W, I = mid_case()
+    model = GpuModel(W)
+    try:
+        runs = []
+        for graph, pdl in ((1, 1), (0, 1), (0, 0), (1, 0)):
+            dr = model.drafter(MID_W.shape, list(W["f_map"]), max_batch=MID_W.batch, max_ctx=int(I["max_ctx"]),
+                               max_new=I["tokens"].shape[1], topk=8)
+            r = run_round(dr, I, n_steps=MID_W.shape.n_steps, topk=8,
+                          options=dict(TCGEN05, use_graph=graph, use_pdl=pdl))
+            dr.close()
+            assert r["flags"] == 0
+            runs.append(r)
+        for r in runs[1:]:
+            for key in ("draft_ids", "topk_ids", "topk_logits", "logits", "hidden_out", "k_cache", "v_cache"):
+                assert np.array_equal(r[key], runs[0][key]), key
+    finally:
+        model.close()
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name,n_sample", [("l3-8b-b1", 1), ("l3-8b-b16", 3)])
+def test_cuda_core_full_size_round(name, n_sample):
+    """Full-size rounds with every projection on the CUDA-core ring kernel."""
+    w = synth.WORKLOADS[name]
+    W, I = synth.make_weights(w), synth.make_round_inputs(w)
+    _, _, rep = _check(w, W, I, sample_seqs(w.batch, n_sample), topk=w.topk, options={"gemv_tcgen05": 0})
+    print(name, rep)
+    assert rep["ids_compared"] >= 1
 
 
 def test_graph_replay_is_repeatable():
