@@ -400,7 +400,7 @@ def run_ours(args, w, world, rank, local):
             "kernel_ms_per_round": kind_total,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-            "gpu_launches": 8 * K * args.steps,
+            "gpu_launches": len(prof[0]) * args.steps,
             "clocks": clk,
             "device_error_word": flags,
         }

@@ -204,15 +204,20 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * the tcgen05 kernel, TMA tensor loads into tensor-memory accumulators; 0:
  * every projection on the kernels below), "gemv_cuda_core" (for projections
  * not on the tcgen05 kernel: 1, the default, the CUDA-core TMA-ring kernel;
- * 0: the warp-level mma.sync kernel).  Changing an option drops cached
- * graphs.  Errors: INVALID_ARG (unknown name or value out of range). */
+ * 0: the warp-level mma.sync kernel), "attn_fused" (1, the default: RoPE,
+ * KV append and attention run as one kernel, a cluster of up to 8 CTAs per
+ * sequence and KV head merging through distributed shared memory; 0: a
+ * RoPE/append kernel, then split-KV attention with a last-CTA merge).
+ * Changing an option drops cached graphs.  Errors: INVALID_ARG (unknown name
+ * or value out of range). */
 prism_status prism_set_option(prism_ctx *ctx, const char *name, int32_t value);
 
 /* Instrumented round for measurement: the same work as prism_draft_round
  * launched eagerly with a CUDA event recorded before and after every kernel.
  * kernel_ms[i] receives the duration of kernel i in launch order (capacity
  * max_kernels); *n_kernels receives the count; kernel_kind[i] (may be NULL)
- * receives a code: 0 fusion, 1 qkv, 2 rope/append, 3 attention, 4 o-proj,
+ * receives a code: 0 fusion, 1 qkv, 2 rope/append, 3 attention (with the
+ * fused option: RoPE, append and attention; no code-2 kernel then), 4 o-proj,
  * 5 gate/up, 6 down, 7 LM head + selection.  Synchronises the stream. */
 prism_status prism_profile_round(prism_ctx *ctx, int32_t batch, const int32_t *tokens,
                                  const void *hidden, const int32_t *n_new, const int32_t *kv_len,

@@ -317,6 +317,793 @@ __global__ void accept_kernel(const AcceptArgs a) {
     a.kv_len[b] += a.n_new[b];
 }
 
+// ------------------------------------------------------------------ fused
+// RoPE + KV append + attention for one query row per sequence, one thread-
+// block cluster of CS CTAs per (sequence b, KV head g).  CTA rank r owns the
+// key range [r P / CS, (r+1) P / CS) of the causal window [0, P):
+//   * cache rows below the committed length L are never written during a
+//     round, so the first two chunks of them are requested (cp.async) before
+//     griddepcontrol.wait, overlapping the QKV projection's tail;
+//   * after the wait, the CTA whose range holds a new position rotates that
+//     row's key and stores key and value in the cache; every CTA rotates the
+//     query heads of g (scaled by 1/sqrt(D)) into shared memory;
+//   * keys stream in chunks of C rows through two shared-memory buffers, K
+//     stored transposed (16-byte vector v of key j at [v][j]) so that a warp
+//     reads 32 consecutive keys without bank conflicts while every lane reads
+//     the same query element; V stays row-major (a warp reads consecutive
+//     dims of one row).  An online softmax keeps the running max, sum and
+//     unnormalised output of each head;
+//   * the CS partial results are merged through distributed shared memory:
+//     after a cluster barrier, rank r combines its slice of the (head, dim)
+//     outputs from every rank, in rank order, and writes the bf16-rounded
+//     attention output.  A second cluster barrier keeps every rank's shared
+//     memory alive until all reads are done.
+constexpr int kFusedThreads = 512;
+constexpr int kMaxCluster = 16;
+constexpr long kAttnWaitLimit = 1L << 22;
+
+template <typename WT, int D> struct FusedCfg {
+    static constexpr int C = sizeof(WT) * D <= 256 ? 128 : 64;   // keys per chunk
+    static constexpr int kVecs = D * (int)sizeof(WT) / 16;       // 16-byte vectors per row
+    static constexpr int kPerVec = 16 / (int)sizeof(WT);         // elements per vector
+};
+
+__device__ __forceinline__ uint32_t sa(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ float dsmem_ld(const float *local, uint32_t rank) {
+    uint32_t remote;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(sa(local)), "r"(rank));
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
+    return v;
+}
+__device__ __forceinline__ bool fa_try(uint64_t *b, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+                 : "=r"(ok) : "r"(sa(b)), "r"(parity) : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Request chunk [j, j + cnt) of head (b, g): K transposed into kt, V row-major
+// into vb (16-byte pieces, one per thread in turn).  The caller commits.
+template <typename WT, int D>
+__device__ __forceinline__ void fa_load(const FusedAttnArgs &a, int b, int g, int j, int cnt, uint4 *kt, WT *vb) {
+    using Cf = FusedCfg<WT, D>;
+    constexpr int C = Cf::C, NV = Cf::kVecs;
+    const size_t off = (((size_t)b * a.Hkv + g) * a.max_ctx + j) * D;
+    const uint4 *ks = (const uint4 *)((const WT *)a.k_cache + off);
+    const uint4 *vs = (const uint4 *)((const WT *)a.v_cache + off);
+    for (int e = threadIdx.x; e < cnt * NV; e += kFusedThreads) {
+        const int jj = e / NV, v = e % NV;
+        cp_async16(kt + v * C + jj, ks + e);
+        cp_async16((uint4 *)vb + e, vs + e);
+    }
+}
+
+// p4[i % 4] += q[i] * k[i] over one 16-byte vector of keys (q broadcast).
+template <typename WT>
+__device__ __forceinline__ void dot4(float (&p4)[4], const float *q, const uint4 &k);
+template <>
+__device__ __forceinline__ void dot4<uint16_t>(float (&p4)[4], const float *q, const uint4 &k) {
+    const float4 q0 = *(const float4 *)q, q1 = *(const float4 *)(q + 4);
+    p4[0] = fmaf(q0.x, bf16lo(k.x), p4[0]);
+    p4[1] = fmaf(q0.y, bf16hi(k.x), p4[1]);
+    p4[2] = fmaf(q0.z, bf16lo(k.y), p4[2]);
+    p4[3] = fmaf(q0.w, bf16hi(k.y), p4[3]);
+    p4[0] = fmaf(q1.x, bf16lo(k.z), p4[0]);
+    p4[1] = fmaf(q1.y, bf16hi(k.z), p4[1]);
+    p4[2] = fmaf(q1.z, bf16lo(k.w), p4[2]);
+    p4[3] = fmaf(q1.w, bf16hi(k.w), p4[3]);
+}
+template <>
+__device__ __forceinline__ void dot4<float>(float (&p4)[4], const float *q, const uint4 &k) {
+    const float4 q0 = *(const float4 *)q;
+    p4[0] = fmaf(q0.x, __uint_as_float(k.x), p4[0]);
+    p4[1] = fmaf(q0.y, __uint_as_float(k.y), p4[1]);
+    p4[2] = fmaf(q0.z, __uint_as_float(k.z), p4[2]);
+    p4[3] = fmaf(q0.w, __uint_as_float(k.w), p4[3]);
+}
+
+template <typename WT, int D>
+__global__ void __launch_bounds__(kFusedThreads, 1) fused_attention_kernel(const FusedAttnArgs a) {
+    using Cf = FusedCfg<WT, D>;
+    constexpr int C = Cf::C, NV = Cf::kVecs;
+    extern __shared__ __align__(128) uint8_t smem_raw[];
+    __shared__ float s_m[16], s_l[16], s_alpha[16];
+    const int G = a.Hq / a.Hkv;
+    uint4 *kt = (uint4 *)smem_raw;                   // [2][NV][C] transposed keys
+    WT *vbuf = (WT *)(kt + 2 * NV * C);              // [2][C][D]
+    float *qs = (float *)(vbuf + 2 * C * D);         // [G][D] rotated, scaled queries
+    float *ps = qs + G * D;                          // [G][C] scores, then probabilities
+    float *po = ps + G * C;                          // [G][D] this rank's unnormalised output
+    float *pm = po + G * D;                          // [16] this rank's running max
+    float *pl = pm + 16;                             // [16] this rank's running sum
+
+    const int r = blockIdx.x, g = blockIdx.y, b = blockIdx.z, CS = a.cs;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int half = D / 2, H = a.Hq + 2 * a.Hkv;
+    pdl_trigger();
+
+    // ranges (n_new and kv_len are inputs of the round, stable throughout it)
+    const int n = clamp_n(a.n_new, b, a.max_new, a.err);
+    const int L = a.kv_len[b];
+    const int qp = query_pos(a.prefill, L, n, a.step);
+    int P = qp + 1;
+    if (P > a.max_ctx) P = a.max_ctx;
+    if (P < 1) P = 1;
+    const int j0 = (int)((long)r * P / CS), j1 = (int)((long)(r + 1) * P / CS);
+    const int nch = (j1 - j0 + C - 1) / C;
+    const int L_old = L < P ? (L > 0 ? L : 0) : P;   // rows below L_old are immutable
+    auto chunk = [&](int i, int &j, int &cnt) {
+        j = j0 + i * C;
+        cnt = j1 - j < C ? j1 - j : C;
+    };
+    // chunk 1 holds later positions than chunk 0, so "chunk 1 old" implies "chunk 0 old"
+    int pre = 0;                                      // chunks requested before the wait
+    for (int i = 0; i < 2 && i < nch; ++i) {
+        int j, cnt;
+        chunk(i, j, cnt);
+        if (j + cnt > L_old) break;
+        fa_load<WT, D>(a, b, g, j, cnt, kt + i * NV * C, vbuf + i * C * D);
+        cp_commit();
+        ++pre;
+    }
+    pdl_wait();
+
+    // append the new rows this rank owns: positions L .. L+n-1 (prefill) or qp
+    const int first_new = a.prefill ? L : qp, n_rows = a.prefill ? n : 1;
+    for (int i = 0; i < n_rows; ++i) {
+        const int pos = first_new + i;
+        if (pos < 0 || pos >= a.max_ctx) {              // no rank owns it: rank 0 reports
+            if (r == 0 && tid == 0) set_err(a.err, kErrCache);
+            continue;
+        }
+        if (pos < j0 || pos >= j1) continue;
+        const int row = a.prefill ? b * a.max_new + i : b;
+        const float *xk = a.qkv + (size_t)row * H * D + (size_t)(a.Hq + g) * D;
+        const float *xv = a.qkv + (size_t)row * H * D + (size_t)(a.Hq + a.Hkv + g) * D;
+        WT *kc = (WT *)a.k_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + pos) * D;
+        WT *vc = (WT *)a.v_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + pos) * D;
+        for (int j = tid; j < half; j += kFusedThreads) {
+            const float c = a.rope_cos[(size_t)pos * half + j], sn = a.rope_sin[(size_t)pos * half + j];
+            const float x0 = xk[j], x1 = xk[j + half];
+            Elem<WT>::store(kc, j, x0 * c - x1 * sn);
+            Elem<WT>::store(kc, j + half, x1 * c + x0 * sn);
+        }
+        for (int j = tid; j < D; j += kFusedThreads) Elem<WT>::store(vc, j, xv[j]);
+    }
+    // rotated queries of the heads sharing g, at qp, scaled by 1/sqrt(D)
+    {
+        const int row = a.prefill ? b * a.max_new + n - 1 : b;
+        const int pc = qp >= 0 && qp < a.max_ctx ? qp : 0;
+        const float scale = 1.0f / sqrtf((float)D);
+        for (int e = tid; e < G * half; e += kFusedThreads) {
+            const int h = e / half, j = e % half;
+            const float *xq = a.qkv + (size_t)row * H * D + (size_t)(g * G + h) * D;
+            const float c = a.rope_cos[(size_t)pc * half + j], sn = a.rope_sin[(size_t)pc * half + j];
+            const float x0 = xq[j], x1 = xq[j + half];
+            qs[h * D + j] = (x0 * c - x1 * sn) * scale;
+            qs[h * D + j + half] = (x1 * c + x0 * sn) * scale;
+        }
+    }
+    if (tid < 16) { s_m[tid] = -INFINITY; s_l[tid] = 0.f; }
+    __syncthreads();                                  // new cache rows written, queries ready
+    for (int i = pre; i < 2 && i < nch; ++i) {
+        int j, cnt;
+        chunk(i, j, cnt);
+        fa_load<WT, D>(a, b, g, j, cnt, kt + i * NV * C, vbuf + i * C * D);
+        cp_commit();
+    }
+
+    // per-thread outputs: e = tid + 512 i  ->  (head e / D, dim e % D)
+    constexpr int kMaxOut = (16 * D + kFusedThreads - 1) / kFusedThreads;
+    float acc[kMaxOut];
+#pragma unroll
+    for (int i = 0; i < kMaxOut; ++i) acc[i] = 0.f;
+    const int n_out = G * D;
+    constexpr int NHG = kFusedThreads / C;            // head groups in the score pass
+
+    for (int ci = 0; ci < nch; ++ci) {
+        const int bi = ci & 1;
+        int j, cnt;
+        chunk(ci, j, cnt);
+        const uint4 *kb = kt + bi * NV * C;
+        const WT *vb = vbuf + bi * C * D;
+        // this chunk's copies are the oldest outstanding group
+        if (ci + 1 < nch) cp_wait<1>(); else cp_wait<0>();
+        __syncthreads();
+        // scores: thread -> key jl = tid % C, heads tid / C + NHG i; four partial sums
+        {
+            const int jl = tid % C;
+            for (int h = tid / C; h < G; h += NHG) {
+                float dot = -INFINITY;
+                if (jl < cnt) {
+                    float p4[4] = {0.f, 0.f, 0.f, 0.f};
+                    const float *q = qs + h * D;
+#pragma unroll 4
+                    for (int v = 0; v < NV; ++v) dot4<WT>(p4, q + v * Cf::kPerVec, kb[v * C + jl]);
+                    dot = (p4[0] + p4[1]) + (p4[2] + p4[3]);
+                }
+                ps[h * C + jl] = dot;
+            }
+        }
+        __syncthreads();
+        // online softmax: warp w takes heads w, w + 16
+        for (int h = warp; h < G; h += kFusedThreads / 32) {
+            float mx = -INFINITY;
+            for (int jl = lane; jl < cnt; jl += 32) mx = fmaxf(mx, ps[h * C + jl]);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
+            const float m_old = s_m[h];
+            const float m_new = fmaxf(m_old, mx);
+            float sum = 0.f;
+            for (int jl = lane; jl < cnt; jl += 32) {
+                const float pv = m_new == -INFINITY ? 0.f : expf(ps[h * C + jl] - m_new);
+                ps[h * C + jl] = pv;
+                sum += pv;
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+            if (lane == 0) {
+                const float alpha = m_old == -INFINITY ? 0.f : expf(m_old - m_new);
+                s_alpha[h] = alpha;
+                s_l[h] = s_l[h] * alpha + sum;
+                s_m[h] = m_new;
+            }
+        }
+        __syncthreads();
+        // PV: acc(h, d) = acc * alpha_h + sum_j p_hj V_jd; keys unrolled by 8 in two chains
+#pragma unroll
+        for (int i = 0; i < kMaxOut; ++i) {
+            const int e = tid + kFusedThreads * i;
+            if (e >= n_out) break;
+            const int h = e / D, d = e % D;
+            const float *ph = ps + h * C;
+            float x0 = acc[i] * s_alpha[h], x1 = 0.f;
+            int jl = 0;
+            for (; jl + 8 <= cnt; jl += 8) {
+#pragma unroll
+                for (int u = 0; u < 8; u += 2) {
+                    x0 = fmaf(ph[jl + u], Elem<WT>::load(vb, (size_t)(jl + u) * D + d), x0);
+                    x1 = fmaf(ph[jl + u + 1], Elem<WT>::load(vb, (size_t)(jl + u + 1) * D + d), x1);
+                }
+            }
+            for (; jl < cnt; ++jl) x0 = fmaf(ph[jl], Elem<WT>::load(vb, (size_t)jl * D + d), x0);
+            acc[i] = x0 + x1;
+        }
+        __syncthreads();                              // buffer bi and ps free
+        if (ci + 2 < nch) {
+            int jn, cn;
+            chunk(ci + 2, jn, cn);
+            fa_load<WT, D>(a, b, g, jn, cn, kt + bi * NV * C, vbuf + bi * C * D);
+            cp_commit();
+        }
+    }
+    cp_wait<0>();
+
+    // publish this rank's partial, then merge across the cluster
+#pragma unroll
+    for (int i = 0; i < kMaxOut; ++i) {
+        const int e = tid + kFusedThreads * i;
+        if (e < n_out) po[e] = acc[i];
+    }
+    if (tid < G) { pm[tid] = s_m[tid]; pl[tid] = s_l[tid]; }
+    cluster_sync_all();
+    {
+        const int e0 = (int)((long)r * n_out / CS), e1 = (int)((long)(r + 1) * n_out / CS);
+        for (int e = e0 + tid; e < e1; e += kFusedThreads) {
+            const int h = e / D;
+            // every remote load of this output issued before any is used
+            float mq[kMaxCluster], lq[kMaxCluster], oq[kMaxCluster];
+#pragma unroll
+            for (int q = 0; q < kMaxCluster; ++q) {
+                if (q < CS) {
+                    mq[q] = dsmem_ld(pm + h, (uint32_t)q);
+                    lq[q] = dsmem_ld(pl + h, (uint32_t)q);
+                    oq[q] = dsmem_ld(po + e, (uint32_t)q);
+                } else {
+                    mq[q] = -INFINITY;
+                    lq[q] = oq[q] = 0.f;
+                }
+            }
+            float M = -INFINITY;
+#pragma unroll
+            for (int q = 0; q < kMaxCluster; ++q) M = fmaxf(M, mq[q]);
+            float num = 0.f, den = 0.f;
+#pragma unroll
+            for (int q = 0; q < kMaxCluster; ++q) {
+                const float w = mq[q] == -INFINITY ? 0.f : expf(mq[q] - M);
+                den = fmaf(w, lq[q], den);
+                num = fmaf(w, oq[q], num);
+            }
+            WT *o = (WT *)a.o_out + (size_t)b * a.Hq * D + (size_t)g * G * D;
+            Elem<WT>::store(o, e, den > 0.f ? num / den : 0.f);
+        }
+    }
+    cluster_sync_all();
+}
+
+// Tensor-core variant for bf16 caches: S = Q K^T and O += P V as mma.sync
+// m16n8k16 tiles (16 rows = the query heads of g, padded).  The contract keeps
+// q and the probabilities in fp32, so each enters the product as a bf16 pair
+// hi + lo (hi = bf16(x), lo = bf16(x - hi)): two MMAs per tile, an error near
+// 2^-17 of the operand, with K and V exact.  Every shared-memory operand tile
+// (keys, values, hi/lo queries and probabilities) is stored with its 16-byte
+// pieces XOR-swizzled by row, so ldmatrix reads are free of bank conflicts.
+constexpr int kMmaC = 160;                            // keys per chunk (multiple of 32)
+constexpr int kMmaPS = (kMmaC + 63) / 64 * 64;        // probability row stride: whole 8-piece groups
+
+__device__ __forceinline__ uint32_t swz(int row, int slot) { return (uint32_t)(slot ^ (row & 7)); }
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+                 "{%8, %9}, {%0, %1, %2, %3};"
+                 : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+                 : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+// bf16 hi/lo split of two floats, packed (low half = first element).
+__device__ __forceinline__ void split2(float x, float y, uint32_t &hi, uint32_t &lo) {
+    const uint16_t hx = f32_to_bf16(x), hy = f32_to_bf16(y);
+    hi = (uint32_t)hx | ((uint32_t)hy << 16);
+    lo = (uint32_t)f32_to_bf16(x - bf16_to_f32(hx)) | ((uint32_t)f32_to_bf16(y - bf16_to_f32(hy)) << 16);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kFusedThreads, 1)
+    fused_attention_mma_kernel(const FusedAttnArgs a, const __grid_constant__ CUtensorMap tk,
+                               const __grid_constant__ CUtensorMap tv) {
+    constexpr int C = kMmaC;
+    constexpr int NH = D / 64;                        // 64-column boxes per row
+    constexpr uint32_t kBox = C * 128;                // one box: C rows x 128 bytes
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full[2];
+    __shared__ float s_m[16], s_l[16], s_alpha[16];
+    __shared__ float red_max[kFusedThreads / 32][16], red_sum[kFusedThreads / 32][16];
+    const int G = a.Hq / a.Hkv;
+    // K and V chunks as TMA wrote them: per buffer NH boxes of C rows x 128 B,
+    // 16-byte piece c of row r at (c ^ (r % 8)) (128-byte swizzle, 1 KB atoms)
+    uint8_t *base = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint16_t *kbuf = (uint16_t *)base;                // [2][NH][C][64]
+    uint16_t *vbuf = kbuf + 2 * C * D;                // [2][NH][C][64]
+    uint16_t *qhi = vbuf + 2 * C * D;                 // [16][D] swizzled
+    uint16_t *qlo = qhi + 16 * D;
+    uint16_t *phi = qlo + 16 * D;                     // [16][kMmaPS] swizzled
+    uint16_t *plo = phi + 16 * kMmaPS;
+    float *qs = (float *)(plo + 16 * kMmaPS);         // [16][D] rotated, scaled queries
+    float *po = qs + 16 * D;                          // [16][D] this rank's unnormalised output
+    float *pm = po + 16 * D;                          // [16]
+    float *pl = pm + 16;                              // [16]
+
+    const int r = blockIdx.x, g = blockIdx.y, b = blockIdx.z, CS = a.cs;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int half = D / 2, H = a.Hq + 2 * a.Hkv;
+    pdl_trigger();
+
+    const int n = clamp_n(a.n_new, b, a.max_new, a.err);
+    const int L = a.kv_len[b];
+    const int qp = query_pos(a.prefill, L, n, a.step);
+    int P = qp + 1;
+    if (P > a.max_ctx) P = a.max_ctx;
+    if (P < 1) P = 1;
+    const int j0 = (int)((long)r * P / CS), j1 = (int)((long)(r + 1) * P / CS);
+    const int nch = (j1 - j0 + C - 1) / C;
+    const int L_old = L < P ? (L > 0 ? L : 0) : P;
+    auto chunk = [&](int i, int &j, int &cnt) {
+        j = j0 + i * C;
+        cnt = j1 - j < C ? j1 - j : C;
+    };
+    // request chunk i into buffer i & 1: 2 NH boxes (K and V) of C rows from
+    // position j of head (b, g); rows past max_ctx arrive as zeros (thread 0)
+    int n_iss0 = 0, n_iss1 = 0;
+    auto load = [&](int i) {
+        int j, cnt;
+        chunk(i, j, cnt);
+        uint64_t *bar = &full[i & 1];
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(sa(bar)), "r"(2 * NH * kBox)
+                     : "memory");
+        const int z = b * a.Hkv + g;
+        const uint32_t kd = sa(kbuf + (i & 1) * C * D), vd = sa(vbuf + (i & 1) * C * D);
+#pragma unroll
+        for (int h = 0; h < NH; ++h) {
+            asm volatile(
+                "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
+                "%4}], [%5];" ::"r"(kd + h * kBox), "l"((uint64_t)&tk), "r"(h * 64), "r"(j), "r"(z), "r"(sa(bar))
+                : "memory");
+            asm volatile(
+                "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
+                "%4}], [%5];" ::"r"(vd + h * kBox), "l"((uint64_t)&tv), "r"(h * 64), "r"(j), "r"(z), "r"(sa(bar))
+                : "memory");
+        }
+        if (i & 1) ++n_iss1; else ++n_iss0;
+    };
+    if (tid == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(sa(&full[0])));
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(sa(&full[1])));
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tk) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tv) : "memory");
+    }
+    __syncthreads();
+    int pre = 0;
+    for (int i = 0; i < 2 && i < nch; ++i) {
+        int j, cnt;
+        chunk(i, j, cnt);
+        if (j + cnt > L_old) break;
+        if (tid == 0) load(i);
+        ++pre;
+    }
+    pdl_wait();
+
+    // append the new rows this rank owns
+    const int first_new = a.prefill ? L : qp, n_rows = a.prefill ? n : 1;
+    for (int i = 0; i < n_rows; ++i) {
+        const int pos = first_new + i;
+        if (pos < 0 || pos >= a.max_ctx) {
+            if (r == 0 && tid == 0) set_err(a.err, kErrCache);
+            continue;
+        }
+        if (pos < j0 || pos >= j1) continue;
+        const int row = a.prefill ? b * a.max_new + i : b;
+        const float *xk = a.qkv + (size_t)row * H * D + (size_t)(a.Hq + g) * D;
+        const float *xv = a.qkv + (size_t)row * H * D + (size_t)(a.Hq + a.Hkv + g) * D;
+        uint16_t *kc = (uint16_t *)a.k_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + pos) * D;
+        uint16_t *vc = (uint16_t *)a.v_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + pos) * D;
+        for (int j = tid; j < half; j += kFusedThreads) {
+            const float c = a.rope_cos[(size_t)pos * half + j], sn = a.rope_sin[(size_t)pos * half + j];
+            const float x0 = xk[j], x1 = xk[j + half];
+            kc[j] = f32_to_bf16(x0 * c - x1 * sn);
+            kc[j + half] = f32_to_bf16(x1 * c + x0 * sn);
+        }
+        for (int j = tid; j < D; j += kFusedThreads) vc[j] = f32_to_bf16(xv[j]);
+    }
+    // queries (rows >= G zero), rotated and scaled, fp32 and split hi/lo
+    {
+        const int row = a.prefill ? b * a.max_new + n - 1 : b;
+        const int pc = qp >= 0 && qp < a.max_ctx ? qp : 0;
+        const float scale = 1.0f / sqrtf((float)D);
+        for (int e = tid; e < 16 * half; e += kFusedThreads) {
+            const int h = e / half, j = e % half;
+            float y0 = 0.f, y1 = 0.f;
+            if (h < G) {
+                const float *xq = a.qkv + (size_t)row * H * D + (size_t)(g * G + h) * D;
+                const float c = a.rope_cos[(size_t)pc * half + j], sn = a.rope_sin[(size_t)pc * half + j];
+                const float x0 = xq[j], x1 = xq[j + half];
+                y0 = (x0 * c - x1 * sn) * scale;
+                y1 = (x1 * c + x0 * sn) * scale;
+            }
+            qs[h * D + j] = y0;
+            qs[h * D + j + half] = y1;
+        }
+    }
+    if (tid < 16) { s_m[tid] = -INFINITY; s_l[tid] = 0.f; }
+    __syncthreads();
+    for (int e = tid; e < 16 * D / 2; e += kFusedThreads) {      // pairs of dims
+        const int h = e / (D / 2), d = 2 * (e % (D / 2));
+        uint32_t hi, lo;
+        split2(qs[h * D + d], qs[h * D + d + 1], hi, lo);
+        const uint32_t o = (uint32_t)(h * D + swz(h, d / 8) * 8 + d % 8);
+        *(uint32_t *)(qhi + o) = hi;
+        *(uint32_t *)(qlo + o) = lo;
+    }
+    // the async proxy reads rows this kernel just wrote: order those writes first
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+    __syncthreads();
+    if (tid == 0)
+        for (int i = pre; i < 2 && i < nch; ++i) load(i);
+    bool dead = false;
+
+    float oq4[4][4] = {};                             // O tile: rows lane/4 (+8), dims of this warp,
+                                                      // in four chains (hi / lo x even / odd keys)
+    const int g4 = lane >> 2, t4 = lane & 3;
+    for (int ci = 0; ci < nch; ++ci) {
+        const int bi = ci & 1;
+        int j, cnt;
+        chunk(ci, j, cnt);
+        const uint16_t *kb = kbuf + bi * C * D, *vb = vbuf + bi * C * D;
+        if (!dead) {
+            bool ok = false;
+            for (long it = 0; it < kAttnWaitLimit && !ok; ++it) ok = fa_try(&full[bi], (uint32_t)((ci >> 1) & 1));
+            if (!ok) {
+                if (tid == 0) set_err(a.err, kErrTimeout);
+                dead = true;
+            }
+        }
+        // value rows past the chunk end hold other positions' data: zero them
+        // (their probabilities are zero, and 0 * NaN would not be)
+        if (cnt < C)
+            for (int e = tid; e < (C - cnt) * (D / 8); e += kFusedThreads) {
+                const int row = cnt + e / (D / 8), sl = e % (D / 8);
+                *(uint4 *)((uint8_t *)vb + (sl >> 3) * kBox + row * 128 + (((sl & 7) ^ (row & 7)) << 4)) =
+                    make_uint4(0, 0, 0, 0);
+            }
+        __syncthreads();
+        // S tiles of this warp: 16 rows x keys 8 nt .. 8 nt + 7 for nt = w, w + 16,
+        // each as four independent accumulation chains (hi / lo x even / odd k-steps)
+        constexpr int NT = C / 8, NTW = (NT + 15) / 16;
+        float sv[NTW][4];
+#pragma unroll
+        for (int t = 0; t < NTW; ++t) {
+            const int nt = warp + 16 * t;
+            float sq[4][4] = {};
+            if (nt < NT) {
+                const int kn = nt * 8;
+#pragma unroll
+                for (int ks = 0; ks < D / 16; ks += 2) {
+                    uint32_t b0, b1, b2, b3, a0, a1, a2, a3;
+                    {
+                        const int key = kn + (lane & 7), slot = 2 * ks + (lane >> 3);
+                        ldsm_x4(sa(kb) + (slot >> 3) * kBox + key * 128 + (((slot & 7) ^ (key & 7)) << 4), b0, b1,
+                                b2, b3);
+                    }
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        const int kk = ks + u;
+                        const int qrow = (lane & 7) + ((lane >> 3) & 1) * 8, qslot = 2 * kk + (lane >> 4);
+                        const uint32_t qo = (uint32_t)(qrow * D + swz(qrow, qslot) * 8);
+                        const uint32_t bb0 = u ? b2 : b0, bb1 = u ? b3 : b1;
+                        ldsm_x4(sa(qhi + qo), a0, a1, a2, a3);
+                        mma16816(sq[2 * u], a0, a1, a2, a3, bb0, bb1);
+                        ldsm_x4(sa(qlo + qo), a0, a1, a2, a3);
+                        mma16816(sq[2 * u + 1], a0, a1, a2, a3, bb0, bb1);
+                    }
+                }
+            }
+            // rows g4 and g4 + 8, keys 8 nt + 2 t4 + {0, 1}; keys past the chunk are -inf
+            const int key0 = nt * 8 + 2 * t4;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float v = (sq[0][q] + sq[1][q]) + (sq[2][q] + sq[3][q]);
+                sv[t][q] = nt < NT && key0 + (q & 1) < cnt ? v : -INFINITY;
+            }
+        }
+        // online softmax over the chunk
+        float m0 = -INFINITY, m1 = -INFINITY;
+#pragma unroll
+        for (int t = 0; t < NTW; ++t) {
+            m0 = fmaxf(m0, fmaxf(sv[t][0], sv[t][1]));
+            m1 = fmaxf(m1, fmaxf(sv[t][2], sv[t][3]));
+        }
+#pragma unroll
+        for (int o = 1; o <= 2; o <<= 1) {
+            m0 = fmaxf(m0, __shfl_xor_sync(0xFFFFFFFFu, m0, o));
+            m1 = fmaxf(m1, __shfl_xor_sync(0xFFFFFFFFu, m1, o));
+        }
+        if (t4 == 0) { red_max[warp][g4] = m0; red_max[warp][g4 + 8] = m1; }
+        __syncthreads();
+        float mn0 = s_m[g4], mn1 = s_m[g4 + 8];
+#pragma unroll
+        for (int w = 0; w < kFusedThreads / 32; ++w) {
+            mn0 = fmaxf(mn0, red_max[w][g4]);
+            mn1 = fmaxf(mn1, red_max[w][g4 + 8]);
+        }
+        float r0s = 0.f, r1s = 0.f;
+#pragma unroll
+        for (int t = 0; t < NTW; ++t) {
+            const int nt = warp + 16 * t;
+            if (nt >= NT) continue;
+            float pv[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float mq = q < 2 ? mn0 : mn1;
+                pv[q] = (sv[t][q] == -INFINITY || mq == -INFINITY) ? 0.f : expf(sv[t][q] - mq);
+            }
+            if (g4 >= G) pv[0] = pv[1] = 0.f;
+            if (g4 + 8 >= G) pv[2] = pv[3] = 0.f;
+            const int key0 = nt * 8 + 2 * t4;
+            uint32_t hi, lo;
+            const uint32_t o0 = (uint32_t)(g4 * kMmaPS + swz(g4, key0 / 8) * 8 + key0 % 8);
+            const uint32_t o1 = (uint32_t)((g4 + 8) * kMmaPS + swz(g4 + 8, key0 / 8) * 8 + key0 % 8);
+            split2(pv[0], pv[1], hi, lo);
+            *(uint32_t *)(phi + o0) = hi;
+            *(uint32_t *)(plo + o0) = lo;
+            split2(pv[2], pv[3], hi, lo);
+            *(uint32_t *)(phi + o1) = hi;
+            *(uint32_t *)(plo + o1) = lo;
+            r0s += pv[0] + pv[1];
+            r1s += pv[2] + pv[3];
+        }
+#pragma unroll
+        for (int o = 1; o <= 2; o <<= 1) {
+            r0s += __shfl_xor_sync(0xFFFFFFFFu, r0s, o);
+            r1s += __shfl_xor_sync(0xFFFFFFFFu, r1s, o);
+        }
+        if (t4 == 0) { red_sum[warp][g4] = r0s; red_sum[warp][g4 + 8] = r1s; }
+        __syncthreads();
+        if (tid < 16) {
+            float mx = s_m[tid], sum = 0.f;
+            for (int w = 0; w < kFusedThreads / 32; ++w) {
+                mx = fmaxf(mx, red_max[w][tid]);
+                sum += red_sum[w][tid];
+            }
+            const float alpha = s_m[tid] == -INFINITY ? 0.f : expf(s_m[tid] - mx);
+            s_alpha[tid] = alpha;
+            s_l[tid] = s_l[tid] * alpha + sum;
+            s_m[tid] = mx;
+        }
+        __syncthreads();
+        // O tile of this warp: dims 8w .. 8w+7 (warps past D/8 idle)
+        if (warp < D / 8) {
+            const float al0 = s_alpha[g4], al1 = s_alpha[g4 + 8];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                oq4[c][0] *= al0;
+                oq4[c][1] *= al0;
+                oq4[c][2] *= al1;
+                oq4[c][3] *= al1;
+            }
+#pragma unroll
+            for (int kk = 0; kk < C / 16; kk += 2) {
+                uint32_t b0, b1, b2, b3, a0, a1, a2, a3;
+                {
+                    const int key = kk * 16 + lane;
+                    ldsm_x4_t(sa(vb) + (warp >> 3) * kBox + key * 128 + (((warp & 7) ^ (key & 7)) << 4), b0, b1,
+                              b2, b3);
+                }
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int k16 = kk + u;
+                    const int prow = (lane & 7) + ((lane >> 3) & 1) * 8, pslot = 2 * k16 + (lane >> 4);
+                    const uint32_t pofs = (uint32_t)(prow * kMmaPS + swz(prow, pslot) * 8);
+                    const uint32_t bb0 = u ? b2 : b0, bb1 = u ? b3 : b1;
+                    ldsm_x4(sa(phi + pofs), a0, a1, a2, a3);
+                    mma16816(oq4[2 * u], a0, a1, a2, a3, bb0, bb1);
+                    ldsm_x4(sa(plo + pofs), a0, a1, a2, a3);
+                    mma16816(oq4[2 * u + 1], a0, a1, a2, a3, bb0, bb1);
+                }
+            }
+        }
+        __syncthreads();                              // buffer bi, p tiles free
+        if (tid == 0 && ci + 2 < nch && !dead) load(ci + 2);
+    }
+    // after a timeout, copies issued but never waited for land before exit
+    if (dead && tid == 0) {
+        for (long it = 0; it < kAttnWaitLimit && n_iss0 > 0 && !fa_try(&full[0], (uint32_t)((n_iss0 - 1) & 1)); ++it) {}
+        for (long it = 0; it < kAttnWaitLimit && n_iss1 > 0 && !fa_try(&full[1], (uint32_t)((n_iss1 - 1) & 1)); ++it) {}
+    }
+
+    // publish this rank's partial, then merge across the cluster
+    if (warp < D / 8) {
+        float oacc[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) oacc[q] = (oq4[0][q] + oq4[1][q]) + (oq4[2][q] + oq4[3][q]);
+        const int d0 = warp * 8 + 2 * t4;
+        if (g4 < G) { po[g4 * D + d0] = oacc[0]; po[g4 * D + d0 + 1] = oacc[1]; }
+        if (g4 + 8 < G) { po[(g4 + 8) * D + d0] = oacc[2]; po[(g4 + 8) * D + d0 + 1] = oacc[3]; }
+    }
+    if (tid < 16) { pm[tid] = s_m[tid]; pl[tid] = s_l[tid]; }
+    cluster_sync_all();
+    {
+        const int n_out = G * D;
+        const int e0 = (int)((long)r * n_out / CS), e1 = (int)((long)(r + 1) * n_out / CS);
+        for (int e = e0 + tid; e < e1; e += kFusedThreads) {
+            const int h = e / D;
+            float mq[kMaxCluster], lq[kMaxCluster], oq[kMaxCluster];
+#pragma unroll
+            for (int q = 0; q < kMaxCluster; ++q) {
+                if (q < CS) {
+                    mq[q] = dsmem_ld(pm + h, (uint32_t)q);
+                    lq[q] = dsmem_ld(pl + h, (uint32_t)q);
+                    oq[q] = dsmem_ld(po + e, (uint32_t)q);
+                } else {
+                    mq[q] = -INFINITY;
+                    lq[q] = oq[q] = 0.f;
+                }
+            }
+            float M = -INFINITY;
+#pragma unroll
+            for (int q = 0; q < kMaxCluster; ++q) M = fmaxf(M, mq[q]);
+            float num = 0.f, den = 0.f;
+#pragma unroll
+            for (int q = 0; q < kMaxCluster; ++q) {
+                const float w = mq[q] == -INFINITY ? 0.f : expf(mq[q] - M);
+                den = fmaf(w, lq[q], den);
+                num = fmaf(w, oq[q], num);
+            }
+            uint16_t *o = (uint16_t *)a.o_out + (size_t)b * a.Hq * D + (size_t)g * G * D;
+            o[e] = f32_to_bf16(den > 0.f ? num / den : 0.f);
+        }
+    }
+    cluster_sync_all();
+}
+
+template <int D>
+size_t fused_mma_smem() {
+    return 1024 + (size_t)4 * kMmaC * D * 2 + (size_t)2 * 16 * D * 2 + (size_t)2 * 16 * kMmaPS * 2 +
+           (size_t)2 * 16 * D * 4 + 32 * 4;
+}
+
+template <typename WT, int D>
+size_t fused_smem(int G) {
+    using Cf = FusedCfg<WT, D>;
+    return (size_t)4 * Cf::C * D * sizeof(WT) + (size_t)G * D * 4 * 2 + (size_t)G * Cf::C * 4 + 32 * 4;
+}
+static_assert(kFusedThreads % 128 == 0, "score pass maps threads to (key, head group)");
+
+template <typename Kern, typename... Args>
+cudaError_t launch_cluster(Kern k, size_t smem, const FusedAttnArgs &a, cudaStream_t s, bool pdl, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(a.cs, a.Hkv, a.B);
+    cfg.blockDim = dim3(kFusedThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = a.cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 2 : 1;
+    return cudaLaunchKernelEx(&cfg, k, args...);
+}
+
+template <typename WT, int D>
+cudaError_t launch_fused_t(const FusedAttnArgs &a, cudaStream_t s, bool pdl, const CUtensorMap *tk,
+                           const CUtensorMap *tv) {
+    if constexpr (sizeof(WT) == 2) {
+        if (tk && tv) return launch_cluster(fused_attention_mma_kernel<D>, fused_mma_smem<D>(), a, s, pdl, a, *tk, *tv);
+    }
+    return launch_cluster(fused_attention_kernel<WT, D>, fused_smem<WT, D>(a.Hq / a.Hkv), a, s, pdl, a);
+}
+
+// Clusters of 16 are a non-portable size: allowed only where the occupancy
+// query confirms that `need` of them can be resident at once.
+template <typename Kern>
+int max_cluster_for(Kern k, size_t smem, int need) {
+    if (cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+        cudaGetLastError();
+        return 8;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(16, 1, 1);
+    cfg.blockDim = dim3(kFusedThreads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 16;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return 8;
+    }
+    return n >= need ? 16 : 8;
+}
+
+template <typename WT, int D>
+cudaError_t prepare_fused_t(int G, int need, int *max_cs) {
+    cudaError_t e;
+    if constexpr (sizeof(WT) == 2) {
+        if (G > 16 || fused_mma_smem<D>() > (size_t)200 * 1024) return cudaErrorInvalidValue;
+        e = cudaFuncSetAttribute(fused_attention_mma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 200 * 1024);
+        if (e == cudaSuccess && max_cs) *max_cs = max_cluster_for(fused_attention_mma_kernel<D>, fused_mma_smem<D>(), need);
+    } else {
+        if (G > 16 || fused_smem<WT, D>(G) > (size_t)200 * 1024) return cudaErrorInvalidValue;
+        e = cudaFuncSetAttribute(fused_attention_kernel<WT, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 200 * 1024);
+        if (e == cudaSuccess && max_cs) *max_cs = max_cluster_for(fused_attention_kernel<WT, D>, fused_smem<WT, D>(G), need);
+    }
+    return e;
+}
+
 template <typename WT, int D>
 size_t attn_smem(int chunk, int G, int splits) {
     constexpr int RS = D + Elem<WT>::kPerVec;
@@ -360,6 +1147,28 @@ cudaError_t prepare_attention_kernel(bool bf16, int D, int chunk, int G, int spl
 size_t attention_smem_bytes(bool bf16, int D, int chunk, int G, int splits) {
     if (bf16) return D == 64 ? attn_smem<uint16_t, 64>(chunk, G, splits) : attn_smem<uint16_t, 128>(chunk, G, splits);
     return D == 64 ? attn_smem<float, 64>(chunk, G, splits) : attn_smem<float, 128>(chunk, G, splits);
+}
+
+int fused_attention_chunk() { return kMmaC; }
+
+cudaError_t launch_fused_attention(const FusedAttnArgs &a, bool bf16, cudaStream_t s, bool pdl,
+                                   const CUtensorMap *tk, const CUtensorMap *tv) {
+    if (a.cs < 1 || a.cs > kMaxCluster || a.Hq / a.Hkv > 16) return cudaErrorInvalidValue;
+    if (bf16)
+        return a.D == 64 ? launch_fused_t<uint16_t, 64>(a, s, pdl, tk, tv)
+                         : launch_fused_t<uint16_t, 128>(a, s, pdl, tk, tv);
+    return a.D == 64 ? launch_fused_t<float, 64>(a, s, pdl, nullptr, nullptr)
+                     : launch_fused_t<float, 128>(a, s, pdl, nullptr, nullptr);
+}
+
+cudaError_t prepare_fused_attention(bool bf16, int D, int G, int need, int *max_cs) {
+    if (bf16) return D == 64 ? prepare_fused_t<uint16_t, 64>(G, need, max_cs) : prepare_fused_t<uint16_t, 128>(G, need, max_cs);
+    return D == 64 ? prepare_fused_t<float, 64>(G, need, max_cs) : prepare_fused_t<float, 128>(G, need, max_cs);
+}
+
+size_t fused_attention_smem_bytes(bool bf16, int D, int G) {
+    if (bf16) return D == 64 ? fused_mma_smem<64>() : fused_mma_smem<128>();
+    return D == 64 ? fused_smem<float, 64>(G) : fused_smem<float, 128>(G);
 }
 
 cudaError_t launch_accept(const AcceptArgs &a, cudaStream_t s) {

@@ -202,6 +202,18 @@ struct AttnArgs {
     int *err;
 };
 
+// Fused RoPE + KV append + attention (one cluster of `cs` CTAs per sequence
+// and KV head).
+struct FusedAttnArgs {
+    const float *qkv;                  // [rows, (Hq + 2Hkv) D]
+    void *k_cache, *v_cache;           // [B, Hkv, max_ctx, D]
+    void *o_out;                       // [B, Hq * D] wtype
+    const float *rope_cos, *rope_sin;  // [max_ctx, D/2]
+    const int32_t *n_new, *kv_len;
+    int B, max_new, prefill, step, Hq, Hkv, D, max_ctx, cs;
+    int *err;
+};
+
 struct AcceptArgs {
     const int32_t *draft, *target, *n_new;
     int32_t *kv_len, *accept_len, *out_tokens;
@@ -235,6 +247,19 @@ int gemv_tc_tiles(const GemvArgs &a);
 cudaError_t launch_gemv_tc(const GemvArgs &a, const CUtensorMap &m, int sms, float *part, int *tile_ctr,
                            cudaStream_t s, bool pdl);
 cudaError_t prepare_attention_kernel(bool bf16, int D, int chunk, int G, int splits);
+// Sets kernel attributes; *max_cs receives the largest cluster size (8 or 16)
+// for which `need` clusters can be resident at once.
+cudaError_t prepare_fused_attention(bool bf16, int D, int G, int need, int *max_cs);
+size_t fused_attention_smem_bytes(bool bf16, int D, int G);
+// K or V cache [heads, max_ctx, D] bf16 as a TMA tensor map of
+// rows_per_box x 64-column boxes in the 128-byte swizzle (D a multiple of 64).
+cudaError_t make_cache_map(CUtensorMap *m, const void *cache, int heads, int max_ctx, int D, int rows_per_box);
+// Keys per chunk of the tensor-core attention kernel (the box height it needs).
+int fused_attention_chunk();
+// tk / tv: cache tensor maps; the bf16 tensor-core kernel runs when both are
+// given, the CUDA-core kernel otherwise.
+cudaError_t launch_fused_attention(const FusedAttnArgs &a, bool bf16, cudaStream_t s, bool pdl,
+                                   const CUtensorMap *tk, const CUtensorMap *tv);
 size_t attention_smem_bytes(bool bf16, int D, int chunk, int G, int splits);
 
 // Launch with optional programmatic stream serialization.

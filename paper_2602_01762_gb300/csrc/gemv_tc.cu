@@ -781,6 +781,20 @@ cudaError_t make_weight_map(CUtensorMap *m, const void *W, int rows, int kin) {
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+cudaError_t make_cache_map(CUtensorMap *m, const void *cache, int heads, int max_ctx, int D, int rows_per_box) {
+    if (!g_encode) return cudaErrorNotSupported;
+    if (((uintptr_t)cache & 15) || (D % 64) || heads < 1 || max_ctx < 1 || rows_per_box < 1 || rows_per_box > 256)
+        return cudaErrorInvalidValue;
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)max_ctx, (cuuint64_t)heads};
+    cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)max_ctx * D * 2};
+    cuuint32_t box[3] = {64, (cuuint32_t)rows_per_box, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(cache), dims, strides, box,
+                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 bool gemv_tc_supported(const GemvArgs &a, int sms) {
     TcPlan p{};
     int grid;

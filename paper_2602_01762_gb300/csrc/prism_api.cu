@@ -70,6 +70,8 @@ struct prism_ctx {
     int gemv_chunk = 0, gemv_smem = 0, gemv_groups = 0;   // projection ring knobs (0 = built-in default)
     int gemv_cuda_core = 1;                               // 1: bf16 projections on CUDA cores
     int gemv_tcgen05 = 1;                                 // 1: bf16 projections on tcgen05 where they fit
+    int attn_fused = 1;                                   // 1: fused RoPE/append/attention cluster kernel
+    int attn_max_cs = 8;                                  // largest cluster the device co-schedules
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
     bool tc_ready = false;
     CUtensorMap tm_lm;
@@ -180,6 +182,12 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         return launch_gemv(g, c->bf16, grid, s, pdl_here);
     };
 
+    // the caches as TMA tensor maps for the tensor-core attention kernel
+    CUtensorMap tmk, tmv;
+    const bool cache_maps = c->attn_fused && c->bf16 && c->tc_ready &&
+                            make_cache_map(&tmk, r.k_cache, r.B * Hkv, f.max_ctx, D, fused_attention_chunk()) == cudaSuccess &&
+                            make_cache_map(&tmv, r.v_cache, r.B * Hkv, f.max_ctx, D, fused_attention_chunk()) == cudaSuccess;
+
     for (int k = 1; k <= K && e == cudaSuccess; ++k) {
         const prism_step_weights &w = c->steps[k - 1];
         const CUtensorMap *tms = c->tm_step_ok[k - 1] ? c->tm_step[k - 1] : nullptr;
@@ -220,6 +228,32 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         after(1);
         if (e != cudaSuccess) break;
 
+        if (c->attn_fused) {
+            // RoPE + KV append + attention in one cluster launch per (sequence, KV head)
+            FusedAttnArgs fa{};
+            fa.qkv = c->qkv;
+            fa.k_cache = r.k_cache;
+            fa.v_cache = r.v_cache;
+            fa.o_out = c->o_buf;
+            fa.rope_cos = c->rope_cos;
+            fa.rope_sin = c->rope_sin;
+            fa.n_new = r.n_new;
+            fa.kv_len = r.kv_len;
+            fa.B = r.B;
+            fa.max_new = f.max_new;
+            fa.prefill = prefill;
+            fa.step = k;
+            fa.Hq = Hq;
+            fa.Hkv = Hkv;
+            fa.D = D;
+            fa.max_ctx = f.max_ctx;
+            fa.cs = c->attn_max_cs;
+            while (fa.cs > 1 && (long long)r.B * Hkv * fa.cs > 2LL * c->sms) fa.cs /= 2;
+            fa.err = c->err;
+            e = launch_fused_attention(fa, c->bf16, s, pdl, cache_maps ? &tmk : nullptr, cache_maps ? &tmv : nullptr);
+            after(3);
+            if (e != cudaSuccess) break;
+        } else {
         // RoPE + KV append (+ rotated q of the query rows)
         RopeArgs ra{};
         ra.qkv = c->qkv;
@@ -269,6 +303,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         e = launch_attention(aa, c->bf16, s, pdl);
         after(3);
         if (e != cudaSuccess) break;
+        }
 
         // O projection + residual
         g = base;
@@ -510,6 +545,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         return fail(nullptr, PRISM_ERR_INVALID_ARG, "max_ctx too large for the attention combine");
     }
     if (e == cudaSuccess) e = prepare_attention_kernel(c->bf16, D, c->attn_chunk, Hq / Hkv, c->attn_splits);
+    if (e == cudaSuccess) e = prepare_fused_attention(c->bf16, D, Hq / Hkv, Hkv, &c->attn_max_cs);
     if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking);
     if (e != cudaSuccess) {
         prism_status st = cuda_fail(nullptr, e, "context setup");
@@ -577,6 +613,7 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
                                                    value == 8 || value == 16)) c->gemv_groups = value;
     else if (!std::strcmp(name, "gemv_cuda_core")) c->gemv_cuda_core = value != 0;
     else if (!std::strcmp(name, "gemv_tcgen05")) c->gemv_tcgen05 = value != 0;
+    else if (!std::strcmp(name, "attn_fused")) c->attn_fused = value != 0;
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);
     return PRISM_OK;

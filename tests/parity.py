@@ -85,7 +85,9 @@ def compare_round(gpu: dict, orc: dict, inputs: dict, seqs, K: int, topk: int, *
                 gaps = -np.diff(o_top)           # gaps[r] = top[r] - top[r+1]
                 for r in range(topk):
                     lo = gaps[r - 1] if r > 0 else np.inf
-                    hi = gaps[r] if r < len(gaps) else np.inf
+                    # without the oracle's next candidate the gap below rank r is
+                    # unknown, so that rank cannot qualify
+                    hi = gaps[r] if r < len(gaps) else 0.0
                     if min(lo, hi) > thr:
                         assert gpu["topk_ids"][b, k, r] == orc["topk_ids"][j, k, r], (
                             f"seq {b} step {k + 1}: top-{r + 1} id differs")

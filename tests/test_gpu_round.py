@@ -42,7 +42,9 @@ def _check(w, W, I, seqs, *, topk, options=None):
     try:
         g = gpu_round(w, W, I, topk=topk, model=model, options=options)
         assert g["flags"] == 0, f"device error word {g['flags']}"
-        o = oracle.draft_round(w.shape, W, I, topk=max(2, topk), want_logits=True, seqs=seqs)
+        # one candidate more than is compared: the margin of the last compared
+        # rank is its gap to the next one
+        o = oracle.draft_round(w.shape, W, I, topk=topk + 1, want_logits=True, seqs=seqs)
         rep = compare_round(g, o, I, seqs, K, topk, chain=True)
         compare_cache(g["k_cache"], g["v_cache"], o["k_cache"], o["v_cache"], I, seqs, K)
         forced = {}
@@ -131,6 +133,22 @@ def test_tcgen05_projection_path_matches_oracle(case):
         seqs = [0]
     _, _, rep = _check(w, W, I, seqs, topk=8, options=TCGEN05)
     print(case, rep)
+    assert rep["ids_compared"] >= 1
+
+
+@pytest.mark.parametrize("case", ["tiny-bf16", "tiny-f32", "mid"])
+def test_split_attention_path_matches_oracle(case):
+    """Attention as two kernels (RoPE/append, then split-KV attention with a
+    last-CTA combine) instead of the fused cluster kernel."""
+    if case == "mid":
+        w = MID_W
+        W, I = mid_case()
+        seqs = [0, 1, 2]
+    else:
+        w = synth.WORKLOADS[case]
+        W, I = synth.make_weights(w), synth.make_round_inputs(w)
+        seqs = [0]
+    _, _, rep = _check(w, W, I, seqs, topk=4, options={"attn_fused": 0})
     assert rep["ids_compared"] >= 1
 
 
