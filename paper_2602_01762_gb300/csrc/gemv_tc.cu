@@ -312,16 +312,20 @@ __device__ void stage_x_tc(const GemvArgs &a, int kb0, int kb1, uint8_t *X, floa
     }
 }
 
-// Top 8 under `better` of candidates spread over a warp: kRounds rounds of a
-// warp-wide argmax over the lanes' best remaining candidate; the winning lane
+// Top `rounds` (<= 8) under `better` of candidates spread over a warp: one
+// warp-wide argmax per rank over the lanes' best remaining candidate; the winning lane
 // retires it.  Each lane holds C candidates (cv, ci); ties between equal
 // entries break by lane, so the winner is warp-uniform.  The result goes to
 // out_v/out_i (written by lane 0).  Compact code on purpose: it runs cold.
 template <int C>
-__device__ void warp_top8(float (&cv)[C], int (&ci)[C], float *out_v, int *out_i) {
+__device__ void warp_top8(float (&cv)[C], int (&ci)[C], float *out_v, int *out_i, int rounds) {
     const int lane = threadIdx.x & 31;
+    // only the ranks the caller keeps are selected; the rest of the list is
+    // filled with sentinels (below every candidate under `better`)
+    if (lane == 0)
+        for (int r = rounds; r < kTopK; ++r) { out_v[r] = -INFINITY; out_i[r] = 0x7FFFFFFF; }
 #pragma unroll 1
-    for (int r = 0; r < kTopK; ++r) {
+    for (int r = 0; r < rounds; ++r) {
         float bv = cv[0];
         int bi = ci[0], bs = 0;
 #pragma unroll
@@ -556,10 +560,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             const float zv = __shfl_sync(0xFFFFFFFFu, z, src);
                             const int uv = __shfl_sync(0xFFFFFFFFu, u, src);
                             if (!better(zv, uv, thr_v[t], thr_i[t])) continue;
+                            // a list of the a.topk best (the rest of it stays at sentinels)
                             if (lane == 0) {
                                 float *lv = s_val[ew][t];
                                 int *li = s_id[ew][t];
-                                int pos = kTopK - 1;
+                                int pos = a.topk - 1;
                                 while (pos > 0 && better(zv, uv, lv[pos - 1], li[pos - 1])) {
                                     lv[pos] = lv[pos - 1];
                                     li[pos] = li[pos - 1];
@@ -569,8 +574,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                 li[pos] = uv;
                             }
                             __syncwarp();
-                            thr_v[t] = s_val[ew][t][kTopK - 1];
-                            thr_i[t] = s_id[ew][t][kTopK - 1];
+                            thr_v[t] = s_val[ew][t][a.topk - 1];
+                            thr_i[t] = s_id[ew][t][a.topk - 1];
                             __syncwarp();
                         }
                     }
@@ -621,7 +626,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     float cv[1] = {s_val[lane / kTopK][t][lane % kTopK]};
                     int ci[1] = {s_id[lane / kTopK][t][lane % kTopK]};
                     const size_t o = ((size_t)t * gridDim.x + blockIdx.x) * kTopK;
-                    warp_top8<1>(cv, ci, a.lm_part + o, a.lm_part_id + o);
+                    warp_top8<1>(cv, ci, a.lm_part + o, a.lm_part_id + o, a.topk);
                 }
                 __threadfence();
                 epi_sync();
@@ -646,12 +651,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             cv[u] = c < hi ? __ldcg(a.lm_part + b0 + c) : -INFINITY;
                             ci[u] = c < hi ? __ldcg(a.lm_part_id + b0 + c) : 0x7FFFFFFF;
                         }
-                        warp_top8<kC>(cv, ci, s_val[ew][0], s_id[ew][0]);
+                        warp_top8<kC>(cv, ci, s_val[ew][0], s_id[ew][0], a.topk);
                         epi_sync();
                         if (ew == 0) {
                             float fv[1] = {s_val[lane / kTopK][0][lane % kTopK]};
                             int fi[1] = {s_id[lane / kTopK][0][lane % kTopK]};
-                            warp_top8<1>(fv, fi, s_fin_v, s_fin_i);
+                            warp_top8<1>(fv, fi, s_fin_v, s_fin_i, a.topk);
                             __syncwarp();
                             if (lane < a.topk) {
                                 const size_t o = (size_t)t * a.K + a.step - 1;
