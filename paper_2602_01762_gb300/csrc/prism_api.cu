@@ -172,8 +172,12 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
 
     // a projection on the tensor-core kernel when enabled and it fits, else on
     // the CUDA-core ring kernel
+    // (gate/up + SwiGLU stays on the CUDA-core kernel unless gemv_tcgen05 = 2:
+    // with 112 unit tiles it needs split-K on the tensor-core kernel, and
+    // measured slower there)
     auto proj = [&](const GemvArgs &g, const CUtensorMap *tm, int grid, bool pdl_here) -> cudaError_t {
-        if (tm && c->gemv_tcgen05 && c->tc_ready && c->bf16 && gemv_tc_supported(g, c->sms)) {
+        const bool want = c->gemv_tcgen05 == 2 || (c->gemv_tcgen05 == 1 && g.epi != kEpiSwiGLU);
+        if (tm && want && c->tc_ready && c->bf16 && gemv_tc_supported(g, c->sms)) {
             // split-K launches need the partial-sum workspace and one ticket per tile
             const size_t ws = gemv_tc_workspace_floats(g, c->sms);
             if (ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n))
@@ -444,12 +448,14 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         const int units[] = {d, c->qkv_rows, d, F, d};
         const int kins[] = {2 * d, d, Hq * D, d, F};
         const int epis[] = {kEpiStore, kEpiStore, kEpiResid, kEpiSwiGLU, kEpiResid};
+        const int pros[] = {kProFuseDecode, kProNorm, kProCopy, kProNorm, kProCopy};
         for (int i = 0; i < 5; ++i)
             for (int T : {(int)T1, (int)B}) {
                 GemvArgs g{};
                 g.n_units = units[i];
                 g.kin = kins[i];
                 g.epi = epis[i];
+                g.pro = pros[i];
                 g.T = T;
                 const size_t need = gemv_tc_workspace_floats(g, c->sms);
                 if (need > tc_floats) tc_floats = need;
@@ -612,7 +618,7 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "gemv_groups") && (value == 0 || value == 1 || value == 2 || value == 4 ||
                                                    value == 8 || value == 16)) c->gemv_groups = value;
     else if (!std::strcmp(name, "gemv_cuda_core")) c->gemv_cuda_core = value != 0;
-    else if (!std::strcmp(name, "gemv_tcgen05")) c->gemv_tcgen05 = value != 0;
+    else if (!std::strcmp(name, "gemv_tcgen05") && value >= 0 && value <= 2) c->gemv_tcgen05 = value;
     else if (!std::strcmp(name, "attn_fused")) c->attn_fused = value != 0;
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);

@@ -115,7 +115,7 @@ def test_fallback_projection_kernels_match_oracle(options):
     compare_cache(g["k_cache"], g["v_cache"], o["k_cache"], o["v_cache"], I, [0, 1, 2], MID_W.shape.n_steps)
 
 
-TCGEN05 = {"gemv_tcgen05": 1}
+TCGEN05 = {"gemv_tcgen05": 2}      # every projection, gate/up included, on the tcgen05 kernel
 
 
 @pytest.mark.parametrize("case", ["tiny-bf16", "mid"])
