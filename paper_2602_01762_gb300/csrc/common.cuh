@@ -246,6 +246,14 @@ size_t gemv_tc_workspace_floats(const GemvArgs &a, int sms);
 int gemv_tc_tiles(const GemvArgs &a);
 cudaError_t launch_gemv_tc(const GemvArgs &a, const CUtensorMap &m, int sms, float *part, int *tile_ctr,
                            cudaStream_t s, bool pdl);
+// Streamed variant for many activation rows (up to 256; 128 for SwiGLU, 64
+// for top-k): prep kernel for the activation rows (into xbuf, bf16
+// [T][kin], unless the prologue is a copy), the projection, and for top-k
+// the cross-CTA merge kernel.
+bool gemv_tcs_supported(const GemvArgs &a, int sms);
+size_t gemv_tcs_workspace_floats(const GemvArgs &a, int sms);
+cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, float *part, int *tile_ctr,
+                            uint16_t *xbuf, cudaStream_t s, bool pdl);
 cudaError_t prepare_attention_kernel(bool bf16, int D, int chunk, int G, int splits);
 // Sets kernel attributes; *max_cs receives the largest cluster size (8 or 16)
 // for which `need` clusters can be resident at once.

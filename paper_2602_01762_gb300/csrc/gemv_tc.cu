@@ -27,6 +27,7 @@
 //   * every wait is bounded; on expiry the kernel sets the timeout bit of the
 //     device error word, stops waiting, drains its copies and MMAs, frees its
 //     tensor memory and returns.
+#include <algorithm>
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -681,6 +682,378 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols));
 }
 
+// ------------------------------------------------------------------ streamed
+// Variant for many activation rows (T > 16): the B operand is not staged
+// whole but streams through the ring next to W.  Each stage holds, per K
+// block, the RPW boxes of W and one box of the activation rows X (NB rows x
+// 64 columns, the same 128-byte swizzle), fetched by TMA from a bf16 X
+// buffer that a prep kernel (or the previous projection, for the copy
+// prologue) has written.  MMA N = NB (16 .. 256); rows of X past T arrive as
+// zeros.  The epilogue reads the NB accumulator columns 16 at a time.  With
+// top-k, the per-row merge across CTAs is left to topk_merge_kernel.
+template <int NB, int RPW, bool TOPK>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    gemv_tcs_kernel(const GemvArgs a, const TcPlan p, const __grid_constant__ CUtensorMap tmW,
+                    const __grid_constant__ CUtensorMap tmX) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full[kTcMaxStages], empty[kTcMaxStages], acc_full[2], acc_empty[2], mma_done;
+    __shared__ uint32_t s_tmem;
+    __shared__ float s_val[TOPK ? 4 : 1][TOPK ? NB : 1][kTopK];
+    __shared__ int s_id[TOPK ? 4 : 1][TOPK ? NB : 1][kTopK];
+    __shared__ int s_last;
+    constexpr uint32_t kXBox = NB * 128;                              // one X box
+    constexpr uint32_t kColsNeed = 2 * RPW * NB;
+    constexpr uint32_t kCols = kColsNeed <= 32 ? 32 : kColsNeed <= 64 ? 64 : kColsNeed <= 128 ? 128
+                               : kColsNeed <= 256 ? 256 : 512;
+    static_assert(kColsNeed <= 512, "accumulators exceed tensor memory");
+    constexpr uint32_t kIdescN = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(NB >> 3) << 17) |
+                                 ((uint32_t)(kTileM >> 4) << 24);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint8_t *ring = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const int S = p.stages;
+    const uint32_t kb_bytes = RPW * kBoxBytes + kXBox;                // one K block in a stage
+    const int ks = blockIdx.x % p.splits;
+    const int tiles_step = gridDim.x / p.splits;
+    const int kb0 = (int)((long)ks * p.nkb / p.splits), kb1 = (int)((long)(ks + 1) * p.nkb / p.splits);
+    const int n_kst = (kb1 - kb0 + p.kb_per_stage - 1) / p.kb_per_stage;
+    int my_tiles = 0;
+    for (int tile = blockIdx.x / p.splits; tile < p.n_tiles; tile += tiles_step) ++my_tiles;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&acc_full[i], 1);
+            mbar_init(&acc_empty[i], 4);
+        }
+        mbar_init(&mma_done, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmW) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmX) : "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(&s_tmem)),
+                     "r"(kCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+    pdl_trigger();
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            int s = 0, issued = 0;
+            uint32_t ph = 0;
+            bool dead = false;
+            bool x_ready = false;      // X is the previous kernel's output: wait before the first X box
+            for (int i = 0; i < my_tiles && !dead; ++i) {
+                const int tile = blockIdx.x / p.splits + i * tiles_step;
+                for (int q = 0; q < n_kst; ++q) {
+                    if (!mbar_wait(&empty[s], ph ^ 1)) {
+                        set_err(a.err, kErrTimeout);
+                        dead = true;
+                        break;
+                    }
+                    if (!x_ready) {
+                        pdl_wait();
+                        x_ready = true;
+                    }
+                    const int kbs = kb0 + q * p.kb_per_stage;
+                    const int nkb = kb1 - kbs < p.kb_per_stage ? kb1 - kbs : p.kb_per_stage;
+                    mbar_arrive_tx(&full[s], (uint32_t)nkb * kb_bytes);
+                    const uint32_t st = saddr(ring) + (uint32_t)s * p.stage_bytes;
+                    for (int j = 0; j < nkb; ++j) {
+#pragma unroll
+                        for (int r = 0; r < RPW; ++r)
+                            tma_load_2d(st + (uint32_t)j * kb_bytes + (uint32_t)r * kBoxBytes, &tmW, (kbs + j) * kBoxK,
+                                        tile * kTileM + r * a.pair_offset, &full[s]);
+                        tma_load_2d(st + (uint32_t)j * kb_bytes + RPW * kBoxBytes, &tmX, (kbs + j) * kBoxK, 0,
+                                    &full[s]);
+                    }
+                    ++issued;
+                    if (++s == S) { s = 0; ph ^= 1; }
+                }
+            }
+            const int first = issued > S ? issued - S : 0;
+            for (int i = first; i < issued; ++i)
+                if (!mbar_wait(&full[i % S], (uint32_t)((i / S) & 1))) set_err(a.err, kErrTimeout);
+        }
+    } else {
+        pdl_wait();
+        if (warp == 1) {
+            // ------------------------------------------------------------ MMA
+            if (lane == 0) {
+                int s = 0;
+                uint32_t ph = 0;
+                bool dead = false;
+                for (int i = 0; i < my_tiles && !dead; ++i) {
+                    const int ab = i & 1;
+                    if (!mbar_wait(&acc_empty[ab], ((i >> 1) & 1) ^ 1)) {
+                        set_err(a.err, kErrTimeout);
+                        dead = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    for (int q = 0; q < n_kst; ++q) {
+                        if (!mbar_wait(&full[s], ph)) {
+                            set_err(a.err, kErrTimeout);
+                            dead = true;
+                            break;
+                        }
+                        tc_fence_after();
+                        const int kbs = kb0 + q * p.kb_per_stage;
+                        const int nkb = kb1 - kbs < p.kb_per_stage ? kb1 - kbs : p.kb_per_stage;
+                        const uint32_t st = saddr(ring) + (uint32_t)s * p.stage_bytes;
+                        for (int j = 0; j < nkb; ++j) {
+                            const uint32_t xa = st + (uint32_t)j * kb_bytes + RPW * kBoxBytes;
+#pragma unroll
+                            for (int kk = 0; kk < kBoxK / 16; ++kk) {
+                                const uint64_t bd = sw128_desc(xa + kk * 32, 1024);
+#pragma unroll
+                                for (int r = 0; r < RPW; ++r) {
+                                    const uint64_t ad =
+                                        sw128_desc(st + (uint32_t)j * kb_bytes + (uint32_t)r * kBoxBytes + kk * 32, 1024);
+                                    const uint32_t acc = (q | j | kk) != 0 ? 1u : 0u;
+                                    asm volatile(
+                                        "{\n\t.reg .pred pp;\n\tsetp.ne.b32 pp, %4, 0;\n\t"
+                                        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, pp;\n\t}"
+                                        ::"r"(tmem + (uint32_t)((ab * RPW + r) * NB)), "l"(ad), "l"(bd),
+                                        "r"(kIdescN), "r"(acc));
+                                }
+                            }
+                        }
+                        mma_commit(&empty[s]);
+                        if (++s == S) { s = 0; ph ^= 1; }
+                    }
+                    if (!dead) mma_commit(&acc_full[ab]);
+                }
+                mma_commit(&mma_done);
+                if (!mbar_wait(&mma_done, 0)) set_err(a.err, kErrTimeout);
+            }
+            __syncwarp();
+        } else {
+            // ------------------------------------------------------------ epilogue
+            const int ew = warp - 2;
+            const int quarter = warp & 3;
+            const int row = quarter * 32 + lane;
+            const int T = a.T;
+            if constexpr (TOPK) {
+                for (int t = lane; t < NB; t += 32)
+#pragma unroll
+                    for (int i = 0; i < kTopK; ++i) { s_val[ew][t][i] = -INFINITY; s_id[ew][t][i] = 0x7FFFFFFF; }
+                __syncwarp();
+            }
+            bool dead = false;
+            for (int i = 0; i < my_tiles; ++i) {
+                const int tile = blockIdx.x / p.splits + i * tiles_step;
+                const int ab = i & 1;
+                if (!dead && !mbar_wait_warp(&acc_full[ab], (i >> 1) & 1)) {
+                    if (lane == 0) set_err(a.err, kErrTimeout);
+                    dead = true;
+                }
+                const int u = tile * kTileM + row;
+                const bool valid = !dead && u < a.n_units;
+                // accumulator columns 16 at a time (all RPW sets of one chunk together)
+                for (int c0 = 0; c0 < NB; c0 += 16) {
+                    float acc[RPW][16];
+                    if (!dead) {
+                        tc_fence_after();
+#pragma unroll
+                        for (int r = 0; r < RPW; ++r)
+                            tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((ab * RPW + r) * NB + c0),
+                                      acc[r]);
+                    }
+                    if (c0 >= T) continue;
+                    if constexpr (TOPK) {
+#pragma unroll
+                        for (int tt = 0; tt < 16; ++tt) {
+                            const int t = c0 + tt;
+                            if (t >= T) break;
+                            const float z = dead ? -INFINITY : acc[0][tt];
+                            if (valid && a.logits) a.logits[((size_t)t * a.K + a.step - 1) * a.vocab + u] = z;
+                            const float thv = s_val[ew][t][a.topk - 1];
+                            const int thi = s_id[ew][t][a.topk - 1];
+                            unsigned m = __ballot_sync(0xFFFFFFFFu, valid && better(z, u, thv, thi));
+                            while (m) {
+                                const int src = __ffs(m) - 1;
+                                m &= m - 1;
+                                const float zv = __shfl_sync(0xFFFFFFFFu, z, src);
+                                const int uv = __shfl_sync(0xFFFFFFFFu, u, src);
+                                if (lane == 0) {
+                                    float *lv = s_val[ew][t];
+                                    int *li = s_id[ew][t];
+                                    if (better(zv, uv, lv[a.topk - 1], li[a.topk - 1])) {
+                                        int pos = a.topk - 1;
+                                        while (pos > 0 && better(zv, uv, lv[pos - 1], li[pos - 1])) {
+                                            lv[pos] = lv[pos - 1];
+                                            li[pos] = li[pos - 1];
+                                            --pos;
+                                        }
+                                        lv[pos] = zv;
+                                        li[pos] = uv;
+                                    }
+                                }
+                                __syncwarp();
+                            }
+                        }
+                    } else if (p.splits == 1) {
+                        if (valid) {
+#pragma unroll
+                            for (int tt = 0; tt < 16; ++tt) {
+                                if (c0 + tt >= T) break;
+                                finish_unit<RPW>(a, c0 + tt, u, acc[0][tt], acc[RPW - 1][tt]);
+                            }
+                        }
+                    } else if (valid) {
+#pragma unroll
+                        for (int r = 0; r < RPW; ++r)
+#pragma unroll
+                            for (int tt = 0; tt < 16; ++tt) {
+                                if (c0 + tt >= T) break;
+                                p.part[(((size_t)ks * RPW + r) * T + c0 + tt) * a.n_units + u] = acc[r][tt];
+                            }
+                    }
+                }
+                if (!dead) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&acc_empty[ab]);
+                }
+                if constexpr (!TOPK) {
+                    if (p.splits > 1) {
+                        __threadfence();
+                        epi_sync();
+                        if (threadIdx.x == 64) s_last = atomicAdd(&p.tile_ctr[tile], 1) == p.splits - 1;
+                        epi_sync();
+                        if (s_last) {
+                            __threadfence();
+                            if (valid) {
+                                for (int t = 0; t < T; ++t) {
+                                    float v0 = 0.f, v1 = 0.f;
+                                    for (int k2 = 0; k2 < p.splits; ++k2) {
+                                        v0 += __ldcg(&p.part[(((size_t)k2 * RPW + 0) * T + t) * a.n_units + u]);
+                                        if (RPW == 2) v1 += __ldcg(&p.part[(((size_t)k2 * RPW + 1) * T + t) * a.n_units + u]);
+                                    }
+                                    finish_unit<RPW>(a, t, u, v0, v1);
+                                }
+                            }
+                            if (threadIdx.x == 64) p.tile_ctr[tile] = 0;
+                        }
+                        epi_sync();
+                    }
+                }
+            }
+            if constexpr (TOPK) {
+                // this CTA's top-k of every row; the cross-CTA merge is a separate kernel
+                epi_sync();
+                for (int t = ew; t < T; t += 4) {
+                    float cv[1] = {s_val[lane / kTopK][t][lane % kTopK]};
+                    int ci[1] = {s_id[lane / kTopK][t][lane % kTopK]};
+                    const size_t o = ((size_t)t * gridDim.x + blockIdx.x) * kTopK;
+                    warp_top8<1>(cv, ci, a.lm_part + o, a.lm_part_id + o, a.topk);
+                }
+            }
+        }
+    }
+
+    if (warp == 0) return;
+    tc_fence_before();
+    stage_sync();
+    tc_fence_after();
+    if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols));
+}
+
+// Cross-CTA top-k merge of the streamed LM head: one CTA (4 warps) per row.
+__global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int grid) {
+    __shared__ float s_v[4][kTopK];
+    __shared__ int s_i[4][kTopK];
+    __shared__ float f_v[kTopK];
+    __shared__ int f_i[kTopK];
+    pdl_trigger();
+    pdl_wait();
+    const int t = blockIdx.x, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int kC = 16;                                        // grids up to 256 CTAs
+    const int ncand = grid * kTopK, lo = w * ncand / 4, hi = (w + 1) * ncand / 4;
+    float cv[kC];
+    int ci[kC];
+    const size_t b0 = (size_t)t * ncand;
+#pragma unroll
+    for (int u = 0; u < kC; ++u) {
+        const int c = lo + lane + 32 * u;
+        cv[u] = c < hi ? __ldcg(a.lm_part + b0 + c) : -INFINITY;
+        ci[u] = c < hi ? __ldcg(a.lm_part_id + b0 + c) : 0x7FFFFFFF;
+    }
+    warp_top8<kC>(cv, ci, s_v[w], s_i[w], a.topk);
+    __syncthreads();
+    if (w == 0) {
+        float fv[1] = {s_v[lane / kTopK][lane % kTopK]};
+        int fi[1] = {s_i[lane / kTopK][lane % kTopK]};
+        warp_top8<1>(fv, fi, f_v, f_i, a.topk);
+        __syncwarp();
+        if (lane < a.topk) {
+            const size_t o = (size_t)t * a.K + a.step - 1;
+            if (lane == 0) a.draft_out[o] = f_i[0];
+            if (a.topk_ids) a.topk_ids[o * a.topk + lane] = f_i[lane];
+            if (a.topk_logits) a.topk_logits[o * a.topk + lane] = f_v[lane];
+        }
+    }
+}
+
+// Activation rows of a projection as a bf16 buffer X [T][kin] (the streamed
+// kernel's B operand): embedding gather and concatenation, or RMSNorm with
+// its gain, rounded to bf16.  One CTA of 256 threads per row.
+__global__ void __launch_bounds__(256) prep_x_kernel(const GemvArgs a, uint16_t *X) {
+    __shared__ float red[8];
+    pdl_trigger();
+    pdl_wait();
+    const int t = blockIdx.x, tid = threadIdx.x;
+    const int d = a.d, kin = a.kin;
+    uint16_t *xr = X + (size_t)t * kin;
+    if (a.pro == kProNorm) {
+        const int sr = a.src_prefill_rows ? (t * a.max_new + clamp_n(a, t) - 1) : t;
+        const float *src = a.src + (size_t)sr * d;
+        float inv = 1.f;
+        if (a.gain) {
+            float ss = 0.f;
+            for (int c = tid; c < d; c += 256) ss = fmaf(src[c], src[c], ss);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
+            if ((tid & 31) == 0) red[tid >> 5] = ss;
+            __syncthreads();
+            float tot = 0.f;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) tot += red[i];
+            inv = 1.0f / sqrtf(tot / (float)d + a.eps);
+        }
+        const uint16_t *g = (const uint16_t *)a.gain;
+        for (int c = tid; c < d; c += 256) xr[c] = f32_to_bf16(a.gain ? src[c] * inv * bf16_to_f32(g[c]) : src[c]);
+    } else if (a.pro == kProFuseDecode) {
+        const int tok = token_ok(a, a.draft[t * a.K + a.step - 2]);
+        const uint16_t *e = (const uint16_t *)a.embed + (size_t)tok * d;
+        const float *h = a.src + (size_t)t * d;
+        for (int c = tid; c < d; c += 256) {
+            xr[c] = e[c];
+            xr[d + c] = f32_to_bf16(h[c]);
+        }
+    } else if (a.pro == kProFusePrefill) {
+        const int b = t / a.max_new, r = t % a.max_new;
+        const bool valid = r < clamp_n(a, b);
+        const int tok = valid ? token_ok(a, a.tokens[b * a.max_new + r]) : 0;
+        const uint16_t *e = (const uint16_t *)a.embed + (size_t)tok * d;
+        const uint16_t *h = (const uint16_t *)a.hidden_in + ((size_t)b * a.max_new + r) * d;
+        for (int c = tid; c < d; c += 256) {
+            xr[c] = valid ? e[c] : (uint16_t)0;
+            xr[d + c] = valid ? h[c] : (uint16_t)0;
+        }
+    }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 template <int NB>
@@ -759,6 +1132,74 @@ bool tc_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem) {
 
 }  // namespace
 
+template <int NB, int RPW, bool TOPK>
+cudaError_t set_tcs_attr(int bytes) {
+    return cudaFuncSetAttribute(gemv_tcs_kernel<NB, RPW, TOPK>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+}
+
+int tcs_nb(int T, int RPW, bool topk) {
+    int nb = 16;
+    while (nb < T) nb *= 2;
+    const int cap = topk ? 64 : (RPW == 2 ? 128 : 256);
+    return nb <= cap ? nb : 0;
+}
+
+// static shared memory of a streamed kernel (barriers, top-k lists)
+size_t tcs_static(int NB, bool topk) { return 512 + (topk ? (size_t)4 * NB * kTopK * 8 : 64); }
+
+bool tcs_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem, int &NB) {
+    const bool topk = a.epi == kEpiTopK;
+    const int RPW = a.epi == kEpiSwiGLU ? 2 : 1;
+    if (a.T < 1 || a.kin % 8 || a.n_units < 1) return false;
+    NB = tcs_nb(a.T, RPW, topk);
+    if (!NB) return false;
+    const int nkb = (a.kin + kBoxK - 1) / kBoxK;
+    const int n_tiles = (a.n_units + kTileM - 1) / kTileM;
+    const int max_s = topk ? 1 : kMaxSplits;
+    long best = -1;
+    int best_s = 0, best_ctas = 0;
+    for (int sp = 1; sp <= max_s && sp <= nkb; ++sp) {
+        const int per = (nkb + sp - 1) / sp;
+        int ctas = sms / sp;
+        if (ctas > n_tiles) ctas = n_tiles;
+        if (ctas < 1) break;
+        const long cost = (long)((n_tiles + ctas - 1) / ctas) * per;
+        if (best < 0 || cost < best) { best = cost; best_s = sp; best_ctas = ctas; }
+    }
+    if (best < 0) return false;
+    const size_t kb_bytes = (size_t)RPW * kBoxBytes + (size_t)NB * 128;
+    const size_t budget = (size_t)220 * 1024 - tcs_static(NB, topk);
+    const size_t dyn = budget < kTcSmem ? budget : kTcSmem;
+    const size_t room = dyn - 1024;
+    p.n_tiles = n_tiles;
+    p.nkb = nkb;
+    p.splits = best_s;
+    p.kb_per_stage = kb_bytes <= 20 * 1024 && room >= 4 * 2 * kb_bytes ? 2 : 1;
+    p.stage_bytes = (uint32_t)(p.kb_per_stage * kb_bytes);
+    p.x_bytes = 0;
+    p.stages = (int)(room / p.stage_bytes);
+    if (p.stages > kTcMaxStages) p.stages = kTcMaxStages;
+    if (p.stages < 2) return false;
+    grid = best_ctas * best_s;
+    smem = 1024 + (size_t)p.stages * p.stage_bytes;
+    return true;
+}
+
+template <int NB>
+cudaError_t dispatch_tcs(const GemvArgs &a, const TcPlan &p, const CUtensorMap &mw, const CUtensorMap &mx, int grid,
+                         size_t smem, cudaStream_t s, bool pdl) {
+    const dim3 g(grid), b(kTcThreads);
+    if (a.epi == kEpiTopK) {
+        if constexpr (NB <= 64) return launch_k(gemv_tcs_kernel<NB, 1, true>, g, b, smem, s, pdl, a, p, mw, mx);
+        return cudaErrorInvalidValue;
+    }
+    if (a.epi == kEpiSwiGLU) {
+        if constexpr (NB <= 128) return launch_k(gemv_tcs_kernel<NB, 2, false>, g, b, smem, s, pdl, a, p, mw, mx);
+        return cudaErrorInvalidValue;
+    }
+    return launch_k(gemv_tcs_kernel<NB, 1, false>, g, b, smem, s, pdl, a, p, mw, mx);
+}
+
 cudaError_t prepare_gemv_tc_kernels() {
     if (!g_encode) {
         void *fn = nullptr;
@@ -770,6 +1211,15 @@ cudaError_t prepare_gemv_tc_kernels() {
     }
     cudaError_t e = set_tc_attrs<8>((int)kTcSmem);
     if (e == cudaSuccess) e = set_tc_attrs<16>((int)kTcSmem);
+    const int b = (int)kTcSmem;
+    // per instance: what the 220 KB budget leaves after its static shared memory
+#define PRISM_TCS(NB, RPW, TK)                                                                          \
+    if (e == cudaSuccess)                                                                               \
+        e = set_tcs_attr<NB, RPW, TK>((int)std::min((size_t)b, (size_t)220 * 1024 - tcs_static(NB, TK)));
+    PRISM_TCS(16, 1, false) PRISM_TCS(32, 1, false) PRISM_TCS(64, 1, false) PRISM_TCS(128, 1, false)
+    PRISM_TCS(256, 1, false) PRISM_TCS(16, 2, false) PRISM_TCS(32, 2, false) PRISM_TCS(64, 2, false)
+    PRISM_TCS(128, 2, false) PRISM_TCS(16, 1, true) PRISM_TCS(32, 1, true) PRISM_TCS(64, 1, true)
+#undef PRISM_TCS
     return e;
 }
 
@@ -808,6 +1258,67 @@ bool gemv_tc_supported(const GemvArgs &a, int sms) {
 }
 
 int gemv_tc_tiles(const GemvArgs &a) { return (a.n_units + kTileM - 1) / kTileM; }
+
+bool gemv_tcs_supported(const GemvArgs &a, int sms) {
+    TcPlan p{};
+    int grid, NB;
+    size_t smem;
+    return tcs_plan(a, sms, p, grid, smem, NB);
+}
+
+size_t gemv_tcs_workspace_floats(const GemvArgs &a, int sms) {
+    TcPlan p{};
+    int grid, NB;
+    size_t smem;
+    if (!tcs_plan(a, sms, p, grid, smem, NB) || p.splits == 1) return 0;
+    return (size_t)p.splits * (a.epi == kEpiSwiGLU ? 2 : 1) * a.T * a.n_units;
+}
+
+cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, float *part, int *tile_ctr,
+                            uint16_t *xbuf, cudaStream_t s, bool pdl) {
+    TcPlan p{};
+    int grid, NB;
+    size_t smem;
+    if (!tcs_plan(a, sms, p, grid, smem, NB)) return cudaErrorInvalidValue;
+    p.part = part;
+    p.tile_ctr = tile_ctr;
+    if (p.splits > 1 && (!part || !tile_ctr)) return cudaErrorInvalidValue;
+    if (a.epi == kEpiTopK && grid > 256) return cudaErrorInvalidValue;
+    // the activation rows as a bf16 [T][kin] buffer: the copy prologue's
+    // source as it is, otherwise written by prep_x_kernel
+    const void *x = a.act;
+    cudaError_t e = cudaSuccess;
+    if (a.pro != kProCopy) {
+        if (!xbuf) return cudaErrorInvalidValue;
+        e = launch_k(prep_x_kernel, dim3(a.T), dim3(256), 0, s, pdl, a, xbuf);
+        if (e != cudaSuccess) return e;
+        x = xbuf;
+        pdl = true;
+    }
+    CUtensorMap mx;
+    if (!g_encode) return cudaErrorNotSupported;
+    {
+        cuuint64_t dims[2] = {(cuuint64_t)a.kin, (cuuint64_t)a.T};
+        cuuint64_t strides[1] = {(cuuint64_t)a.kin * 2};
+        cuuint32_t box[2] = {(cuuint32_t)kBoxK, (cuuint32_t)NB};
+        cuuint32_t estr[2] = {1, 1};
+        if (((uintptr_t)x & 15) ||
+            g_encode(&mx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(x), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    switch (NB) {
+        case 16: e = dispatch_tcs<16>(a, p, mw, mx, grid, smem, s, pdl); break;
+        case 32: e = dispatch_tcs<32>(a, p, mw, mx, grid, smem, s, pdl); break;
+        case 64: e = dispatch_tcs<64>(a, p, mw, mx, grid, smem, s, pdl); break;
+        case 128: e = dispatch_tcs<128>(a, p, mw, mx, grid, smem, s, pdl); break;
+        default: e = dispatch_tcs<256>(a, p, mw, mx, grid, smem, s, pdl); break;
+    }
+    if (e == cudaSuccess && a.epi == kEpiTopK)
+        e = launch_k(topk_merge_kernel, dim3(a.T), dim3(128), 0, s, true, a, grid);
+    return e;
+}
 
 size_t gemv_tc_workspace_floats(const GemvArgs &a, int sms) {
     TcPlan p{};

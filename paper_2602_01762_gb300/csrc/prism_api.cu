@@ -82,6 +82,7 @@ struct prism_ctx {
     size_t tc_part_floats = 0;
     int *tc_ctr = nullptr;
     int tc_ctr_n = 0;
+    uint16_t *xbuf = nullptr;                             // bf16 activation rows of the streamed kernel
     std::vector<GraphEntry> graphs;
     unsigned long long tick = 0;
     std::string error;
@@ -176,7 +177,12 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
     // with 112 unit tiles it needs split-K on the tensor-core kernel, and
     // measured slower there)
     auto proj = [&](const GemvArgs &g, const CUtensorMap *tm, int grid, bool pdl_here) -> cudaError_t {
-        const bool want = c->gemv_tcgen05 == 2 || (c->gemv_tcgen05 == 1 && g.epi != kEpiSwiGLU);
+        const bool want = c->gemv_tcgen05 == 2 || (c->gemv_tcgen05 == 1 && (g.epi != kEpiSwiGLU || g.T > 2));
+        if (tm && want && c->tc_ready && c->bf16 && g.T > 16 && gemv_tcs_supported(g, c->sms)) {
+            const size_t ws = gemv_tcs_workspace_floats(g, c->sms);
+            if (ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n))
+                return launch_gemv_tcs(g, *tm, c->sms, c->tc_part, c->tc_ctr, c->xbuf, s, pdl_here);
+        }
         if (tm && want && c->tc_ready && c->bf16 && gemv_tc_supported(g, c->sms)) {
             // split-K launches need the partial-sum workspace and one ticket per tile
             const size_t ws = gemv_tc_workspace_floats(g, c->sms);
@@ -457,7 +463,9 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
                 g.epi = epis[i];
                 g.pro = pros[i];
                 g.T = T;
-                const size_t need = gemv_tc_workspace_floats(g, c->sms);
+                size_t need = gemv_tc_workspace_floats(g, c->sms);
+                if (need > tc_floats) tc_floats = need;
+                need = gemv_tcs_workspace_floats(g, c->sms);
                 if (need > tc_floats) tc_floats = need;
                 if (gemv_tc_tiles(g) > tc_tiles) tc_tiles = gemv_tc_tiles(g);
             }
@@ -479,6 +487,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         32,                                                        // error word (+ checked-build record)
         tc_floats * 4,                                             // tensor-core split-K partials
         (size_t)tc_tiles * 4,                                      // tensor-core tile tickets
+        T1 * 2 * d * es,                                           // streamed-kernel activation rows
     };
     size_t total = 0;
     for (size_t s : sizes) total += align256(s);
@@ -509,6 +518,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     c->tc_part_floats = tc_floats;
     c->tc_ctr = (int *)slot[15];
     c->tc_ctr_n = tc_tiles;
+    c->xbuf = (uint16_t *)slot[16];
 
     // rotary tables: angle p * theta^(-2j/D), computed in double, stored as float
     std::vector<float> cs((size_t)f.max_ctx * (D / 2)), sn((size_t)f.max_ctx * (D / 2));
