@@ -367,6 +367,38 @@ __device__ __forceinline__ void finish_unit(const GemvArgs &a, int t, int u, flo
     }
 }
 
+// Merge this warp's new candidates (lane's (z, u) where ok) into the warp's
+// list for one row (lv / li: the topk best so far, best first, sentinels
+// after): topk rounds of a warp-wide argmax over every lane's new candidate
+// and the old list entries, ties between equal entries broken by lane.
+// Warp-uniform call.  Kept out of line: it runs rarely, and inlined into
+// the unrolled epilogue loop it cost the top-1 path measurable time.
+__device__ __noinline__ void warp_list_merge(float *lv, int *li, int topk, bool ok, float z, int u) {
+    const int lane = threadIdx.x & 31;
+    float c0v = ok ? z : -INFINITY, c1v = lane < topk ? lv[lane] : -INFINITY;
+    int c0i = ok ? u : 0x7FFFFFFF, c1i = lane < topk ? li[lane] : 0x7FFFFFFF;
+    __syncwarp();
+#pragma unroll 1
+    for (int r = 0; r < topk; ++r) {
+        const bool first = better(c0v, c0i, c1v, c1i);
+        float wv = first ? c0v : c1v;
+        int wi = first ? c0i : c1i, wl = lane;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float xv = __shfl_xor_sync(0xFFFFFFFFu, wv, o);
+            const int xi = __shfl_xor_sync(0xFFFFFFFFu, wi, o);
+            const int xl = __shfl_xor_sync(0xFFFFFFFFu, wl, o);
+            if (better(xv, xi, wv, wi) || (xv == wv && xi == wi && xl < wl)) { wv = xv; wi = xi; wl = xl; }
+        }
+        if (lane == wl) {
+            if (first) { c0v = -INFINITY; c0i = 0x7FFFFFFF; }
+            else { c1v = -INFINITY; c1i = 0x7FFFFFFF; }
+        }
+        if (lane == 0) { lv[r] = wv; li[r] = wi; }
+    }
+    __syncwarp();
+}
+
 template <int NB, int RPW, bool TOPK, int PRO>
 __global__ void __launch_bounds__(kTcThreads, 1)
     gemv_tc_kernel(const GemvArgs a, const TcPlan p, const __grid_constant__ CUtensorMap tmW) {
@@ -510,7 +542,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int quarter = warp & 3;              // TMEM lanes 32*quarter .. +31
             const int row = quarter * 32 + lane;
             const int T = a.T;
-            float thr_v[NB];
+            float thr_v[NB];                           // k-th best of each row's list, cached
             int thr_i[NB];
             if constexpr (TOPK) {
 #pragma unroll
@@ -554,30 +586,29 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         if (t >= T) break;
                         const float z = acc[0][t];
                         if (valid && a.logits) a.logits[((size_t)t * a.K + a.step - 1) * a.vocab + u] = z;
-                        unsigned m = __ballot_sync(0xFFFFFFFFu, valid && better(z, u, thr_v[t], thr_i[t]));
-                        while (m) {
-                            const int src = __ffs(m) - 1;
-                            m &= m - 1;
-                            const float zv = __shfl_sync(0xFFFFFFFFu, z, src);
-                            const int uv = __shfl_sync(0xFFFFFFFFu, u, src);
-                            if (!better(zv, uv, thr_v[t], thr_i[t])) continue;
-                            // a list of the a.topk best (the rest of it stays at sentinels)
-                            if (lane == 0) {
-                                float *lv = s_val[ew][t];
-                                int *li = s_id[ew][t];
-                                int pos = a.topk - 1;
-                                while (pos > 0 && better(zv, uv, lv[pos - 1], li[pos - 1])) {
-                                    lv[pos] = lv[pos - 1];
-                                    li[pos] = li[pos - 1];
-                                    --pos;
+                        const bool ok = valid && better(z, u, thr_v[t], thr_i[t]);
+                        if (a.topk == 1) {
+                            // top-1: insert the qualifying lanes in turn (measured faster than the merge)
+                            unsigned m = __ballot_sync(0xFFFFFFFFu, ok);
+                            while (m) {
+                                const int src = __ffs(m) - 1;
+                                m &= m - 1;
+                                const float zv = __shfl_sync(0xFFFFFFFFu, z, src);
+                                const int uv = __shfl_sync(0xFFFFFFFFu, u, src);
+                                if (!better(zv, uv, thr_v[t], thr_i[t])) continue;
+                                if (lane == 0) {
+                                    s_val[ew][t][0] = zv;
+                                    s_id[ew][t][0] = uv;
                                 }
-                                lv[pos] = zv;
-                                li[pos] = uv;
+                                __syncwarp();
+                                thr_v[t] = s_val[ew][t][0];
+                                thr_i[t] = s_id[ew][t][0];
+                                __syncwarp();
                             }
-                            __syncwarp();
+                        } else if (__any_sync(0xFFFFFFFFu, ok)) {
+                            warp_list_merge(s_val[ew][t], s_id[ew][t], a.topk, ok, z, u);
                             thr_v[t] = s_val[ew][t][a.topk - 1];
                             thr_i[t] = s_id[ew][t][a.topk - 1];
-                            __syncwarp();
                         }
                     }
                 } else if (p.splits == 1) {
@@ -877,30 +908,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             if (t >= T) break;
                             const float z = dead ? -INFINITY : acc[0][tt];
                             if (valid && a.logits) a.logits[((size_t)t * a.K + a.step - 1) * a.vocab + u] = z;
-                            const float thv = s_val[ew][t][a.topk - 1];
-                            const int thi = s_id[ew][t][a.topk - 1];
-                            unsigned m = __ballot_sync(0xFFFFFFFFu, valid && better(z, u, thv, thi));
-                            while (m) {
-                                const int src = __ffs(m) - 1;
-                                m &= m - 1;
-                                const float zv = __shfl_sync(0xFFFFFFFFu, z, src);
-                                const int uv = __shfl_sync(0xFFFFFFFFu, u, src);
-                                if (lane == 0) {
-                                    float *lv = s_val[ew][t];
-                                    int *li = s_id[ew][t];
-                                    if (better(zv, uv, lv[a.topk - 1], li[a.topk - 1])) {
-                                        int pos = a.topk - 1;
-                                        while (pos > 0 && better(zv, uv, lv[pos - 1], li[pos - 1])) {
-                                            lv[pos] = lv[pos - 1];
-                                            li[pos] = li[pos - 1];
-                                            --pos;
-                                        }
-                                        lv[pos] = zv;
-                                        li[pos] = uv;
-                                    }
-                                }
-                                __syncwarp();
-                            }
+                            const bool ok = valid && better(z, u, s_val[ew][t][a.topk - 1], s_id[ew][t][a.topk - 1]);
+                            if (__any_sync(0xFFFFFFFFu, ok))
+                                warp_list_merge(s_val[ew][t], s_id[ew][t], a.topk, ok, z, u);
                         }
                     } else if (p.splits == 1) {
                         if (valid) {
