@@ -170,6 +170,7 @@ struct GemvArgs {
     float *lm_part;          // [T, grid, 8] values (LM head)
     int *lm_part_id;         // [T, grid, 8] ids
     int *counter;            // LM head last-CTA counter
+    unsigned long long *best;  // [T] packed (value, id) of the best logit so far, for top-1 (zero: none)
     int32_t *draft_out;      // [B, K]
     int32_t *topk_ids;       // [B, K, topk] or null
     float *topk_logits;      // [B, K, topk] or null

@@ -367,6 +367,20 @@ __device__ __forceinline__ void finish_unit(const GemvArgs &a, int t, int u, flo
     }
 }
 
+// Top-1 as one 64-bit key: an order-preserving image of the fp32 logit in
+// the high word and the inverted id in the low word, so that the numeric
+// maximum is the best candidate under `better` (larger logit, then lower id).
+__device__ __forceinline__ unsigned long long pack_best(float v, int id) {
+    const uint32_t b = __float_as_uint(v);
+    const uint32_t k = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+    return ((unsigned long long)k << 32) | (uint32_t)(0xFFFFFFFFu - (uint32_t)id);
+}
+__device__ __forceinline__ void unpack_best(unsigned long long key, float &v, int &id) {
+    const uint32_t k = (uint32_t)(key >> 32);
+    v = __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+    id = (int)(0xFFFFFFFFu - (uint32_t)key);
+}
+
 // Merge this warp's new candidates (lane's (z, u) where ok) into the warp's
 // list for one row (lv / li: the topk best so far, best first, sentinels
 // after): topk rounds of a warp-wide argmax over every lane's new candidate
@@ -652,6 +666,35 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
             }
             if constexpr (TOPK) {
+              if (a.topk == 1 && a.best) {
+                // top-1: this CTA's best of each row joins a 64-bit atomic maximum;
+                // the last CTA to finish reads and clears it
+                epi_sync();
+                if (ew == 0 && lane < T) {
+                    float bv = s_val[0][lane][0];
+                    int bi = s_id[0][lane][0];
+#pragma unroll
+                    for (int w = 1; w < 4; ++w)
+                        if (better(s_val[w][lane][0], s_id[w][lane][0], bv, bi)) { bv = s_val[w][lane][0]; bi = s_id[w][lane][0]; }
+                    if (bi != 0x7FFFFFFF) atomicMax(a.best + lane, pack_best(bv, bi));
+                }
+                __threadfence();
+                epi_sync();
+                if (threadIdx.x == 64) s_last = atomicAdd(a.counter, 1) == (int)gridDim.x - 1;
+                epi_sync();
+                if (s_last && ew == 0 && lane < T) {
+                    __threadfence();
+                    const unsigned long long key = atomicExch(a.best + lane, 0ull);
+                    float v;
+                    int id;
+                    unpack_best(key, v, id);
+                    const size_t o = (size_t)lane * a.K + a.step - 1;
+                    a.draft_out[o] = id;
+                    if (a.topk_ids) a.topk_ids[o] = id;
+                    if (a.topk_logits) a.topk_logits[o] = v;
+                }
+                if (s_last && threadIdx.x == 64) *a.counter = 0;
+              } else {
                 // per-CTA merge of the four epilogue warps' lists, then the last CTA merges all CTAs
                 epi_sync();
                 for (int t = ew; t < T; t += 4) {
@@ -701,6 +744,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                     if (threadIdx.x == 64) *a.counter = 0;
                 }
+              }
             }
         }
     }

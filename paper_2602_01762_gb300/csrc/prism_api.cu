@@ -63,6 +63,7 @@ struct prism_ctx {
     float *lm_val = nullptr;
     int *lm_id = nullptr;
     int *counters = nullptr;  // [max_batch * Hkv] attention + [1] LM head
+    unsigned long long *lm_best = nullptr;  // [max_batch] LM head top-1 keys (left at zero)
     int *err = nullptr;
     // execution
     cudaStream_t cap_stream = nullptr;
@@ -384,6 +385,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.lm_part = c->lm_val;
         g.lm_part_id = c->lm_id;
         g.counter = c->counters + (size_t)f.max_batch * Hkv;
+        g.best = c->lm_best;
         g.draft_out = r.draft;
         g.topk_ids = r.topk_ids;
         g.topk_logits = r.topk_logits;
@@ -484,6 +486,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         B * (size_t)c->lm_grid * kTopK * 4,                        // LM partial values
         B * (size_t)c->lm_grid * kTopK * 4,                        // LM partial ids
         (B * Hkv + 1) * 4,                                         // counters
+        B * 8,                                                     // LM head packed top-1 keys
         32,                                                        // error word (+ checked-build record)
         tc_floats * 4,                                             // tensor-core split-K partials
         (size_t)tc_tiles * 4,                                      // tensor-core tile tickets
@@ -513,12 +516,13 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     c->lm_val = (float *)slot[10];
     c->lm_id = (int *)slot[11];
     c->counters = (int *)slot[12];
-    c->err = (int *)slot[13];
-    c->tc_part = (float *)slot[14];
+    c->lm_best = (unsigned long long *)slot[13];
+    c->err = (int *)slot[14];
+    c->tc_part = (float *)slot[15];
     c->tc_part_floats = tc_floats;
-    c->tc_ctr = (int *)slot[15];
+    c->tc_ctr = (int *)slot[16];
     c->tc_ctr_n = tc_tiles;
-    c->xbuf = (uint16_t *)slot[16];
+    c->xbuf = (uint16_t *)slot[17];
 
     // rotary tables: angle p * theta^(-2j/D), computed in double, stored as float
     std::vector<float> cs((size_t)f.max_ctx * (D / 2)), sn((size_t)f.max_ctx * (D / 2));
