@@ -200,11 +200,14 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * 0 = default), "gemv_smem_kb" (shared-memory budget of the projection
  * ring, 0..200, 0 = default), "gemv_groups" (consumer warp groups of the
  * projection kernels: 1, 2, 4, 8 or 16; 0 = default), "gemv_tcgen05"
- * (1, the default: bf16 projections with at most 16 activation rows run on
- * the tcgen05 kernel, TMA tensor loads into tensor-memory accumulators,
- * except gate/up + SwiGLU, which measures faster on the CUDA-core kernel;
+ * (1, the default: bf16 projections run on the tcgen05 kernels, TMA tensor
+ * loads into tensor-memory accumulators, except gate/up + SwiGLU with at
+ * most 2 activation rows, which measures faster on the CUDA-core kernel;
  * 2: gate/up as well; 0: every projection on the kernels below),
- * "gemv_cuda_core" (for projections
+ * "tc_stream_rows" (>= 1, default 17: a tcgen05 projection with at least
+ * this many activation rows streams them through the TMA ring beside the
+ * weights instead of staging them whole in shared memory; at most 16 rows
+ * can be staged), "gemv_cuda_core" (for projections
  * not on the tcgen05 kernel: 1, the default, the CUDA-core TMA-ring kernel;
  * 0: the warp-level mma.sync kernel), "attn_fused" (1, the default: RoPE,
  * KV append and attention run as one kernel, a cluster of up to 8 CTAs per

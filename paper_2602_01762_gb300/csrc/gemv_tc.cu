@@ -313,43 +313,6 @@ __device__ void stage_x_tc(const GemvArgs &a, int kb0, int kb1, uint8_t *X, floa
     }
 }
 
-// Top `rounds` (<= 8) under `better` of candidates spread over a warp: one
-// warp-wide argmax per rank over the lanes' best remaining candidate; the winning lane
-// retires it.  Each lane holds C candidates (cv, ci); ties between equal
-// entries break by lane, so the winner is warp-uniform.  The result goes to
-// out_v/out_i (written by lane 0).  Compact code on purpose: it runs cold.
-template <int C>
-__device__ void warp_top8(float (&cv)[C], int (&ci)[C], float *out_v, int *out_i, int rounds) {
-    const int lane = threadIdx.x & 31;
-    // only the ranks the caller keeps are selected; the rest of the list is
-    // filled with sentinels (below every candidate under `better`)
-    if (lane == 0)
-        for (int r = rounds; r < kTopK; ++r) { out_v[r] = -INFINITY; out_i[r] = 0x7FFFFFFF; }
-#pragma unroll 1
-    for (int r = 0; r < rounds; ++r) {
-        float bv = cv[0];
-        int bi = ci[0], bs = 0;
-#pragma unroll
-        for (int u = 1; u < C; ++u)
-            if (better(cv[u], ci[u], bv, bi)) { bv = cv[u]; bi = ci[u]; bs = u; }
-        float wv = bv;
-        int wi = bi, wl = lane;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float xv = __shfl_xor_sync(0xFFFFFFFFu, wv, o);
-            const int xi = __shfl_xor_sync(0xFFFFFFFFu, wi, o);
-            const int xl = __shfl_xor_sync(0xFFFFFFFFu, wl, o);
-            if (better(xv, xi, wv, wi) || (xv == wv && xi == wi && xl < wl)) { wv = xv; wi = xi; wl = xl; }
-        }
-        if (lane == wl) {
-#pragma unroll
-            for (int u = 0; u < C; ++u)
-                if (u == bs) { cv[u] = -INFINITY; ci[u] = 0x7FFFFFFF; }
-        }
-        if (lane == 0) { out_v[r] = wv; out_i[r] = wi; }
-    }
-}
-
 // Final epilogue of one output unit u for activation row t, given its
 // accumulators (RPW = 2: gate, up).
 template <int RPW>
@@ -381,36 +344,152 @@ __device__ __forceinline__ void unpack_best(unsigned long long key, float &v, in
     id = (int)(0xFFFFFFFFu - (uint32_t)key);
 }
 
-// Merge this warp's new candidates (lane's (z, u) where ok) into the warp's
-// list for one row (lv / li: the topk best so far, best first, sentinels
-// after): topk rounds of a warp-wide argmax over every lane's new candidate
-// and the old list entries, ties between equal entries broken by lane.
-// Warp-uniform call.  Kept out of line: it runs rarely, and inlined into
-// the unrolled epilogue loop it cost the top-1 path measurable time.
-__device__ __noinline__ void warp_list_merge(float *lv, int *li, int topk, bool ok, float z, int u) {
-    const int lane = threadIdx.x & 31;
-    float c0v = ok ? z : -INFINITY, c1v = lane < topk ? lv[lane] : -INFINITY;
-    int c0i = ok ? u : 0x7FFFFFFF, c1i = lane < topk ? li[lane] : 0x7FFFFFFF;
-    __syncwarp();
-#pragma unroll 1
-    for (int r = 0; r < topk; ++r) {
-        const bool first = better(c0v, c0i, c1v, c1i);
-        float wv = first ? c0v : c1v;
-        int wi = first ? c0i : c1i, wl = lane;
+// ---------------------------------------------------------------- top-k lists
+// A candidate list is kTopK packed keys (pack_best) in registers, best first;
+// key 0 is the empty slot (below every real candidate).  Each epilogue thread
+// keeps one list, for one activation row: with NB rows, P = 128 / NB threads
+// share a row and each scans 128 / P of a tile's 128 logits.  The logits
+// reach the scanning threads through a transposed shared-memory copy of one
+// 16-column accumulator chunk at a time, so a scan is one compare per logit
+// (a list changes only when a logit beats its last entry).  The P lists of a
+// row are merged pairwise across lanes (bitonic merge), and the per-CTA lists
+// of all CTAs once at the end.
+constexpr int kTrMax = kTileM + 8;   // floats per transposed row, largest P
+
+using Key = unsigned long long;
+
+__device__ __forceinline__ void key_clear(Key (&l)[kTopK]) {
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float xv = __shfl_xor_sync(0xFFFFFFFFu, wv, o);
-            const int xi = __shfl_xor_sync(0xFFFFFFFFu, wi, o);
-            const int xl = __shfl_xor_sync(0xFFFFFFFFu, wl, o);
-            if (better(xv, xi, wv, wi) || (xv == wv && xi == wi && xl < wl)) { wv = xv; wi = xi; wl = xl; }
-        }
-        if (lane == wl) {
-            if (first) { c0v = -INFINITY; c0i = 0x7FFFFFFF; }
-            else { c1v = -INFINITY; c1i = 0x7FFFFFFF; }
-        }
-        if (lane == 0) { lv[r] = wv; li[r] = wi; }
+    for (int i = 0; i < kTopK; ++i) l[i] = 0ull;
+}
+
+// Insert k into the sorted list l (static indices: l stays in registers).
+__device__ __forceinline__ void key_insert(Key (&l)[kTopK], Key k) {
+    if (k <= l[kTopK - 1]) return;
+    l[kTopK - 1] = k;
+#pragma unroll
+    for (int s = kTopK - 1; s > 0; --s) {
+        const Key x = l[s - 1], y = l[s];
+        l[s - 1] = x > y ? x : y;
+        l[s] = x > y ? y : x;
     }
-    __syncwarp();
+}
+
+// Lanes lane and lane ^ m both end with the best kTopK keys of their two
+// lists: the element-wise maximum of one list and the other reversed is that
+// set as a bitonic sequence, sorted by three half-cleaner stages.  Every lane
+// of the warp takes part.
+__device__ __forceinline__ void key_merge_xor(Key (&l)[kTopK], int m) {
+    Key c[kTopK];
+#pragma unroll
+    for (int i = 0; i < kTopK; ++i) {
+        const Key o = __shfl_xor_sync(0xFFFFFFFFu, l[kTopK - 1 - i], m);
+        c[i] = l[i] > o ? l[i] : o;
+    }
+#pragma unroll
+    for (int d = kTopK / 2; d > 0; d >>= 1)
+#pragma unroll
+        for (int i = 0; i < kTopK; ++i)
+            if ((i & d) == 0) {
+                const Key x = c[i], y = c[i + d];
+                c[i] = x > y ? x : y;
+                c[i + d] = x > y ? y : x;
+            }
+#pragma unroll
+    for (int i = 0; i < kTopK; ++i) l[i] = c[i];
+}
+
+// Entry r of a register list without a dynamic index.
+__device__ __forceinline__ Key key_at(const Key (&l)[kTopK], int r) {
+    Key k = l[0];
+#pragma unroll
+    for (int i = 1; i < kTopK; ++i)
+        if (r == i) k = l[i];
+    return k;
+}
+
+// One 16-column accumulator chunk (columns c0 .. c0 + 15) of a finished tile
+// into the lists.  The four epilogue warps write their TMEM rows transposed
+// (tr[j][row]: column j becomes a row of 128 logits), then the threads of
+// those columns' rows scan them.  A transposed row is 128 + P floats long, so
+// the 32 lanes of a scanning warp read 32 distinct banks.
+template <int P>
+__device__ __forceinline__ void chunk_to_lists(const float (&acc)[16], int row, float *tr, int tile, int c0, int T,
+                                               int n_units, bool dead, Key (&l)[kTopK]) {
+    constexpr int S = kTileM + P;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) tr[j * S + row] = acc[j];
+    epi_sync();
+    const int e = threadIdx.x - 64, t = e / P, q = e % P;
+    if (!dead && t >= c0 && t < c0 + 16 && t < T) {
+        const float *src = tr + (t - c0) * S;
+#pragma unroll 4
+        for (int i = 0; i < kTileM / P; ++i) {
+            const int r = i * P + q, u = tile * kTileM + r;
+            if (u < n_units) key_insert(l, pack_best(src[r], u));
+        }
+    }
+    epi_sync();
+}
+
+// The CTA's list of each row: the P threads of a row merge theirs and write
+// it to the per-CTA partial lists ([row][CTA][kTopK] values and ids; id -1
+// marks an empty slot), thread q the entries q, q + P, ...
+template <int P>
+__device__ __forceinline__ void lists_publish(const GemvArgs &a, Key (&l)[kTopK], int T) {
+#pragma unroll
+    for (int m = 1; m < P; m <<= 1) key_merge_xor(l, m);
+    const int e = threadIdx.x - 64, t = e / P, q = e % P;
+    if (t < T) {
+#pragma unroll
+        for (int r0 = 0; r0 < kTopK; r0 += P) {
+            float v;
+            int id;
+            unpack_best(key_at(l, r0 + q), v, id);
+            const size_t o = ((size_t)t * gridDim.x + blockIdx.x) * kTopK + r0 + q;
+            a.lm_part[o] = v;
+            a.lm_part_id[o] = id;
+        }
+    }
+}
+
+// This thread's share (candidates first, first + stride, ...) of row t's
+// partial lists, as a sorted list.  Loads are issued 16 at a time.
+__device__ __forceinline__ void gather_keys(const GemvArgs &a, int t, int grid, int first, int stride, Key (&l)[kTopK]) {
+    constexpr int kBatch = 16;
+    const int ncand = grid * kTopK;
+    const float *pv = a.lm_part + (size_t)t * ncand;
+    const int *pi = a.lm_part_id + (size_t)t * ncand;
+    key_clear(l);
+#pragma unroll 1
+    for (int c = first; c < ncand; c += kBatch * stride) {
+        float v[kBatch];
+        int id[kBatch];
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b) {
+            const int cc = c + b * stride;
+            v[b] = cc < ncand ? __ldcg(pv + cc) : 0.f;
+            id[b] = cc < ncand ? __ldcg(pi + cc) : -1;
+        }
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b)
+            if (id[b] >= 0) key_insert(l, pack_best(v[b], id[b]));
+    }
+}
+
+// Row t's final top-k from a list every lane of the warp holds: lane r < topk
+// writes rank r.
+__device__ __forceinline__ void write_row(const GemvArgs &a, int t, const Key (&l)[kTopK]) {
+    const int lane = threadIdx.x & 31;
+    if (lane < a.topk) {
+        float v;
+        int id;
+        unpack_best(key_at(l, lane), v, id);
+        const size_t o = (size_t)t * a.K + a.step - 1;
+        if (lane == 0) a.draft_out[o] = id;
+        if (a.topk_ids) a.topk_ids[o * a.topk + lane] = id;
+        if (a.topk_logits) a.topk_logits[o * a.topk + lane] = v;
+    }
 }
 
 template <int NB, int RPW, bool TOPK, int PRO>
@@ -420,10 +499,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     __shared__ __align__(8) uint64_t full[kTcMaxStages], empty[kTcMaxStages], acc_full[2], acc_empty[2], mma_done;
     __shared__ uint32_t s_tmem;
     __shared__ float red[kStageThreads / 32];
-    __shared__ float s_fin_v[TOPK ? kTopK : 1];
-    __shared__ int s_fin_i[TOPK ? kTopK : 1];
-    __shared__ float s_val[TOPK ? 4 : 1][TOPK ? NB : 1][kTopK];
-    __shared__ int s_id[TOPK ? 4 : 1][TOPK ? NB : 1][kTopK];
+    __shared__ float s_val[TOPK ? 4 : 1][TOPK ? NB : 1];   // top-1: each epilogue warp's best per row
+    __shared__ int s_id[TOPK ? 4 : 1][TOPK ? NB : 1];
+    __shared__ float s_tr[TOPK ? 16 : 1][TOPK ? kTrMax : 1];
     __shared__ int s_last;
     constexpr uint32_t kCols = RPW == 1 ? 32 : 64;   // two accumulator buffers x RPW x 16 columns
 
@@ -556,15 +634,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int quarter = warp & 3;              // TMEM lanes 32*quarter .. +31
             const int row = quarter * 32 + lane;
             const int T = a.T;
-            float thr_v[NB];                           // k-th best of each row's list, cached
+            // top-1 with the 64-bit atomic maximum: per warp and row the best so
+            // far (thr, cached in registers); otherwise the register lists
+            const bool top1 = a.topk == 1 && a.best != nullptr;
+            float thr_v[NB];
             int thr_i[NB];
+            Key lst[kTopK];
             if constexpr (TOPK) {
 #pragma unroll
                 for (int t = 0; t < NB; ++t) { thr_v[t] = -INFINITY; thr_i[t] = 0x7FFFFFFF; }
-                if (lane < NB) {
-#pragma unroll
-                    for (int i = 0; i < kTopK; ++i) { s_val[ew][lane][i] = -INFINITY; s_id[ew][lane][i] = 0x7FFFFFFF; }
-                }
+                if (lane < NB) { s_val[ew][lane] = -INFINITY; s_id[ew][lane] = 0x7FFFFFFF; }
+                key_clear(lst);
                 __syncwarp();
             }
             bool dead = false;
@@ -595,15 +675,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 const int u = tile * kTileM + row;
                 const bool valid = !dead && u < a.n_units;
                 if constexpr (TOPK) {
+                    if (valid && a.logits) {
 #pragma unroll
-                    for (int t = 0; t < NB; ++t) {
-                        if (t >= T) break;
-                        const float z = acc[0][t];
-                        if (valid && a.logits) a.logits[((size_t)t * a.K + a.step - 1) * a.vocab + u] = z;
-                        const bool ok = valid && better(z, u, thr_v[t], thr_i[t]);
-                        if (a.topk == 1) {
-                            // top-1: insert the qualifying lanes in turn (measured faster than the merge)
-                            unsigned m = __ballot_sync(0xFFFFFFFFu, ok);
+                        for (int t = 0; t < NB; ++t)
+                            if (t < T) a.logits[((size_t)t * a.K + a.step - 1) * a.vocab + u] = acc[0][t];
+                    }
+                    if (top1) {
+#pragma unroll
+                        for (int t = 0; t < NB; ++t) {
+                            if (t >= T) break;
+                            const float z = acc[0][t];
+                            // insert the qualifying lanes in turn
+                            unsigned m = __ballot_sync(0xFFFFFFFFu, valid && better(z, u, thr_v[t], thr_i[t]));
                             while (m) {
                                 const int src = __ffs(m) - 1;
                                 m &= m - 1;
@@ -611,19 +694,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                 const int uv = __shfl_sync(0xFFFFFFFFu, u, src);
                                 if (!better(zv, uv, thr_v[t], thr_i[t])) continue;
                                 if (lane == 0) {
-                                    s_val[ew][t][0] = zv;
-                                    s_id[ew][t][0] = uv;
+                                    s_val[ew][t] = zv;
+                                    s_id[ew][t] = uv;
                                 }
                                 __syncwarp();
-                                thr_v[t] = s_val[ew][t][0];
-                                thr_i[t] = s_id[ew][t][0];
+                                thr_v[t] = s_val[ew][t];
+                                thr_i[t] = s_id[ew][t];
                                 __syncwarp();
                             }
-                        } else if (__any_sync(0xFFFFFFFFu, ok)) {
-                            warp_list_merge(s_val[ew][t], s_id[ew][t], a.topk, ok, z, u);
-                            thr_v[t] = s_val[ew][t][a.topk - 1];
-                            thr_i[t] = s_id[ew][t][a.topk - 1];
                         }
+                    } else {
+                        chunk_to_lists<8>(acc[0], row, &s_tr[0][0], tile, 0, T, a.n_units, dead, lst);
                     }
                 } else if (p.splits == 1) {
                     if (valid) {
@@ -666,42 +747,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
             }
             if constexpr (TOPK) {
-              if (a.topk == 1 && a.best) {
-                // top-1: this CTA's best of each row joins a 64-bit atomic maximum;
-                // the last CTA to finish reads and clears it
-                epi_sync();
-                if (ew == 0 && lane < T) {
-                    float bv = s_val[0][lane][0];
-                    int bi = s_id[0][lane][0];
+                if (top1) {
+                    // this CTA's best of each row joins a 64-bit atomic maximum;
+                    // the last CTA to finish reads and clears it
+                    epi_sync();
+                    if (ew == 0 && lane < T) {
+                        float bv = s_val[0][lane];
+                        int bi = s_id[0][lane];
 #pragma unroll
-                    for (int w = 1; w < 4; ++w)
-                        if (better(s_val[w][lane][0], s_id[w][lane][0], bv, bi)) { bv = s_val[w][lane][0]; bi = s_id[w][lane][0]; }
-                    if (bi != 0x7FFFFFFF) atomicMax(a.best + lane, pack_best(bv, bi));
-                }
-                __threadfence();
-                epi_sync();
-                if (threadIdx.x == 64) s_last = atomicAdd(a.counter, 1) == (int)gridDim.x - 1;
-                epi_sync();
-                if (s_last && ew == 0 && lane < T) {
-                    __threadfence();
-                    const unsigned long long key = atomicExch(a.best + lane, 0ull);
-                    float v;
-                    int id;
-                    unpack_best(key, v, id);
-                    const size_t o = (size_t)lane * a.K + a.step - 1;
-                    a.draft_out[o] = id;
-                    if (a.topk_ids) a.topk_ids[o] = id;
-                    if (a.topk_logits) a.topk_logits[o] = v;
-                }
-                if (s_last && threadIdx.x == 64) *a.counter = 0;
-              } else {
-                // per-CTA merge of the four epilogue warps' lists, then the last CTA merges all CTAs
-                epi_sync();
-                for (int t = ew; t < T; t += 4) {
-                    float cv[1] = {s_val[lane / kTopK][t][lane % kTopK]};
-                    int ci[1] = {s_id[lane / kTopK][t][lane % kTopK]};
-                    const size_t o = ((size_t)t * gridDim.x + blockIdx.x) * kTopK;
-                    warp_top8<1>(cv, ci, a.lm_part + o, a.lm_part_id + o, a.topk);
+                        for (int w = 1; w < 4; ++w)
+                            if (better(s_val[w][lane], s_id[w][lane], bv, bi)) { bv = s_val[w][lane]; bi = s_id[w][lane]; }
+                        if (bi != 0x7FFFFFFF) atomicMax(a.best + lane, pack_best(bv, bi));
+                    }
+                } else {
+                    lists_publish<8>(a, lst, T);
                 }
                 __threadfence();
                 epi_sync();
@@ -709,42 +768,28 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 epi_sync();
                 if (s_last) {
                     __threadfence();
-                    // each warp takes a quarter of every row's candidates (all
-                    // loads of a lane issued together), then one warp merges
-                    // the four partial lists
-                    constexpr int kC = 12;                         // grids up to 192 CTAs
-                    const int ncand = (int)gridDim.x * kTopK;
-                    const int lo = ew * ncand / 4, hi = (ew + 1) * ncand / 4;
-#pragma unroll 1
-                    for (int t = 0; t < T; ++t) {
-                        float cv[kC];
-                        int ci[kC];
-                        const size_t b0 = (size_t)t * ncand;
+                    if (top1) {
+                        if (ew == 0 && lane < T) {
+                            const Key key = atomicExch(a.best + lane, 0ull);
+                            float v;
+                            int id;
+                            unpack_best(key, v, id);
+                            const size_t o = (size_t)lane * a.K + a.step - 1;
+                            a.draft_out[o] = id;
+                            if (a.topk_ids) a.topk_ids[o] = id;
+                            if (a.topk_logits) a.topk_logits[o] = v;
+                        }
+                    } else {
+                        // one warp per row over every CTA's list
+                        for (int t = ew; t < T; t += 4) {
+                            gather_keys(a, t, gridDim.x, lane, 32, lst);
 #pragma unroll
-                        for (int u = 0; u < kC; ++u) {
-                            const int c = lo + lane + 32 * u;
-                            cv[u] = c < hi ? __ldcg(a.lm_part + b0 + c) : -INFINITY;
-                            ci[u] = c < hi ? __ldcg(a.lm_part_id + b0 + c) : 0x7FFFFFFF;
+                            for (int m = 1; m < 32; m <<= 1) key_merge_xor(lst, m);
+                            write_row(a, t, lst);
                         }
-                        warp_top8<kC>(cv, ci, s_val[ew][0], s_id[ew][0], a.topk);
-                        epi_sync();
-                        if (ew == 0) {
-                            float fv[1] = {s_val[lane / kTopK][0][lane % kTopK]};
-                            int fi[1] = {s_id[lane / kTopK][0][lane % kTopK]};
-                            warp_top8<1>(fv, fi, s_fin_v, s_fin_i, a.topk);
-                            __syncwarp();
-                            if (lane < a.topk) {
-                                const size_t o = (size_t)t * a.K + a.step - 1;
-                                if (lane == 0) a.draft_out[o] = s_fin_i[0];
-                                if (a.topk_ids) a.topk_ids[o * a.topk + lane] = s_fin_i[lane];
-                                if (a.topk_logits) a.topk_logits[o * a.topk + lane] = s_fin_v[lane];
-                            }
-                        }
-                        epi_sync();
                     }
                     if (threadIdx.x == 64) *a.counter = 0;
                 }
-              }
             }
         }
     }
@@ -773,8 +818,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full[kTcMaxStages], empty[kTcMaxStages], acc_full[2], acc_empty[2], mma_done;
     __shared__ uint32_t s_tmem;
-    __shared__ float s_val[TOPK ? 4 : 1][TOPK ? NB : 1][kTopK];
-    __shared__ int s_id[TOPK ? 4 : 1][TOPK ? NB : 1][kTopK];
+    __shared__ float s_tr[TOPK ? 16 : 1][TOPK ? kTrMax : 1];
     __shared__ int s_last;
     constexpr uint32_t kXBox = NB * 128;                              // one X box
     constexpr uint32_t kColsNeed = 2 * RPW * NB;
@@ -918,12 +962,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int quarter = warp & 3;
             const int row = quarter * 32 + lane;
             const int T = a.T;
-            if constexpr (TOPK) {
-                for (int t = lane; t < NB; t += 32)
-#pragma unroll
-                    for (int i = 0; i < kTopK; ++i) { s_val[ew][t][i] = -INFINITY; s_id[ew][t][i] = 0x7FFFFFFF; }
-                __syncwarp();
-            }
+            constexpr int kP = NB <= 128 ? kTileM / NB : 1;     // threads per activation row
+            Key lst[kTopK];
+            if constexpr (TOPK) key_clear(lst);
             bool dead = false;
             for (int i = 0; i < my_tiles; ++i) {
                 const int tile = blockIdx.x / p.splits + i * tiles_step;
@@ -934,8 +975,27 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
                 const int u = tile * kTileM + row;
                 const bool valid = !dead && u < a.n_units;
+                if constexpr (TOPK) {
+#pragma unroll 1
+                    for (int c0 = 0; c0 < NB && c0 < T; c0 += 16) {
+                        float acc[16];
+                        if (!dead) {
+                            tc_fence_after();
+                            tmem_ld16(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(ab * NB + c0), acc);
+                        } else {
+#pragma unroll
+                            for (int tt = 0; tt < 16; ++tt) acc[tt] = 0.f;
+                        }
+                        if (valid && a.logits) {
+#pragma unroll
+                            for (int tt = 0; tt < 16; ++tt)
+                                if (c0 + tt < T) a.logits[((size_t)(c0 + tt) * a.K + a.step - 1) * a.vocab + u] = acc[tt];
+                        }
+                        chunk_to_lists<kP>(acc, row, &s_tr[0][0], tile, c0, T, a.n_units, dead, lst);
+                    }
+                }
                 // accumulator columns 16 at a time (all RPW sets of one chunk together)
-                for (int c0 = 0; c0 < NB; c0 += 16) {
+                for (int c0 = 0; c0 < (TOPK ? 0 : NB); c0 += 16) {
                     float acc[RPW][16];
                     if (!dead) {
                         tc_fence_after();
@@ -945,18 +1005,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                       acc[r]);
                     }
                     if (c0 >= T) continue;
-                    if constexpr (TOPK) {
-#pragma unroll
-                        for (int tt = 0; tt < 16; ++tt) {
-                            const int t = c0 + tt;
-                            if (t >= T) break;
-                            const float z = dead ? -INFINITY : acc[0][tt];
-                            if (valid && a.logits) a.logits[((size_t)t * a.K + a.step - 1) * a.vocab + u] = z;
-                            const bool ok = valid && better(z, u, s_val[ew][t][a.topk - 1], s_id[ew][t][a.topk - 1]);
-                            if (__any_sync(0xFFFFFFFFu, ok))
-                                warp_list_merge(s_val[ew][t], s_id[ew][t], a.topk, ok, z, u);
-                        }
-                    } else if (p.splits == 1) {
+                    if (p.splits == 1) {
                         if (valid) {
 #pragma unroll
                             for (int tt = 0; tt < 16; ++tt) {
@@ -1004,14 +1053,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
             }
             if constexpr (TOPK) {
-                // this CTA's top-k of every row; the cross-CTA merge is a separate kernel
-                epi_sync();
-                for (int t = ew; t < T; t += 4) {
-                    float cv[1] = {s_val[lane / kTopK][t][lane % kTopK]};
-                    int ci[1] = {s_id[lane / kTopK][t][lane % kTopK]};
-                    const size_t o = ((size_t)t * gridDim.x + blockIdx.x) * kTopK;
-                    warp_top8<1>(cv, ci, a.lm_part + o, a.lm_part_id + o, a.topk);
-                }
+                // this CTA's list of every row; the cross-CTA merge is a separate kernel
+                lists_publish<kP>(a, lst, T);
             }
         }
     }
@@ -1023,39 +1066,29 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols));
 }
 
-// Cross-CTA top-k merge of the streamed LM head: one CTA (4 warps) per row.
+// Cross-CTA top-k merge of the streamed LM head: one CTA (4 warps) per row;
+// each warp merges a quarter of the row's candidates, warp 0 the four lists.
 __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int grid) {
-    __shared__ float s_v[4][kTopK];
-    __shared__ int s_i[4][kTopK];
-    __shared__ float f_v[kTopK];
-    __shared__ int f_i[kTopK];
+    __shared__ Key s_k[4][kTopK];
     pdl_trigger();
     pdl_wait();
     const int t = blockIdx.x, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    constexpr int kC = 16;                                        // grids up to 256 CTAs
-    const int ncand = grid * kTopK, lo = w * ncand / 4, hi = (w + 1) * ncand / 4;
-    float cv[kC];
-    int ci[kC];
-    const size_t b0 = (size_t)t * ncand;
+    Key l[kTopK];
+    gather_keys(a, t, grid, threadIdx.x, 128, l);
 #pragma unroll
-    for (int u = 0; u < kC; ++u) {
-        const int c = lo + lane + 32 * u;
-        cv[u] = c < hi ? __ldcg(a.lm_part + b0 + c) : -INFINITY;
-        ci[u] = c < hi ? __ldcg(a.lm_part_id + b0 + c) : 0x7FFFFFFF;
+    for (int m = 1; m < 32; m <<= 1) key_merge_xor(l, m);
+    if (lane == 0) {
+#pragma unroll
+        for (int i = 0; i < kTopK; ++i) s_k[w][i] = l[i];
     }
-    warp_top8<kC>(cv, ci, s_v[w], s_i[w], a.topk);
     __syncthreads();
     if (w == 0) {
-        float fv[1] = {s_v[lane / kTopK][lane % kTopK]};
-        int fi[1] = {s_i[lane / kTopK][lane % kTopK]};
-        warp_top8<1>(fv, fi, f_v, f_i, a.topk);
-        __syncwarp();
-        if (lane < a.topk) {
-            const size_t o = (size_t)t * a.K + a.step - 1;
-            if (lane == 0) a.draft_out[o] = f_i[0];
-            if (a.topk_ids) a.topk_ids[o * a.topk + lane] = f_i[lane];
-            if (a.topk_logits) a.topk_logits[o * a.topk + lane] = f_v[lane];
-        }
+#pragma unroll
+        for (int i = 0; i < kTopK; ++i) l[i] = lane < 4 ? s_k[lane][i] : 0ull;
+        // every lane ends with the merged list (write_row reads rank r from lane r)
+#pragma unroll
+        for (int m = 1; m < 32; m <<= 1) key_merge_xor(l, m);
+        write_row(a, t, l);
     }
 }
 
@@ -1162,7 +1195,6 @@ bool tc_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem) {
         if ((size_t)NB * 128 * per > kXBudget) continue;
         int ctas = sms / sp;
         if (ctas > n_tiles) ctas = n_tiles;
-        if (a.epi == kEpiTopK && ctas > 192) ctas = 192;   // candidates the final merge holds
         if (ctas < 1) break;
         const long cost = (long)((n_tiles + ctas - 1) / ctas) * per;
         if (best < 0 || cost < best) { best = cost; best_s = sp; best_ctas = ctas; }
@@ -1199,7 +1231,7 @@ int tcs_nb(int T, int RPW, bool topk) {
 }
 
 // static shared memory of a streamed kernel (barriers, top-k lists)
-size_t tcs_static(int NB, bool topk) { return 512 + (topk ? (size_t)4 * NB * kTopK * 8 : 64); }
+size_t tcs_static(int NB, bool topk) { return 512 + (topk ? (size_t)16 * kTrMax * 4 : 64); }
 
 bool tcs_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem, int &NB) {
     const bool topk = a.epi == kEpiTopK;
@@ -1337,7 +1369,6 @@ cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, f
     p.part = part;
     p.tile_ctr = tile_ctr;
     if (p.splits > 1 && (!part || !tile_ctr)) return cudaErrorInvalidValue;
-    if (a.epi == kEpiTopK && grid > 256) return cudaErrorInvalidValue;
     // the activation rows as a bf16 [T][kin] buffer: the copy prologue's
     // source as it is, otherwise written by prep_x_kernel
     const void *x = a.act;

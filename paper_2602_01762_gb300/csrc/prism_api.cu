@@ -72,6 +72,7 @@ struct prism_ctx {
     int gemv_cuda_core = 1;                               // 1: bf16 projections on CUDA cores
     int gemv_tcgen05 = 1;                                 // 1: bf16 projections on tcgen05 where they fit
     int attn_fused = 1;                                   // 1: fused RoPE/append/attention cluster kernel
+    int tc_stream_rows = 17;                              // tcgen05 projections with this many rows or more stream X
     int attn_max_cs = 8;                                  // largest cluster the device co-schedules
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
     bool tc_ready = false;
@@ -179,7 +180,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
     // measured slower there)
     auto proj = [&](const GemvArgs &g, const CUtensorMap *tm, int grid, bool pdl_here) -> cudaError_t {
         const bool want = c->gemv_tcgen05 == 2 || (c->gemv_tcgen05 == 1 && (g.epi != kEpiSwiGLU || g.T > 2));
-        if (tm && want && c->tc_ready && c->bf16 && g.T > 16 && gemv_tcs_supported(g, c->sms)) {
+        if (tm && want && c->tc_ready && c->bf16 && g.T >= c->tc_stream_rows && gemv_tcs_supported(g, c->sms)) {
             const size_t ws = gemv_tcs_workspace_floats(g, c->sms);
             if (ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n))
                 return launch_gemv_tcs(g, *tm, c->sms, c->tc_part, c->tc_ctr, c->xbuf, s, pdl_here);
@@ -634,6 +635,7 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "gemv_cuda_core")) c->gemv_cuda_core = value != 0;
     else if (!std::strcmp(name, "gemv_tcgen05") && value >= 0 && value <= 2) c->gemv_tcgen05 = value;
     else if (!std::strcmp(name, "attn_fused")) c->attn_fused = value != 0;
+    else if (!std::strcmp(name, "tc_stream_rows") && value >= 1) c->tc_stream_rows = value;
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);
     return PRISM_OK;
