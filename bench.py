@@ -322,6 +322,7 @@ def run_ours(args, w, world, rank, local):
     ms_local = ev0.elapsed_time(ev1)
     ms = dist_reduce(ms_local, "max", world, dev if world > 1 else None)
     flags = dr.sync_status(stream)
+    launches_per_round = dr.round_launches()
     tokens_total = B * K * args.steps * world
     value = tokens_total / (ms / 1e3)
     per_round_ms = ms / args.steps
@@ -400,7 +401,7 @@ def run_ours(args, w, world, rank, local):
             "kernel_ms_per_round": kind_total,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-            "gpu_launches": len(prof[0]) * args.steps,
+            "gpu_launches": launches_per_round * args.steps,
             "clocks": clk,
             "device_error_word": flags,
         }

@@ -204,7 +204,7 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * loads into tensor-memory accumulators, except gate/up + SwiGLU with at
  * most 2 activation rows, which measures faster on the CUDA-core kernel;
  * 2: gate/up as well; 0: every projection on the kernels below),
- * "tc_stream_rows" (>= 1, default 17: a tcgen05 projection with at least
+ * "tc_stream_rows" (>= 1, default 9: a tcgen05 projection with at least
  * this many activation rows streams them through the TMA ring beside the
  * weights instead of staging them whole in shared memory; at most 16 rows
  * can be staged), "gemv_cuda_core" (for projections
@@ -216,6 +216,13 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * Changing an option drops cached graphs.  Errors: INVALID_ARG (unknown name
  * or value out of range). */
 prism_status prism_set_option(prism_ctx *ctx, const char *name, int32_t value);
+
+/* Kernel launches of one round: the kernel nodes of the CUDA graph that the
+ * most recent prism_draft_round call (with "use_graph" on) replayed.  The
+ * count depends on the batch and the options (a projection may take one to
+ * three kernels).  Errors: INVALID_ARG (null argument, or no round replayed
+ * from a graph yet). */
+prism_status prism_round_launches(prism_ctx *ctx, int32_t *n_launches);
 
 /* Instrumented round for measurement: the same work as prism_draft_round
  * launched eagerly with a CUDA event recorded before and after every kernel.

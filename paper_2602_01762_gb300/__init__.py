@@ -64,11 +64,12 @@ def library() -> ctypes.CDLL:
         lib.prism_profile_round.argtypes = [vp, i32] + [vp] * 10 + [P(ctypes.c_float), P(i32), i32, P(i32)]
         lib.prism_lm_head_topk_static.argtypes = [i32] * 5 + [ctypes.c_float] + [vp] * 9
         lib.prism_get_error.argtypes = [vp]
+        lib.prism_round_launches.argtypes = [vp, P(i32)]
         lib.prism_get_error.restype = ctypes.c_char_p
         lib.prism_version.restype = ctypes.c_char_p
         for f in ("prism_create", "prism_destroy", "prism_load_shared_weights", "prism_load_step_weights",
                   "prism_draft_round", "prism_accept_greedy", "prism_sync_status", "prism_set_option",
-                  "prism_profile_round", "prism_lm_head_topk_static"):
+                  "prism_profile_round", "prism_lm_head_topk_static", "prism_round_launches"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -191,6 +192,12 @@ class Drafter:
             self.h, B, _ptr(tokens), _ptr(hidden), _ptr(n_new), _ptr(kv_len), _ptr(k_cache),
             _ptr(v_cache), _ptr(draft_ids), _ptr(topk_ids), _ptr(topk_logits), _ptr(logits),
             _ptr(hidden_out), _stream(stream)))
+
+    def round_launches(self) -> int:
+        """Kernel launches of the last round replayed from a CUDA graph."""
+        n = ctypes.c_int32(0)
+        self._check(self.lib.prism_round_launches(self.h, ctypes.byref(n)))
+        return int(n.value)
 
     def profile_round(self, tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids,
                       topk_ids=None, topk_logits=None, stream=None):

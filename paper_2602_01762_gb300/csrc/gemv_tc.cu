@@ -175,6 +175,7 @@ struct TcPlan {
     uint32_t stage_bytes, x_bytes;
     float *part;        // split-K partial sums [splits][RPW][T][n_units]
     int *tile_ctr;      // per-tile arrival tickets (left at zero)
+    int defer;          // split-K sums finished by splitk_finish_kernel, not the tile's last CTA
 };
 
 // X rows (bf16, swizzled K-major operand layout) for the K blocks [kb0, kb1).
@@ -342,6 +343,58 @@ __device__ __forceinline__ void unpack_best(unsigned long long key, float &v, in
     const uint32_t k = (uint32_t)(key >> 32);
     v = __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
     id = (int)(0xFFFFFFFFu - (uint32_t)key);
+}
+
+// Split-K: the last CTA of a tile adds the K slices of unit u for every
+// activation row, in slice order, and finishes the unit.  The partial sums
+// come from other SMs through L2, so the loads of several rows and all their
+// slices (32 values; SB bounds the slice count) are issued before any is
+// used: the round trips are T / C rather than T x splits.
+template <int RPW, int SB>
+__device__ __forceinline__ void reduce_slices_sb(const GemvArgs &a, const TcPlan &p, int T, int u) {
+    constexpr int C = 32 / (SB * RPW);             // rows per batch of loads
+    const int splits = p.splits;
+#pragma unroll 1
+    for (int t0 = 0; t0 < T; t0 += C) {
+        float v[C][SB][RPW];
+#pragma unroll
+        for (int c = 0; c < C; ++c)
+#pragma unroll
+            for (int k = 0; k < SB; ++k)
+#pragma unroll
+                for (int r = 0; r < RPW; ++r)
+                    v[c][k][r] = (t0 + c < T && k < splits)
+                                     ? __ldcg(&p.part[(((size_t)k * RPW + r) * T + t0 + c) * a.n_units + u])
+                                     : 0.f;
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+            if (t0 + c >= T) break;
+            float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+            for (int k = 0; k < SB; ++k)
+                if (k < splits) {
+                    s0 += v[c][k][0];
+                    s1 += v[c][k][RPW - 1];
+                }
+            finish_unit<RPW>(a, t0 + c, u, s0, s1);
+        }
+    }
+}
+template <int RPW>
+__device__ __forceinline__ void reduce_slices(const GemvArgs &a, const TcPlan &p, int T, int u) {
+    if (T <= 4) {
+        // few rows: the short loop (this code runs cold, once per tile)
+        for (int t = 0; t < T; ++t) {
+            float v0 = 0.f, v1 = 0.f;
+            for (int k = 0; k < p.splits; ++k) {
+                v0 += __ldcg(&p.part[(((size_t)k * RPW + 0) * T + t) * a.n_units + u]);
+                if (RPW == 2) v1 += __ldcg(&p.part[(((size_t)k * RPW + 1) * T + t) * a.n_units + u]);
+            }
+            finish_unit<RPW>(a, t, u, v0, v1);
+        }
+    } else if (p.splits <= 2) reduce_slices_sb<RPW, 2>(a, p, T, u);
+    else if (p.splits <= 4) reduce_slices_sb<RPW, 4>(a, p, T, u);
+    else reduce_slices_sb<RPW, kMaxSplits>(a, p, T, u);
 }
 
 // ---------------------------------------------------------------- top-k lists
@@ -731,16 +784,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     epi_sync();
                     if (s_last) {
                         __threadfence();
-                        if (valid) {
-                            for (int t = 0; t < T; ++t) {
-                                float v0 = 0.f, v1 = 0.f;
-                                for (int k2 = 0; k2 < p.splits; ++k2) {
-                                    v0 += __ldcg(&p.part[(((size_t)k2 * RPW + 0) * T + t) * a.n_units + u]);
-                                    if (RPW == 2) v1 += __ldcg(&p.part[(((size_t)k2 * RPW + 1) * T + t) * a.n_units + u]);
-                                }
-                                finish_unit<RPW>(a, t, u, v0, v1);
-                            }
-                        }
+                        if (valid) reduce_slices<RPW>(a, p, T, u);
                         if (threadIdx.x == 64) p.tile_ctr[tile] = 0;
                     }
                     epi_sync();
@@ -1029,23 +1073,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     if (lane == 0) mbar_arrive(&acc_empty[ab]);
                 }
                 if constexpr (!TOPK) {
-                    if (p.splits > 1) {
+                    if (p.splits > 1 && !p.defer) {
                         __threadfence();
                         epi_sync();
                         if (threadIdx.x == 64) s_last = atomicAdd(&p.tile_ctr[tile], 1) == p.splits - 1;
                         epi_sync();
                         if (s_last) {
                             __threadfence();
-                            if (valid) {
-                                for (int t = 0; t < T; ++t) {
-                                    float v0 = 0.f, v1 = 0.f;
-                                    for (int k2 = 0; k2 < p.splits; ++k2) {
-                                        v0 += __ldcg(&p.part[(((size_t)k2 * RPW + 0) * T + t) * a.n_units + u]);
-                                        if (RPW == 2) v1 += __ldcg(&p.part[(((size_t)k2 * RPW + 1) * T + t) * a.n_units + u]);
-                                    }
-                                    finish_unit<RPW>(a, t, u, v0, v1);
-                                }
-                            }
+                            if (valid) reduce_slices<RPW>(a, p, T, u);
                             if (threadIdx.x == 64) p.tile_ctr[tile] = 0;
                         }
                         epi_sync();
@@ -1064,6 +1099,36 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     stage_sync();
     tc_fence_after();
     if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kCols));
+}
+
+// Split-K sums of a streamed projection with many activation rows: the
+// projection kernel only publishes its slices, and this kernel adds them, one
+// thread per (row t, unit u) with all slices loaded at once, in slice order
+// (the same sums as the last-CTA path), and finishes the unit.  Inline in the
+// projection, the last CTA of a tile would read T x 128 x splits partial sums
+// through L2 while the tile's other work waits behind it.
+template <int RPW>
+__global__ void __launch_bounds__(256) splitk_finish_kernel(const GemvArgs a, const float *part, int splits) {
+    pdl_trigger();
+    pdl_wait();
+    const long total = (long)a.T * a.n_units;
+    const long e = (long)blockIdx.x * 256 + threadIdx.x;
+    if (e >= total) return;
+    const int t = (int)(e / a.n_units), u = (int)(e % a.n_units);
+    float v[kMaxSplits][RPW];
+#pragma unroll
+    for (int k = 0; k < kMaxSplits; ++k)
+#pragma unroll
+        for (int r = 0; r < RPW; ++r)
+            v[k][r] = k < splits ? __ldcg(&part[(((size_t)k * RPW + r) * a.T + t) * a.n_units + u]) : 0.f;
+    float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+    for (int k = 0; k < kMaxSplits; ++k)
+        if (k < splits) {
+            s0 += v[k][0];
+            s1 += v[k][RPW - 1];
+        }
+    finish_unit<RPW>(a, t, u, s0, s1);
 }
 
 // Cross-CTA top-k merge of the streamed LM head: one CTA (4 warps) per row;
@@ -1368,6 +1433,7 @@ cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, f
     if (!tcs_plan(a, sms, p, grid, smem, NB)) return cudaErrorInvalidValue;
     p.part = part;
     p.tile_ctr = tile_ctr;
+    p.defer = p.splits > 1;
     if (p.splits > 1 && (!part || !tile_ctr)) return cudaErrorInvalidValue;
     // the activation rows as a bf16 [T][kin] buffer: the copy prologue's
     // source as it is, otherwise written by prep_x_kernel
@@ -1402,6 +1468,11 @@ cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, f
     }
     if (e == cudaSuccess && a.epi == kEpiTopK)
         e = launch_k(topk_merge_kernel, dim3(a.T), dim3(128), 0, s, true, a, grid);
+    if (e == cudaSuccess && p.defer) {
+        const dim3 fg((unsigned)(((long)a.T * a.n_units + 255) / 256));
+        e = a.epi == kEpiSwiGLU ? launch_k(splitk_finish_kernel<2>, fg, dim3(256), 0, s, true, a, (const float *)part, p.splits)
+                                : launch_k(splitk_finish_kernel<1>, fg, dim3(256), 0, s, true, a, (const float *)part, p.splits);
+    }
     return e;
 }
 

@@ -33,6 +33,7 @@ struct GraphEntry {
     bool pdl;
     cudaGraphExec_t exec;
     unsigned long long used;
+    int kernels;        // kernel nodes of the captured round
 };
 
 thread_local std::string g_error;
@@ -72,7 +73,7 @@ struct prism_ctx {
     int gemv_cuda_core = 1;                               // 1: bf16 projections on CUDA cores
     int gemv_tcgen05 = 1;                                 // 1: bf16 projections on tcgen05 where they fit
     int attn_fused = 1;                                   // 1: fused RoPE/append/attention cluster kernel
-    int tc_stream_rows = 17;                              // tcgen05 projections with this many rows or more stream X
+    int tc_stream_rows = 9;                               // tcgen05 projections with this many rows or more stream X
     int attn_max_cs = 8;                                  // largest cluster the device co-schedules
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
     bool tc_ready = false;
@@ -86,6 +87,7 @@ struct prism_ctx {
     int tc_ctr_n = 0;
     uint16_t *xbuf = nullptr;                             // bf16 activation rows of the streamed kernel
     std::vector<GraphEntry> graphs;
+    int last_round_kernels = -1;                          // kernel launches of the last replayed round
     unsigned long long tick = 0;
     std::string error;
 };
@@ -677,16 +679,35 @@ prism_status prism_draft_round(prism_ctx *c, int32_t batch, const int32_t *token
             return cuda_fail(c, le, "kernel launch during capture");
         }
         if (e != cudaSuccess) return cuda_fail(c, e, "cudaStreamEndCapture");
+        // the round's kernel launches, as the graph holds them
+        int kernels = 0;
+        size_t n_nodes = 0;
+        if (cudaGraphGetNodes(graph, nullptr, &n_nodes) == cudaSuccess && n_nodes > 0) {
+            std::vector<cudaGraphNode_t> nodes(n_nodes);
+            if (cudaGraphGetNodes(graph, nodes.data(), &n_nodes) == cudaSuccess)
+                for (size_t i = 0; i < n_nodes; ++i) {
+                    cudaGraphNodeType t;
+                    if (cudaGraphNodeGetType(nodes[i], &t) == cudaSuccess && t == cudaGraphNodeTypeKernel) ++kernels;
+                }
+        }
         cudaGraphExec_t exec = nullptr;
         e = cudaGraphInstantiate(&exec, graph, 0);
         cudaGraphDestroy(graph);
         if (e != cudaSuccess) return cuda_fail(c, e, "cudaGraphInstantiate");
-        c->graphs.push_back(GraphEntry{r, c->use_pdl, exec, 0});
+        c->graphs.push_back(GraphEntry{r, c->use_pdl, exec, 0, kernels});
         hit = &c->graphs.back();
     }
     hit->used = ++c->tick;
+    c->last_round_kernels = hit->kernels;
     e = cudaGraphLaunch(hit->exec, s);
     return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "cudaGraphLaunch");
+}
+
+prism_status prism_round_launches(prism_ctx *c, int32_t *n_launches) {
+    if (!c || !n_launches) return fail(c, PRISM_ERR_INVALID_ARG, "null argument");
+    if (c->last_round_kernels < 0) return fail(c, PRISM_ERR_INVALID_ARG, "no round has been replayed from a graph");
+    *n_launches = c->last_round_kernels;
+    return PRISM_OK;
 }
 
 prism_status prism_profile_round(prism_ctx *c, int32_t batch, const int32_t *tokens, const void *hidden,
