@@ -628,31 +628,50 @@ __global__ void __launch_bounds__(kFusedThreads, 1) fused_attention_kernel(const
     cluster_sync_all();
 }
 
-// Tensor-core variant for bf16 caches: S = Q K^T and O += P V as mma.sync
-// m16n8k16 tiles (16 rows = the query heads of g, padded).  The contract keeps
-// q and the probabilities in fp32, so each enters the product as a bf16 pair
-// hi + lo (hi = bf16(x), lo = bf16(x - hi)): two MMAs per tile, an error near
-// 2^-17 of the operand, with K and V exact.  Every shared-memory operand tile
-// (keys, values, hi/lo queries and probabilities) is stored with its 16-byte
-// pieces XOR-swizzled by row, so ldmatrix reads are free of bank conflicts.
-constexpr int kMmaC = 160;                            // keys per chunk (multiple of 32)
-constexpr int kMmaPS = (kMmaC + 63) / 64 * 64;        // probability row stride: whole 8-piece groups
+// Tensor-core variant for bf16 caches, with the products transposed so that
+// keys fill the MMA's 16-row M dimension and the G <= 8 query heads of g its
+// 8-column N dimension:
+//   S^T[key][h]  = K[key][:] . q[h][:]       A = 16 keys of K (ldmatrix),
+//                                            B = q^T, held in registers;
+//   O^T[d][h]   += V^T[d][keys] P^T[keys][h]  A = V^T (transposing ldmatrix),
+//                                            B = P^T (movmatrix of the S^T tile).
+// The contract keeps q and the probabilities in fp32, so each enters a product
+// as a bf16 pair hi + lo (hi = bf16(x), lo = bf16(x - hi)): two MMAs per tile,
+// an error near 2^-17 of the operand, with K and V exact.  Shared memory holds
+// only K and V as TMA wrote them (128-byte swizzle), and each of their bytes is
+// read once.
+//   * Keys stream through a ring of kTaStages stages of kTaC rows, filled by
+//     one producer warp with TMA tensor loads; stages made only of rows
+//     committed before the round are requested before griddepcontrol.wait;
+//   * compute warp w owns keys 16w .. 16w + 15 of every stage and keeps its own
+//     online softmax (running max, sum and O^T per head), so a stage needs no
+//     block-wide barrier: each warp releases it through an mbarrier;
+//   * at the end the warps' states merge in shared memory (log-sum-exp rule,
+//     warp order), then the cluster's ranks merge through distributed shared
+//     memory as in the CUDA-core kernel.
+constexpr int kTaWarps = 8;                           // compute warps; one more warp issues loads
+constexpr int kTaThreads = (kTaWarps + 1) * 32;
+constexpr int kTaC = kTaWarps * 16;                   // keys per stage
+constexpr int kTaStages = 3;
 
-__device__ __forceinline__ uint32_t swz(int row, int slot) { return (uint32_t)(slot ^ (row & 7)); }
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(addr));
 }
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t (&r)[4]) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(addr));
 }
-__device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
-                                         uint32_t b0, uint32_t b1) {
+__device__ __forceinline__ uint32_t movm_t(uint32_t x) {
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
+}
+__device__ __forceinline__ void mma16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
     asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
                  "{%8, %9}, {%0, %1, %2, %3};"
                  : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-                 : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 // bf16 hi/lo split of two floats, packed (low half = first element).
 __device__ __forceinline__ void split2(float x, float y, uint32_t &hi, uint32_t &lo) {
@@ -660,36 +679,48 @@ __device__ __forceinline__ void split2(float x, float y, uint32_t &hi, uint32_t 
     hi = (uint32_t)hx | ((uint32_t)hy << 16);
     lo = (uint32_t)f32_to_bf16(x - bf16_to_f32(hx)) | ((uint32_t)f32_to_bf16(y - bf16_to_f32(hy)) << 16);
 }
+// Whole-warp bounded wait on an mbarrier phase: lane 0 polls, every lane then
+// observes the completed phase itself.  Warp-uniform result.
+__device__ __forceinline__ bool ta_wait_warp(uint64_t *bar, uint32_t parity) {
+    bool ok = true;
+    if ((threadIdx.x & 31) == 0) {
+        ok = false;
+        for (long it = 0; it < kAttnWaitLimit && !ok; ++it) ok = fa_try(bar, parity);
+    }
+    ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+    if (ok) fa_try(bar, parity);
+    return ok;
+}
+// Shared-memory address of 16-byte piece `chunk` (8 dims) of row `row` of a
+// stage buffer: D / 64 boxes of kTaC rows x 128 bytes, pieces XOR-swizzled by
+// row (the TMA 128-byte swizzle).
+__device__ __forceinline__ uint32_t ta_piece(uint32_t buf, int row, int chunk) {
+    return buf + (uint32_t)(chunk >> 3) * (kTaC * 128) + (uint32_t)row * 128 + ((uint32_t)((chunk & 7) ^ (row & 7)) << 4);
+}
 
 template <int D>
-__global__ void __launch_bounds__(kFusedThreads, 1)
-    fused_attention_mma_kernel(const FusedAttnArgs a, const __grid_constant__ CUtensorMap tk,
-                               const __grid_constant__ CUtensorMap tv) {
-    constexpr int C = kMmaC;
+__global__ void __launch_bounds__(kTaThreads, 1)
+    fused_attention_tc_kernel(const FusedAttnArgs a, const __grid_constant__ CUtensorMap tk,
+                              const __grid_constant__ CUtensorMap tv) {
     constexpr int NH = D / 64;                        // 64-column boxes per row
-    constexpr uint32_t kBox = C * 128;                // one box: C rows x 128 bytes
+    constexpr uint32_t kBox = kTaC * 128;
+    constexpr uint32_t kStage = 2 * NH * kBox;        // K boxes, then V boxes
+    constexpr int NT = D / 16;                        // 16-dim tiles
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full[2];
-    __shared__ float s_m[16], s_l[16], s_alpha[16];
-    __shared__ float red_max[kFusedThreads / 32][16], red_sum[kFusedThreads / 32][16];
-    const int G = a.Hq / a.Hkv;
-    // K and V chunks as TMA wrote them: per buffer NH boxes of C rows x 128 B,
-    // 16-byte piece c of row r at (c ^ (r % 8)) (128-byte swizzle, 1 KB atoms)
-    uint8_t *base = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint16_t *kbuf = (uint16_t *)base;                // [2][NH][C][64]
-    uint16_t *vbuf = kbuf + 2 * C * D;                // [2][NH][C][64]
-    uint16_t *qhi = vbuf + 2 * C * D;                 // [16][D] swizzled
-    uint16_t *qlo = qhi + 16 * D;
-    uint16_t *phi = qlo + 16 * D;                     // [16][kMmaPS] swizzled
-    uint16_t *plo = phi + 16 * kMmaPS;
-    float *qs = (float *)(plo + 16 * kMmaPS);         // [16][D] rotated, scaled queries
-    float *po = qs + 16 * D;                          // [16][D] this rank's unnormalised output
-    float *pm = po + 16 * D;                          // [16]
-    float *pl = pm + 16;                              // [16]
+    __shared__ __align__(8) uint64_t full[kTaStages], empty[kTaStages];
+    uint8_t *ring = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    float *qs = (float *)(ring + kTaStages * kStage);  // [8][D] rotated, scaled queries (heads >= G zero)
+    float *po = qs + 8 * D;                            // [G][D] this rank's unnormalised output
+    float *pm = po + 8 * D;                            // [8]
+    float *pl = pm + 8;                                // [8]
+    // after the key loop the ring holds the warps' states
+    float *wo = (float *)ring;                         // [warp][8][D]
+    float *wm = wo + kTaWarps * 8 * D;                 // [warp][8]
+    float *wl = wm + kTaWarps * 8;                     // [warp][8]
 
     const int r = blockIdx.x, g = blockIdx.y, b = blockIdx.z, CS = a.cs;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int half = D / 2, H = a.Hq + 2 * a.Hkv;
+    const int half = D / 2, H = a.Hq + 2 * a.Hkv, G = a.Hq / a.Hkv;
     pdl_trigger();
 
     const int n = clamp_n(a.n_new, b, a.max_new, a.err);
@@ -699,52 +730,45 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
     if (P > a.max_ctx) P = a.max_ctx;
     if (P < 1) P = 1;
     const int j0 = (int)((long)r * P / CS), j1 = (int)((long)(r + 1) * P / CS);
-    const int nch = (j1 - j0 + C - 1) / C;
+    const int nst = (j1 - j0 + kTaC - 1) / kTaC;
     const int L_old = L < P ? (L > 0 ? L : 0) : P;
-    auto chunk = [&](int i, int &j, int &cnt) {
-        j = j0 + i * C;
-        cnt = j1 - j < C ? j1 - j : C;
-    };
-    // request chunk i into buffer i & 1: 2 NH boxes (K and V) of C rows from
-    // position j of head (b, g); rows past max_ctx arrive as zeros (thread 0)
-    int n_iss0 = 0, n_iss1 = 0;
+    const uint32_t ring_s = sa(ring);
+
+    // stage i -> ring slot i % kTaStages: NH boxes of K and NH of V from row
+    // j0 + i * kTaC of head (b, g); rows past max_ctx arrive as zeros
     auto load = [&](int i) {
-        int j, cnt;
-        chunk(i, j, cnt);
-        uint64_t *bar = &full[i & 1];
-        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(sa(bar)), "r"(2 * NH * kBox)
+        const int s = i % kTaStages, j = j0 + i * kTaC, z = b * a.Hkv + g;
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(sa(&full[s])), "r"(kStage)
                      : "memory");
-        const int z = b * a.Hkv + g;
-        const uint32_t kd = sa(kbuf + (i & 1) * C * D), vd = sa(vbuf + (i & 1) * C * D);
+        const uint32_t kd = ring_s + (uint32_t)s * kStage, vd = kd + NH * kBox;
 #pragma unroll
         for (int h = 0; h < NH; ++h) {
             asm volatile(
                 "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
-                "%4}], [%5];" ::"r"(kd + h * kBox), "l"((uint64_t)&tk), "r"(h * 64), "r"(j), "r"(z), "r"(sa(bar))
+                "%4}], [%5];" ::"r"(kd + h * kBox), "l"((uint64_t)&tk), "r"(h * 64), "r"(j), "r"(z), "r"(sa(&full[s]))
                 : "memory");
             asm volatile(
                 "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
-                "%4}], [%5];" ::"r"(vd + h * kBox), "l"((uint64_t)&tv), "r"(h * 64), "r"(j), "r"(z), "r"(sa(bar))
+                "%4}], [%5];" ::"r"(vd + h * kBox), "l"((uint64_t)&tv), "r"(h * 64), "r"(j), "r"(z), "r"(sa(&full[s]))
                 : "memory");
         }
-        if (i & 1) ++n_iss1; else ++n_iss0;
     };
-    if (tid == 0) {
-        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(sa(&full[0])));
-        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(sa(&full[1])));
+    const bool producer = tid == kTaWarps * 32;
+    if (producer) {
+        for (int s = 0; s < kTaStages; ++s) {
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(sa(&full[s])));
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(sa(&empty[s])), "r"(kTaWarps));
+        }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tk) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tv) : "memory");
     }
     __syncthreads();
+    // stages made only of committed rows do not wait for the QKV projection
     int pre = 0;
-    for (int i = 0; i < 2 && i < nch; ++i) {
-        int j, cnt;
-        chunk(i, j, cnt);
-        if (j + cnt > L_old) break;
-        if (tid == 0) load(i);
-        ++pre;
-    }
+    while (pre < kTaStages && pre < nst && min(j0 + (pre + 1) * kTaC, j1) <= L_old) ++pre;
+    if (producer)
+        for (int i = 0; i < pre; ++i) load(i);
     pdl_wait();
 
     // append the new rows this rank owns
@@ -761,20 +785,20 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
         const float *xv = a.qkv + (size_t)row * H * D + (size_t)(a.Hq + a.Hkv + g) * D;
         uint16_t *kc = (uint16_t *)a.k_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + pos) * D;
         uint16_t *vc = (uint16_t *)a.v_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + pos) * D;
-        for (int j = tid; j < half; j += kFusedThreads) {
+        for (int j = tid; j < half; j += kTaThreads) {
             const float c = a.rope_cos[(size_t)pos * half + j], sn = a.rope_sin[(size_t)pos * half + j];
             const float x0 = xk[j], x1 = xk[j + half];
             kc[j] = f32_to_bf16(x0 * c - x1 * sn);
             kc[j + half] = f32_to_bf16(x1 * c + x0 * sn);
         }
-        for (int j = tid; j < D; j += kFusedThreads) vc[j] = f32_to_bf16(xv[j]);
+        for (int j = tid; j < D; j += kTaThreads) vc[j] = f32_to_bf16(xv[j]);
     }
-    // queries (rows >= G zero), rotated and scaled, fp32 and split hi/lo
+    // queries (heads >= G zero), rotated and scaled by 1/sqrt(D)
     {
         const int row = a.prefill ? b * a.max_new + n - 1 : b;
         const int pc = qp >= 0 && qp < a.max_ctx ? qp : 0;
         const float scale = 1.0f / sqrtf((float)D);
-        for (int e = tid; e < 16 * half; e += kFusedThreads) {
+        for (int e = tid; e < 8 * half; e += kTaThreads) {
             const int h = e / half, j = e % half;
             float y0 = 0.f, y1 = 0.f;
             if (h < G) {
@@ -788,207 +812,191 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
             qs[h * D + j + half] = y1;
         }
     }
-    if (tid < 16) { s_m[tid] = -INFINITY; s_l[tid] = 0.f; }
-    __syncthreads();
-    for (int e = tid; e < 16 * D / 2; e += kFusedThreads) {      // pairs of dims
-        const int h = e / (D / 2), d = 2 * (e % (D / 2));
-        uint32_t hi, lo;
-        split2(qs[h * D + d], qs[h * D + d + 1], hi, lo);
-        const uint32_t o = (uint32_t)(h * D + swz(h, d / 8) * 8 + d % 8);
-        *(uint32_t *)(qhi + o) = hi;
-        *(uint32_t *)(qlo + o) = lo;
-    }
     // the async proxy reads rows this kernel just wrote: order those writes first
     asm volatile("fence.proxy.async.global;" ::: "memory");
     __syncthreads();
-    if (tid == 0)
-        for (int i = pre; i < 2 && i < nch; ++i) load(i);
-    bool dead = false;
 
-    float oq4[4][4] = {};                             // O tile: rows lane/4 (+8), dims of this warp,
-                                                      // in four chains (hi / lo x even / odd keys)
-    const int g4 = lane >> 2, t4 = lane & 3;
-    for (int ci = 0; ci < nch; ++ci) {
-        const int bi = ci & 1;
-        int j, cnt;
-        chunk(ci, j, cnt);
-        const uint16_t *kb = kbuf + bi * C * D, *vb = vbuf + bi * C * D;
-        if (!dead) {
-            bool ok = false;
-            for (long it = 0; it < kAttnWaitLimit && !ok; ++it) ok = fa_try(&full[bi], (uint32_t)((ci >> 1) & 1));
-            if (!ok) {
-                if (tid == 0) set_err(a.err, kErrTimeout);
+    bool dead = false;
+    // compute-warp state: entries for keys lane / 4 (+ 8) of the warp's 16 and
+    // heads h0 = 2 (lane % 4), h1 = h0 + 1; O^T for dims 16 t + lane / 4 (+ 8)
+    constexpr int NTO = NT;
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+    float o[NTO][4];
+#pragma unroll
+    for (int t = 0; t < NTO; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
+    if (warp == kTaWarps) {
+        // ---------------------------------------------------------------- producer
+        if (producer) {
+            int issued = pre;
+            for (int i = pre; i < nst && !dead; ++i) {
+                if (i >= kTaStages) {
+                    // slot i % S is free once every warp has released stage i - S
+                    bool ok = false;
+                    const uint32_t par = (uint32_t)((i / kTaStages - 1) & 1);
+                    for (long it = 0; it < kAttnWaitLimit && !ok; ++it) ok = fa_try(&empty[i % kTaStages], par);
+                    if (!ok) {
+                        set_err(a.err, kErrTimeout);
+                        dead = true;
+                        break;
+                    }
+                }
+                load(i);
+                issued = i + 1;
+            }
+            // every copy issued lands before the ring is reused or the CTA exits
+            for (int i = issued > kTaStages ? issued - kTaStages : 0; i < issued; ++i) {
+                bool ok = false;
+                for (long it = 0; it < kAttnWaitLimit && !ok; ++it)
+                    ok = fa_try(&full[i % kTaStages], (uint32_t)((i / kTaStages) & 1));
+                if (!ok) set_err(a.err, kErrTimeout);
+            }
+        }
+    } else {
+        // ---------------------------------------------------------------- compute warps
+        // q^T as B fragments: b0 = q[h][16 ks + 2 (lane % 4) + {0, 1}], b1 = the same dims + 8, h = lane / 4
+        uint32_t qh[NT][2], ql[NT][2];
+#pragma unroll
+        for (int ks = 0; ks < NT; ++ks)
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const float *src = qs + (lane >> 2) * D + 16 * ks + 2 * (lane & 3) + 8 * u;
+                split2(src[0], src[1], qh[ks][u], ql[ks][u]);
+            }
+        const int kr = 16 * warp;                     // this warp's first row in a stage
+        for (int i = 0; i < nst; ++i) {
+            const int s = i % kTaStages;
+            if (!dead && !ta_wait_warp(&full[s], (uint32_t)((i / kTaStages) & 1))) {
+                if (lane == 0) set_err(a.err, kErrTimeout);
                 dead = true;
             }
-        }
-        // value rows past the chunk end hold other positions' data: zero them
-        // (their probabilities are zero, and 0 * NaN would not be)
-        if (cnt < C)
-            for (int e = tid; e < (C - cnt) * (D / 8); e += kFusedThreads) {
-                const int row = cnt + e / (D / 8), sl = e % (D / 8);
-                *(uint4 *)((uint8_t *)vb + (sl >> 3) * kBox + row * 128 + (((sl & 7) ^ (row & 7)) << 4)) =
-                    make_uint4(0, 0, 0, 0);
-            }
-        __syncthreads();
-        // S tiles of this warp: 16 rows x keys 8 nt .. 8 nt + 7 for nt = w, w + 16,
-        // each as four independent accumulation chains (hi / lo x even / odd k-steps)
-        constexpr int NT = C / 8, NTW = (NT + 15) / 16;
-        float sv[NTW][4];
-#pragma unroll
-        for (int t = 0; t < NTW; ++t) {
-            const int nt = warp + 16 * t;
-            float sq[4][4] = {};
-            if (nt < NT) {
-                const int kn = nt * 8;
-#pragma unroll
-                for (int ks = 0; ks < D / 16; ks += 2) {
-                    uint32_t b0, b1, b2, b3, a0, a1, a2, a3;
-                    {
-                        const int key = kn + (lane & 7), slot = 2 * ks + (lane >> 3);
-                        ldsm_x4(sa(kb) + (slot >> 3) * kBox + key * 128 + (((slot & 7) ^ (key & 7)) << 4), b0, b1,
-                                b2, b3);
+            const int key0 = j0 + i * kTaC + kr;     // position of the warp's first key
+            const int cnt = min(16, j1 - key0);       // valid keys of the warp (may be <= 0)
+            if (!dead && cnt > 0) {
+                const uint32_t kb = ring_s + (uint32_t)s * kStage, vb = kb + NH * kBox;
+                // value rows past the range hold other positions' data: zero them
+                // (their probabilities are zero, and 0 * NaN would not be)
+                if (cnt < 16) {
+                    for (int e = lane; e < (16 - cnt) * NH * 8; e += 32) {
+                        const int row = kr + cnt + e / (NH * 8), piece = e % (NH * 8);
+                        asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" ::"r"(ta_piece(vb, row, piece)), "r"(0)
+                                     : "memory");
                     }
-#pragma unroll
-                    for (int u = 0; u < 2; ++u) {
-                        const int kk = ks + u;
-                        const int qrow = (lane & 7) + ((lane >> 3) & 1) * 8, qslot = 2 * kk + (lane >> 4);
-                        const uint32_t qo = (uint32_t)(qrow * D + swz(qrow, qslot) * 8);
-                        const uint32_t bb0 = u ? b2 : b0, bb1 = u ? b3 : b1;
-                        ldsm_x4(sa(qhi + qo), a0, a1, a2, a3);
-                        mma16816(sq[2 * u], a0, a1, a2, a3, bb0, bb1);
-                        ldsm_x4(sa(qlo + qo), a0, a1, a2, a3);
-                        mma16816(sq[2 * u + 1], a0, a1, a2, a3, bb0, bb1);
-                    }
+                    __syncwarp();
                 }
-            }
-            // rows g4 and g4 + 8, keys 8 nt + 2 t4 + {0, 1}; keys past the chunk are -inf
-            const int key0 = nt * 8 + 2 * t4;
+                // S^T for 16 keys x 8 heads, hi and lo queries in separate chains
+                float sh[4] = {0.f, 0.f, 0.f, 0.f}, sl[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const float v = (sq[0][q] + sq[1][q]) + (sq[2][q] + sq[3][q]);
-                sv[t][q] = nt < NT && key0 + (q & 1) < cnt ? v : -INFINITY;
-            }
-        }
-        // online softmax over the chunk
-        float m0 = -INFINITY, m1 = -INFINITY;
-#pragma unroll
-        for (int t = 0; t < NTW; ++t) {
-            m0 = fmaxf(m0, fmaxf(sv[t][0], sv[t][1]));
-            m1 = fmaxf(m1, fmaxf(sv[t][2], sv[t][3]));
-        }
-#pragma unroll
-        for (int o = 1; o <= 2; o <<= 1) {
-            m0 = fmaxf(m0, __shfl_xor_sync(0xFFFFFFFFu, m0, o));
-            m1 = fmaxf(m1, __shfl_xor_sync(0xFFFFFFFFu, m1, o));
-        }
-        if (t4 == 0) { red_max[warp][g4] = m0; red_max[warp][g4 + 8] = m1; }
-        __syncthreads();
-        float mn0 = s_m[g4], mn1 = s_m[g4 + 8];
-#pragma unroll
-        for (int w = 0; w < kFusedThreads / 32; ++w) {
-            mn0 = fmaxf(mn0, red_max[w][g4]);
-            mn1 = fmaxf(mn1, red_max[w][g4 + 8]);
-        }
-        float r0s = 0.f, r1s = 0.f;
-#pragma unroll
-        for (int t = 0; t < NTW; ++t) {
-            const int nt = warp + 16 * t;
-            if (nt >= NT) continue;
-            float pv[4];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const float mq = q < 2 ? mn0 : mn1;
-                pv[q] = (sv[t][q] == -INFINITY || mq == -INFINITY) ? 0.f : expf(sv[t][q] - mq);
-            }
-            if (g4 >= G) pv[0] = pv[1] = 0.f;
-            if (g4 + 8 >= G) pv[2] = pv[3] = 0.f;
-            const int key0 = nt * 8 + 2 * t4;
-            uint32_t hi, lo;
-            const uint32_t o0 = (uint32_t)(g4 * kMmaPS + swz(g4, key0 / 8) * 8 + key0 % 8);
-            const uint32_t o1 = (uint32_t)((g4 + 8) * kMmaPS + swz(g4 + 8, key0 / 8) * 8 + key0 % 8);
-            split2(pv[0], pv[1], hi, lo);
-            *(uint32_t *)(phi + o0) = hi;
-            *(uint32_t *)(plo + o0) = lo;
-            split2(pv[2], pv[3], hi, lo);
-            *(uint32_t *)(phi + o1) = hi;
-            *(uint32_t *)(plo + o1) = lo;
-            r0s += pv[0] + pv[1];
-            r1s += pv[2] + pv[3];
-        }
-#pragma unroll
-        for (int o = 1; o <= 2; o <<= 1) {
-            r0s += __shfl_xor_sync(0xFFFFFFFFu, r0s, o);
-            r1s += __shfl_xor_sync(0xFFFFFFFFu, r1s, o);
-        }
-        if (t4 == 0) { red_sum[warp][g4] = r0s; red_sum[warp][g4 + 8] = r1s; }
-        __syncthreads();
-        if (tid < 16) {
-            float mx = s_m[tid], sum = 0.f;
-            for (int w = 0; w < kFusedThreads / 32; ++w) {
-                mx = fmaxf(mx, red_max[w][tid]);
-                sum += red_sum[w][tid];
-            }
-            const float alpha = s_m[tid] == -INFINITY ? 0.f : expf(s_m[tid] - mx);
-            s_alpha[tid] = alpha;
-            s_l[tid] = s_l[tid] * alpha + sum;
-            s_m[tid] = mx;
-        }
-        __syncthreads();
-        // O tile of this warp: dims 8w .. 8w+7 (warps past D/8 idle)
-        if (warp < D / 8) {
-            const float al0 = s_alpha[g4], al1 = s_alpha[g4 + 8];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                oq4[c][0] *= al0;
-                oq4[c][1] *= al0;
-                oq4[c][2] *= al1;
-                oq4[c][3] *= al1;
-            }
-#pragma unroll
-            for (int kk = 0; kk < C / 16; kk += 2) {
-                uint32_t b0, b1, b2, b3, a0, a1, a2, a3;
-                {
-                    const int key = kk * 16 + lane;
-                    ldsm_x4_t(sa(vb) + (warp >> 3) * kBox + key * 128 + (((warp & 7) ^ (key & 7)) << 4), b0, b1,
-                              b2, b3);
+                for (int ks = 0; ks < NT; ++ks) {
+                    uint32_t ka[4];
+                    const int mi = lane >> 3;
+                    ldsm_x4(ta_piece(kb, kr + (mi & 1) * 8 + (lane & 7), 2 * ks + (mi >> 1)), ka);
+                    mma16816(sh, ka, qh[ks][0], qh[ks][1]);
+                    mma16816(sl, ka, ql[ks][0], ql[ks][1]);
                 }
+                float sv[4];
 #pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    const int k16 = kk + u;
-                    const int prow = (lane & 7) + ((lane >> 3) & 1) * 8, pslot = 2 * k16 + (lane >> 4);
-                    const uint32_t pofs = (uint32_t)(prow * kMmaPS + swz(prow, pslot) * 8);
-                    const uint32_t bb0 = u ? b2 : b0, bb1 = u ? b3 : b1;
-                    ldsm_x4(sa(phi + pofs), a0, a1, a2, a3);
-                    mma16816(oq4[2 * u], a0, a1, a2, a3, bb0, bb1);
-                    ldsm_x4(sa(plo + pofs), a0, a1, a2, a3);
-                    mma16816(oq4[2 * u + 1], a0, a1, a2, a3, bb0, bb1);
+                for (int q = 0; q < 4; ++q) {
+                    const int key = (lane >> 2) + (q >> 1) * 8;
+                    sv[q] = key < cnt ? sh[q] + sl[q] : -INFINITY;
                 }
-            }
-        }
-        __syncthreads();                              // buffer bi, p tiles free
-        if (tid == 0 && ci + 2 < nch && !dead) load(ci + 2);
-    }
-    // after a timeout, copies issued but never waited for land before exit
-    if (dead && tid == 0) {
-        for (long it = 0; it < kAttnWaitLimit && n_iss0 > 0 && !fa_try(&full[0], (uint32_t)((n_iss0 - 1) & 1)); ++it) {}
-        for (long it = 0; it < kAttnWaitLimit && n_iss1 > 0 && !fa_try(&full[1], (uint32_t)((n_iss1 - 1) & 1)); ++it) {}
-    }
-
-    // publish this rank's partial, then merge across the cluster
-    if (warp < D / 8) {
-        float oacc[4];
+                // online softmax of this warp: heads h0 = 2 (lane % 4) (entries 0, 2), h1 (1, 3)
+                float c0 = fmaxf(sv[0], sv[2]), c1 = fmaxf(sv[1], sv[3]);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) oacc[q] = (oq4[0][q] + oq4[1][q]) + (oq4[2][q] + oq4[3][q]);
-        const int d0 = warp * 8 + 2 * t4;
-        if (g4 < G) { po[g4 * D + d0] = oacc[0]; po[g4 * D + d0 + 1] = oacc[1]; }
-        if (g4 + 8 < G) { po[(g4 + 8) * D + d0] = oacc[2]; po[(g4 + 8) * D + d0 + 1] = oacc[3]; }
+                for (int off = 4; off < 32; off <<= 1) {
+                    c0 = fmaxf(c0, __shfl_xor_sync(0xFFFFFFFFu, c0, off));
+                    c1 = fmaxf(c1, __shfl_xor_sync(0xFFFFFFFFu, c1, off));
+                }
+                const float n0 = fmaxf(m0, c0), n1 = fmaxf(m1, c1);
+                const float al0 = m0 == -INFINITY ? 0.f : expf(m0 - n0), al1 = m1 == -INFINITY ? 0.f : expf(m1 - n1);
+                float p[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float mq = (q & 1) ? n1 : n0;
+                    p[q] = (sv[q] == -INFINITY || mq == -INFINITY) ? 0.f : expf(sv[q] - mq);
+                }
+                l0 = l0 * al0 + (p[0] + p[2]);
+                l1 = l1 * al1 + (p[1] + p[3]);
+                m0 = n0;
+                m1 = n1;
+#pragma unroll
+                for (int t = 0; t < NT; ++t) {
+                    o[t][0] *= al0;
+                    o[t][1] *= al1;
+                    o[t][2] *= al0;
+                    o[t][3] *= al1;
+                }
+                // P^T as B fragments: the S^T tile's 8 x 8 halves, transposed in registers
+                uint32_t h01, l01, h23, l23;
+                split2(p[0], p[1], h01, l01);
+                split2(p[2], p[3], h23, l23);
+                const uint32_t pb_h0 = movm_t(h01), pb_h1 = movm_t(h23), pb_l0 = movm_t(l01), pb_l1 = movm_t(l23);
+                // O^T += V^T P^T, one 16-dim tile at a time
+#pragma unroll
+                for (int t = 0; t < NT; ++t) {
+                    uint32_t va[4];
+                    const int mi = lane >> 3;
+                    ldsm_x4_t(ta_piece(vb, kr + (mi >> 1) * 8 + (lane & 7), 2 * t + (mi & 1)), va);
+                    mma16816(o[t], va, pb_h0, pb_h1);
+                    mma16816(o[t], va, pb_l0, pb_l1);
+                }
+                // zeros written above precede the next TMA write of this slot
+                if (cnt < 16) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            }
+            __syncwarp();
+            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(sa(&empty[s])) : "memory");
+        }
+        // the warp's sums over its lanes' keys
+#pragma unroll
+        for (int off = 4; off < 32; off <<= 1) {
+            l0 += __shfl_xor_sync(0xFFFFFFFFu, l0, off);
+            l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, off);
+        }
     }
-    if (tid < 16) { pm[tid] = s_m[tid]; pl[tid] = s_l[tid]; }
+    __syncthreads();                                  // every copy landed, every warp done with the ring
+    if (warp < kTaWarps) {
+        const int h0 = 2 * (lane & 3), d0 = lane >> 2;
+        if (lane < 4) {
+            wm[warp * 8 + h0] = m0;
+            wm[warp * 8 + h0 + 1] = m1;
+            wl[warp * 8 + h0] = l0;
+            wl[warp * 8 + h0 + 1] = l1;
+        }
+        float *w0 = wo + (size_t)(warp * 8 + h0) * D, *w1 = w0 + D;
+#pragma unroll
+        for (int t = 0; t < NTO; ++t) {
+            w0[16 * t + d0] = o[t][0];
+            w1[16 * t + d0] = o[t][1];
+            w0[16 * t + d0 + 8] = o[t][2];
+            w1[16 * t + d0 + 8] = o[t][3];
+        }
+    }
+    __syncthreads();
+    // this rank's partial: the warps' states merged in warp order
+    for (int e = tid; e < G * D; e += kTaThreads) {
+        const int h = e / D, d = e % D;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < kTaWarps; ++w) M = fmaxf(M, wm[w * 8 + h]);
+        float num = 0.f, den = 0.f;
+#pragma unroll
+        for (int w = 0; w < kTaWarps; ++w) {
+            const float mw = wm[w * 8 + h];
+            const float f = mw == -INFINITY ? 0.f : expf(mw - M);
+            den = fmaf(f, wl[w * 8 + h], den);
+            num = fmaf(f, wo[(size_t)(w * 8 + h) * D + d], num);
+        }
+        po[h * D + d] = num;
+        if (d == 0) {
+            pm[h] = M;
+            pl[h] = den;
+        }
+    }
     cluster_sync_all();
+    // rank r combines its slice of the (head, dim) outputs from every rank, in rank order
     {
         const int n_out = G * D;
         const int e0 = (int)((long)r * n_out / CS), e1 = (int)((long)(r + 1) * n_out / CS);
-        for (int e = e0 + tid; e < e1; e += kFusedThreads) {
+        for (int e = e0 + tid; e < e1; e += kTaThreads) {
             const int h = e / D;
             float mq[kMaxCluster], lq[kMaxCluster], oq[kMaxCluster];
 #pragma unroll
@@ -1012,18 +1020,21 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
                 den = fmaf(w, lq[q], den);
                 num = fmaf(w, oq[q], num);
             }
-            uint16_t *o = (uint16_t *)a.o_out + (size_t)b * a.Hq * D + (size_t)g * G * D;
-            o[e] = f32_to_bf16(den > 0.f ? num / den : 0.f);
+            uint16_t *out = (uint16_t *)a.o_out + (size_t)b * a.Hq * D + (size_t)g * G * D;
+            out[e] = f32_to_bf16(den > 0.f ? num / den : 0.f);
         }
     }
     cluster_sync_all();
 }
 
 template <int D>
-size_t fused_mma_smem() {
-    return 1024 + (size_t)4 * kMmaC * D * 2 + (size_t)2 * 16 * D * 2 + (size_t)2 * 16 * kMmaPS * 2 +
-           (size_t)2 * 16 * D * 4 + 32 * 4;
+constexpr size_t fused_tc_smem_bound() {
+    return 1024 + (size_t)kTaStages * 2 * (D / 64) * kTaC * 128 + (size_t)2 * 8 * D * 4 + 16 * 4;
 }
+template <int D>
+size_t fused_tc_smem() { return fused_tc_smem_bound<D>(); }
+static_assert((size_t)kTaWarps * 8 * 128 * 4 + 2 * kTaWarps * 8 * 4 <= (size_t)kTaStages * 2 * 2 * kTaC * 128,
+              "the warps' states fit in the ring");
 
 template <typename WT, int D>
 size_t fused_smem(int G) {
@@ -1033,10 +1044,11 @@ size_t fused_smem(int G) {
 static_assert(kFusedThreads % 128 == 0, "score pass maps threads to (key, head group)");
 
 template <typename Kern, typename... Args>
-cudaError_t launch_cluster(Kern k, size_t smem, const FusedAttnArgs &a, cudaStream_t s, bool pdl, Args... args) {
+cudaError_t launch_cluster(Kern k, size_t smem, int threads, const FusedAttnArgs &a, cudaStream_t s, bool pdl,
+                           Args... args) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(a.cs, a.Hkv, a.B);
-    cfg.blockDim = dim3(kFusedThreads);
+    cfg.blockDim = dim3(threads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[2];
@@ -1055,22 +1067,23 @@ template <typename WT, int D>
 cudaError_t launch_fused_t(const FusedAttnArgs &a, cudaStream_t s, bool pdl, const CUtensorMap *tk,
                            const CUtensorMap *tv) {
     if constexpr (sizeof(WT) == 2) {
-        if (tk && tv) return launch_cluster(fused_attention_mma_kernel<D>, fused_mma_smem<D>(), a, s, pdl, a, *tk, *tv);
+        if (tk && tv && a.Hq / a.Hkv <= 8)
+            return launch_cluster(fused_attention_tc_kernel<D>, fused_tc_smem<D>(), kTaThreads, a, s, pdl, a, *tk, *tv);
     }
-    return launch_cluster(fused_attention_kernel<WT, D>, fused_smem<WT, D>(a.Hq / a.Hkv), a, s, pdl, a);
+    return launch_cluster(fused_attention_kernel<WT, D>, fused_smem<WT, D>(a.Hq / a.Hkv), kFusedThreads, a, s, pdl, a);
 }
 
 // Clusters of 16 are a non-portable size: allowed only where the occupancy
 // query confirms that `need` of them can be resident at once.
 template <typename Kern>
-int max_cluster_for(Kern k, size_t smem, int need) {
+int max_cluster_for(Kern k, size_t smem, int threads, int need) {
     if (cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
         cudaGetLastError();
         return 8;
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(16, 1, 1);
-    cfg.blockDim = dim3(kFusedThreads);
+    cfg.blockDim = dim3(threads);
     cfg.dynamicSmemBytes = smem;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -1089,17 +1102,21 @@ int max_cluster_for(Kern k, size_t smem, int need) {
 
 template <typename WT, int D>
 cudaError_t prepare_fused_t(int G, int need, int *max_cs) {
-    cudaError_t e;
+    // the CUDA-core kernel serves every cache type (and bf16 caches without
+    // tensor maps); the tensor-core kernel bf16 caches with G <= 8
+    if (G > 16 || fused_smem<WT, D>(G) > (size_t)200 * 1024) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(fused_attention_kernel<WT, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         200 * 1024);
+    if (e == cudaSuccess && max_cs)
+        *max_cs = max_cluster_for(fused_attention_kernel<WT, D>, fused_smem<WT, D>(G), kFusedThreads, need);
     if constexpr (sizeof(WT) == 2) {
-        if (G > 16 || fused_mma_smem<D>() > (size_t)200 * 1024) return cudaErrorInvalidValue;
-        e = cudaFuncSetAttribute(fused_attention_mma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 200 * 1024);
-        if (e == cudaSuccess && max_cs) *max_cs = max_cluster_for(fused_attention_mma_kernel<D>, fused_mma_smem<D>(), need);
-    } else {
-        if (G > 16 || fused_smem<WT, D>(G) > (size_t)200 * 1024) return cudaErrorInvalidValue;
-        e = cudaFuncSetAttribute(fused_attention_kernel<WT, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 200 * 1024);
-        if (e == cudaSuccess && max_cs) *max_cs = max_cluster_for(fused_attention_kernel<WT, D>, fused_smem<WT, D>(G), need);
+        if (e == cudaSuccess && G <= 8) {
+            static_assert(fused_tc_smem_bound<D>() <= (size_t)227 * 1024, "tensor-core attention shared memory");
+            e = cudaFuncSetAttribute(fused_attention_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)fused_tc_smem<D>());
+            if (e == cudaSuccess && max_cs)
+                *max_cs = max_cluster_for(fused_attention_tc_kernel<D>, fused_tc_smem<D>(), kTaThreads, need);
+        }
     }
     return e;
 }
@@ -1149,7 +1166,7 @@ size_t attention_smem_bytes(bool bf16, int D, int chunk, int G, int splits) {
     return D == 64 ? attn_smem<float, 64>(chunk, G, splits) : attn_smem<float, 128>(chunk, G, splits);
 }
 
-int fused_attention_chunk() { return kMmaC; }
+int fused_attention_chunk() { return kTaC; }
 
 cudaError_t launch_fused_attention(const FusedAttnArgs &a, bool bf16, cudaStream_t s, bool pdl,
                                    const CUtensorMap *tk, const CUtensorMap *tv) {
@@ -1167,7 +1184,8 @@ cudaError_t prepare_fused_attention(bool bf16, int D, int G, int need, int *max_
 }
 
 size_t fused_attention_smem_bytes(bool bf16, int D, int G) {
-    if (bf16) return D == 64 ? fused_mma_smem<64>() : fused_mma_smem<128>();
+    if (bf16 && G <= 8) return D == 64 ? fused_tc_smem<64>() : fused_tc_smem<128>();
+    if (bf16) return D == 64 ? fused_smem<uint16_t, 64>(G) : fused_smem<uint16_t, 128>(G);
     return D == 64 ? fused_smem<float, 64>(G) : fused_smem<float, 128>(G);
 }
 
