@@ -204,10 +204,12 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * loads into tensor-memory accumulators, except gate/up + SwiGLU with at
  * most 2 activation rows, which measures faster on the CUDA-core kernel;
  * 2: gate/up as well; 0: every projection on the kernels below),
- * "tc_stream_rows" (>= 1, default 9: a tcgen05 projection with at least
+ * "tc_stream_rows" (>= 1, default 8: a tcgen05 projection with at least
  * this many activation rows streams them through the TMA ring beside the
  * weights instead of staging them whole in shared memory; at most 16 rows
- * can be staged), "gemv_cuda_core" (for projections
+ * can be staged), "attn_ctas_per_sm" (1..64, default 2: the fused attention
+ * kernel's cluster size halves while batch x KV heads x cluster size exceeds
+ * this many CTAs per SM), "gemv_cuda_core" (for projections
  * not on the tcgen05 kernel: 1, the default, the CUDA-core TMA-ring kernel;
  * 0: the warp-level mma.sync kernel), "attn_fused" (1, the default: RoPE,
  * KV append and attention run as one kernel, a cluster of up to 8 CTAs per

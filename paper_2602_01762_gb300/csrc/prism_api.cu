@@ -73,7 +73,8 @@ struct prism_ctx {
     int gemv_cuda_core = 1;                               // 1: bf16 projections on CUDA cores
     int gemv_tcgen05 = 1;                                 // 1: bf16 projections on tcgen05 where they fit
     int attn_fused = 1;                                   // 1: fused RoPE/append/attention cluster kernel
-    int tc_stream_rows = 9;                               // tcgen05 projections with this many rows or more stream X
+    int attn_ctas_per_sm = 2;                             // fused attention: clusters shrink until B*Hkv*cs <= this * SMs
+    int tc_stream_rows = 8;                               // tcgen05 projections with this many rows or more stream X
     int attn_max_cs = 8;                                  // largest cluster the device co-schedules
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
     bool tc_ready = false;
@@ -262,7 +263,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
             fa.D = D;
             fa.max_ctx = f.max_ctx;
             fa.cs = c->attn_max_cs;
-            while (fa.cs > 1 && (long long)r.B * Hkv * fa.cs > 2LL * c->sms) fa.cs /= 2;
+            while (fa.cs > 1 && (long long)r.B * Hkv * fa.cs > (long long)c->attn_ctas_per_sm * c->sms) fa.cs /= 2;
             fa.err = c->err;
             e = launch_fused_attention(fa, c->bf16, s, pdl, cache_maps ? &tmk : nullptr, cache_maps ? &tmv : nullptr);
             after(3);
@@ -638,6 +639,7 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "gemv_tcgen05") && value >= 0 && value <= 2) c->gemv_tcgen05 = value;
     else if (!std::strcmp(name, "attn_fused")) c->attn_fused = value != 0;
     else if (!std::strcmp(name, "tc_stream_rows") && value >= 1) c->tc_stream_rows = value;
+    else if (!std::strcmp(name, "attn_ctas_per_sm") && value >= 1 && value <= 64) c->attn_ctas_per_sm = value;
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);
     return PRISM_OK;
