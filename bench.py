@@ -157,16 +157,17 @@ def dist_reduce(x: float, op: str, world: int, device=None) -> float:
     return float(t.item())
 
 
-def traffic_from_profile(kernel_src: str):
+def traffic_from_profile(kernel_src: str, workload: str):
     """dram bytes per LM-head launch from the committed ncu summary, or None
-    when the kernel source changed since that capture."""
+    when the kernel source changed since that capture or the summary is of
+    another workload."""
     path = os.path.join(ROOT, "profiles", "lm_head_traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)
         with open(kernel_src, "rb") as f:
             digest = hashlib.sha256(f.read()).hexdigest()
-        if rec.get("kernel_sha256") != digest:
+        if rec.get("kernel_sha256") != digest or rec.get("workload") != workload:
             return None
         return float(rec["dram_bytes_per_launch_full_size"])
     except Exception:
@@ -395,7 +396,7 @@ def run_ours(args, w, world, rank, local):
                     "frac_of_measured": total_bytes / (per_round_ms / 1e3) / 1e9 / peak},
             "roofline": {"kernel": "LM head GEMV + top-k selection", "bound": "hbm", "achieved": achieved,
                          "peak": peak, "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
-                         "traffic": traffic_from_profile(kernel_src), "bytes_per_launch": lm_b,
+                         "traffic": traffic_from_profile(kernel_src, w.name), "bytes_per_launch": lm_b,
                          "avg_launch_ms": lm_ms},
             "kernel_time_share": shares,
             "kernel_ms_per_round": kind_total,
