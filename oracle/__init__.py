@@ -64,6 +64,19 @@ def _bind(path: str):
     lib.orc_draft_round.argtypes = [ctypes.POINTER(_Config), vp, vp, ctypes.POINTER(_Module),
                                     i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
     lib.orc_draft_round.restype = ctypes.c_int
+    u64 = ctypes.c_uint64
+    lib.orc_draft_round_sampled.argtypes = [ctypes.POINTER(_Config), vp, vp, ctypes.POINTER(_Module),
+                                            i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp,
+                                            dbl, u64, vp, vp, vp]
+    lib.orc_draft_round_sampled.restype = ctypes.c_int
+    lib.orc_splitmix_at.argtypes = [u64, u64]
+    lib.orc_splitmix_at.restype = u64
+    lib.orc_uniform.argtypes = [u64, i32, i64, i64, i64]
+    lib.orc_uniform.restype = dbl
+    lib.orc_sample_gumbel.argtypes = [vp, i64, dbl, u64, i64, i64, vp, vp, vp]
+    lib.orc_sample_gumbel.restype = None
+    lib.orc_accept_sampled.argtypes = [i32, i32, i64, vp, vp, vp, vp, dbl, vp, u64, vp, vp, vp, vp]
+    lib.orc_accept_sampled.restype = None
     lib.orc_accept_greedy.argtypes = [i32, i32, vp, vp, vp, vp, vp, vp]
     lib.orc_num_threads.restype = ctypes.c_int
     lib.orc_round_bf16_bits.argtypes = [vp, i64, vp]
@@ -176,7 +189,7 @@ def config_of(shape, *, topk: int, max_ctx: int, round_acts: bool | None = None,
 
 def draft_round(shape, weights: dict, inputs: dict, *, topk: int = 1, round_acts: bool | None = None,
                 final_norm: bool = True, want_logits: bool = False, want_hidden: bool = True,
-                seqs=None) -> dict:
+                seqs=None, temperature: float = 0.0, seed: int = 0) -> dict:
     """Run one draft round on the host.
 
     ``weights``: {"embed", "lm_head", "modules": {m: {...}}, "f_map"} as made
@@ -184,7 +197,10 @@ def draft_round(shape, weights: dict, inputs: dict, *, topk: int = 1, round_acts
     ``inputs``: {"tokens", "hidden", "n_new", "kv_len", "k_cache", "v_cache", "max_ctx"}.
     ``seqs``: optional list of sequence indices to compute (sequences are
     independent); outputs then cover only those sequences, in that order.
-    The caches in ``inputs`` are not modified; updated copies are returned."""
+    The caches in ``inputs`` are not modified; updated copies are returned.
+    ``temperature`` > 0: each draft token is drawn from softmax(z / T) with
+    the random streams of ``seed`` (sequence numbers are the indices in the
+    full batch); the result then also holds ``draft_lse`` and ``draft_margin``."""
     lib = _load()
     bf = shape.dtype == "bf16"
     wdt = np.uint16 if bf else np.float32
@@ -214,15 +230,23 @@ def draft_round(shape, weights: dict, inputs: dict, *, topk: int = 1, round_acts
     tvals = np.empty((B, K, topk), dtype=np.float64)
     logits = np.empty((B, K, shape.vocab), dtype=np.float64) if want_logits else None
     hout = np.empty((B, K, shape.hidden), dtype=np.float64) if want_hidden else None
-    rc = lib.orc_draft_round(ctypes.byref(cfg), embed.ctypes.data, lm.ctypes.data, mods, B, max_new,
-                             tokens.ctypes.data, hidden.ctypes.data, n_new.ctypes.data,
-                             kv_len.ctypes.data, k_cache.ctypes.data, v_cache.ctypes.data,
-                             draft.ctypes.data, tids.ctypes.data, tvals.ctypes.data,
-                             _ptr(logits), _ptr(hout))
+    seq_index = _c(np.asarray(sel), np.int32)
+    lse = np.empty((B, K), dtype=np.float64)
+    margin = np.empty((B, K), dtype=np.float64)
+    rc = lib.orc_draft_round_sampled(ctypes.byref(cfg), embed.ctypes.data, lm.ctypes.data, mods, B, max_new,
+                                     tokens.ctypes.data, hidden.ctypes.data, n_new.ctypes.data,
+                                     kv_len.ctypes.data, k_cache.ctypes.data, v_cache.ctypes.data,
+                                     draft.ctypes.data, tids.ctypes.data, tvals.ctypes.data,
+                                     _ptr(logits), _ptr(hout), float(temperature), int(seed),
+                                     seq_index.ctypes.data, lse.ctypes.data, margin.ctypes.data)
     if rc != 0:
         raise ValueError(f"oracle draft round rejected its input (code {rc})")
-    return {"draft_ids": draft, "topk_ids": tids, "topk_logits": tvals, "logits": logits,
-            "hidden_out": hout, "k_cache": k_cache, "v_cache": v_cache}
+    out = {"draft_ids": draft, "topk_ids": tids, "topk_logits": tvals, "logits": logits,
+           "hidden_out": hout, "k_cache": k_cache, "v_cache": v_cache}
+    if temperature > 0:
+        out["draft_lse"] = lse
+        out["draft_margin"] = margin
+    return out
 
 
 def accept_greedy(draft: np.ndarray, target: np.ndarray, n_new: np.ndarray, kv_len: np.ndarray) -> dict:
@@ -234,4 +258,49 @@ def accept_greedy(draft: np.ndarray, target: np.ndarray, n_new: np.ndarray, kv_l
     out = np.empty((B, K + 1), dtype=np.int32)
     _load().orc_accept_greedy(B, K, draft.ctypes.data, target.ctypes.data, _c(n_new, np.int32).ctypes.data,
                               kv.ctypes.data, acc.ctypes.data, out.ctypes.data)
+    return {"accept_len": acc, "out_tokens": out, "kv_len": kv}
+
+
+# ------------------------------------------------------------------ sampling (temperature > 0)
+
+def splitmix_at(seed: int, n: int) -> int:
+    """The n-th output of SplitMix64 started from state ``seed``."""
+    return int(_load().orc_splitmix_at(int(seed) & (2 ** 64 - 1), int(n)))
+
+
+def uniform(seed: int, stream: int, b: int, k: int, i: int) -> float:
+    """The random number of (stream, sequence b, position k, index i), in (0, 1)."""
+    return float(_load().orc_uniform(int(seed) & (2 ** 64 - 1), stream, b, k, i))
+
+
+def sample_gumbel(z: np.ndarray, tau: float, seed: int, b: int, k: int):
+    """One draw from softmax(z / tau): (token, log-sum-exp of z / tau, Gumbel margin)."""
+    z = _c(z, np.float64)
+    tok = ctypes.c_int32(0)
+    lse = ctypes.c_double(0.0)
+    margin = ctypes.c_double(0.0)
+    _load().orc_sample_gumbel(z.ctypes.data, z.size, float(tau), int(seed) & (2 ** 64 - 1), b, k,
+                              ctypes.byref(tok), ctypes.byref(lse), ctypes.byref(margin))
+    return int(tok.value), float(lse.value), float(margin.value)
+
+
+def accept_sampled(draft: np.ndarray, logits: np.ndarray, lse: np.ndarray, tau: float, target_probs: np.ndarray,
+                   seed: int, n_new: np.ndarray, kv_len: np.ndarray, seq_index=None) -> dict:
+    """Speculative-sampling acceptance: draft [B, K], logits [B, K, V], lse [B, K],
+    target_probs [B, K + 1, V]."""
+    draft = _c(draft, np.int32)
+    B, K = draft.shape
+    z = _c(logits, np.float64)
+    lse = _c(lse, np.float64)
+    pt = _c(target_probs, np.float64)
+    V = z.shape[-1]
+    assert z.shape == (B, K, V) and pt.shape == (B, K + 1, V) and lse.shape == (B, K)
+    idx = _c(np.arange(B) if seq_index is None else seq_index, np.int32)
+    kv = _c(kv_len, np.int32).copy()
+    acc = np.empty(B, dtype=np.int32)
+    out = np.empty((B, K + 1), dtype=np.int32)
+    _load().orc_accept_sampled(B, K, V, idx.ctypes.data, draft.ctypes.data, z.ctypes.data, lse.ctypes.data,
+                               float(tau), pt.ctypes.data, int(seed) & (2 ** 64 - 1),
+                               _c(n_new, np.int32).ctypes.data, kv.ctypes.data, acc.ctypes.data,
+                               out.ctypes.data)
     return {"accept_len": acc, "out_tokens": out, "kv_len": kv}

@@ -17,6 +17,11 @@
  *   greedy acceptance (Sec. 2 "Speculative Decoding", the rejection rule at
  *     temperature 0): the longest prefix on which draft and target agree,
  *     followed by the target's token at the first disagreement.
+ *   sampled drafting and acceptance (Sec. 2, at a temperature tau > 0): each
+ *     step draws x^_k from p_draft = softmax(z / tau) instead of taking the
+ *     argmax; a draft token x is accepted when r < min(1, p_target(x) /
+ *     p_draft(x)), and the first rejected position draws its replacement from
+ *     max(0, p_target - p_draft) normalised.
  *
  * Readings where the paper is silent (each is a reading, not a quote):
  *   fusion F = one bias-free linear map W_fuse [d, 2d] applied to the
@@ -268,6 +273,119 @@ static void select_tokens(const orc_config *c, const void *lm_head, const orc_mo
     }
 }
 
+/* ---------------------------------------------------------------- sampling */
+
+/* Random numbers of sampled drafting and acceptance: the n-th output of
+ * SplitMix64 (Steele, Lea and Flood, OOPSLA 2014) started from state `seed`,
+ * i.e. the finaliser applied to seed + (n + 1) * gamma, with the counter
+ * n = (stream << 60) | (b << 40) | (k << 32) | i (b < 2^20, k < 2^8,
+ * i < 2^32).  Mapped to the open interval (0, 1) as ((x >> 40) + 1/2) / 2^24,
+ * a value that float32 holds exactly.  Streams: 1 = draft sampling (i = token
+ * id), 2 = the acceptance test of position k, 3 = the replacement or extra
+ * token drawn at position k. */
+uint64_t orc_splitmix_at(uint64_t seed, uint64_t n) {
+    uint64_t z = seed + (n + 1) * 0x9E3779B97F4A7C15ULL;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+    return z ^ (z >> 31);
+}
+
+double orc_uniform(uint64_t seed, int32_t stream, int64_t b, int64_t k, int64_t i) {
+    const uint64_t n = ((uint64_t)stream << 60) | ((uint64_t)b << 40) | ((uint64_t)k << 32) | (uint64_t)i;
+    return ((double)(orc_splitmix_at(seed, n) >> 40) + 0.5) / 16777216.0;
+}
+
+/* One draw from p_draft = softmax(z / tau) over V logits by the Gumbel-max
+ * rule (the argmax of z_i / tau + G_i, G_i = -log(-log U_i) independent
+ * standard Gumbel variables, is distributed as softmax(z / tau)); ties go to
+ * the lower id.  lse = log sum_i exp(z_i / tau), so p_draft(x) =
+ * exp(z_x / tau - lse).  margin = best minus second-best perturbed score. */
+void orc_sample_gumbel(const double *z, int64_t V, double tau, uint64_t seed, int64_t b, int64_t k,
+                       int32_t *token, double *lse, double *margin) {
+    double m = -INFINITY;
+    for (int64_t i = 0; i < V; ++i) m = fmax(m, z[i] / tau);
+    double s = 0.0;
+    for (int64_t i = 0; i < V; ++i) s += exp(z[i] / tau - m);
+    *lse = m + log(s);
+    double best = -INFINITY, second = -INFINITY;
+    int32_t arg = 0;
+    for (int64_t i = 0; i < V; ++i) {
+        const double v = z[i] / tau - log(-log(orc_uniform(seed, 1, b, k, i)));
+        if (v > best) {
+            second = best;
+            best = v;
+            arg = (int32_t)i;
+        } else if (v > second) {
+            second = v;
+        }
+    }
+    *token = arg;
+    *margin = best - second;
+}
+
+/* Inverse-CDF draw from the non-negative weights w[0..V) (not necessarily
+ * normalised): the first i whose running sum exceeds u * total. */
+static int32_t draw_cdf(const double *w, int64_t V, double u) {
+    double total = 0.0;
+    for (int64_t i = 0; i < V; ++i) total += w[i];
+    const double t = u * total;
+    double c = 0.0;
+    int32_t last = 0;
+    for (int64_t i = 0; i < V; ++i) {
+        if (w[i] > 0.0) last = (int32_t)i;
+        c += w[i];
+        if (c > t) return (int32_t)i;
+    }
+    return last;
+}
+
+/* Speculative-sampling acceptance (Sec. 2) of B sequences with K drafted
+ * tokens each.  z: the draft logits [B, K, V]; lse: log sum exp(z / tau) per
+ * (b, k); pt: the target's distributions [B, K + 1, V] (rows sum to 1);
+ * seq_index[b]: the sequence's index in the random streams.  For k = 0..K-1
+ * in turn, x = draft[b, k] is accepted when r * p_draft(x) < p_target(x)
+ * (r < min(1, p_target / p_draft) without the division), r = uniform(2, b,
+ * k).  At the first rejected position k the replacement is drawn from
+ * max(0, p_target - p_draft) (uniform(3, b, k)); if that residual is zero
+ * everywhere, from p_target.  When all K are accepted, the extra token is
+ * drawn from p_target at position K (uniform(3, b, K)).  accept_len[b] = the
+ * accepted count a; out_tokens[b] = the a accepted drafts followed by the
+ * drawn token, the rest -1; kv_len[b] += n_new[b]. */
+void orc_accept_sampled(int32_t B, int32_t K, int64_t V, const int32_t *seq_index, const int32_t *draft,
+                        const double *z, const double *lse, double tau, const double *pt, uint64_t seed,
+                        const int32_t *n_new, int32_t *kv_len, int32_t *accept_len, int32_t *out_tokens) {
+    double *w = malloc(sizeof(double) * (size_t)V);
+    for (int32_t b = 0; b < B; ++b) {
+        const int64_t sb = seq_index ? seq_index[b] : b;
+        int32_t a = 0, extra = -1;
+        for (; a < K; ++a) {
+            const int32_t x = draft[b * K + a];
+            const double *zk = z + ((int64_t)b * K + a) * V, *pk = pt + ((int64_t)b * (K + 1) + a) * V;
+            const double pd = exp(zk[x] / tau - lse[b * K + a]);
+            const double r = orc_uniform(seed, 2, sb, a, 0);
+            if (r * pd < pk[x]) continue;
+            double tot = 0.0;
+            for (int64_t i = 0; i < V; ++i) {
+                w[i] = fmax(0.0, pk[i] - exp(zk[i] / tau - lse[b * K + a]));
+                tot += w[i];
+            }
+            const double u = orc_uniform(seed, 3, sb, a, 0);
+            extra = tot > 0.0 ? draw_cdf(w, V, u) : draw_cdf(pk, V, u);
+            break;
+        }
+        if (a == K) extra = draw_cdf(pt + ((int64_t)b * (K + 1) + K) * V, V, orc_uniform(seed, 3, sb, K, 0));
+        accept_len[b] = a;
+        for (int32_t j = 0; j <= K; ++j) {
+            int32_t v = -1;
+            if (j < a) v = draft[b * K + j];
+            else if (j == a) v = extra;
+            out_tokens[b * (K + 1) + j] = v;
+        }
+        kv_len[b] = kv_len[b] + n_new[b];
+    }
+    free(w);
+}
+
 /* ---------------------------------------------------------------- round */
 
 /* Returns 0 on success; 1 bad argument; 2 token id out of range; 3 cache
@@ -275,12 +393,17 @@ static void select_tokens(const orc_config *c, const void *lm_head, const orc_mo
  * steps[k] is the module of draft step k+1 (the surjection f_map applied).
  * Outputs: draft_ids [B, K]; topk_ids/topk_logits [B, K, topk];
  * logits [B, K, V] and hidden_out [B, K, d] when non-NULL. */
-int orc_draft_round(const orc_config *c, const void *embed, const void *lm_head,
-                    const orc_module *steps, int32_t B, int32_t max_new,
-                    const int32_t *tokens, const void *hidden, const int32_t *n_new,
-                    const int32_t *kv_len, void *k_cache, void *v_cache,
-                    int32_t *draft_ids, int32_t *topk_ids, double *topk_logits,
-                    double *logits, double *hidden_out) {
+/* The round with sampled drafting when tau > 0 (see orc_sample_gumbel):
+ * seq_index[b] names sequence b in the random streams (NULL: b itself);
+ * draft_lse / draft_margin [B, K] receive lse and the Gumbel margin of each
+ * draw when non-NULL.  With tau <= 0 this is the greedy round. */
+int orc_draft_round_sampled(const orc_config *c, const void *embed, const void *lm_head,
+                            const orc_module *steps, int32_t B, int32_t max_new,
+                            const int32_t *tokens, const void *hidden, const int32_t *n_new,
+                            const int32_t *kv_len, void *k_cache, void *v_cache,
+                            int32_t *draft_ids, int32_t *topk_ids, double *topk_logits,
+                            double *logits, double *hidden_out, double tau, uint64_t seed,
+                            const int32_t *seq_index, double *draft_lse, double *draft_margin) {
     const int64_t d = c->hidden, V = c->vocab, K = c->n_steps, F = c->ffn;
     const int64_t Hq = c->n_q_heads, Hkv = c->n_kv_heads, D = c->head_dim;
     const int bf = c->bf16;
@@ -334,6 +457,12 @@ int orc_draft_round(const orc_config *c, const void *embed, const void *lm_head,
             memcpy(hhat, w.y, sizeof(double) * (size_t)d);
             select_tokens(c, lm_head, m, hhat, z, order, &w, tid, tval);
             prev = tid[0];
+            if (tau > 0.0) {
+                double lse, margin;
+                orc_sample_gumbel(z, V, tau, seed, seq_index ? seq_index[b] : b, k - 1, &prev, &lse, &margin);
+                if (draft_lse) draft_lse[b * K + (k - 1)] = lse;
+                if (draft_margin) draft_margin[b * K + (k - 1)] = margin;
+            }
             draft_ids[b * K + (k - 1)] = prev;
             for (int32_t r = 0; r < c->topk; ++r) {
                 if (topk_ids) topk_ids[(b * K + (k - 1)) * c->topk + r] = tid[r];
@@ -347,6 +476,17 @@ int orc_draft_round(const orc_config *c, const void *embed, const void *lm_head,
     free(w.mm); free(w.y); free(w.g_attn); free(w.g_mlp); free(w.g_final);
     free(u); free(hhat); free(z); free(order); free(tid); free(tval);
     return 0;
+}
+
+int orc_draft_round(const orc_config *c, const void *embed, const void *lm_head,
+                    const orc_module *steps, int32_t B, int32_t max_new,
+                    const int32_t *tokens, const void *hidden, const int32_t *n_new,
+                    const int32_t *kv_len, void *k_cache, void *v_cache,
+                    int32_t *draft_ids, int32_t *topk_ids, double *topk_logits,
+                    double *logits, double *hidden_out) {
+    return orc_draft_round_sampled(c, embed, lm_head, steps, B, max_new, tokens, hidden, n_new, kv_len,
+                                   k_cache, v_cache, draft_ids, topk_ids, topk_logits, logits, hidden_out,
+                                   0.0, 0, NULL, NULL, NULL);
 }
 
 /* Greedy acceptance (temperature 0).  accept_len[b] = largest a in [0, K]
