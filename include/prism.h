@@ -153,6 +153,54 @@ prism_status prism_accept_greedy(prism_ctx *ctx, int32_t batch, const int32_t *d
                                  const int32_t *target, const int32_t *n_new, int32_t *kv_len,
                                  int32_t *accept_len, int32_t *out_tokens, void *stream);
 
+/* Random numbers of the sampled calls below: the n-th output x of SplitMix64
+ * (Steele, Lea and Flood, OOPSLA 2014) started from state *seed, with
+ * n = (stream << 60) | (b << 40) | (k << 32) | i, taken as
+ * ((x >> 41) + 1/2) / 2^23 in (0, 1).  Streams: 1 the draft draw of sequence
+ * b at step k + 1 (i = token id), 2 the acceptance test of position k, 3 the
+ * token drawn at position k (k = K: the extra token after a full accept).
+ * `seed` is a device pointer, read when the kernels run, so a captured round
+ * replays with a new seed written between rounds. */
+
+/* One draft round with sampled drafting (Sec. 2: the draft model draws its
+ * candidates from p_draft; here p_draft = softmax(z / temperature)): the same
+ * round as prism_draft_round, except that x^_k is drawn from softmax(z / T)
+ * of step k's logits (Gumbel-max rule, stream 1) and feeds step k + 1.
+ *   temperature  > 0, finite
+ *   seed         uint64 device word (8-byte aligned)
+ *   logits       float [batch, K, V] out, required (the acceptance reads them)
+ *   draft_lse    float [batch, K] out: log sum_i exp(z_i / T), so that
+ *                p_draft(x) = exp(z_x / T - lse)
+ *   draft_ids    the drawn tokens; topk_ids / topk_logits stay the argmax list
+ * Other arguments as prism_draft_round.  Errors: INVALID_ARG (temperature,
+ * null seed / logits / draft_lse, and as prism_draft_round), CAPACITY (also
+ * max_batch >= 2^20 or K > 255, the counter's fields), NOT_LOADED, CUDA. */
+prism_status prism_draft_round_sampled(prism_ctx *ctx, int32_t batch, const int32_t *tokens,
+                                       const void *hidden, const int32_t *n_new, const int32_t *kv_len,
+                                       void *k_cache, void *v_cache, float temperature, const uint64_t *seed,
+                                       int32_t *draft_ids, int32_t *topk_ids, float *topk_logits,
+                                       float *logits, float *draft_lse, float *hidden_out, void *stream);
+
+/* Speculative-sampling acceptance (Sec. 2): for k = 0..K-1 in turn, the draft
+ * token x = draft[b, k] is accepted when r < min(1, p_target(x) / p_draft(x))
+ * (r from stream 2, evaluated as r * p_draft < p_target); the first rejected
+ * position's replacement is drawn from max(0, p_target - p_draft) normalised
+ * (stream 3; from p_target if that residual is zero everywhere); after a full
+ * accept the extra token is drawn from p_target at position K.  p_draft(x) =
+ * exp(logits[b, k, x] / T - draft_lse[b, k]).
+ *   draft int32 [batch, K], logits float [batch, K, V], draft_lse float
+ *   [batch, K] (as written by prism_draft_round_sampled), temperature the
+ *   round's, target_probs float [batch, K+1, V] (rows sum to 1), seed uint64
+ *   device word, n_new int32 [batch], kv_len int32 [batch] in/out (+= n_new),
+ *   accept_len int32 [batch] out, out_tokens int32 [batch, K+1] out (the
+ *   accepted drafts, the drawn token, then -1).
+ * A draft id outside [0, V) sets the token bit of the device error word.
+ * Errors: INVALID_ARG, CAPACITY (batch > max_batch), CUDA. */
+prism_status prism_accept_sampled(prism_ctx *ctx, int32_t batch, const int32_t *draft, const float *logits,
+                                  const float *draft_lse, float temperature, const float *target_probs,
+                                  const uint64_t *seed, const int32_t *n_new, int32_t *kv_len,
+                                  int32_t *accept_len, int32_t *out_tokens, void *stream);
+
 /* LM-head selection that allocates nothing.  The paper has no counterpart to
  * this entry point; it serves callers that cannot call cudaMalloc, so cannot
  * own a prism_ctx workspace: an inference server whose caching allocator has
@@ -232,7 +280,8 @@ prism_status prism_round_launches(prism_ctx *ctx, int32_t *n_launches);
  * max_kernels); *n_kernels receives the count; kernel_kind[i] (may be NULL)
  * receives a code: 0 fusion, 1 qkv, 2 rope/append, 3 attention (with the
  * fused option: RoPE, append and attention; no code-2 kernel then), 4 o-proj,
- * 5 gate/up, 6 down, 7 LM head + selection.  Synchronises the stream. */
+ * 5 gate/up, 6 down, 7 LM head + selection, 8 sampled draw (sampled rounds
+ * only; this call profiles the greedy round).  Synchronises the stream. */
 prism_status prism_profile_round(prism_ctx *ctx, int32_t batch, const int32_t *tokens,
                                  const void *hidden, const int32_t *n_new, const int32_t *kv_len,
                                  void *k_cache, void *v_cache, int32_t *draft_ids,

@@ -18,7 +18,7 @@ __all__ = ["Drafter", "PrismError", "library", "lm_head_topk_static", "STEP_TENS
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.environ.get("PRISM_LIB") or os.path.join(_HERE, "libprism.so")
 STEP_TENSORS = ("w_fuse", "g_attn", "w_qkv", "w_o", "g_mlp", "w_gate_up", "w_down", "g_final")
-KERNEL_KINDS = ("fusion", "qkv", "rope_append", "attention", "o_proj", "gate_up", "down", "lm_head")
+KERNEL_KINDS = ("fusion", "qkv", "rope_append", "attention", "o_proj", "gate_up", "down", "lm_head", "sample")
 _STATUS = ["OK", "INVALID_ARG", "SHAPE", "CAPACITY", "NOT_LOADED", "CUDA", "OOM", "DEVICE_FLAG", "TIMEOUT"]
 
 
@@ -65,11 +65,15 @@ def library() -> ctypes.CDLL:
         lib.prism_lm_head_topk_static.argtypes = [i32] * 5 + [ctypes.c_float] + [vp] * 9
         lib.prism_get_error.argtypes = [vp]
         lib.prism_round_launches.argtypes = [vp, P(i32)]
+        flt = ctypes.c_float
+        lib.prism_draft_round_sampled.argtypes = [vp, i32] + [vp] * 6 + [flt] + [vp] * 8
+        lib.prism_accept_sampled.argtypes = [vp, i32, vp, vp, vp, flt] + [vp] * 7
         lib.prism_get_error.restype = ctypes.c_char_p
         lib.prism_version.restype = ctypes.c_char_p
         for f in ("prism_create", "prism_destroy", "prism_load_shared_weights", "prism_load_step_weights",
                   "prism_draft_round", "prism_accept_greedy", "prism_sync_status", "prism_set_option",
-                  "prism_profile_round", "prism_lm_head_topk_static", "prism_round_launches"):
+                  "prism_profile_round", "prism_lm_head_topk_static", "prism_round_launches",
+                  "prism_draft_round_sampled", "prism_accept_sampled"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -193,6 +197,43 @@ class Drafter:
             _ptr(v_cache), _ptr(draft_ids), _ptr(topk_ids), _ptr(topk_logits), _ptr(logits),
             _ptr(hidden_out), _stream(stream)))
 
+    def draft_round_sampled(self, tokens, hidden, n_new, kv_len, k_cache, v_cache, temperature: float, seed,
+                            draft_ids, logits, draft_lse, topk_ids=None, topk_logits=None, hidden_out=None,
+                            stream=None):
+        """Draft round with every x^_k drawn from softmax(z / temperature).
+        ``seed``: uint64 device tensor of one element (int64 storage), read when
+        the round runs; ``logits`` [B, K, V] and ``draft_lse`` [B, K] are required."""
+        B = self._round_args(tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids,
+                             topk_ids, topk_logits)
+        self._tensor(logits, (B, self.n_steps, self.vocab), torch.float32, "logits")
+        self._tensor(draft_lse, (B, self.n_steps), torch.float32, "draft_lse")
+        self._tensor(seed, (1,), torch.int64, "seed")
+        if hidden_out is not None:
+            self._tensor(hidden_out, (B, self.n_steps, self.hidden), torch.float32, "hidden_out")
+        self._check(self.lib.prism_draft_round_sampled(
+            self.h, B, _ptr(tokens), _ptr(hidden), _ptr(n_new), _ptr(kv_len), _ptr(k_cache),
+            _ptr(v_cache), float(temperature), _ptr(seed), _ptr(draft_ids), _ptr(topk_ids), _ptr(topk_logits),
+            _ptr(logits), _ptr(draft_lse), _ptr(hidden_out), _stream(stream)))
+
+    def accept_sampled(self, draft, logits, draft_lse, temperature: float, target_probs, seed, n_new, kv_len,
+                       accept_len, out_tokens, stream=None):
+        """Speculative-sampling acceptance against target_probs [B, K + 1, V]."""
+        B = draft.shape[0]
+        K, V = self.n_steps, self.vocab
+        i32 = torch.int32
+        self._tensor(draft, (B, K), i32, "draft")
+        self._tensor(logits, (B, K, V), torch.float32, "logits")
+        self._tensor(draft_lse, (B, K), torch.float32, "draft_lse")
+        self._tensor(target_probs, (B, K + 1, V), torch.float32, "target_probs")
+        self._tensor(seed, (1,), torch.int64, "seed")
+        self._tensor(n_new, (B,), i32, "n_new")
+        self._tensor(kv_len, (B,), i32, "kv_len")
+        self._tensor(accept_len, (B,), i32, "accept_len")
+        self._tensor(out_tokens, (B, K + 1), i32, "out_tokens")
+        self._check(self.lib.prism_accept_sampled(
+            self.h, B, _ptr(draft), _ptr(logits), _ptr(draft_lse), float(temperature), _ptr(target_probs),
+            _ptr(seed), _ptr(n_new), _ptr(kv_len), _ptr(accept_len), _ptr(out_tokens), _stream(stream)))
+
     def round_launches(self) -> int:
         """Kernel launches of the last round replayed from a CUDA graph."""
         n = ctypes.c_int32(0)
@@ -205,7 +246,7 @@ class Drafter:
         (kind, milliseconds) in launch order."""
         B = self._round_args(tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids,
                              topk_ids, topk_logits)
-        cap = 8 * self.n_steps + 8
+        cap = 9 * self.n_steps + 8
         ms = (ctypes.c_float * cap)()
         kinds = (ctypes.c_int32 * cap)()
         n = ctypes.c_int32(0)

@@ -221,6 +221,34 @@ struct AcceptArgs {
     int B, K;
 };
 
+// Sampled drafting (Sec. 2 at a temperature T > 0): the draw of step `step`
+// from the logits that step's LM head wrote.
+constexpr int kSampleMaxBlocks = 128;   // CTAs per row of logits
+struct SampleArgs {
+    const float *logits;       // [B, K, V] fp32
+    const uint64_t *seed;      // device word: the round's random-stream seed
+    int32_t *draft;            // [B, K]: the drawn token replaces the argmax
+    float *lse;                // [B, K]: log sum exp(z / T)
+    float *part;               // [B, kSampleMaxBlocks, 4] per-CTA partials
+    int *counter;              // [B] last-CTA tickets (left at zero)
+    float temperature;
+    int V, K, step, chunk, max_blocks;
+};
+// Speculative-sampling acceptance of B sequences with K drafted tokens each.
+struct AcceptSampledArgs {
+    const int32_t *draft;      // [B, K]
+    const float *logits;       // [B, K, V] draft logits
+    const float *lse;          // [B, K]
+    const float *target;       // [B, K + 1, V] target probabilities
+    const uint64_t *seed;
+    const int32_t *n_new;
+    int32_t *kv_len, *accept_len, *out_tokens;
+    int *err;
+    float temperature;
+    int B, K, V;
+};
+int sample_blocks(int V, int *chunk);
+
 // Host launchers (return cudaGetLastError of the launch).
 cudaError_t launch_gemv(const GemvArgs &a, bool bf16, int grid, cudaStream_t s, bool pdl);
 size_t gemv_smem_bytes(const GemvArgs &a, bool bf16, int tc);
@@ -228,6 +256,8 @@ int gemv_rows_per_pass(const GemvArgs &a, bool bf16);
 cudaError_t launch_rope_append(const RopeArgs &a, bool bf16, cudaStream_t s, bool pdl);
 cudaError_t launch_attention(const AttnArgs &a, bool bf16, cudaStream_t s, bool pdl);
 cudaError_t launch_accept(const AcceptArgs &a, cudaStream_t s);
+cudaError_t launch_sample(const SampleArgs &a, int B, cudaStream_t s, bool pdl);
+cudaError_t launch_accept_sampled(const AcceptSampledArgs &a, cudaStream_t s);
 // One-time kernel attribute setup (maximum dynamic shared memory); must run
 // before any stream capture.
 cudaError_t prepare_gemv_kernels();

@@ -14,7 +14,7 @@ using namespace prism;
 namespace {
 
 constexpr int kGraphCache = 8;
-constexpr int kMaxProfileKernels = 8 * kMaxSteps + 8;
+constexpr int kMaxProfileKernels = 9 * kMaxSteps + 8;
 
 struct RoundArgs {
     int B;
@@ -25,8 +25,32 @@ struct RoundArgs {
     int32_t *draft;
     int32_t *topk_ids;
     float *topk_logits, *logits, *hidden_out;
+    float temperature;             // > 0: sampled drafting (then logits, seed and lse are set)
+    const uint64_t *seed;
+    float *lse;
     bool operator==(const RoundArgs &o) const { return std::memcmp(this, &o, sizeof(RoundArgs)) == 0; }
 };
+
+// Zero-filled (padding included: graphs are looked up by memcmp of the arguments).
+RoundArgs round_args(int B, const int32_t *tokens, const void *hidden, const int32_t *n_new, const int32_t *kv_len,
+                     void *k_cache, void *v_cache, int32_t *draft, int32_t *topk_ids, float *topk_logits,
+                     float *logits, float *hidden_out) {
+    RoundArgs r;
+    std::memset(&r, 0, sizeof r);
+    r.B = B;
+    r.tokens = tokens;
+    r.hidden = hidden;
+    r.n_new = n_new;
+    r.kv_len = kv_len;
+    r.k_cache = k_cache;
+    r.v_cache = v_cache;
+    r.draft = draft;
+    r.topk_ids = topk_ids;
+    r.topk_logits = topk_logits;
+    r.logits = logits;
+    r.hidden_out = hidden_out;
+    return r;
+}
 
 struct GraphEntry {
     RoundArgs key;
@@ -65,6 +89,8 @@ struct prism_ctx {
     int *lm_id = nullptr;
     int *counters = nullptr;  // [max_batch * Hkv] attention + [1] LM head
     unsigned long long *lm_best = nullptr;  // [max_batch] LM head top-1 keys (left at zero)
+    float *sample_part = nullptr;           // [max_batch, kSampleMaxBlocks, 4] sampled-draft partials
+    int *sample_ctr = nullptr;              // [max_batch] sampled-draft tickets (left at zero)
     int *err = nullptr;
     // execution
     cudaStream_t cap_stream = nullptr;
@@ -395,6 +421,24 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.topk_logits = r.topk_logits;
         e = proj(g, c->tm_lm_ok ? &c->tm_lm : nullptr, c->lm_grid, pdl);
         after(7);
+        if (e != cudaSuccess) break;
+
+        if (r.temperature > 0.f) {
+            // x^_k drawn from softmax(z / T): replaces the argmax before the next step reads it
+            SampleArgs sa{};
+            sa.logits = r.logits;
+            sa.seed = r.seed;
+            sa.draft = r.draft;
+            sa.lse = r.lse;
+            sa.part = c->sample_part;
+            sa.counter = c->sample_ctr;
+            sa.temperature = r.temperature;
+            sa.V = V;
+            sa.K = K;
+            sa.step = k;
+            e = launch_sample(sa, r.B, s, pdl);
+            after(8);
+        }
     }
     if (n_kernels) *n_kernels = nk;
     return e;
@@ -495,6 +539,8 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         tc_floats * 4,                                             // tensor-core split-K partials
         (size_t)tc_tiles * 4,                                      // tensor-core tile tickets
         T1 * 2 * d * es,                                           // streamed-kernel activation rows
+        B * (size_t)kSampleMaxBlocks * 4 * 4,                      // sampled-draft partials
+        B * 4,                                                     // sampled-draft tickets
     };
     size_t total = 0;
     for (size_t s : sizes) total += align256(s);
@@ -527,6 +573,8 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     c->tc_ctr = (int *)slot[16];
     c->tc_ctr_n = tc_tiles;
     c->xbuf = (uint16_t *)slot[17];
+    c->sample_part = (float *)slot[18];
+    c->sample_ctr = (int *)slot[19];
 
     // rotary tables: angle p * theta^(-2j/D), computed in double, stored as float
     std::vector<float> cs((size_t)f.max_ctx * (D / 2)), sn((size_t)f.max_ctx * (D / 2));
@@ -645,12 +693,12 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     return PRISM_OK;
 }
 
-prism_status prism_draft_round(prism_ctx *c, int32_t batch, const int32_t *tokens, const void *hidden,
-                               const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
-                               int32_t *draft_ids, int32_t *topk_ids, float *topk_logits, float *logits,
-                               float *hidden_out, void *stream) {
-    RoundArgs r{batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids, topk_ids, topk_logits,
-                logits, hidden_out};
+}  // extern "C"
+
+namespace {
+
+// One round, as a replayed graph (captured on first use per argument set) or eagerly.
+prism_status run_round(prism_ctx *c, const RoundArgs &r, void *stream) {
     prism_status st = check_round_args(c, r);
     if (st != PRISM_OK) return st;
     cudaStream_t s = (cudaStream_t)stream;
@@ -705,6 +753,38 @@ prism_status prism_draft_round(prism_ctx *c, int32_t batch, const int32_t *token
     return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "cudaGraphLaunch");
 }
 
+}  // namespace
+
+extern "C" {
+
+prism_status prism_draft_round(prism_ctx *c, int32_t batch, const int32_t *tokens, const void *hidden,
+                               const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
+                               int32_t *draft_ids, int32_t *topk_ids, float *topk_logits, float *logits,
+                               float *hidden_out, void *stream) {
+    return run_round(c, round_args(batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids, topk_ids,
+                                   topk_logits, logits, hidden_out), stream);
+}
+
+prism_status prism_draft_round_sampled(prism_ctx *c, int32_t batch, const int32_t *tokens, const void *hidden,
+                                       const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
+                                       float temperature, const uint64_t *seed, int32_t *draft_ids,
+                                       int32_t *topk_ids, float *topk_logits, float *logits, float *draft_lse,
+                                       float *hidden_out, void *stream) {
+    if (!c) return fail(c, PRISM_ERR_INVALID_ARG, "null context");
+    if (!(temperature > 0.f) || !std::isfinite(temperature))
+        return fail(c, PRISM_ERR_INVALID_ARG, "temperature must be a finite value > 0");
+    if (!seed || ((uintptr_t)seed & 7) || !logits || !draft_lse)
+        return fail(c, PRISM_ERR_INVALID_ARG, "sampled rounds need seed (8-byte aligned), logits and draft_lse");
+    if (c->cfg.max_batch >= (1 << 20) || c->cfg.n_steps > 255)
+        return fail(c, PRISM_ERR_CAPACITY, "random-stream counter: batch below 2^20, steps below 256");
+    RoundArgs r = round_args(batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids, topk_ids,
+                             topk_logits, logits, hidden_out);
+    r.temperature = temperature;
+    r.seed = seed;
+    r.lse = draft_lse;
+    return run_round(c, r, stream);
+}
+
 prism_status prism_round_launches(prism_ctx *c, int32_t *n_launches) {
     if (!c || !n_launches) return fail(c, PRISM_ERR_INVALID_ARG, "null argument");
     if (c->last_round_kernels < 0) return fail(c, PRISM_ERR_INVALID_ARG, "no round has been replayed from a graph");
@@ -717,8 +797,8 @@ prism_status prism_profile_round(prism_ctx *c, int32_t batch, const int32_t *tok
                                  int32_t *draft_ids, int32_t *topk_ids, float *topk_logits, void *stream,
                                  float *kernel_ms, int32_t *kernel_kind, int32_t max_kernels,
                                  int32_t *n_kernels) {
-    RoundArgs r{batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids, topk_ids, topk_logits,
-                nullptr, nullptr};
+    const RoundArgs r = round_args(batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids, topk_ids,
+                                   topk_logits, nullptr, nullptr);
     prism_status st = check_round_args(c, r);
     if (st != PRISM_OK) return st;
     if (!kernel_ms || !n_kernels || max_kernels < 1) return fail(c, PRISM_ERR_INVALID_ARG, "null output");
@@ -754,6 +834,38 @@ prism_status prism_accept_greedy(prism_ctx *c, int32_t batch, const int32_t *dra
     AcceptArgs a{draft, target, n_new, kv_len, accept_len, out_tokens, batch, c->cfg.n_steps};
     cudaError_t e = launch_accept(a, (cudaStream_t)stream);
     return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "accept kernel launch");
+}
+
+prism_status prism_accept_sampled(prism_ctx *c, int32_t batch, const int32_t *draft, const float *logits,
+                                  const float *draft_lse, float temperature, const float *target_probs,
+                                  const uint64_t *seed, const int32_t *n_new, int32_t *kv_len, int32_t *accept_len,
+                                  int32_t *out_tokens, void *stream) {
+    if (!c) return fail(c, PRISM_ERR_INVALID_ARG, "null context");
+    if (!draft || !logits || !draft_lse || !target_probs || !seed || !n_new || !kv_len || !accept_len || !out_tokens)
+        return fail(c, PRISM_ERR_INVALID_ARG, "null tensor argument");
+    if ((uintptr_t)seed & 7) return fail(c, PRISM_ERR_INVALID_ARG, "seed must be 8-byte aligned");
+    if (!(temperature > 0.f) || !std::isfinite(temperature))
+        return fail(c, PRISM_ERR_INVALID_ARG, "temperature must be a finite value > 0");
+    if (batch < 1) return fail(c, PRISM_ERR_SHAPE, "batch must be >= 1");
+    if (batch > c->cfg.max_batch) return fail(c, PRISM_ERR_CAPACITY, "batch exceeds max_batch");
+    cudaSetDevice(c->device);
+    AcceptSampledArgs a{};
+    a.draft = draft;
+    a.logits = logits;
+    a.lse = draft_lse;
+    a.target = target_probs;
+    a.seed = seed;
+    a.n_new = n_new;
+    a.kv_len = kv_len;
+    a.accept_len = accept_len;
+    a.out_tokens = out_tokens;
+    a.err = c->err;
+    a.temperature = temperature;
+    a.B = batch;
+    a.K = c->cfg.n_steps;
+    a.V = c->cfg.vocab;
+    cudaError_t e = launch_accept_sampled(a, (cudaStream_t)stream);
+    return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "sampled accept kernel launch");
 }
 
 prism_status prism_sync_status(prism_ctx *c, void *stream, int32_t *flags) {

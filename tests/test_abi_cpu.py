@@ -65,4 +65,11 @@ def test_null_context_calls_return_invalid_arg(lib):
         f = getattr(lib, name)
         f.argtypes = [ctypes.c_void_p, ctypes.c_int32] + [ctypes.c_void_p] * (n - 2)
         assert f(None, 1, *([None] * (n - 2))) == 1
+    vp, f32 = ctypes.c_void_p, ctypes.c_float
+    f = lib.prism_draft_round_sampled
+    f.argtypes = [vp, ctypes.c_int32] + [vp] * 6 + [f32] + [vp] * 8
+    assert f(None, 1, *([None] * 6), 0.8, *([None] * 8)) == 1
+    f = lib.prism_accept_sampled
+    f.argtypes = [vp, ctypes.c_int32, vp, vp, vp, f32] + [vp] * 7
+    assert f(None, 1, None, None, None, 0.8, *([None] * 7)) == 1
     assert lib.prism_destroy(None) == 0

@@ -37,10 +37,11 @@ def test_random_numbers_are_the_published_splitmix64_sequence():
             if x.strip() and not x.startswith("#")]
     seed, outs = vals[0], vals[1:]
     assert [oracle.splitmix_at(seed, n) for n in range(len(outs))] == outs
-    # counter 0..4 of stream 0, sequence 0, position 0: the top 24 bits, centred in their cell
+    # counter 0..4 of stream 0, sequence 0, position 0: the top 23 bits, centred in their cell
     for n, x in enumerate(outs):
         u = oracle.uniform(seed, 0, 0, 0, n)
-        assert 0.0 < u < 1.0 and u * 2 ** 24 - 0.5 == x >> 40
+        assert 0.0 < u < 1.0 and u * 2 ** 23 - 0.5 == x >> 41
+        assert float(np.float32(u)) == u          # exact in float32
 
 
 def test_uniforms_are_uniform_and_streams_differ():
