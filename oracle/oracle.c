@@ -279,8 +279,9 @@ static void select_tokens(const orc_config *c, const void *lm_head, const orc_mo
  * SplitMix64 (Steele, Lea and Flood, OOPSLA 2014) started from state `seed`,
  * i.e. the finaliser applied to seed + (n + 1) * gamma, with the counter
  * n = (stream << 60) | (b << 40) | (k << 32) | i (b < 2^20, k < 2^8,
- * i < 2^32).  Mapped to the open interval (0, 1) as ((x >> 40) + 1/2) / 2^24,
- * a value that float32 holds exactly.  Streams: 1 = draft sampling (i = token
+ * i < 2^32).  Mapped to the open interval (0, 1) as ((x >> 41) + 1/2) / 2^23:
+ * 24 significant bits, so float32 holds the value exactly and a float32
+ * implementation draws the very same numbers.  Streams: 1 = draft sampling (i = token
  * id), 2 = the acceptance test of position k, 3 = the replacement or extra
  * token drawn at position k. */
 uint64_t orc_splitmix_at(uint64_t seed, uint64_t n) {
@@ -292,7 +293,7 @@ uint64_t orc_splitmix_at(uint64_t seed, uint64_t n) {
 
 double orc_uniform(uint64_t seed, int32_t stream, int64_t b, int64_t k, int64_t i) {
     const uint64_t n = ((uint64_t)stream << 60) | ((uint64_t)b << 40) | ((uint64_t)k << 32) | (uint64_t)i;
-    return ((double)(orc_splitmix_at(seed, n) >> 40) + 0.5) / 16777216.0;
+    return ((double)(orc_splitmix_at(seed, n) >> 41) + 0.5) / 8388608.0;
 }
 
 /* One draw from p_draft = softmax(z / tau) over V logits by the Gumbel-max
