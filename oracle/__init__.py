@@ -78,6 +78,12 @@ def _bind(path: str):
     lib.orc_accept_sampled.argtypes = [i32, i32, i64, vp, vp, vp, vp, dbl, vp, u64, vp, vp, vp, vp]
     lib.orc_accept_sampled.restype = None
     lib.orc_accept_greedy.argtypes = [i32, i32, vp, vp, vp, vp, vp, vp]
+    lib.orc_draft_tree.argtypes = [ctypes.POINTER(_Config), vp, vp, ctypes.POINTER(_Module), i32, i32,
+                                   vp, vp, vp, vp, vp, vp, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp,
+                                   vp, vp, vp, vp, vp]
+    lib.orc_draft_tree.restype = ctypes.c_int
+    lib.orc_accept_tree.argtypes = [i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
+    lib.orc_accept_tree.restype = None
     lib.orc_num_threads.restype = ctypes.c_int
     lib.orc_round_bf16_bits.argtypes = [vp, i64, vp]
     lib.orc_round_bf16_bits.restype = None
@@ -304,3 +310,93 @@ def accept_sampled(draft: np.ndarray, logits: np.ndarray, lse: np.ndarray, tau: 
                                _c(n_new, np.int32).ctypes.data, kv.ctypes.data, acc.ctypes.data,
                                out.ctypes.data)
     return {"accept_len": acc, "out_tokens": out, "kv_len": kv}
+
+
+# ------------------------------------------------------------------ tree drafting
+
+def pool_size(n_steps: int, width: int) -> int:
+    """Candidates of one tree round: w at depth 1, then w * w per later step."""
+    return width + (n_steps - 1) * width * width
+
+
+def draft_tree(shape, weights: dict, inputs: dict, *, width: int, n_nodes: int, follow: dict | None = None,
+               round_acts: bool | None = None, final_norm: bool = True, want_logits: bool = True,
+               want_hidden: bool = False, seqs=None) -> dict:
+    """One tree-drafting round on the host (``orc_draft_tree``).
+
+    ``follow``: {"pool_tokens" [B, P], "frontier" [B, K, w]} over the same
+    sequences as ``seqs`` (or the full batch): recompute that tree instead of
+    choosing candidates and frontiers.  Returns the pool (tokens, parents,
+    scores), the frontier chosen after each step, per-row logits / lse
+    ([B, K, w, ...]; step 1 fills row 0 only), the verified tree and the
+    updated caches."""
+    lib = _load()
+    bf = shape.dtype == "bf16"
+    wdt = np.uint16 if bf else np.float32
+    K, V, d = shape.n_steps, shape.vocab, shape.hidden
+    sel = list(range(inputs["tokens"].shape[0])) if seqs is None else list(seqs)
+    B = len(sel)
+    P = pool_size(K, width)
+    tokens = _c(inputs["tokens"][sel], np.int32)
+    max_new = tokens.shape[1]
+    hidden = _c(inputs["hidden"][sel], wdt)
+    n_new = _c(inputs["n_new"][sel], np.int32)
+    kv_len = _c(inputs["kv_len"][sel], np.int32)
+    k_cache = _c(inputs["k_cache"][sel], wdt).copy()
+    v_cache = _c(inputs["v_cache"][sel], wdt).copy()
+    cfg = config_of(shape, topk=width, max_ctx=int(inputs["max_ctx"]), round_acts=round_acts,
+                    final_norm=final_norm)
+    keep = []
+    mods = (_Module * K)()
+    for k in range(K):
+        mod = weights["modules"][weights["f_map"][k]]
+        arrs = [_c(mod[n], wdt) for n in STEP_TENSORS]
+        keep.extend(arrs)
+        mods[k] = _Module(*[a.ctypes.data for a in arrs])
+    embed = _c(weights["embed"], wdt)
+    lm = _c(weights["lm_head"], wdt)
+    ft = ff = None
+    if follow is not None:
+        ft = _c(follow["pool_tokens"], np.int32)
+        ff = _c(follow["frontier"], np.int32)
+        assert ft.shape == (B, P) and ff.shape == (B, K, width)
+    out = {
+        "pool_tokens": np.empty((B, P), np.int32), "pool_parent": np.empty((B, P), np.int32),
+        "pool_score": np.empty((B, P), np.float64), "frontier": np.empty((B, K, width), np.int32),
+        "row_logits": np.empty((B, K, width, V), np.float64) if want_logits else None,
+        "row_lse": np.empty((B, K, width), np.float64),
+        "row_hidden": np.empty((B, K, width, d), np.float64) if want_hidden else None,
+        "tree_tokens": np.empty((B, n_nodes), np.int32), "tree_parent": np.empty((B, n_nodes), np.int32),
+        "tree_depth": np.empty((B, n_nodes), np.int32), "tree_score": np.empty((B, n_nodes), np.float64),
+        "tree_pool": np.empty((B, n_nodes), np.int32),
+    }
+    rc = lib.orc_draft_tree(ctypes.byref(cfg), embed.ctypes.data, lm.ctypes.data, mods, B, max_new,
+                            tokens.ctypes.data, hidden.ctypes.data, n_new.ctypes.data, kv_len.ctypes.data,
+                            k_cache.ctypes.data, v_cache.ctypes.data, int(width), int(n_nodes), _ptr(ft), _ptr(ff),
+                            out["pool_tokens"].ctypes.data, out["pool_parent"].ctypes.data,
+                            out["pool_score"].ctypes.data, out["frontier"].ctypes.data, _ptr(out["row_logits"]),
+                            out["row_lse"].ctypes.data, _ptr(out["row_hidden"]), out["tree_tokens"].ctypes.data,
+                            out["tree_parent"].ctypes.data, out["tree_depth"].ctypes.data,
+                            out["tree_score"].ctypes.data, out["tree_pool"].ctypes.data)
+    if rc != 0:
+        raise ValueError(f"oracle tree round rejected its input (code {rc})")
+    out["k_cache"], out["v_cache"] = k_cache, v_cache
+    return out
+
+
+def accept_tree(tree_tokens: np.ndarray, tree_parent: np.ndarray, target_next: np.ndarray, n_new: np.ndarray,
+                kv_len: np.ndarray, n_steps: int) -> dict:
+    """Greedy acceptance of a draft tree (``orc_accept_tree``)."""
+    tt = _c(tree_tokens, np.int32)
+    tp = _c(tree_parent, np.int32)
+    tn = _c(target_next, np.int32)
+    B, m = tt.shape
+    assert tn.shape == (B, m + 1)
+    kv = _c(kv_len, np.int32).copy()
+    acc = np.empty(B, np.int32)
+    nodes = np.empty((B, n_steps), np.int32)
+    out = np.empty((B, n_steps + 1), np.int32)
+    _load().orc_accept_tree(B, m, n_steps, tt.ctypes.data, tp.ctypes.data, tn.ctypes.data,
+                            _c(n_new, np.int32).ctypes.data, kv.ctypes.data, acc.ctypes.data,
+                            nodes.ctypes.data, out.ctypes.data)
+    return {"accept_len": acc, "accept_nodes": nodes, "out_tokens": out, "kv_len": kv}

@@ -191,11 +191,15 @@ static void widen(const void *p, int bf16, int64_t n, double *out) {
     for (int64_t i = 0; i < n; ++i) out[i] = load_el(p, i, bf16);
 }
 
-/* One row through fusion + transformer layer of module m at cache position
- * pos.  u = [E(x); h] (already rounded per the contract).  Writes this row's
- * K/V at pos of sequence b's cache and the layer output to y. */
-static void layer_row(const orc_config *c, const orc_module *m, const double *u, int64_t pos,
-                      void *kc_b, void *vc_b, scratch *w) {
+/* One row through fusion + transformer layer of module m.  u = [E(x); h]
+ * (already rounded per the contract).  The row's q and k are rotated at
+ * position pos and its K/V are stored at cache slot `slot` of sequence b's
+ * cache.  Attention runs over the cache slots vis[0..n_vis) in that order, or
+ * over [0, pos] when vis is NULL (the chain, where slot == pos).  Writes the
+ * layer output to y. */
+static void layer_row_at(const orc_config *c, const orc_module *m, const double *u, int64_t pos,
+                         int64_t slot, const int64_t *vis, int64_t n_vis, void *kc_b, void *vc_b,
+                         scratch *w) {
     const int64_t d = c->hidden, Hq = c->n_q_heads, Hkv = c->n_kv_heads, D = c->head_dim, F = c->ffn;
     const int bf = c->bf16, ra = c->round_acts;
     const int64_t group = Hq / Hkv;
@@ -213,16 +217,33 @@ static void layer_row(const orc_config *c, const orc_module *m, const double *u,
     for (int64_t g = 0; g < Hkv; ++g) orc_rope(k + g * D, (int32_t)D, pos, c->rope_theta);
     for (int64_t g = 0; g < Hkv; ++g)
         for (int64_t t = 0; t < D; ++t) {
-            int64_t idx = (g * c->max_ctx + pos) * D + t;
+            int64_t idx = (g * c->max_ctx + slot) * D + t;
             store_el(kc_b, idx, bf, k[g * D + t]);
             store_el(vc_b, idx, bf, v[g * D + t]);
         }
+    const size_t el = bf ? 2 : 4;
+    if (!vis) {
 #pragma omp parallel for schedule(static) if (pos > 256)
-    for (int64_t h = 0; h < Hq; ++h) {
-        int64_t g = h / group;
-        const char *kb = (const char *)kc_b + (size_t)(g * c->max_ctx * D) * (bf ? 2 : 4);
-        const char *vb = (const char *)vc_b + (size_t)(g * c->max_ctx * D) * (bf ? 2 : 4);
-        orc_attend(q + h * D, kb, vb, bf, D, pos + 1, (int32_t)D, w->o + h * D);
+        for (int64_t h = 0; h < Hq; ++h) {
+            int64_t g = h / group;
+            const char *kb = (const char *)kc_b + (size_t)(g * c->max_ctx * D) * el;
+            const char *vb = (const char *)vc_b + (size_t)(g * c->max_ctx * D) * el;
+            orc_attend(q + h * D, kb, vb, bf, D, pos + 1, (int32_t)D, w->o + h * D);
+        }
+    } else {
+        /* gather the visible rows of each KV head, then plain softmax attention */
+        char *kt = malloc((size_t)(n_vis * D) * el), *vt = malloc((size_t)(n_vis * D) * el);
+        for (int64_t g = 0; g < Hkv; ++g) {
+            for (int64_t i = 0; i < n_vis; ++i) {
+                const size_t src = (size_t)((g * c->max_ctx + vis[i]) * D) * el;
+                memcpy(kt + (size_t)(i * D) * el, (const char *)kc_b + src, (size_t)D * el);
+                memcpy(vt + (size_t)(i * D) * el, (const char *)vc_b + src, (size_t)D * el);
+            }
+            for (int64_t h = g * group; h < (g + 1) * group; ++h)
+                orc_attend(q + h * D, kt, vt, bf, D, n_vis, (int32_t)D, w->o + h * D);
+        }
+        free(kt);
+        free(vt);
     }
     round_vec(w->o, Hq * D, ra);
     orc_matvec(m->w_o, bf, d, Hq * D, w->o, w->a);
@@ -237,6 +258,12 @@ static void layer_row(const orc_config *c, const orc_module *m, const double *u,
     round_vec(w->mm, F, ra);
     orc_matvec(m->w_down, bf, d, F, w->mm, w->y);
     for (int64_t i = 0; i < d; ++i) w->y[i] += w->a[i];
+}
+
+/* The chain's row: rotary position = cache slot = pos, causal window [0, pos]. */
+static void layer_row(const orc_config *c, const orc_module *m, const double *u, int64_t pos,
+                      void *kc_b, void *vc_b, scratch *w) {
+    layer_row_at(c, m, u, pos, pos, NULL, 0, kc_b, vc_b, w);
 }
 
 /* ---------------------------------------------------------------- selection */
@@ -507,6 +534,254 @@ void orc_accept_greedy(int32_t B, int32_t K, const int32_t *draft, const int32_t
             else if (j == a) v = target[b * (K + 1) + a];
             out_tokens[b * (K + 1) + j] = v;
         }
+        kv_len[b] += n_new[b];
+    }
+}
+
+/* ---------------------------------------------------------------- tree drafting */
+
+/* Tree-structured drafting.  PRISM states that its step-wise modules work
+ * unchanged with tree-shaped drafts (Sec. 3.2, after the recurrence), and
+ * evaluates a 6-step, 4-branch tree with at most 16 verified tokens (Sec. 4).
+ * The paper does not spell the tree out; this oracle reads it as the dynamic
+ * top-w expansion of EAGLE-2, where a candidate's score is the sum of the
+ * draft log-probabilities along its path:
+ *   step 1: the prefill as in the chain gives h^_0 and logits z; the w best
+ *     tokens of z are the depth-1 candidates, score = z_x - lse(z).  All w
+ *     form the first frontier.
+ *   step k = 2..K: frontier node j (token t, emitted by a row with output
+ *     h^) is processed by step k's module as its own row: input
+ *     [E(t); h^], rotary position L + n + k - 2 (its depth), K/V stored at
+ *     cache slot L + n + (k - 2) w + j, attention over the committed rows
+ *     [0, L + n) plus the slots of the rows that processed its ancestors and
+ *     its own slot.  The row's w best tokens become candidates with score =
+ *     parent score + z_x - lse(z).  The next frontier is the w best of these
+ *     w^2 candidates (score descending, then pool index ascending).
+ *   end: the verified tree is the n_nodes best candidates of the whole pool
+ *     (score descending, then pool index ascending), listed in pool order.
+ *     The pool lists shallower entries first and log-probabilities are <= 0,
+ *     so a parent always ranks before its children: every chosen node's
+ *     parent is chosen too, and parents precede children in the list.
+ * Pool layout per sequence: P = w + (K - 1) w^2 entries; depth-1 candidate r
+ * at index r; candidate r of row j at step k at w + (k - 2) w^2 + j w + r.
+ *
+ * follow_tokens [B, P] / follow_frontier [B, K, w] (both or neither): use
+ * these candidate tokens and frontier choices instead of the oracle's own
+ * (scores are still the oracle's), so that another implementation's tree can
+ * be recomputed node by node.
+ * Outputs: pool_tokens / pool_parent (pool index, -1 = root) / pool_score
+ * [B, P]; frontier [B, K, w] (pool indices chosen after each step);
+ * row_logits [B, K, w, V], row_lse [B, K, w] and row_hidden [B, K, w, d]
+ * when non-NULL (step 1 fills only row 0); tree_* [B, n_nodes] (tree_parent
+ * is the parent's position in the tree, -1 = root; tree_pool the pool index).
+ * Returns 0; 1 bad argument; 2 token id out of range; 3 cache capacity
+ * (kv_len + n_new + (K - 1) w > max_ctx); 4 invalid follow input. */
+static const double *g_tree_score;
+static int cmp_tree(const void *pa, const void *pb) {
+    int32_t a = *(const int32_t *)pa, b = *(const int32_t *)pb;
+    if (g_tree_score[a] > g_tree_score[b]) return -1;
+    if (g_tree_score[a] < g_tree_score[b]) return 1;
+    return (a > b) - (a < b);
+}
+
+static double log_sum_exp(const double *z, int64_t V) {
+    double m = -INFINITY;
+    for (int64_t i = 0; i < V; ++i) m = fmax(m, z[i]);
+    double s = 0.0;
+    for (int64_t i = 0; i < V; ++i) s += exp(z[i] - m);
+    return m + log(s);
+}
+
+int orc_draft_tree(const orc_config *c, const void *embed, const void *lm_head, const orc_module *steps,
+                   int32_t B, int32_t max_new, const int32_t *tokens, const void *hidden,
+                   const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
+                   int32_t width, int32_t n_nodes, const int32_t *follow_tokens,
+                   const int32_t *follow_frontier, int32_t *pool_tokens, int32_t *pool_parent,
+                   double *pool_score, int32_t *frontier, double *row_logits, double *row_lse,
+                   double *row_hidden, int32_t *tree_tokens, int32_t *tree_parent, int32_t *tree_depth,
+                   double *tree_score, int32_t *tree_pool) {
+    const int64_t d = c->hidden, V = c->vocab, K = c->n_steps, F = c->ffn;
+    const int64_t Hq = c->n_q_heads, Hkv = c->n_kv_heads, D = c->head_dim;
+    const int64_t w_ = width, P = width + (K - 1) * (int64_t)width * width;
+    const int bf = c->bf16;
+    if (K < 1 || width < 1 || width > V || n_nodes < 1 || n_nodes > P || Hq % Hkv != 0 || D % 2 != 0) return 1;
+    if ((follow_tokens == NULL) != (follow_frontier == NULL)) return 1;
+    for (int32_t b = 0; b < B; ++b) {
+        if (n_new[b] < 1 || n_new[b] > max_new || kv_len[b] < 0) return 1;
+        if ((int64_t)kv_len[b] + n_new[b] + (K - 1) * w_ > c->max_ctx) return 3;
+        for (int32_t i = 0; i < n_new[b]; ++i)
+            if (tokens[b * max_new + i] < 0 || tokens[b * max_new + i] >= V) return 2;
+    }
+    scratch w;
+    w.x0 = calloc((size_t)d, 8); w.n1 = calloc((size_t)d, 8);
+    w.qkv = calloc((size_t)((Hq + 2 * Hkv) * D), 8); w.o = calloc((size_t)(Hq * D), 8);
+    w.a = calloc((size_t)d, 8); w.n2 = calloc((size_t)d, 8);
+    w.gu = calloc((size_t)(2 * F), 8); w.mm = calloc((size_t)F, 8); w.y = calloc((size_t)d, 8);
+    w.g_attn = calloc((size_t)d, 8); w.g_mlp = calloc((size_t)d, 8); w.g_final = calloc((size_t)d, 8);
+    double *u = calloc((size_t)(2 * d), 8);
+    double *z = calloc((size_t)V, 8);
+    int32_t *order = calloc((size_t)V, 4);
+    int32_t *tid = calloc((size_t)width, 4);
+    double *tval = calloc((size_t)width, 8);
+    /* h^ of every row of the round: row 0 = the prefill's last row, then
+     * (k - 2) w + j + 1 for row j of step k */
+    double *H = calloc((size_t)((1 + (K - 1) * w_) * d), 8);
+    /* cache-slot offsets (from L + n) of each row's own and ancestors' rows */
+    int64_t *anc = calloc((size_t)((1 + (K - 1) * w_) * K), 8);
+    int32_t *n_anc = calloc((size_t)(1 + (K - 1) * w_), 4);
+    int64_t *vis = calloc((size_t)(c->max_ctx), 8);
+    int32_t *idx = calloc((size_t)P, 4), *depth = calloc((size_t)P, 4), *pos_in_tree = calloc((size_t)P, 4);
+    orc_config ct = *c;
+    ct.topk = width;
+    const size_t el = bf ? 2 : 4;
+    const int64_t cache_seq = Hkv * (int64_t)c->max_ctx * D;
+    int rc = 0;
+
+    for (int64_t e = 0; e < P; ++e) depth[e] = e < w_ ? 1 : (int32_t)(2 + (e - w_) / (w_ * w_));
+    for (int32_t b = 0; b < B && rc == 0; ++b) {
+        void *kc_b = (char *)k_cache + (size_t)(b * cache_seq) * el;
+        void *vc_b = (char *)v_cache + (size_t)(b * cache_seq) * el;
+        const int64_t L = kv_len[b], n = n_new[b];
+        int32_t *ptok = pool_tokens + (int64_t)b * P, *ppar = pool_parent + (int64_t)b * P;
+        double *psc = pool_score + (int64_t)b * P;
+        int32_t *front = frontier + (int64_t)b * K * w_;
+        if (row_logits) memset(row_logits + (int64_t)b * K * w_ * V, 0, sizeof(double) * (size_t)(K * w_ * V));
+        if (row_lse) memset(row_lse + (int64_t)b * K * w_, 0, sizeof(double) * (size_t)(K * w_));
+        if (row_hidden) memset(row_hidden + (int64_t)b * K * w_ * d, 0, sizeof(double) * (size_t)(K * w_ * d));
+        for (int64_t k = 1; k <= K && rc == 0; ++k) {
+            const orc_module *m = &steps[k - 1];
+            const int64_t rows = k == 1 ? 1 : w_;
+            const int64_t base = k == 1 ? 0 : w_ + (k - 2) * w_ * w_;
+            for (int64_t j = 0; j < rows && rc == 0; ++j) {
+                const int64_t row = k == 1 ? 0 : 1 + (k - 2) * w_ + j;
+                int64_t parent = -1;
+                if (k == 1) {
+                    for (int64_t i = 0; i < n; ++i) {
+                        int32_t x = tokens[b * max_new + i];
+                        for (int64_t t = 0; t < d; ++t) {
+                            u[t] = load_el(embed, (int64_t)x * d + t, bf);
+                            u[d + t] = load_el(hidden, ((int64_t)b * max_new + i) * d + t, bf);
+                        }
+                        round_vec(u, 2 * d, c->round_acts);
+                        layer_row(c, m, u, L + i, kc_b, vc_b, &w);
+                    }
+                    n_anc[row] = 0;
+                } else {
+                    parent = front[(k - 2) * w_ + j];
+                    /* the row that emitted the parent candidate */
+                    const int64_t erow = parent < w_ ? 0 : 1 + (k - 3) * w_ + (parent - (w_ + (k - 3) * w_ * w_)) / w_;
+                    const int64_t slot_off = (k - 2) * w_ + j;
+                    n_anc[row] = n_anc[erow] + 1;
+                    for (int32_t i = 0; i < n_anc[erow]; ++i) anc[row * K + i] = anc[erow * K + i];
+                    anc[row * K + n_anc[erow]] = slot_off;
+                    const int32_t x = ptok[parent];
+                    for (int64_t t = 0; t < d; ++t) {
+                        u[t] = load_el(embed, (int64_t)x * d + t, bf);
+                        u[d + t] = H[erow * d + t];
+                    }
+                    round_vec(u, 2 * d, c->round_acts);
+                    int64_t nv = 0;
+                    for (int64_t p = 0; p < L + n; ++p) vis[nv++] = p;
+                    for (int32_t i = 0; i < n_anc[row]; ++i) vis[nv++] = L + n + anc[row * K + i];
+                    layer_row_at(c, m, u, L + n + k - 2, L + n + slot_off, vis, nv, kc_b, vc_b, &w);
+                }
+                memcpy(H + row * d, w.y, sizeof(double) * (size_t)d);
+                select_tokens(&ct, lm_head, m, w.y, z, order, &w, tid, tval);
+                const double lse = log_sum_exp(z, V);
+                const int64_t ri = ((int64_t)b * K + (k - 1)) * w_ + j;
+                if (row_logits) memcpy(row_logits + ri * V, z, sizeof(double) * (size_t)V);
+                if (row_lse) row_lse[ri] = lse;
+                if (row_hidden) memcpy(row_hidden + ri * d, w.y, sizeof(double) * (size_t)d);
+                for (int64_t r = 0; r < w_; ++r) {
+                    const int64_t e = base + j * w_ + r;
+                    int32_t x = tid[r];
+                    if (follow_tokens) {
+                        x = follow_tokens[(int64_t)b * P + e];
+                        if (x < 0 || x >= V) { rc = 4; break; }
+                        for (int64_t r2 = 0; r2 < r; ++r2)
+                            if (ptok[base + j * w_ + r2] == x) rc = 4;
+                    }
+                    ptok[e] = x;
+                    ppar[e] = (int32_t)parent;
+                    psc[e] = (parent < 0 ? 0.0 : psc[parent]) + (z[x] - lse);
+                }
+            }
+            if (rc) break;
+            /* the next frontier: the w best of this step's candidates */
+            const int64_t ncand = rows * w_;
+            for (int64_t e = 0; e < ncand; ++e) idx[e] = (int32_t)(base + e);
+            g_tree_score = psc;
+            qsort(idx, (size_t)ncand, sizeof(int32_t), cmp_tree);
+            for (int64_t j = 0; j < w_; ++j) {
+                int32_t e = idx[j];
+                if (follow_frontier) {
+                    e = follow_frontier[((int64_t)b * K + (k - 1)) * w_ + j];
+                    if (e < base || e >= base + ncand) rc = 4;
+                    for (int64_t j2 = 0; j2 < j; ++j2)
+                        if (front[(k - 1) * w_ + j2] == e) rc = 4;
+                }
+                front[(k - 1) * w_ + j] = e;
+            }
+        }
+        if (rc) break;
+        /* the verified tree: the n_nodes best of the pool, listed in pool order */
+        for (int64_t e = 0; e < P; ++e) idx[e] = (int32_t)e;
+        g_tree_score = psc;
+        qsort(idx, (size_t)P, sizeof(int32_t), cmp_tree);
+        for (int64_t e = 0; e < P; ++e) pos_in_tree[e] = -1;
+        for (int64_t i = 0; i < n_nodes; ++i) pos_in_tree[idx[i]] = 0;
+        int32_t np = 0;
+        for (int64_t e = 0; e < P; ++e)
+            if (pos_in_tree[e] == 0) pos_in_tree[e] = np++;
+        for (int64_t e = 0; e < P; ++e) {
+            if (pos_in_tree[e] < 0) continue;
+            const int64_t o = (int64_t)b * n_nodes + pos_in_tree[e];
+            tree_pool[o] = (int32_t)e;
+            tree_tokens[o] = ptok[e];
+            tree_depth[o] = depth[e];
+            tree_score[o] = psc[e];
+            tree_parent[o] = ppar[e] < 0 ? -1 : pos_in_tree[ppar[e]];
+            if (ppar[e] >= 0 && pos_in_tree[ppar[e]] < 0) rc = 4;   /* cannot happen: see above */
+        }
+    }
+    free(w.x0); free(w.n1); free(w.qkv); free(w.o); free(w.a); free(w.n2); free(w.gu);
+    free(w.mm); free(w.y); free(w.g_attn); free(w.g_mlp); free(w.g_final);
+    free(u); free(z); free(order); free(tid); free(tval); free(H); free(anc); free(n_anc); free(vis);
+    free(idx); free(depth); free(pos_in_tree);
+    return rc;
+}
+
+/* Greedy acceptance of a draft tree (Sec. 2's temperature-0 rule applied
+ * along the tree, as in tree-based verification): target_next[b, 0] is the
+ * target's token after the last accepted token (the root) and
+ * target_next[b, 1 + i] its token after tree node i.  From the root, repeatedly
+ * accept the child whose token equals the target's token at the current node;
+ * stop when no child matches.  accept_len[b] = accepted nodes a (0..K);
+ * accept_nodes[b, 0:a] their tree positions (rest -1); out_tokens[b] = their
+ * tokens followed by the target's token at the last accepted node (rest -1);
+ * kv_len[b] += n_new[b]. */
+void orc_accept_tree(int32_t B, int32_t n_nodes, int32_t K, const int32_t *tree_tokens,
+                     const int32_t *tree_parent, const int32_t *target_next, const int32_t *n_new,
+                     int32_t *kv_len, int32_t *accept_len, int32_t *accept_nodes, int32_t *out_tokens) {
+    for (int32_t b = 0; b < B; ++b) {
+        const int32_t *tok = tree_tokens + (int64_t)b * n_nodes, *par = tree_parent + (int64_t)b * n_nodes;
+        const int32_t *tn = target_next + (int64_t)b * (n_nodes + 1);
+        int32_t cur = -1, a = 0;
+        for (int32_t j = 0; j < K; ++j) accept_nodes[b * K + j] = -1;
+        for (int32_t j = 0; j <= K; ++j) out_tokens[b * (K + 1) + j] = -1;
+        while (a < K) {
+            const int32_t want = tn[cur + 1];
+            int32_t next = -1;
+            for (int32_t i = 0; i < n_nodes && next < 0; ++i)
+                if (par[i] == cur && tok[i] == want) next = i;
+            if (next < 0) break;
+            accept_nodes[b * K + a] = next;
+            out_tokens[b * (K + 1) + a] = tok[next];
+            ++a;
+            cur = next;
+        }
+        out_tokens[b * (K + 1) + a] = tn[cur + 1];
+        accept_len[b] = a;
         kv_len[b] += n_new[b];
     }
 }

@@ -112,9 +112,9 @@ def bf16_to_f32(a: np.ndarray) -> np.ndarray:
 
 
 from .workloads import (Shape, Workload, WORKLOADS, make_weights,  # noqa: E402
-                        make_round_inputs, make_targets, max_ctx_of)
+                        make_round_inputs, make_targets, make_tree_targets, max_ctx_of)
 
 __all__ = ["build", "tag", "normal", "uniform_int", "uniform01", "raw",
            "splitmix64_sequence", "bf16_to_f32", "Shape", "Workload",
            "WORKLOADS", "make_weights", "make_round_inputs", "make_targets",
-           "max_ctx_of"]
+           "make_tree_targets", "max_ctx_of"]

@@ -62,6 +62,8 @@ class Workload:
     weight_sigma: float = 0.02
     gain_sigma: float = 0.0
     f_map: tuple = field(default=())   # module index of each step; () = one module per step
+    tree_width: int = 0     # > 0: tree drafting with this many branches per node
+    tree_nodes: int = 0     # verified tree size of a tree round
 
     def modules(self) -> tuple:
         return self.f_map if self.f_map else tuple(range(self.shape.n_steps))
@@ -86,12 +88,19 @@ WORKLOADS = {
     "l3-8b-b64": Workload("l3-8b-b64", L3_8B, 64, 512, 4096, 1, 8, 2),
     "l2-7b-b8": Workload("l2-7b-b8", L2_7B, 8, 1024, 1024, 1, 1, 3),
     "l3-70b-b32": Workload("l3-70b-b32", L3_70B, 32, 4096, 4096, 1, 1, 4),
+    # tree drafting: w branches per node, the n best candidates verified
+    "tiny-bf16-tree": Workload("tiny-bf16-tree", replace(TINY_BF16, name="tiny-bf16-k4", n_steps=4), 3, 16, 40, 3,
+                               1, 0, gain_sigma=0.1, tree_width=4, tree_nodes=16),
+    # the tree the paper evaluates (Sec. 4): 6 steps, 4 branches, 16 verified tokens, batch 1
+    "l3-8b-b1-tree": Workload("l3-8b-b1-tree", replace(L3_8B, name="llama3-8b-k6", n_steps=6), 1, 2048, 2048, 1,
+                              1, 1, tree_width=4, tree_nodes=16),
 }
 
 
 def max_ctx_of(w: Workload) -> int:
-    """Cache capacity: longest committed context + new rows + draft rows, rounded up to 16."""
-    need = w.ctx_hi + w.n_new + w.shape.n_steps
+    """Cache capacity: longest committed context + new rows + draft rows (K for
+    the chain, (K - 1) * width for a tree), rounded up to 16."""
+    need = w.ctx_hi + w.n_new + max(w.shape.n_steps, (w.shape.n_steps - 1) * w.tree_width)
     return (need + 15) // 16 * 16
 
 
@@ -182,3 +191,22 @@ def make_targets(w: Workload, draft_ids: np.ndarray) -> np.ndarray:
     tgt = rnd.copy()
     tgt[:, :K] = np.where(u < 0.5, draft_ids, rnd[:, :K])
     return tgt.astype(np.int32)
+
+
+def make_tree_targets(w: Workload, tree_tokens: np.ndarray, tree_parent: np.ndarray) -> np.ndarray:
+    """Target tokens [B, n + 1] for greedy tree acceptance: entry 0 is the
+    target's token after the root, entry 1 + i its token after tree node i.
+    Each entry is, with probability 1/2, the token of a uniformly chosen child
+    of that node (when it has one), else a uniform id."""
+    B, n = tree_tokens.shape
+    V = w.shape.vocab
+    u = uniform01(w.seed, "tree_target_u", (B, n + 1))
+    pick = uniform01(w.seed, "tree_target_pick", (B, n + 1))
+    rnd = uniform_int(w.seed, "tree_target_tok", (B, n + 1), 0, V - 1)
+    out = rnd.copy()
+    for b in range(B):
+        for node in range(-1, n):
+            kids = [i for i in range(n) if tree_parent[b, i] == node]
+            if kids and u[b, node + 1] < 0.5:
+                out[b, node + 1] = tree_tokens[b, kids[int(pick[b, node + 1] * len(kids))]]
+    return out.astype(np.int32)

@@ -42,7 +42,9 @@ def _rope(x: torch.Tensor, pos: torch.Tensor, theta: float) -> torch.Tensor:
     return torch.cat([z.real, z.imag], dim=-1)
 
 
-def reference_round(shape, weights, inputs, *, topk=1, round_acts=False, final_norm=True):
+def reference_round(shape, weights, inputs, *, topk=1, round_acts=False, final_norm=True, forced=None):
+    """``forced`` [B, K-1]: tokens fed to steps 2..K in place of the previous
+    step's argmax (a chain that follows a given path)."""
     d, Hq, Hkv, D, F = shape.hidden, shape.n_q_heads, shape.n_kv_heads, shape.head_dim, shape.ffn
     K, eps = shape.n_steps, shape.rms_eps
     grp = Hq // Hkv
@@ -100,6 +102,8 @@ def reference_round(shape, weights, inputs, *, topk=1, round_acts=False, final_n
             order = np.lexsort((np.arange(zs.size), -zs))
             prev = int(order[0])
             out_ids[b, k - 1] = prev
+            if forced is not None and k < K:
+                prev = int(forced[b, k - 1])
             out_top[b, k - 1] = order[:topk]
             out_logits[b, k - 1] = zs
             out_hidden[b, k - 1] = hhat.numpy()
