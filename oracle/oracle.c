@@ -581,7 +581,7 @@ static int cmp_tree(const void *pa, const void *pb) {
     int32_t a = *(const int32_t *)pa, b = *(const int32_t *)pb;
     if (g_tree_score[a] > g_tree_score[b]) return -1;
     if (g_tree_score[a] < g_tree_score[b]) return 1;
-    return (a > b) - (a < b);
+    return a < b ? -1 : (a > b);   /* equal scores: lower pool index first */
 }
 
 static double log_sum_exp(const double *z, int64_t V) {
@@ -782,6 +782,6 @@ void orc_accept_tree(int32_t B, int32_t n_nodes, int32_t K, const int32_t *tree_
         }
         out_tokens[b * (K + 1) + a] = tn[cur + 1];
         accept_len[b] = a;
-        kv_len[b] += n_new[b];
+        kv_len[b] = kv_len[b] + n_new[b];   /* only the step-1 rows are committed */
     }
 }

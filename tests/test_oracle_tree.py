@@ -276,6 +276,7 @@ TREE_MUTANTS = [
     ("tree-final-size", "for (int64_t i = 0; i < n_nodes; ++i) pos_in_tree[idx[i]] = 0;",
      "for (int64_t i = 0; i < n_nodes; ++i) pos_in_tree[idx[i + (i + 1 < n_nodes ? 0 : 1)]] = 0;"),
     ("accept-tree-wrong-target", "const int32_t want = tn[cur + 1];", "const int32_t want = tn[a];"),
+    ("accept-tree-commit", "kv_len[b] = kv_len[b] + n_new[b];   /* only", "kv_len[b] = kv_len[b] + n_new[b] + a;   /* only"),
     ("accept-tree-bonus", "out_tokens[b * (K + 1) + a] = tn[cur + 1];", "out_tokens[b * (K + 1) + a] = tn[a];"),
 ]
 
