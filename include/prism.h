@@ -68,13 +68,17 @@ typedef enum { PRISM_F32 = 0, PRISM_BF16 = 1 } prism_dtype;
  * positions per sequence) and max_new (accepted tokens per sequence fed to
  * step 1) size the workspace.  topk in 1..8 candidates are reported per step
  * (the chained token is the first).  final_norm: 1 applies RMSNorm with the
- * step's g_final before the LM head.  rope_theta and rms_eps as in Llama. */
+ * step's g_final before the LM head.  rope_theta and rms_eps as in Llama.
+ * max_tree_width: 0 (no tree rounds), or the largest width w (1..8) that
+ * prism_draft_tree will be called with; the workspace then holds w rows per
+ * sequence for the draft steps. */
 typedef struct {
     int32_t hidden, n_q_heads, n_kv_heads, head_dim, ffn, vocab, n_steps;
     int32_t dtype;
     int32_t max_batch, max_ctx, max_new, topk;
     float rope_theta, rms_eps;
     int32_t final_norm;
+    int32_t max_tree_width;
 } prism_config;
 
 /* One processing module (Sec. 3.2: a fully connected fusion layer and a
@@ -200,6 +204,79 @@ prism_status prism_accept_sampled(prism_ctx *ctx, int32_t batch, const int32_t *
                                   const float *draft_lse, float temperature, const float *target_probs,
                                   const uint64_t *seed, const int32_t *n_new, int32_t *kv_len,
                                   int32_t *accept_len, int32_t *out_tokens, void *stream);
+
+/* Outputs of a tree round (prism_draft_tree), all device pointers:
+ *   tokens, parents, depths  int32 [batch, n_nodes]  the verified tree in
+ *                 candidate-pool order (parents before children); parents[i]
+ *                 is the position of node i's parent in the list, -1 for a
+ *                 child of the root (the last accepted token); depth 1..K
+ *   scores        float [batch, n_nodes]  summed draft log-probabilities of
+ *                 each node's path
+ *   pool_tokens, pool_parents, pool_scores  [batch, P], P = w + (K - 1) w^2:
+ *                 every candidate of the round (or NULL).  Depth-1 candidate
+ *                 r sits at r; candidate r of frontier row j at step k at
+ *                 w + (k - 2) w^2 + j w + r; parents are pool indices
+ *   frontier      int32 [batch, K, w]  pool indices of the frontier chosen
+ *                 after each step (or NULL)
+ *   row_logits    float [K, batch, w, V]  every processed row's logits (or
+ *                 NULL); step 1 has one row per sequence, written at j = 0 */
+typedef struct {
+    int32_t *tokens, *parents, *depths;
+    float *scores;
+    int32_t *pool_tokens, *pool_parents;
+    float *pool_scores;
+    int32_t *frontier;
+    float *row_logits;
+} prism_tree_outputs;
+
+/* One tree-drafting round.  PRISM's step modules apply unchanged to
+ * tree-shaped drafts (Sec. 3.2, after the recurrence), and the paper
+ * evaluates a 6-step, 4-branch tree verifying at most 16 tokens (Sec. 4).
+ * This is the dynamic top-w expansion of that tree:
+ *   step 1: the prefill of prism_draft_round; the w best tokens of its
+ *     logits are the depth-1 candidates and the first frontier;
+ *   step k = 2..K: each of the w frontier nodes of a sequence is one row of
+ *     step k's module: input [E(token); h^ of the row whose LM head proposed
+ *     it], rotary position kv_len + n_new + k - 2, K/V stored at cache slot
+ *     kv_len + n_new + (k - 2) w + j, attention over the rows
+ *     [0, kv_len + n_new) and the slots of the node's ancestors and itself.
+ *     Each row's w best tokens are candidates whose score is the parent's
+ *     score plus the token's draft log-probability (logit - log-sum-exp);
+ *     the next frontier is the w best of the w^2 new candidates;
+ *   end: the verified tree is the n_nodes best candidates of the round.
+ * Orders: top-w by logit, then id; frontiers and the tree by score
+ * descending, then pool index ascending.
+ *   width        1..max_tree_width; (K - 1) * width <= 64; P <= 1024
+ *   n_nodes      1..P
+ *   out          see prism_tree_outputs (tokens, parents, depths, scores
+ *                required)
+ * Other arguments as prism_draft_round; cache rows kv_len .. kv_len + n_new +
+ * (K - 1) w - 1 are written (a row beyond max_ctx sets the cache-range bit
+ * and is skipped).  With width 1 and n_nodes K the tree is the greedy chain.
+ * Captured as a CUDA graph per argument set, like prism_draft_round.
+ * Errors: INVALID_ARG (null or misaligned argument, width or n_nodes out of
+ * range), CAPACITY (batch > max_batch, width > max_tree_width), NOT_LOADED,
+ * CUDA. */
+prism_status prism_draft_tree(prism_ctx *ctx, int32_t batch, const int32_t *tokens, const void *hidden,
+                              const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
+                              int32_t width, int32_t n_nodes, const prism_tree_outputs *out, void *stream);
+
+/* Greedy acceptance of a draft tree (Sec. 2's temperature-0 rule applied
+ * along the tree, as in tree verification): starting at the root, accept the
+ * child whose token equals the target's token at the current node, until no
+ * child matches or K nodes are accepted.
+ *   tree_tokens, tree_parents int32 [batch, n_nodes] (as prism_draft_tree
+ *   writes them); target_next int32 [batch, n_nodes + 1]: entry 0 the
+ *   target's token after the root, entry 1 + i its token after node i;
+ *   n_new int32 [batch]; kv_len int32 [batch] in/out (+= n_new);
+ *   accept_len int32 [batch] out; accept_nodes int32 [batch, K] out (the
+ *   accepted nodes' positions, then -1); out_tokens int32 [batch, K+1] out
+ *   (their tokens, the target's token at the last accepted node, then -1).
+ * Errors: INVALID_ARG, CAPACITY, CUDA. */
+prism_status prism_accept_tree(prism_ctx *ctx, int32_t batch, int32_t n_nodes, const int32_t *tree_tokens,
+                               const int32_t *tree_parents, const int32_t *target_next, const int32_t *n_new,
+                               int32_t *kv_len, int32_t *accept_len, int32_t *accept_nodes,
+                               int32_t *out_tokens, void *stream);
 
 /* LM-head selection that allocates nothing.  The paper has no counterpart to
  * this entry point; it serves callers that cannot call cudaMalloc, so cannot

@@ -18,7 +18,8 @@ __all__ = ["Drafter", "PrismError", "library", "lm_head_topk_static", "STEP_TENS
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.environ.get("PRISM_LIB") or os.path.join(_HERE, "libprism.so")
 STEP_TENSORS = ("w_fuse", "g_attn", "w_qkv", "w_o", "g_mlp", "w_gate_up", "w_down", "g_final")
-KERNEL_KINDS = ("fusion", "qkv", "rope_append", "attention", "o_proj", "gate_up", "down", "lm_head", "sample")
+KERNEL_KINDS = ("fusion", "qkv", "rope_append", "attention", "o_proj", "gate_up", "down", "lm_head", "sample",
+                "tree_gather", "tree_lse", "tree_select")
 _STATUS = ["OK", "INVALID_ARG", "SHAPE", "CAPACITY", "NOT_LOADED", "CUDA", "OOM", "DEVICE_FLAG", "TIMEOUT"]
 
 
@@ -33,7 +34,14 @@ class _Config(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "hidden", "n_q_heads", "n_kv_heads", "head_dim", "ffn", "vocab", "n_steps", "dtype",
         "max_batch", "max_ctx", "max_new", "topk")] + [
-        ("rope_theta", ctypes.c_float), ("rms_eps", ctypes.c_float), ("final_norm", ctypes.c_int32)]
+        ("rope_theta", ctypes.c_float), ("rms_eps", ctypes.c_float), ("final_norm", ctypes.c_int32),
+        ("max_tree_width", ctypes.c_int32)]
+
+
+class _TreeOutputs(ctypes.Structure):
+    _fields_ = [("tokens", ctypes.c_void_p), ("parents", ctypes.c_void_p), ("depths", ctypes.c_void_p),
+                ("scores", ctypes.c_void_p), ("pool_tokens", ctypes.c_void_p), ("pool_parents", ctypes.c_void_p),
+                ("pool_scores", ctypes.c_void_p), ("frontier", ctypes.c_void_p), ("row_logits", ctypes.c_void_p)]
 
 
 class _StepWeights(ctypes.Structure):
@@ -68,12 +76,14 @@ def library() -> ctypes.CDLL:
         flt = ctypes.c_float
         lib.prism_draft_round_sampled.argtypes = [vp, i32] + [vp] * 6 + [flt] + [vp] * 8
         lib.prism_accept_sampled.argtypes = [vp, i32, vp, vp, vp, flt] + [vp] * 7
+        lib.prism_draft_tree.argtypes = [vp, i32] + [vp] * 6 + [i32, i32, P(_TreeOutputs), vp]
+        lib.prism_accept_tree.argtypes = [vp, i32, i32] + [vp] * 9
         lib.prism_get_error.restype = ctypes.c_char_p
         lib.prism_version.restype = ctypes.c_char_p
         for f in ("prism_create", "prism_destroy", "prism_load_shared_weights", "prism_load_step_weights",
                   "prism_draft_round", "prism_accept_greedy", "prism_sync_status", "prism_set_option",
                   "prism_profile_round", "prism_lm_head_topk_static", "prism_round_launches",
-                  "prism_draft_round_sampled", "prism_accept_sampled"):
+                  "prism_draft_round_sampled", "prism_accept_sampled", "prism_draft_tree", "prism_accept_tree"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -95,17 +105,18 @@ class Drafter:
 
     def __init__(self, *, hidden, n_q_heads, n_kv_heads, head_dim, ffn, vocab, n_steps,
                  dtype="bf16", max_batch=1, max_ctx=4096, max_new=1, topk=1,
-                 rope_theta=10000.0, rms_eps=1e-5, final_norm=True, device=0):
+                 rope_theta=10000.0, rms_eps=1e-5, final_norm=True, max_tree_width=0, device=0):
         self.lib = library()
         self.dtype = dtype
         self.tdtype = torch.bfloat16 if dtype == "bf16" else torch.float32
         self.device = torch.device("cuda", device)
         self.cfg = _Config(hidden, n_q_heads, n_kv_heads, head_dim, ffn, vocab, n_steps,
                            1 if dtype == "bf16" else 0, max_batch, max_ctx, max_new, topk,
-                           rope_theta, rms_eps, int(final_norm))
+                           rope_theta, rms_eps, int(final_norm), int(max_tree_width))
         self.hidden, self.n_steps, self.vocab, self.topk = hidden, n_steps, vocab, topk
         self.max_batch, self.max_ctx, self.max_new = max_batch, max_ctx, max_new
         self.n_kv_heads, self.head_dim = n_kv_heads, head_dim
+        self.max_tree_width = max_tree_width
         self._shapes = {
             "w_fuse": (hidden, 2 * hidden), "g_attn": (hidden,),
             "w_qkv": ((n_q_heads + 2 * n_kv_heads) * head_dim, hidden),
@@ -118,12 +129,13 @@ class Drafter:
         self.h = h
 
     @classmethod
-    def from_shape(cls, shape, *, max_batch, max_ctx, max_new, topk=1, final_norm=True, device=0):
+    def from_shape(cls, shape, *, max_batch, max_ctx, max_new, topk=1, final_norm=True, max_tree_width=0,
+                   device=0):
         return cls(hidden=shape.hidden, n_q_heads=shape.n_q_heads, n_kv_heads=shape.n_kv_heads,
                    head_dim=shape.head_dim, ffn=shape.ffn, vocab=shape.vocab, n_steps=shape.n_steps,
                    dtype=shape.dtype, max_batch=max_batch, max_ctx=max_ctx, max_new=max_new,
                    topk=topk, rope_theta=shape.rope_theta, rms_eps=shape.rms_eps,
-                   final_norm=final_norm, device=device)
+                   final_norm=final_norm, max_tree_width=max_tree_width, device=device)
 
     # ------------------------------------------------------------ helpers
     def _check(self, status, h="self"):
@@ -177,7 +189,8 @@ class Drafter:
             raise ValueError("k_cache holds fewer sequences than the batch")
         self._tensor(k_cache, cshape, self.tdtype, "k_cache")
         self._tensor(v_cache, cshape, self.tdtype, "v_cache")
-        self._tensor(draft_ids, (B, self.n_steps), i32, "draft_ids")
+        if draft_ids is not None:
+            self._tensor(draft_ids, (B, self.n_steps), i32, "draft_ids")
         if topk_ids is not None:
             self._tensor(topk_ids, (B, self.n_steps, self.topk), i32, "topk_ids")
         if topk_logits is not None:
@@ -234,6 +247,52 @@ class Drafter:
             self.h, B, _ptr(draft), _ptr(logits), _ptr(draft_lse), float(temperature), _ptr(target_probs),
             _ptr(seed), _ptr(n_new), _ptr(kv_len), _ptr(accept_len), _ptr(out_tokens), _stream(stream)))
 
+    def tree_pool_size(self, width: int) -> int:
+        """Candidates of one tree round of this width: w + (K - 1) w^2."""
+        return width + (self.n_steps - 1) * width * width
+
+    def draft_tree(self, tokens, hidden, n_new, kv_len, k_cache, v_cache, width: int, tree_tokens, tree_parents,
+                   tree_depths, tree_scores, pool_tokens=None, pool_parents=None, pool_scores=None, frontier=None,
+                   row_logits=None, stream=None):
+        """Tree-drafting round (``prism_draft_tree``): the verified tree goes to
+        tree_tokens / tree_parents / tree_depths (int32 [B, n]) and tree_scores
+        (fp32 [B, n]), n = tree_tokens.shape[1]; the candidate pool
+        ([B, P]), the frontiers ([B, K, w]) and every row's logits
+        ([K, B, w, V]) are optional outputs."""
+        B = self._round_args(tokens, hidden, n_new, kv_len, k_cache, v_cache, None, None, None)
+        n = tree_tokens.shape[1]
+        P = self.tree_pool_size(width)
+        i32, f32 = torch.int32, torch.float32
+        for t, shp, dt, name in ((tree_tokens, (B, n), i32, "tree_tokens"), (tree_parents, (B, n), i32, "tree_parents"),
+                                 (tree_depths, (B, n), i32, "tree_depths"), (tree_scores, (B, n), f32, "tree_scores"),
+                                 (pool_tokens, (B, P), i32, "pool_tokens"), (pool_parents, (B, P), i32, "pool_parents"),
+                                 (pool_scores, (B, P), f32, "pool_scores"),
+                                 (frontier, (B, self.n_steps, width), i32, "frontier"),
+                                 (row_logits, (self.n_steps, B, width, self.vocab), f32, "row_logits")):
+            if t is not None:
+                self._tensor(t, shp, dt, name)
+        out = _TreeOutputs(*[None if t is None else t.data_ptr() for t in (
+            tree_tokens, tree_parents, tree_depths, tree_scores, pool_tokens, pool_parents, pool_scores, frontier,
+            row_logits)])
+        self._check(self.lib.prism_draft_tree(
+            self.h, B, _ptr(tokens), _ptr(hidden), _ptr(n_new), _ptr(kv_len), _ptr(k_cache), _ptr(v_cache),
+            int(width), int(n), ctypes.byref(out), _stream(stream)))
+
+    def accept_tree(self, tree_tokens, tree_parents, target_next, n_new, kv_len, accept_len, accept_nodes,
+                    out_tokens, stream=None):
+        """Greedy tree acceptance (``prism_accept_tree``); target_next int32 [B, n + 1]."""
+        B, n = tree_tokens.shape
+        K = self.n_steps
+        i32 = torch.int32
+        for t, shp, name in ((tree_tokens, (B, n), "tree_tokens"), (tree_parents, (B, n), "tree_parents"),
+                             (target_next, (B, n + 1), "target_next"), (n_new, (B,), "n_new"),
+                             (kv_len, (B,), "kv_len"), (accept_len, (B,), "accept_len"),
+                             (accept_nodes, (B, K), "accept_nodes"), (out_tokens, (B, K + 1), "out_tokens")):
+            self._tensor(t, shp, i32, name)
+        self._check(self.lib.prism_accept_tree(
+            self.h, B, n, _ptr(tree_tokens), _ptr(tree_parents), _ptr(target_next), _ptr(n_new), _ptr(kv_len),
+            _ptr(accept_len), _ptr(accept_nodes), _ptr(out_tokens), _stream(stream)))
+
     def round_launches(self) -> int:
         """Kernel launches of the last round replayed from a CUDA graph."""
         n = ctypes.c_int32(0)
@@ -246,7 +305,7 @@ class Drafter:
         (kind, milliseconds) in launch order."""
         B = self._round_args(tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids,
                              topk_ids, topk_logits)
-        cap = 9 * self.n_steps + 8
+        cap = 12 * self.n_steps + 8
         ms = (ctypes.c_float * cap)()
         kinds = (ctypes.c_int32 * cap)()
         n = ctypes.c_int32(0)

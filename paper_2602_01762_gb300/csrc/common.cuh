@@ -249,6 +249,64 @@ struct AcceptSampledArgs {
 };
 int sample_blocks(int V, int *chunk);
 
+// Tree drafting (tree.cu): the frontier of each sequence is w rows b * w + j.
+constexpr int kTreeMaxWidth = 8;      // branches per node (the top-k lists hold 8)
+constexpr int kTreeMaxPool = 1024;    // candidates per sequence and round
+constexpr int kTreeMaskBits = 64;     // draft slots a row's ancestor mask can name
+struct TreeArgs {
+    int B, w, K, step, R;             // R: rows per sequence this step (1 at step 1, else w)
+    int d, V, Hq, Hkv, D, max_ctx, max_new, n_nodes, P;
+    const int32_t *n_new, *kv_len;
+    int *err;
+    // fusion input rows
+    const void *embed;                // [V, d] wtype
+    const float *hhat;                // h^ rows [*, d]
+    void *u_out;                      // [B*w, 2d] wtype
+    // frontier (rows b*w + j): token, h^ row that emitted it, pool index,
+    // score, ancestor slot mask of the row that will process it
+    int32_t *front_tok, *front_row, *front_pool;
+    float *front_score;
+    unsigned long long *front_mask;
+    // candidate pool [B, P]
+    int32_t *pool_tok, *pool_par;
+    float *pool_score;
+    // this step's LM-head outputs (rows b*w + j)
+    const float *logits;              // [B*w, V]
+    const int32_t *top_ids;           // [B*w, w]
+    const float *top_vals;            // [B*w, w]
+    float *lse;                       // [B*w]
+    float *lse_part;                  // [B*w, kSampleMaxBlocks, 2]
+    int *lse_ctr;                     // [B*w] (left at zero)
+    int lse_chunk, lse_blocks;
+    // RoPE / append / attention
+    const float *qkv;                 // [B*w, (Hq + 2Hkv) D]
+    void *k_cache, *v_cache;          // [B, Hkv, max_ctx, D]
+    float *q;                         // [B*w, Hq, D]
+    const float *rope_cos, *rope_sin;
+    float *attn_part;                 // [B*w, Hq, splits, D + 4]
+    int *attn_ctr;                    // [B, Hkv] (left at zero)
+    void *o_out;                      // [B*w, Hq*D] wtype
+    int chunk, splits;
+    // caller outputs: the verified tree [B, n_nodes]; optional pool [B, P] and frontier [B, K, w]
+    int32_t *tree_tokens, *tree_parents, *tree_depths;
+    float *tree_scores;
+    int32_t *out_pool_tokens, *out_pool_parents, *out_frontier;
+    float *out_pool_scores;
+};
+struct AcceptTreeArgs {
+    const int32_t *tree_tokens, *tree_parents, *target_next, *n_new;  // [B, m], [B, m], [B, m+1], [B]
+    int32_t *kv_len, *accept_len, *accept_nodes, *out_tokens;         // [B], [B], [B, K], [B, K+1]
+    int B, n_nodes, K;
+};
+size_t tree_attention_smem_bytes(bool bf16, int D, int chunk, int G, int w, int splits);
+cudaError_t prepare_tree_kernels(bool bf16, int D, int chunk, int G, int w, int splits);
+cudaError_t launch_tree_gather(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl);
+cudaError_t launch_tree_rope(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl);
+cudaError_t launch_tree_attention(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl);
+cudaError_t launch_tree_lse(const TreeArgs &a, cudaStream_t s, bool pdl);
+cudaError_t launch_tree_select(const TreeArgs &a, cudaStream_t s, bool pdl);
+cudaError_t launch_accept_tree(const AcceptTreeArgs &a, cudaStream_t s);
+
 // Host launchers (return cudaGetLastError of the launch).
 cudaError_t launch_gemv(const GemvArgs &a, bool bf16, int grid, cudaStream_t s, bool pdl);
 size_t gemv_smem_bytes(const GemvArgs &a, bool bf16, int tc);

@@ -1,5 +1,6 @@
 // C ABI of the PRISM draft round: context, workspace, validation, the per-step
 // launch sequence and CUDA-graph capture/replay.  See include/prism.h.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -14,7 +15,7 @@ using namespace prism;
 namespace {
 
 constexpr int kGraphCache = 8;
-constexpr int kMaxProfileKernels = 9 * kMaxSteps + 8;
+constexpr int kMaxProfileKernels = 12 * kMaxSteps + 8;
 
 struct RoundArgs {
     int B;
@@ -28,6 +29,8 @@ struct RoundArgs {
     float temperature;             // > 0: sampled drafting (then logits, seed and lse are set)
     const uint64_t *seed;
     float *lse;
+    int tree_w, tree_m;            // > 0: tree drafting of this width, verifying tree_m nodes
+    prism_tree_outputs tree;
     bool operator==(const RoundArgs &o) const { return std::memcmp(this, &o, sizeof(RoundArgs)) == 0; }
 };
 
@@ -91,6 +94,21 @@ struct prism_ctx {
     unsigned long long *lm_best = nullptr;  // [max_batch] LM head top-1 keys (left at zero)
     float *sample_part = nullptr;           // [max_batch, kSampleMaxBlocks, 4] sampled-draft partials
     int *sample_ctr = nullptr;              // [max_batch] sampled-draft tickets (left at zero)
+    // tree drafting (max_tree_width > 0): w rows per sequence, frontier and candidate pool
+    int tree_rows = 0;                      // max_batch * max(1, max_tree_width)
+    void *tree_u = nullptr;                 // [rows, 2d] wtype fusion inputs
+    float *tree_logits = nullptr;           // [rows, V]
+    int32_t *tree_top_ids = nullptr;        // [rows, 8]
+    float *tree_top_vals = nullptr;         // [rows, 8]
+    int32_t *tree_draft = nullptr;          // [rows] (LM-head top-1, unused by the tree)
+    float *tree_lse = nullptr;              // [rows]
+    float *tree_lse_part = nullptr;         // [rows, kSampleMaxBlocks, 2]
+    int *tree_lse_ctr = nullptr;            // [rows] (left at zero)
+    int32_t *front_tok = nullptr, *front_row = nullptr, *front_pool = nullptr;  // [rows]
+    float *front_score = nullptr;           // [rows]
+    unsigned long long *front_mask = nullptr;  // [rows]
+    int32_t *pool_tok = nullptr, *pool_par = nullptr;  // [max_batch, P_max]
+    float *pool_score = nullptr;
     int *err = nullptr;
     // execution
     cudaStream_t cap_stream = nullptr;
@@ -229,12 +247,80 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
                             make_cache_map(&tmk, r.k_cache, r.B * Hkv, f.max_ctx, D, fused_attention_chunk()) == cudaSuccess &&
                             make_cache_map(&tmv, r.v_cache, r.B * Hkv, f.max_ctx, D, fused_attention_chunk()) == cudaSuccess;
 
+    // tree drafting: w rows per sequence from step 2 on
+    const bool tree = r.tree_w > 0;
+    const int tw = tree ? r.tree_w : 1;
+    TreeArgs ta{};
+    if (tree) {
+        ta.B = r.B;
+        ta.w = tw;
+        ta.K = K;
+        ta.d = d;
+        ta.V = V;
+        ta.Hq = Hq;
+        ta.Hkv = Hkv;
+        ta.D = D;
+        ta.max_ctx = f.max_ctx;
+        ta.max_new = f.max_new;
+        ta.n_nodes = r.tree_m;
+        ta.P = tw + (K - 1) * tw * tw;
+        ta.n_new = r.n_new;
+        ta.kv_len = r.kv_len;
+        ta.err = c->err;
+        ta.embed = c->embed;
+        ta.hhat = c->hhat;
+        ta.u_out = c->tree_u;
+        ta.front_tok = c->front_tok;
+        ta.front_row = c->front_row;
+        ta.front_pool = c->front_pool;
+        ta.front_score = c->front_score;
+        ta.front_mask = c->front_mask;
+        ta.pool_tok = c->pool_tok;
+        ta.pool_par = c->pool_par;
+        ta.pool_score = c->pool_score;
+        ta.top_ids = c->tree_top_ids;
+        ta.top_vals = c->tree_top_vals;
+        ta.lse = c->tree_lse;
+        ta.lse_part = c->tree_lse_part;
+        ta.lse_ctr = c->tree_lse_ctr;
+        ta.qkv = c->qkv;
+        ta.k_cache = r.k_cache;
+        ta.v_cache = r.v_cache;
+        ta.q = c->q;
+        ta.rope_cos = c->rope_cos;
+        ta.rope_sin = c->rope_sin;
+        ta.attn_part = c->attn_part;
+        ta.attn_ctr = c->counters;
+        ta.o_out = c->o_buf;
+        ta.chunk = c->attn_chunk;
+        ta.splits = c->attn_splits;
+        ta.tree_tokens = r.tree.tokens;
+        ta.tree_parents = r.tree.parents;
+        ta.tree_depths = r.tree.depths;
+        ta.tree_scores = r.tree.scores;
+        ta.out_pool_tokens = r.tree.pool_tokens;
+        ta.out_pool_parents = r.tree.pool_parents;
+        ta.out_pool_scores = r.tree.pool_scores;
+        ta.out_frontier = r.tree.frontier;
+    }
+
     for (int k = 1; k <= K && e == cudaSuccess; ++k) {
         const prism_step_weights &w = c->steps[k - 1];
         const CUtensorMap *tms = c->tm_step_ok[k - 1] ? c->tm_step[k - 1] : nullptr;
         const bool prefill = k == 1;
-        const int T1 = prefill ? r.B * f.max_new : r.B;
+        const bool tstep = tree && !prefill;       // a tree step: w rows per sequence
+        const int Trow = tstep ? r.B * tw : r.B;   // rows from attention on
+        const int T1 = prefill ? r.B * f.max_new : Trow;
         const bool p = pdl && !first;
+        ta.step = k;
+        ta.R = prefill ? 1 : tw;
+
+        if (tstep) {
+            // fusion input rows [E(token); round(h^ of the emitting row)]
+            e = launch_tree_gather(ta, c->bf16, s, p);
+            after(9);
+            if (e != cudaSuccess) break;
+        }
 
         // fusion F(E(x), h)
         GemvArgs g = base;
@@ -243,12 +329,13 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.n_units = d;
         g.kin = 2 * d;
         g.T = T1;
-        g.pro = prefill ? kProFusePrefill : kProFuseDecode;
+        g.pro = prefill ? kProFusePrefill : (tstep ? kProCopy : kProFuseDecode);
         g.src = c->hhat;
+        g.act = c->tree_u;
         g.epi = kEpiStore;
         g.out = c->x0;
         g.out_ld = d;
-        e = proj(g, tms ? &tms[0] : nullptr, gemv_grid(c, d), p);
+        e = proj(g, tms ? &tms[0] : nullptr, gemv_grid(c, d), tstep ? pdl : p);
         after(0);
         if (e != cudaSuccess) break;
 
@@ -269,7 +356,16 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         after(1);
         if (e != cudaSuccess) break;
 
-        if (c->attn_fused) {
+        if (tstep) {
+            // RoPE at the node's depth, K/V at its own slot; attention over the
+            // committed rows and the node's ancestors
+            e = launch_tree_rope(ta, c->bf16, s, pdl);
+            after(2);
+            if (e != cudaSuccess) break;
+            e = launch_tree_attention(ta, c->bf16, s, pdl);
+            after(3);
+            if (e != cudaSuccess) break;
+        } else if (c->attn_fused) {
             // RoPE + KV append + attention in one cluster launch per (sequence, KV head)
             FusedAttnArgs fa{};
             fa.qkv = c->qkv;
@@ -352,7 +448,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.W = w.w_o;
         g.n_units = d;
         g.kin = Hq * D;
-        g.T = r.B;
+        g.T = Trow;
         g.pro = kProCopy;
         g.act = c->o_buf;
         g.epi = kEpiResid;
@@ -371,7 +467,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.n_units = F;
         g.pair_offset = F;
         g.kin = d;
-        g.T = r.B;
+        g.T = Trow;
         g.pro = kProNorm;
         g.src = c->a;
         g.gain = w.g_mlp;
@@ -388,14 +484,14 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.W = w.w_down;
         g.n_units = d;
         g.kin = F;
-        g.T = r.B;
+        g.T = Trow;
         g.pro = kProCopy;
         g.act = c->m_buf;
         g.epi = kEpiResid;
         g.resid = c->a;
         g.out = c->hhat;
         g.out_ld = d;
-        g.hidden_out = r.hidden_out;
+        g.hidden_out = tree ? nullptr : r.hidden_out;
         e = proj(g, tms ? &tms[4] : nullptr, gemv_grid(c, d), pdl);
         after(6);
         if (e != cudaSuccess) break;
@@ -406,7 +502,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.W = c->lm_head;
         g.n_units = V;
         g.kin = d;
-        g.T = r.B;
+        g.T = Trow;
         g.pro = kProNorm;
         g.src = c->hhat;
         g.gain = f.final_norm ? w.g_final : nullptr;
@@ -419,9 +515,33 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.draft_out = r.draft;
         g.topk_ids = r.topk_ids;
         g.topk_logits = r.topk_logits;
+        if (tree) {
+            // rows b * w + j of [B * w, .] buffers: at step 1 (one row per
+            // sequence) K = w puts row b at b * w; later steps index by row
+            float *lg = r.tree.row_logits ? r.tree.row_logits + (size_t)(k - 1) * r.B * tw * V : c->tree_logits;
+            g.K = prefill ? tw : 1;
+            g.step = 1;
+            g.topk = tw;
+            g.logits = lg;
+            g.draft_out = c->tree_draft;
+            g.topk_ids = c->tree_top_ids;
+            g.topk_logits = c->tree_top_vals;
+            ta.logits = lg;
+        }
         e = proj(g, c->tm_lm_ok ? &c->tm_lm : nullptr, c->lm_grid, pdl);
         after(7);
         if (e != cudaSuccess) break;
+
+        if (tree) {
+            // draft log-probabilities, candidate scores, next frontier (and the tree after step K)
+            e = launch_tree_lse(ta, s, pdl);
+            after(10);
+            if (e != cudaSuccess) break;
+            e = launch_tree_select(ta, s, pdl);
+            after(11);
+            if (e != cudaSuccess) break;
+            continue;
+        }
 
         if (r.temperature > 0.f) {
             // x^_k drawn from softmax(z / T): replaces the argmax before the next step reads it
@@ -476,7 +596,8 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         (f.head_dim != 64 && f.head_dim != 128) || f.ffn < 8 || f.ffn % 8 || f.vocab < kTopK ||
         f.n_steps < 1 || f.n_steps > kMaxSteps || f.max_batch < 1 || f.max_ctx < 2 || f.max_new < 1 ||
         f.topk < 1 || f.topk > kTopK || (f.dtype != PRISM_F32 && f.dtype != PRISM_BF16) ||
-        f.n_q_heads / f.n_kv_heads > 16 || !(f.rms_eps >= 0.f) || !(f.rope_theta > 0.f))
+        f.n_q_heads / f.n_kv_heads > 16 || !(f.rms_eps >= 0.f) || !(f.rope_theta > 0.f) ||
+        f.max_tree_width < 0 || f.max_tree_width > kTreeMaxWidth)
         return fail(nullptr, PRISM_ERR_INVALID_ARG, "unsupported configuration");
     prism_ctx *c = new prism_ctx();
     c->cfg = f;
@@ -495,7 +616,12 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     while ((f.max_ctx + c->attn_chunk - 1) / c->attn_chunk > 256) c->attn_chunk *= 2;
     c->attn_splits = (f.max_ctx + c->attn_chunk - 1) / c->attn_chunk;
 
-    const size_t T1 = (size_t)f.max_batch * f.max_new, B = f.max_batch;
+    // rows per sequence after step 1: w for tree rounds, else 1
+    const size_t TW = f.max_tree_width > 0 ? (size_t)f.max_tree_width : 1;
+    const size_t Bw = (size_t)f.max_batch * TW;
+    const size_t T1 = std::max((size_t)f.max_batch * f.max_new, Bw), B = Bw, Bseq = f.max_batch;
+    const size_t tree_on = f.max_tree_width > 0 ? 1 : 0;
+    const size_t P_max = TW + (size_t)(f.n_steps - 1) * TW * TW;
     // split-K workspace of the tensor-core projections: the largest need of
     // any projection of this shape
     size_t tc_floats = 0;
@@ -506,7 +632,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         const int epis[] = {kEpiStore, kEpiStore, kEpiResid, kEpiSwiGLU, kEpiResid};
         const int pros[] = {kProFuseDecode, kProNorm, kProCopy, kProNorm, kProCopy};
         for (int i = 0; i < 5; ++i)
-            for (int T : {(int)T1, (int)B}) {
+            for (int T : {(int)T1, (int)B, (int)Bseq}) {
                 GemvArgs g{};
                 g.n_units = units[i];
                 g.kin = kins[i];
@@ -533,7 +659,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         B * F * es,                                                // m
         B * (size_t)c->lm_grid * kTopK * 4,                        // LM partial values
         B * (size_t)c->lm_grid * kTopK * 4,                        // LM partial ids
-        (B * Hkv + 1) * 4,                                         // counters
+        (Bseq * Hkv + 1) * 4,                                      // counters
         B * 8,                                                     // LM head packed top-1 keys
         32,                                                        // error word (+ checked-build record)
         tc_floats * 4,                                             // tensor-core split-K partials
@@ -541,6 +667,17 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         T1 * 2 * d * es,                                           // streamed-kernel activation rows
         B * (size_t)kSampleMaxBlocks * 4 * 4,                      // sampled-draft partials
         B * 4,                                                     // sampled-draft tickets
+        tree_on * Bw * 2 * d * es,                                 // tree fusion inputs
+        tree_on * Bw * f.vocab * 4,                                // tree row logits
+        tree_on * Bw * kTopK * 4,                                  // tree top-w ids
+        tree_on * Bw * kTopK * 4,                                  // tree top-w logits
+        tree_on * Bw * 4,                                          // tree LM-head top-1 (unused)
+        tree_on * Bw * 4,                                          // tree row lse
+        tree_on * Bw * kSampleMaxBlocks * 2 * 4,                   // tree lse partials
+        tree_on * Bw * 4,                                          // tree lse tickets
+        tree_on * Bw * 4 * 4,                                      // frontier token, row, pool index, score
+        tree_on * Bw * 8,                                          // frontier ancestor masks
+        tree_on * Bseq * P_max * 4 * 3,                            // pool tokens, parents, scores
     };
     size_t total = 0;
     for (size_t s : sizes) total += align256(s);
@@ -575,6 +712,23 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     c->xbuf = (uint16_t *)slot[17];
     c->sample_part = (float *)slot[18];
     c->sample_ctr = (int *)slot[19];
+    c->tree_rows = (int)Bw;
+    c->tree_u = slot[20];
+    c->tree_logits = (float *)slot[21];
+    c->tree_top_ids = (int32_t *)slot[22];
+    c->tree_top_vals = (float *)slot[23];
+    c->tree_draft = (int32_t *)slot[24];
+    c->tree_lse = (float *)slot[25];
+    c->tree_lse_part = (float *)slot[26];
+    c->tree_lse_ctr = (int *)slot[27];
+    c->front_tok = (int32_t *)slot[28];
+    c->front_row = c->front_tok + Bw;
+    c->front_pool = c->front_row + Bw;
+    c->front_score = (float *)(c->front_pool + Bw);
+    c->front_mask = (unsigned long long *)slot[29];
+    c->pool_tok = (int32_t *)slot[30];
+    c->pool_par = c->pool_tok + Bseq * P_max;
+    c->pool_score = (float *)(c->pool_par + Bseq * P_max);
 
     // rotary tables: angle p * theta^(-2j/D), computed in double, stored as float
     std::vector<float> cs((size_t)f.max_ctx * (D / 2)), sn((size_t)f.max_ctx * (D / 2));
@@ -603,7 +757,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
             GemvArgs g{};
             g.kin = kins[i];
             g.epi = epis[i];
-            g.T = i < 2 ? T1 : f.max_batch;
+            g.T = i < 2 ? (int)T1 : (int)B;
             if (!gemv_supported(g, c->bf16)) {
                 cudaFree(ws);
                 delete c;
@@ -618,6 +772,14 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
     }
     if (e == cudaSuccess) e = prepare_attention_kernel(c->bf16, D, c->attn_chunk, Hq / Hkv, c->attn_splits);
     if (e == cudaSuccess) e = prepare_fused_attention(c->bf16, D, Hq / Hkv, Hkv, &c->attn_max_cs);
+    if (e == cudaSuccess && tree_on) {
+        if (tree_attention_smem_bytes(c->bf16, D, c->attn_chunk, Hq / Hkv, (int)TW, c->attn_splits) > 200 * 1024) {
+            cudaFree(ws);
+            delete c;
+            return fail(nullptr, PRISM_ERR_INVALID_ARG, "max_ctx too large for the tree attention combine");
+        }
+        e = prepare_tree_kernels(c->bf16, D, c->attn_chunk, Hq / Hkv, (int)TW, c->attn_splits);
+    }
     if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking);
     if (e != cudaSuccess) {
         prism_status st = cuda_fail(nullptr, e, "context setup");
@@ -783,6 +945,46 @@ prism_status prism_draft_round_sampled(prism_ctx *c, int32_t batch, const int32_
     r.seed = seed;
     r.lse = draft_lse;
     return run_round(c, r, stream);
+}
+
+prism_status prism_draft_tree(prism_ctx *c, int32_t batch, const int32_t *tokens, const void *hidden,
+                              const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
+                              int32_t width, int32_t n_nodes, const prism_tree_outputs *out, void *stream) {
+    if (!c) return fail(c, PRISM_ERR_INVALID_ARG, "null context");
+    if (!out || !out->tokens || !out->parents || !out->depths || !out->scores)
+        return fail(c, PRISM_ERR_INVALID_ARG, "tree outputs: tokens, parents, depths and scores are required");
+    if (width < 1 || width > kTreeMaxWidth || width > c->cfg.vocab)
+        return fail(c, PRISM_ERR_INVALID_ARG, "tree width must be in 1..8");
+    if (width > c->cfg.max_tree_width)
+        return fail(c, PRISM_ERR_CAPACITY, "tree width exceeds the context's max_tree_width");
+    const long K = c->cfg.n_steps;
+    const long P = width + (K - 1) * width * width;
+    if ((K - 1) * width > kTreeMaskBits || P > kTreeMaxPool)
+        return fail(c, PRISM_ERR_INVALID_ARG, "tree too large: (K - 1) * width must be <= 64 and the pool <= 1024");
+    if (n_nodes < 1 || n_nodes > P) return fail(c, PRISM_ERR_INVALID_ARG, "n_nodes must be in 1..w + (K - 1) w^2");
+    RoundArgs r = round_args(batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, c->tree_draft, nullptr,
+                             nullptr, nullptr, nullptr);
+    r.tree_w = width;
+    r.tree_m = n_nodes;
+    r.tree = *out;
+    return run_round(c, r, stream);
+}
+
+prism_status prism_accept_tree(prism_ctx *c, int32_t batch, int32_t n_nodes, const int32_t *tree_tokens,
+                               const int32_t *tree_parents, const int32_t *target_next, const int32_t *n_new,
+                               int32_t *kv_len, int32_t *accept_len, int32_t *accept_nodes, int32_t *out_tokens,
+                               void *stream) {
+    if (!c) return fail(c, PRISM_ERR_INVALID_ARG, "null context");
+    if (!tree_tokens || !tree_parents || !target_next || !n_new || !kv_len || !accept_len || !accept_nodes ||
+        !out_tokens)
+        return fail(c, PRISM_ERR_INVALID_ARG, "null tensor argument");
+    if (batch < 1 || n_nodes < 1) return fail(c, PRISM_ERR_SHAPE, "batch and n_nodes must be >= 1");
+    if (batch > c->cfg.max_batch) return fail(c, PRISM_ERR_CAPACITY, "batch exceeds max_batch");
+    cudaSetDevice(c->device);
+    AcceptTreeArgs a{tree_tokens, tree_parents, target_next, n_new, kv_len, accept_len, accept_nodes, out_tokens,
+                     batch, n_nodes, c->cfg.n_steps};
+    cudaError_t e = launch_accept_tree(a, (cudaStream_t)stream);
+    return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "tree accept kernel launch");
 }
 
 prism_status prism_round_launches(prism_ctx *c, int32_t *n_launches) {

@@ -1,0 +1,549 @@
+// Tree drafting for the PRISM draft round (sm_103a).
+//
+// PRISM's step-wise modules work unchanged with tree-shaped drafts (Sec. 3.2,
+// after the recurrence); the paper evaluates a 6-step, 4-branch tree that
+// verifies at most 16 tokens (Sec. 4).  The tree is read as the dynamic top-w
+// expansion: step 1 (the chain's prefill) yields the w best tokens as depth-1
+// candidates; at step k >= 2 every frontier node is processed by step k's
+// module as its own activation row, so the projections and the LM head run on
+// T = B * w rows through the chain's kernels.  A candidate's score is the sum
+// of draft log-probabilities along its path; the next frontier is the w best
+// new candidates, and after step K the verified tree is the n best candidates
+// of the round.  The kernels this file adds:
+//   tree_gather_kernel     fusion input row [E(token); round(h^ of the row
+//                          that emitted the token)];
+//   tree_rope_kernel       rotary embedding at the node's depth, K/V stored at
+//                          the node's own cache slot L + n + (k - 2) w + j;
+//   tree_attention_kernel  split-KV attention over the committed rows [0, L+n)
+//                          plus the draft slots in the row's 64-bit ancestor
+//                          mask, all w rows of a sequence against one staged
+//                          chunk of keys, last-CTA merge in split order;
+//   tree_lse_kernel        log-sum-exp of every row's logits;
+//   tree_select_kernel     candidate scores, the next frontier, and after the
+//                          last step the verified tree (one CTA per sequence);
+//   accept_tree_kernel     greedy acceptance along the tree (Sec. 2's
+//                          temperature-0 rule applied from the root).
+#include "common.cuh"
+
+namespace prism {
+
+namespace {
+
+__device__ __forceinline__ int tree_n(const TreeArgs &a, int b) {
+    int n = a.n_new[b];
+    if (n < 1 || n > a.max_new) {
+        set_err(a.err, kErrNNew);
+        n = n < 1 ? 1 : a.max_new;
+    }
+    return n;
+}
+
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
+    const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+}
+
+// (max, sum of exp(v - max)) of two parts, combined.
+__device__ __forceinline__ void lse_merge(float &m, float &s, float m2, float s2) {
+    if (m2 == -INFINITY) return;
+    if (m == -INFINITY) { m = m2; s = s2; return; }
+    if (m2 > m) { s = s * expf(m - m2) + s2; m = m2; }
+    else s += s2 * expf(m2 - m);
+}
+
+// ------------------------------------------------------------------ gather
+
+template <typename WT>
+__global__ void __launch_bounds__(256) tree_gather_kernel(const TreeArgs a) {
+    pdl_trigger();
+    pdl_wait();
+    const int t = blockIdx.x;              // row b * w + j
+    int tok = a.front_tok[t];
+    if (tok < 0 || tok >= a.V) {
+        if (threadIdx.x == 0) set_err(a.err, kErrToken);
+        tok = tok < 0 ? 0 : a.V - 1;
+    }
+    const WT *e = (const WT *)a.embed + (size_t)tok * a.d;
+    const float *h = a.hhat + (size_t)a.front_row[t] * a.d;
+    WT *u = (WT *)a.u_out + (size_t)t * 2 * a.d;
+    for (int i = threadIdx.x; i < a.d; i += blockDim.x) {
+        u[i] = e[i];
+        Elem<WT>::store(u, a.d + i, h[i]);  // the operand rounding of the fusion input
+    }
+}
+
+// ------------------------------------------------------------------ RoPE + append
+
+template <typename WT>
+__global__ void __launch_bounds__(128) tree_rope_kernel(const TreeArgs a) {
+    pdl_trigger();
+    pdl_wait();
+    const int lane = threadIdx.x & 31;
+    const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int H = a.Hq + 2 * a.Hkv;
+    if (gw >= a.B * a.w * H) return;
+    const int t = gw / H, h = gw % H, b = t / a.w, j = t % a.w;
+    const int n = tree_n(a, b), L = a.kv_len[b];
+    const int pos = L + n + a.step - 2;                  // rotary position: the node's depth
+    const int slot = L + n + (a.step - 2) * a.w + j;     // cache slot: the node's own row (>= pos)
+    const int D = a.D, half = D / 2;
+    const float *x = a.qkv + (size_t)t * H * D + (size_t)h * D;
+    const bool ok = pos >= 0 && slot < a.max_ctx;
+    if (h >= a.Hq && !ok) {
+        if (lane == 0) set_err(a.err, kErrCache);
+        return;
+    }
+    const int pc = ok ? pos : 0;
+    if (h < a.Hq) {
+        float *q = a.q + ((size_t)t * a.Hq + h) * D;
+        for (int i = lane; i < half; i += 32) {
+            const float c = a.rope_cos[(size_t)pc * half + i], s = a.rope_sin[(size_t)pc * half + i];
+            const float x0 = x[i], x1 = x[i + half];
+            q[i] = x0 * c - x1 * s;
+            q[i + half] = x1 * c + x0 * s;
+        }
+    } else if (h < a.Hq + a.Hkv) {
+        WT *k = (WT *)a.k_cache + (((size_t)b * a.Hkv + (h - a.Hq)) * a.max_ctx + slot) * D;
+        for (int i = lane; i < half; i += 32) {
+            const float c = a.rope_cos[(size_t)pos * half + i], s = a.rope_sin[(size_t)pos * half + i];
+            const float x0 = x[i], x1 = x[i + half];
+            Elem<WT>::store(k, i, x0 * c - x1 * s);
+            Elem<WT>::store(k, i + half, x1 * c + x0 * s);
+        }
+    } else {
+        WT *v = (WT *)a.v_cache + (((size_t)b * a.Hkv + (h - a.Hq - a.Hkv)) * a.max_ctx + slot) * D;
+        for (int i = lane; i < D; i += 32) Elem<WT>::store(v, i, x[i]);
+    }
+}
+
+// ------------------------------------------------------------------ attention
+
+// q . k for one key row in shared memory (16-byte vector reads of both).
+template <typename WT, int D>
+__device__ __forceinline__ float dot_row(const float *q, const WT *k) {
+    float acc = 0.f;
+    if constexpr (sizeof(WT) == 2) {
+#pragma unroll 4
+        for (int c = 0; c < D; c += 8) {
+            const uint4 kv = *(const uint4 *)(k + c);
+            const float4 q0 = *(const float4 *)(q + c), q1 = *(const float4 *)(q + c + 4);
+            acc = fmaf(q0.x, bf16lo(kv.x), acc);
+            acc = fmaf(q0.y, bf16hi(kv.x), acc);
+            acc = fmaf(q0.z, bf16lo(kv.y), acc);
+            acc = fmaf(q0.w, bf16hi(kv.y), acc);
+            acc = fmaf(q1.x, bf16lo(kv.z), acc);
+            acc = fmaf(q1.y, bf16hi(kv.z), acc);
+            acc = fmaf(q1.z, bf16lo(kv.w), acc);
+            acc = fmaf(q1.w, bf16hi(kv.w), acc);
+        }
+    } else {
+#pragma unroll 4
+        for (int c = 0; c < D; c += 4) {
+            const float4 kv = *(const float4 *)(k + c), q0 = *(const float4 *)(q + c);
+            acc = fmaf(q0.x, kv.x, acc);
+            acc = fmaf(q0.y, kv.y, acc);
+            acc = fmaf(q0.z, kv.z, acc);
+            acc = fmaf(q0.w, kv.w, acc);
+        }
+    }
+    return acc;
+}
+
+// The DPL consecutive values a lane owns in one V row.
+template <typename WT, int DPL>
+__device__ __forceinline__ void load_run(const WT *p, float (&out)[DPL]) {
+    if constexpr (sizeof(WT) == 2 && DPL == 4) {
+        const uint2 v = *(const uint2 *)p;
+        out[0] = bf16lo(v.x); out[1] = bf16hi(v.x); out[2] = bf16lo(v.y); out[3] = bf16hi(v.y);
+    } else if constexpr (sizeof(WT) == 2 && DPL == 2) {
+        const uint32_t v = *(const uint32_t *)p;
+        out[0] = bf16lo(v); out[1] = bf16hi(v);
+    } else {
+#pragma unroll
+        for (int u = 0; u < DPL; ++u) out[u] = Elem<WT>::load(p, u);
+    }
+}
+
+// Grid (splits, Hkv, B); CTA (s, g, b) stages keys [s C, s C + C) of KV head g
+// once and scores them against the G query heads of g in each of the w rows
+// of sequence b.  Key slot p is visible to row j when p < L + n (committed and
+// step-1 rows) or bit p - (L + n) of the row's ancestor mask is set.
+template <typename WT, int D>
+__global__ void __launch_bounds__(kAttnThreads) tree_attention_kernel(const TreeArgs a) {
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    __shared__ int s_last;
+    constexpr int VEC = Elem<WT>::kPerVec;
+    constexpr int RS = D + VEC;              // padded row stride (elements)
+    constexpr int DPL = D / 32;
+    constexpr int PS = D + 4;                // partial record: D sums, max, sum, 2 pad
+    const int C = a.chunk, G = a.Hq / a.Hkv, NQ = a.w * G;
+    WT *Ks = (WT *)smem_raw;
+    WT *Vs = Ks + (size_t)C * RS;
+    float *qs = (float *)(Vs + (size_t)C * RS);  // [NQ][D], pair (j, hl) at j * G + hl
+    float *ps = qs + (size_t)NQ * D;             // [NQ][C]
+    float *ws = ps + (size_t)NQ * C;             // [NQ][splits]
+    const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
+
+    pdl_trigger();
+    pdl_wait();
+
+    const int n = tree_n(a, b), L = a.kv_len[b];
+    const int base = L + n;
+    int PE = base + (a.step - 1) * a.w;          // keys [0, PE)
+    if (PE > a.max_ctx) PE = a.max_ctx;
+    const int j0 = s * C;
+    const int nk = PE - j0 < C ? PE - j0 : C;
+    const float scale = 1.0f / sqrtf((float)D);
+
+    if (nk > 0 && L >= 0) {
+        const uint4 *kg = (const uint4 *)((const WT *)a.k_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D);
+        const uint4 *vg = (const uint4 *)((const WT *)a.v_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D);
+        constexpr int VPR = D / VEC;
+        for (int e = threadIdx.x; e < nk * VPR; e += blockDim.x) {
+            const int r = e / VPR, c = e % VPR;
+            cp_async16(Ks + (size_t)r * RS + c * VEC, kg + e);
+            cp_async16(Vs + (size_t)r * RS + c * VEC, vg + e);
+        }
+        for (int e = threadIdx.x; e < NQ * D; e += blockDim.x) {
+            const int pr = e / D, c = e % D, j = pr / G, hl = pr % G;
+            qs[e] = a.q[(((size_t)b * a.w + j) * a.Hq + (size_t)g * G + hl) * D + c];
+        }
+        cp_async_wait_all();
+        __syncthreads();
+
+        for (int pr = warp; pr < NQ; pr += nwarp) {
+            const int j = pr / G, hl = pr % G, t = b * a.w + j;
+            const unsigned long long msk = a.front_mask[t];
+            const float *q = qs + (size_t)pr * D;
+            float *pp = ps + (size_t)pr * C;
+            float mloc = -INFINITY;
+            for (int jj = lane; jj < nk; jj += 32) {
+                const int p = j0 + jj;
+                const int off = p - base;
+                const bool vis = off < 0 || (off < kTreeMaskBits && ((msk >> off) & 1ull));
+                float sc = -INFINITY;
+                if (vis) sc = dot_row<WT, D>(q, Ks + (size_t)jj * RS) * scale;
+                pp[jj] = sc;
+                mloc = fmaxf(mloc, sc);
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xFFFFFFFFu, mloc, o));
+            float lsum = 0.f;
+            for (int jj = lane; jj < nk; jj += 32) {
+                const float p = mloc == -INFINITY ? 0.f : expf(pp[jj] - mloc);
+                pp[jj] = p;
+                lsum += p;
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) lsum += __shfl_xor_sync(0xFFFFFFFFu, lsum, o);
+            __syncwarp();
+            float acc[DPL];
+#pragma unroll
+            for (int u = 0; u < DPL; ++u) acc[u] = 0.f;
+            for (int jj = 0; jj < nk; ++jj) {
+                const float p = pp[jj];
+                if (p == 0.f) continue;
+                float vv[DPL];
+                load_run<WT, DPL>(Vs + (size_t)jj * RS + lane * DPL, vv);
+#pragma unroll
+                for (int u = 0; u < DPL; ++u) acc[u] = fmaf(p, vv[u], acc[u]);
+            }
+            float *part = a.attn_part + (((size_t)t * a.Hq + (size_t)g * G + hl) * a.splits + s) * PS;
+#pragma unroll
+            for (int u = 0; u < DPL; ++u) part[lane * DPL + u] = acc[u];
+            if (lane == 0) { part[D] = mloc; part[D + 1] = lsum; }
+        }
+    } else {
+        for (int pr = warp; pr < NQ; pr += nwarp) {
+            const int j = pr / G, hl = pr % G, t = b * a.w + j;
+            float *part = a.attn_part + (((size_t)t * a.Hq + (size_t)g * G + hl) * a.splits + s) * PS;
+#pragma unroll
+            for (int u = 0; u < DPL; ++u) part[lane * DPL + u] = 0.f;
+            if (lane == 0) { part[D] = -INFINITY; part[D + 1] = 0.f; }
+        }
+    }
+
+    // last CTA of (b, g): log-sum-exp merge of the splits in split order
+    __threadfence();
+    __syncthreads();
+    int *ctr = a.attn_ctr + (size_t)b * a.Hkv + g;
+    if (threadIdx.x == 0) s_last = (atomicAdd(ctr, 1) == a.splits - 1);
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    for (int pr = warp; pr < NQ; pr += nwarp) {
+        const int j = pr / G, hl = pr % G, t = b * a.w + j, h = g * G + hl;
+        const float *part = a.attn_part + ((size_t)t * a.Hq + h) * a.splits * PS;
+        float *wh = ws + (size_t)pr * a.splits;
+        constexpr int kMaxPerLane = 8;           // splits <= 256
+        float mv[kMaxPerLane], lv[kMaxPerLane];
+#pragma unroll
+        for (int k = 0; k < kMaxPerLane; ++k) {
+            const int sp = lane + 32 * k;
+            const bool in = sp < a.splits;
+            mv[k] = in ? __ldcg(part + (size_t)sp * PS + D) : -INFINITY;
+            lv[k] = in ? __ldcg(part + (size_t)sp * PS + D + 1) : 0.f;
+        }
+        float M = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < kMaxPerLane; ++k) M = fmaxf(M, mv[k]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xFFFFFFFFu, M, o));
+        float den = 0.f;
+#pragma unroll
+        for (int k = 0; k < kMaxPerLane; ++k) {
+            const int sp = lane + 32 * k;
+            const float wgt = lv[k] > 0.f ? expf(mv[k] - M) : 0.f;
+            if (sp < a.splits) wh[sp] = wgt;
+            den = fmaf(wgt, lv[k], den);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) den += __shfl_xor_sync(0xFFFFFFFFu, den, o);
+        __syncwarp();
+        float acc[DPL];
+#pragma unroll
+        for (int u = 0; u < DPL; ++u) acc[u] = 0.f;
+        for (int sp = 0; sp < a.splits; ++sp) {
+            const float wgt = wh[sp];
+            if (wgt == 0.f) continue;
+            const float *src = part + (size_t)sp * PS + lane * DPL;
+#pragma unroll
+            for (int u = 0; u < DPL; ++u) acc[u] = fmaf(wgt, __ldcg(src + u), acc[u]);
+        }
+        WT *o = (WT *)a.o_out + ((size_t)t * a.Hq + h) * D;
+        const float inv = den > 0.f ? 1.0f / den : 0.f;
+#pragma unroll
+        for (int u = 0; u < DPL; ++u) Elem<WT>::store(o, lane * DPL + u, acc[u] * inv);
+    }
+    if (threadIdx.x == 0) *ctr = 0;
+}
+
+// ------------------------------------------------------------------ log-sum-exp
+
+// Grid (blocks per row, B * R): row t = b * w + j of the LM head's logits.
+__global__ void __launch_bounds__(256) tree_lse_kernel(const TreeArgs a) {
+    __shared__ float s_m[8], s_s[8];
+    pdl_trigger();
+    pdl_wait();
+    const int blk = blockIdx.x, nblk = gridDim.x;
+    const int b = blockIdx.y / a.R, j = blockIdx.y % a.R, t = b * a.w + j;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const float *z = a.logits + (size_t)t * a.V;
+    const int lo = blk * a.lse_chunk, hi = min(a.V, lo + a.lse_chunk);
+    float m = -INFINITY, s = 0.f;
+    for (int i = lo + tid; i < hi; i += blockDim.x) lse_merge(m, s, z[i], 1.f);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, s, o);
+        lse_merge(m, s, m2, s2);
+    }
+    if (lane == 0) { s_m[warp] = m; s_s[warp] = s; }
+    __syncthreads();
+    if (tid != 0) return;
+    for (int q = 1; q < (int)(blockDim.x >> 5); ++q) lse_merge(m, s, s_m[q], s_s[q]);
+    float *part = a.lse_part + ((size_t)t * kSampleMaxBlocks + blk) * 2;
+    part[0] = m;
+    part[1] = s;
+    __threadfence();
+    if (atomicAdd(a.lse_ctr + t, 1) != nblk - 1) return;
+    __threadfence();
+    float M = -INFINITY, S = 0.f;
+    for (int q = 0; q < nblk; ++q) {
+        const float *pq = a.lse_part + ((size_t)t * kSampleMaxBlocks + q) * 2;
+        lse_merge(M, S, __ldcg(pq), __ldcg(pq + 1));
+    }
+    a.lse[t] = M + logf(S);
+    a.lse_ctr[t] = 0;
+}
+
+// ------------------------------------------------------------------ selection
+
+constexpr int kSelectThreads = 256;
+
+// One CTA per sequence.  Candidate c = j * w + r of step k (row j's r-th best
+// token) has pool index base + c and score = frontier score of row j +
+// logit - lse.  Frontier and tree orders: score descending, then pool index
+// ascending (a parent always ranks before its children).
+__global__ void __launch_bounds__(kSelectThreads) tree_select_kernel(const TreeArgs a) {
+    __shared__ float s_fscore[kTreeMaxWidth];
+    __shared__ int s_fpool[kTreeMaxWidth];
+    __shared__ unsigned long long s_fmask[kTreeMaxWidth];
+    __shared__ float s_cs[kTreeMaxWidth * kTreeMaxWidth];
+    __shared__ float s_ps[kTreeMaxPool];
+    __shared__ int s_sel[kTreeMaxPool];
+    __shared__ int s_pos[kTreeMaxPool];
+    pdl_trigger();
+    pdl_wait();
+    const int b = blockIdx.x, tid = threadIdx.x, w = a.w, k = a.step, R = a.R;
+    const int base = k == 1 ? 0 : w + (k - 2) * w * w;
+    const int nc = R * w;
+    if (tid < R) {
+        s_fscore[tid] = k == 1 ? 0.f : a.front_score[b * w + tid];
+        s_fpool[tid] = k == 1 ? -1 : a.front_pool[b * w + tid];
+        s_fmask[tid] = k == 1 ? 0ull : a.front_mask[b * w + tid];
+    }
+    __syncthreads();
+    int tok = 0;
+    float sc = 0.f;
+    if (tid < nc) {
+        const int j = tid / w, r = tid % w, t = b * w + j;
+        tok = a.top_ids[(size_t)t * w + r];
+        sc = s_fscore[j] + (a.top_vals[(size_t)t * w + r] - a.lse[t]);
+        s_cs[tid] = sc;
+        const size_t e = (size_t)b * a.P + base + tid;
+        a.pool_tok[e] = tok;
+        a.pool_par[e] = s_fpool[j];
+        a.pool_score[e] = sc;
+    }
+    __syncthreads();
+    if (tid < nc) {
+        int rank = 0;
+        for (int c = 0; c < nc; ++c) rank += (s_cs[c] > sc) || (s_cs[c] == sc && c < tid);
+        if (rank < w) {
+            const int j = tid / w, o = b * w + rank;
+            a.front_tok[o] = tok;
+            a.front_row[o] = k == 1 ? b : b * w + j;   // the h^ row that emitted the token
+            a.front_pool[o] = base + tid;
+            a.front_score[o] = sc;
+            const int bit = (k - 1) * w + rank;     // the slot offset of the row that processes it next
+            a.front_mask[o] = s_fmask[j] | (bit < kTreeMaskBits ? 1ull << bit : 0ull);
+            if (a.out_frontier) a.out_frontier[((size_t)b * a.K + k - 1) * w + rank] = base + tid;
+        }
+    }
+    if (k < a.K) return;                           // uniform over the CTA
+
+    // the verified tree: the n_nodes best of the pool, listed in pool order
+    __syncthreads();
+    const int P = a.P;
+    const size_t pb = (size_t)b * P;
+    for (int e = tid; e < P; e += kSelectThreads) s_ps[e] = __ldcg(a.pool_score + pb + e);
+    __syncthreads();
+    for (int e = tid; e < P; e += kSelectThreads) {
+        const float se = s_ps[e];
+        int rank = 0;
+        for (int c = 0; c < P; ++c) {
+            const float x = s_ps[c];
+            rank += (x > se) || (x == se && c < e);
+        }
+        s_sel[e] = rank < a.n_nodes;
+    }
+    __syncthreads();
+    for (int e = tid; e < P; e += kSelectThreads) {
+        int p = -1;
+        if (s_sel[e]) {
+            p = 0;
+            for (int c = 0; c < e; ++c) p += s_sel[c];
+        }
+        s_pos[e] = p;
+    }
+    __syncthreads();
+    for (int e = tid; e < P; e += kSelectThreads) {
+        const int tk = __ldcg(a.pool_tok + pb + e), par = __ldcg(a.pool_par + pb + e);
+        if (a.out_pool_tokens) a.out_pool_tokens[pb + e] = tk;
+        if (a.out_pool_parents) a.out_pool_parents[pb + e] = par;
+        if (a.out_pool_scores) a.out_pool_scores[pb + e] = s_ps[e];
+        const int p = s_pos[e];
+        if (p < 0) continue;
+        const size_t o = (size_t)b * a.n_nodes + p;
+        a.tree_tokens[o] = tk;
+        a.tree_depths[o] = e < w ? 1 : 2 + (e - w) / (w * w);
+        a.tree_scores[o] = s_ps[e];
+        a.tree_parents[o] = par < 0 ? -1 : s_pos[par];
+    }
+}
+
+// ------------------------------------------------------------------ acceptance
+
+__global__ void accept_tree_kernel(const AcceptTreeArgs a) {
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b >= a.B) return;
+    const int m = a.n_nodes, K = a.K;
+    const int32_t *tok = a.tree_tokens + (size_t)b * m, *par = a.tree_parents + (size_t)b * m;
+    const int32_t *tn = a.target_next + (size_t)b * (m + 1);
+    for (int j = 0; j < K; ++j) a.accept_nodes[b * K + j] = -1;
+    for (int j = 0; j <= K; ++j) a.out_tokens[b * (K + 1) + j] = -1;
+    int cur = -1, acc = 0;
+    while (acc < K) {
+        const int want = tn[cur + 1];
+        int next = -1;
+        for (int i = 0; i < m; ++i)
+            if (par[i] == cur && tok[i] == want) { next = i; break; }
+        if (next < 0) break;
+        a.accept_nodes[b * K + acc] = next;
+        a.out_tokens[b * (K + 1) + acc] = tok[next];
+        ++acc;
+        cur = next;
+    }
+    a.out_tokens[b * (K + 1) + acc] = tn[cur + 1];
+    a.accept_len[b] = acc;
+    a.kv_len[b] += a.n_new[b];
+}
+
+template <typename WT, int D>
+size_t tree_attn_smem(int chunk, int G, int w, int splits) {
+    constexpr int RS = D + Elem<WT>::kPerVec;
+    const int NQ = w * G;
+    return 2 * (size_t)chunk * RS * sizeof(WT) + ((size_t)NQ * D + (size_t)NQ * chunk + (size_t)NQ * splits) * 4;
+}
+
+template <typename WT, int D>
+cudaError_t launch_tree_attn_t(const TreeArgs &a, cudaStream_t s, bool pdl) {
+    const size_t smem = tree_attn_smem<WT, D>(a.chunk, a.Hq / a.Hkv, a.w, a.splits);
+    return launch_k(tree_attention_kernel<WT, D>, dim3(a.splits, a.Hkv, a.B), dim3(kAttnThreads), smem, s, pdl, a);
+}
+
+template <typename WT, int D>
+cudaError_t prepare_tree_attn_t(int chunk, int G, int w, int splits) {
+    const size_t smem = tree_attn_smem<WT, D>(chunk, G, w, splits);
+    return cudaFuncSetAttribute(tree_attention_kernel<WT, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+}
+
+}  // namespace
+
+size_t tree_attention_smem_bytes(bool bf16, int D, int chunk, int G, int w, int splits) {
+    if (bf16) return D == 64 ? tree_attn_smem<uint16_t, 64>(chunk, G, w, splits) : tree_attn_smem<uint16_t, 128>(chunk, G, w, splits);
+    return D == 64 ? tree_attn_smem<float, 64>(chunk, G, w, splits) : tree_attn_smem<float, 128>(chunk, G, w, splits);
+}
+
+cudaError_t prepare_tree_kernels(bool bf16, int D, int chunk, int G, int w, int splits) {
+    if (bf16) return D == 64 ? prepare_tree_attn_t<uint16_t, 64>(chunk, G, w, splits)
+                             : prepare_tree_attn_t<uint16_t, 128>(chunk, G, w, splits);
+    return D == 64 ? prepare_tree_attn_t<float, 64>(chunk, G, w, splits) : prepare_tree_attn_t<float, 128>(chunk, G, w, splits);
+}
+
+cudaError_t launch_tree_gather(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl) {
+    if (bf16) return launch_k(tree_gather_kernel<uint16_t>, dim3(a.B * a.w), dim3(256), 0, s, pdl, a);
+    return launch_k(tree_gather_kernel<float>, dim3(a.B * a.w), dim3(256), 0, s, pdl, a);
+}
+
+cudaError_t launch_tree_rope(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl) {
+    const int warps = a.B * a.w * (a.Hq + 2 * a.Hkv);
+    const dim3 grid((warps + 3) / 4);
+    if (bf16) return launch_k(tree_rope_kernel<uint16_t>, grid, dim3(128), 0, s, pdl, a);
+    return launch_k(tree_rope_kernel<float>, grid, dim3(128), 0, s, pdl, a);
+}
+
+cudaError_t launch_tree_attention(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl) {
+    if (bf16) return a.D == 64 ? launch_tree_attn_t<uint16_t, 64>(a, s, pdl) : launch_tree_attn_t<uint16_t, 128>(a, s, pdl);
+    return a.D == 64 ? launch_tree_attn_t<float, 64>(a, s, pdl) : launch_tree_attn_t<float, 128>(a, s, pdl);
+}
+
+cudaError_t launch_tree_lse(const TreeArgs &args, cudaStream_t s, bool pdl) {
+    TreeArgs a = args;
+    a.lse_blocks = sample_blocks(a.V, &a.lse_chunk);
+    return launch_k(tree_lse_kernel, dim3(a.lse_blocks, a.B * a.R), dim3(256), 0, s, pdl, a);
+}
+
+cudaError_t launch_tree_select(const TreeArgs &a, cudaStream_t s, bool pdl) {
+    return launch_k(tree_select_kernel, dim3(a.B), dim3(kSelectThreads), 0, s, pdl, a);
+}
+
+cudaError_t launch_accept_tree(const AcceptTreeArgs &a, cudaStream_t s) {
+    return launch_k(accept_tree_kernel, dim3((a.B + 127) / 128), dim3(128), 0, s, false, a);
+}
+
+}  // namespace prism

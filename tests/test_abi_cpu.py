@@ -73,3 +73,21 @@ def test_null_context_calls_return_invalid_arg(lib):
     f.argtypes = [vp, ctypes.c_int32, vp, vp, vp, f32] + [vp] * 7
     assert f(None, 1, None, None, None, 0.8, *([None] * 7)) == 1
     assert lib.prism_destroy(None) == 0
+
+
+def test_tree_entry_points_reject_null_context(lib):
+    vp, i32 = ctypes.c_void_p, ctypes.c_int32
+    f = lib.prism_draft_tree
+    f.argtypes = [vp, i32] + [vp] * 6 + [i32, i32, vp, vp]
+    assert f(None, 1, *([None] * 6), 4, 16, None, None) == 1
+    f = lib.prism_accept_tree
+    f.argtypes = [vp, i32, i32] + [vp] * 9
+    assert f(None, 1, 16, *([None] * 9)) == 1
+
+
+def test_create_rejects_tree_width_above_eight(lib):
+    from paper_2602_01762_gb300 import _Config
+    bad = _Config(256, 4, 4, 64, 688, 4096, 3, 1, 1, 64, 1, 1, 10000.0, 1e-5, 1, 9)
+    out = ctypes.c_void_p()
+    lib.prism_create.argtypes = [ctypes.POINTER(_Config), ctypes.c_int32, ctypes.POINTER(ctypes.c_void_p)]
+    assert lib.prism_create(ctypes.byref(bad), 0, ctypes.byref(out)) == 1
