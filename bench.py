@@ -30,6 +30,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "draft tokens/s and K-step round latency (µs) at 1 GB300; % of HBM roofline"
 UNIT = "draft tokens/s"
+TREE_UNIT = "draft tree tokens/s (verified tree nodes)"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 LM_KIND = "lm_head"
@@ -63,6 +64,27 @@ def round_bytes(w, kv_len):
             p = L + n - 1 if k == 1 else L + n + k - 2
             kv_read += (p + 1) * kv_row
     kv_write = B * (n + K - 1) * kv_row
+    return weights + emb + hid + kv_read + kv_write
+
+
+def tree_round_bytes(w, kv_len):
+    """Algorithmic bytes of one tree round: every step's module weights and
+    the LM head, embedding rows gathered and target hidden states read, the
+    KV rows each step's attention must read once per sequence (the committed
+    rows plus the tree's draft slots so far) and the KV rows written."""
+    s = w.shape
+    es = 2 if s.dtype == "bf16" else 4
+    K, B, n, tw = s.n_steps, w.batch, w.n_new, w.tree_width
+    weights = K * (s.module_params() + s.vocab * s.hidden) * es
+    emb = B * n * s.hidden * es + B * (K - 1) * tw * s.hidden * es
+    hid = B * n * s.hidden * es
+    kv_row = 2 * s.n_kv_heads * s.head_dim * es
+    kv_read = 0
+    for L in kv_len:
+        kv_read += (L + n) * kv_row                      # step 1: the causal window of the last prefill row
+        for k in range(2, K + 1):
+            kv_read += (L + n + (k - 1) * tw) * kv_row   # committed rows + the draft slots up to this step
+    kv_write = B * (n + (K - 1) * tw) * kv_row
     return weights + emb + hid + kv_read + kv_write
 
 
@@ -217,7 +239,10 @@ def main():
             run_reference(args, w)
         return
     world, rank, local = dist_setup()
-    run_ours(args, w, world, rank, local)
+    if w.tree_width > 0:
+        run_tree(args, w, world, rank, local)
+    else:
+        run_ours(args, w, world, rank, local)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
@@ -237,7 +262,7 @@ def run_reference(args, w):
     W1 = dict(W, f_map=tuple(W["f_map"])[:1])
 
     def sample():
-        oracle.draft_round(shape1, W1, I, topk=max(1, w.topk), want_hidden=False, seqs=[0])
+        oracle.draft_round(shape1, W1, I, topk=max(1, w.topk, w.tree_width), want_hidden=False, seqs=[0])
 
     for _ in range(args.warmup):
         sample()
@@ -251,13 +276,21 @@ def run_reference(args, w):
     cores = oracle.num_threads()
     desc = (f"per step, the first draft step of sequence 0 of workload {w.name} (one draft token: "
             f"fusion, transformer block, LM head, selection), fp64 oracle")
+    unit = UNIT
+    if w.tree_width > 0:
+        # a tree round processes 1 + (K - 1) w such rows and yields n_nodes tree tokens
+        rows = 1 + (w.shape.n_steps - 1) * w.tree_width
+        value *= w.tree_nodes / rows
+        unit = TREE_UNIT
+        desc += (f"; scaled to tree tokens: {w.tree_nodes} tokens per round of {rows} processed rows, "
+                 f"each row costing one such step")
     print(json.dumps({
-        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "impl": "reference", "metric": METRIC, "value": value, "unit": unit, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": config_of(w),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc},
-        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "cpu_baseline": {"value": value, "unit": unit, "cores": cores, "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
 
 
@@ -268,7 +301,8 @@ def config_of(w):
             "draft_steps": s.n_steps, "batch": w.batch, "kv_context": [w.ctx_lo, w.ctx_hi],
             "accepted_tokens_in": w.n_new, "topk": w.topk, "modules": len(set(w.modules())),
             "seed": w.seed, "l2": "inputs larger than L2 (whole weight set streamed every round)",
-            "parallelism": "replicas"}
+            "parallelism": "replicas",
+            **({"tree_width": w.tree_width, "tree_nodes": w.tree_nodes} if w.tree_width else {})}
 
 
 def run_ours(args, w, world, rank, local):
@@ -410,6 +444,147 @@ def run_ours(args, w, world, rank, local):
     dr.close()
     del weights_dev
 
+
+def run_tree(args, w, world, rank, local):
+    """Tree-drafting rounds (prism_draft_tree): the same timing contract as
+    the chain; `value` counts verified tree tokens (n_nodes per sequence)."""
+    import numpy as np
+    import torch
+
+    import synth
+    from paper_2602_01762_gb300 import Drafter
+    from paper_2602_01762_gb300.host import bind_weights, to_device
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    s = w.shape
+    W, I = synth.make_weights(w), synth.make_round_inputs(w)
+    B, K, tw, m = w.batch, s.n_steps, w.tree_width, w.tree_nodes
+    dr = Drafter.from_shape(s, max_batch=B, max_ctx=int(I["max_ctx"]), max_new=I["tokens"].shape[1], topk=1,
+                            max_tree_width=tw, device=local)
+    weights_dev = bind_weights(dr, W, device=dev)
+    options = {}
+    for kv in args.opt:
+        name, value = kv.split("=", 1)
+        options[name] = int(value)
+        dr.set_option(name, int(value))
+    t = {n: to_device(I[n], dev) for n in ("tokens", "hidden", "n_new", "kv_len", "k_cache", "v_cache")}
+    tt = torch.empty((B, m), dtype=torch.int32, device=dev)
+    tp = torch.empty((B, m), dtype=torch.int32, device=dev)
+    td = torch.empty((B, m), dtype=torch.int32, device=dev)
+    ts = torch.empty((B, m), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def one_round():
+        dr.draft_tree(t["tokens"], t["hidden"], t["n_new"], t["kv_len"], t["k_cache"], t["v_cache"], tw,
+                      tt, tp, td, ts, stream=stream)
+
+    for _ in range(args.warmup):
+        one_round()
+    assert dr.sync_status(stream) == 0
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.2)
+    dist_barrier(world)
+    torch.cuda.synchronize(dev)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        one_round()
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    dist_barrier(world)
+    clk = clocks.stop()
+    ms = dist_reduce(ev0.elapsed_time(ev1), "max", world, dev if world > 1 else None)
+    flags = dr.sync_status(stream)
+    launches_per_round = dr.round_launches()
+    tokens_total = B * m * args.steps * world
+    value = tokens_total / (ms / 1e3)
+    per_round_ms = ms / args.steps
+
+    prof = [dr.profile_tree(t["tokens"], t["hidden"], t["n_new"], t["kv_len"], t["k_cache"], t["v_cache"], tw,
+                            tt, tp, td, ts, stream=stream) for _ in range(max(3, min(20, args.steps)))]
+    by_kind = {}
+    for rnd in prof[1:]:
+        for kind, kms in rnd:
+            by_kind.setdefault(kind, []).append(kms)
+    kind_total = {k: sum(v) / (len(prof) - 1) for k, v in by_kind.items()}
+    lm_ms = statistics.mean(by_kind.get(LM_KIND, [float("nan")]))
+    es = 2 if s.dtype == "bf16" else 4
+    # LM-head launches of a round: step 1 on B rows, steps 2..K on B * w rows
+    lm_b = s.vocab * s.hidden * es + (B + (K - 1) * B * tw) / K * (s.hidden * 4 + kTOP * 8)
+    peak, peak_src = hbm_peak()
+    achieved = lm_b / (lm_ms / 1e3) / 1e9
+
+    pin = {n: torch.from_numpy(np.ascontiguousarray(
+        I[n].view(np.int16) if I[n].dtype == np.uint16 else I[n])).pin_memory()
+        for n in ("tokens", "hidden", "n_new", "kv_len")}
+    if I["hidden"].dtype == np.uint16:
+        pin["hidden"] = pin["hidden"].view(torch.bfloat16)
+    host_out = [torch.empty((B, m), dtype=torch.int32).pin_memory() for _ in range(2)]
+    h2d = sum(p.numel() * p.element_size() for p in pin.values())
+    d2h = sum(h.numel() * h.element_size() for h in host_out)
+
+    def e2e_round():
+        for n, p in pin.items():
+            t[n].copy_(p, non_blocking=True)
+        one_round()
+        host_out[0].copy_(tt, non_blocking=True)
+        host_out[1].copy_(tp, non_blocking=True)
+
+    for _ in range(args.warmup):
+        e2e_round()
+    torch.cuda.synchronize(dev)
+    dist_barrier(world)
+    e0 = time.perf_counter()
+    for _ in range(args.steps):
+        e2e_round()
+    torch.cuda.synchronize(dev)
+    e_s = dist_reduce(time.perf_counter() - e0, "max", world, dev if world > 1 else None)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        times = []
+        t_end = time.perf_counter() + args.cpu_budget
+        while True:
+            c0 = time.perf_counter()
+            oracle.draft_tree(s, W, I, width=tw, n_nodes=m, want_logits=False, seqs=[0])
+            times.append(time.perf_counter() - c0)
+            if time.perf_counter() >= t_end:
+                break
+        sec = statistics.median(times)
+        cpu = {"value": m / sec, "unit": TREE_UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+               "sample": (f"{len(times)} full tree rounds of sequence 0 of {w.name} "
+                          f"(median {sec:.3f} s per round), fp64 oracle on all host cores")}
+
+    total_bytes = tree_round_bytes(w, [int(x) for x in I["kv_len"]])
+    if rank == 0:
+        shares = {k: v / sum(kind_total.values()) for k, v in kind_total.items()}
+        print(json.dumps({
+            "metric": METRIC, "value": value, "unit": TREE_UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": per_round_ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if s.dtype == "bf16" else "f32",
+            "data": "synthetic", "config": dict(config_of(w), options=options),
+            "round_latency_us": per_round_ms * 1e3,
+            "hbm": {"bytes_per_round": total_bytes,
+                    "achieved_gbs": total_bytes / (per_round_ms / 1e3) / 1e9,
+                    "frac_of_8tbs": total_bytes / (per_round_ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,
+                    "frac_of_measured": total_bytes / (per_round_ms / 1e3) / 1e9 / peak},
+            "roofline": {"kernel": "LM head GEMV + top-w selection", "bound": "hbm", "achieved": achieved,
+                         "peak": peak, "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": None, "bytes_per_launch": lm_b, "avg_launch_ms": lm_ms},
+            "kernel_time_share": shares,
+            "kernel_ms_per_round": kind_total,
+            "cpu_baseline": cpu,
+            "e2e": {"value": B * m * args.steps * world / e_s, "unit": TREE_UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches_per_round * args.steps,
+            "clocks": clk,
+            "device_error_word": flags,
+        }), flush=True)
+    dr.close()
+    del weights_dev
 
 if __name__ == "__main__":
     main()

@@ -78,12 +78,15 @@ def library() -> ctypes.CDLL:
         lib.prism_accept_sampled.argtypes = [vp, i32, vp, vp, vp, flt] + [vp] * 7
         lib.prism_draft_tree.argtypes = [vp, i32] + [vp] * 6 + [i32, i32, P(_TreeOutputs), vp]
         lib.prism_accept_tree.argtypes = [vp, i32, i32] + [vp] * 9
+        lib.prism_profile_tree.argtypes = [vp, i32] + [vp] * 6 + [i32, i32, P(_TreeOutputs), vp,
+                                                                P(ctypes.c_float), P(i32), i32, P(i32)]
         lib.prism_get_error.restype = ctypes.c_char_p
         lib.prism_version.restype = ctypes.c_char_p
         for f in ("prism_create", "prism_destroy", "prism_load_shared_weights", "prism_load_step_weights",
                   "prism_draft_round", "prism_accept_greedy", "prism_sync_status", "prism_set_option",
                   "prism_profile_round", "prism_lm_head_topk_static", "prism_round_launches",
-                  "prism_draft_round_sampled", "prism_accept_sampled", "prism_draft_tree", "prism_accept_tree"):
+                  "prism_draft_round_sampled", "prism_accept_sampled", "prism_draft_tree", "prism_accept_tree",
+                  "prism_profile_tree"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -277,6 +280,26 @@ class Drafter:
         self._check(self.lib.prism_draft_tree(
             self.h, B, _ptr(tokens), _ptr(hidden), _ptr(n_new), _ptr(kv_len), _ptr(k_cache), _ptr(v_cache),
             int(width), int(n), ctypes.byref(out), _stream(stream)))
+
+    def profile_tree(self, tokens, hidden, n_new, kv_len, k_cache, v_cache, width: int, tree_tokens, tree_parents,
+                     tree_depths, tree_scores, stream=None):
+        """Eager tree round with a CUDA event around every kernel; returns a
+        list of (kind, milliseconds) in launch order."""
+        B = self._round_args(tokens, hidden, n_new, kv_len, k_cache, v_cache, None, None, None)
+        n = tree_tokens.shape[1]
+        for t, dt, name in ((tree_tokens, torch.int32, "tree_tokens"), (tree_parents, torch.int32, "tree_parents"),
+                            (tree_depths, torch.int32, "tree_depths"), (tree_scores, torch.float32, "tree_scores")):
+            self._tensor(t, (B, n), dt, name)
+        out = _TreeOutputs(tree_tokens.data_ptr(), tree_parents.data_ptr(), tree_depths.data_ptr(),
+                           tree_scores.data_ptr(), None, None, None, None, None)
+        cap = 12 * self.n_steps + 8
+        ms = (ctypes.c_float * cap)()
+        kinds = (ctypes.c_int32 * cap)()
+        cnt = ctypes.c_int32(0)
+        self._check(self.lib.prism_profile_tree(
+            self.h, B, _ptr(tokens), _ptr(hidden), _ptr(n_new), _ptr(kv_len), _ptr(k_cache), _ptr(v_cache),
+            int(width), int(n), ctypes.byref(out), _stream(stream), ms, kinds, cap, ctypes.byref(cnt)))
+        return [(KERNEL_KINDS[kinds[i]], float(ms[i])) for i in range(cnt.value)]
 
     def accept_tree(self, tree_tokens, tree_parents, target_next, n_new, kv_len, accept_len, accept_nodes,
                     out_tokens, stream=None):

@@ -994,6 +994,11 @@ prism_status prism_round_launches(prism_ctx *c, int32_t *n_launches) {
     return PRISM_OK;
 }
 
+namespace {
+prism_status profile_round(prism_ctx *c, const RoundArgs &r, void *stream, float *kernel_ms, int32_t *kernel_kind,
+                           int32_t max_kernels, int32_t *n_kernels);
+}
+
 prism_status prism_profile_round(prism_ctx *c, int32_t batch, const int32_t *tokens, const void *hidden,
                                  const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
                                  int32_t *draft_ids, int32_t *topk_ids, float *topk_logits, void *stream,
@@ -1001,6 +1006,34 @@ prism_status prism_profile_round(prism_ctx *c, int32_t batch, const int32_t *tok
                                  int32_t *n_kernels) {
     const RoundArgs r = round_args(batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids, topk_ids,
                                    topk_logits, nullptr, nullptr);
+    return profile_round(c, r, stream, kernel_ms, kernel_kind, max_kernels, n_kernels);
+}
+
+prism_status prism_profile_tree(prism_ctx *c, int32_t batch, const int32_t *tokens, const void *hidden,
+                                const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
+                                int32_t width, int32_t n_nodes, const prism_tree_outputs *out, void *stream,
+                                float *kernel_ms, int32_t *kernel_kind, int32_t max_kernels, int32_t *n_kernels) {
+    if (!c) return fail(c, PRISM_ERR_INVALID_ARG, "null context");
+    if (!out || !out->tokens || !out->parents || !out->depths || !out->scores)
+        return fail(c, PRISM_ERR_INVALID_ARG, "tree outputs: tokens, parents, depths and scores are required");
+    const long K = c->cfg.n_steps;
+    const long P = width + (K - 1) * (long)width * width;
+    if (width < 1 || width > c->cfg.max_tree_width || width > c->cfg.vocab || (K - 1) * width > kTreeMaskBits ||
+        P > kTreeMaxPool || n_nodes < 1 || n_nodes > P)
+        return fail(c, PRISM_ERR_INVALID_ARG, "tree width or n_nodes out of range");
+    RoundArgs r = round_args(batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, c->tree_draft, nullptr,
+                             nullptr, nullptr, nullptr);
+    r.tree_w = width;
+    r.tree_m = n_nodes;
+    r.tree = *out;
+    return profile_round(c, r, stream, kernel_ms, kernel_kind, max_kernels, n_kernels);
+}
+
+}  // extern "C"
+
+namespace {
+prism_status profile_round(prism_ctx *c, const RoundArgs &r, void *stream, float *kernel_ms, int32_t *kernel_kind,
+                           int32_t max_kernels, int32_t *n_kernels) {
     prism_status st = check_round_args(c, r);
     if (st != PRISM_OK) return st;
     if (!kernel_ms || !n_kernels || max_kernels < 1) return fail(c, PRISM_ERR_INVALID_ARG, "null output");
@@ -1023,6 +1056,9 @@ prism_status prism_profile_round(prism_ctx *c, int32_t batch, const int32_t *tok
     for (auto &x : ev) cudaEventDestroy(x);
     return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "profiled round");
 }
+}  // namespace
+
+extern "C" {
 
 prism_status prism_accept_greedy(prism_ctx *c, int32_t batch, const int32_t *draft, const int32_t *target,
                                  const int32_t *n_new, int32_t *kv_len, int32_t *accept_len,

@@ -56,23 +56,38 @@ __device__ __forceinline__ void lse_merge(float &m, float &s, float m2, float s2
 
 // ------------------------------------------------------------------ gather
 
+constexpr int kGatherThreads = 128;
+
+// Grid (rows, ceil(d / (VEC * 128))): thread i of CTA (t, c) moves VEC
+// consecutive elements (16 bytes of the embedding row) of both halves of
+// row t, issuing its loads before its stores.
 template <typename WT>
-__global__ void __launch_bounds__(256) tree_gather_kernel(const TreeArgs a) {
+__global__ void __launch_bounds__(kGatherThreads) tree_gather_kernel(const TreeArgs a) {
+    constexpr int VEC = Elem<WT>::kPerVec;
     pdl_trigger();
     pdl_wait();
     const int t = blockIdx.x;              // row b * w + j
+    const int i0 = (blockIdx.y * kGatherThreads + threadIdx.x) * VEC;
+    if (i0 >= a.d) return;
     int tok = a.front_tok[t];
     if (tok < 0 || tok >= a.V) {
-        if (threadIdx.x == 0) set_err(a.err, kErrToken);
+        set_err(a.err, kErrToken);
         tok = tok < 0 ? 0 : a.V - 1;
     }
-    const WT *e = (const WT *)a.embed + (size_t)tok * a.d;
-    const float *h = a.hhat + (size_t)a.front_row[t] * a.d;
-    WT *u = (WT *)a.u_out + (size_t)t * 2 * a.d;
-    for (int i = threadIdx.x; i < a.d; i += blockDim.x) {
-        u[i] = e[i];
-        Elem<WT>::store(u, a.d + i, h[i]);  // the operand rounding of the fusion input
+    const uint4 ev = *(const uint4 *)((const WT *)a.embed + (size_t)tok * a.d + i0);
+    const float *h = a.hhat + (size_t)a.front_row[t] * a.d + i0;
+    float hv[VEC];
+#pragma unroll
+    for (int q = 0; q < VEC; q += 4) {
+        const float4 f = *(const float4 *)(h + q);
+        hv[q] = f.x; hv[q + 1] = f.y; hv[q + 2] = f.z; hv[q + 3] = f.w;
     }
+    WT *u = (WT *)a.u_out + (size_t)t * 2 * a.d;
+    *(uint4 *)(u + i0) = ev;
+    alignas(16) WT r[VEC];
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) Elem<WT>::store(r, q, hv[q]);   // the fusion input's operand rounding
+    *(uint4 *)(u + a.d + i0) = *(const uint4 *)r;
 }
 
 // ------------------------------------------------------------------ RoPE + append
@@ -167,12 +182,14 @@ __device__ __forceinline__ void load_run(const WT *p, float (&out)[DPL]) {
     }
 }
 
+constexpr int kTreeAttnThreads = 512;   // 16 warps: one (row, query head) pair each when w * G = 16
+
 // Grid (splits, Hkv, B); CTA (s, g, b) stages keys [s C, s C + C) of KV head g
 // once and scores them against the G query heads of g in each of the w rows
 // of sequence b.  Key slot p is visible to row j when p < L + n (committed and
 // step-1 rows) or bit p - (L + n) of the row's ancestor mask is set.
 template <typename WT, int D>
-__global__ void __launch_bounds__(kAttnThreads) tree_attention_kernel(const TreeArgs a) {
+__global__ void __launch_bounds__(kTreeAttnThreads) tree_attention_kernel(const TreeArgs a) {
     extern __shared__ __align__(16) uint8_t smem_raw[];
     __shared__ int s_last;
     constexpr int VEC = Elem<WT>::kPerVec;
@@ -307,12 +324,24 @@ __global__ void __launch_bounds__(kAttnThreads) tree_attention_kernel(const Tree
         float acc[DPL];
 #pragma unroll
         for (int u = 0; u < DPL; ++u) acc[u] = 0.f;
-        for (int sp = 0; sp < a.splits; ++sp) {
-            const float wgt = wh[sp];
-            if (wgt == 0.f) continue;
-            const float *src = part + (size_t)sp * PS + lane * DPL;
+        // weighted sum in split order, eight splits' loads in flight at a time
+        // (a split with no visible key has weight 0 and zero sums)
+        constexpr int kBatch = 8;
+        for (int sp0 = 0; sp0 < a.splits; sp0 += kBatch) {
+            float v[kBatch][DPL], wv[kBatch];
 #pragma unroll
-            for (int u = 0; u < DPL; ++u) acc[u] = fmaf(wgt, __ldcg(src + u), acc[u]);
+            for (int i = 0; i < kBatch; ++i) {
+                const int sp = sp0 + i;
+                const bool in = sp < a.splits;
+                wv[i] = in ? wh[sp] : 0.f;
+                const float *src = part + (size_t)(in ? sp : 0) * PS + lane * DPL;
+#pragma unroll
+                for (int u = 0; u < DPL; ++u) v[i][u] = in ? __ldcg(src + u) : 0.f;
+            }
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i)
+#pragma unroll
+                for (int u = 0; u < DPL; ++u) acc[u] = fmaf(wv[i], v[i][u], acc[u]);
         }
         WT *o = (WT *)a.o_out + ((size_t)t * a.Hq + h) * D;
         const float inv = den > 0.f ? 1.0f / den : 0.f;
@@ -327,6 +356,7 @@ __global__ void __launch_bounds__(kAttnThreads) tree_attention_kernel(const Tree
 // Grid (blocks per row, B * R): row t = b * w + j of the LM head's logits.
 __global__ void __launch_bounds__(256) tree_lse_kernel(const TreeArgs a) {
     __shared__ float s_m[8], s_s[8];
+    __shared__ int s_last;
     pdl_trigger();
     pdl_wait();
     const int blk = blockIdx.x, nblk = gridDim.x;
@@ -343,21 +373,40 @@ __global__ void __launch_bounds__(256) tree_lse_kernel(const TreeArgs a) {
     }
     if (lane == 0) { s_m[warp] = m; s_s[warp] = s; }
     __syncthreads();
-    if (tid != 0) return;
-    for (int q = 1; q < (int)(blockDim.x >> 5); ++q) lse_merge(m, s, s_m[q], s_s[q]);
-    float *part = a.lse_part + ((size_t)t * kSampleMaxBlocks + blk) * 2;
-    part[0] = m;
-    part[1] = s;
-    __threadfence();
-    if (atomicAdd(a.lse_ctr + t, 1) != nblk - 1) return;
-    __threadfence();
-    float M = -INFINITY, S = 0.f;
-    for (int q = 0; q < nblk; ++q) {
-        const float *pq = a.lse_part + ((size_t)t * kSampleMaxBlocks + q) * 2;
-        lse_merge(M, S, __ldcg(pq), __ldcg(pq + 1));
+    if (tid == 0) {
+        for (int q = 1; q < (int)(blockDim.x >> 5); ++q) lse_merge(m, s, s_m[q], s_s[q]);
+        float *part = a.lse_part + ((size_t)t * kSampleMaxBlocks + blk) * 2;
+        part[0] = m;
+        part[1] = s;
+        __threadfence();
+        s_last = atomicAdd(a.lse_ctr + t, 1) == nblk - 1;
     }
-    a.lse[t] = M + logf(S);
-    a.lse_ctr[t] = 0;
+    __syncthreads();
+    if (!s_last || warp != 0) return;
+    // the last CTA of the row: lane l merges partials l, l + 32, ... (all
+    // loads issued first), then the lanes merge in a fixed butterfly order
+    __threadfence();
+    constexpr int kPer = kSampleMaxBlocks / 32;
+    float pm[kPer], ps[kPer];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        const int q = lane + 32 * i;
+        const float *pq = a.lse_part + ((size_t)t * kSampleMaxBlocks + q) * 2;
+        pm[i] = q < nblk ? __ldcg(pq) : -INFINITY;
+        ps[i] = q < nblk ? __ldcg(pq + 1) : 0.f;
+    }
+    float M = -INFINITY, S = 0.f;
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) lse_merge(M, S, pm[i], ps[i]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, M, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, S, o);
+        lse_merge(M, S, m2, s2);
+    }
+    if (lane == 0) {
+        a.lse[t] = M + logf(S);
+        a.lse_ctr[t] = 0;
+    }
 }
 
 // ------------------------------------------------------------------ selection
@@ -493,7 +542,8 @@ size_t tree_attn_smem(int chunk, int G, int w, int splits) {
 template <typename WT, int D>
 cudaError_t launch_tree_attn_t(const TreeArgs &a, cudaStream_t s, bool pdl) {
     const size_t smem = tree_attn_smem<WT, D>(a.chunk, a.Hq / a.Hkv, a.w, a.splits);
-    return launch_k(tree_attention_kernel<WT, D>, dim3(a.splits, a.Hkv, a.B), dim3(kAttnThreads), smem, s, pdl, a);
+    return launch_k(tree_attention_kernel<WT, D>, dim3(a.splits, a.Hkv, a.B), dim3(kTreeAttnThreads), smem, s, pdl,
+                    a);
 }
 
 template <typename WT, int D>
@@ -516,8 +566,10 @@ cudaError_t prepare_tree_kernels(bool bf16, int D, int chunk, int G, int w, int 
 }
 
 cudaError_t launch_tree_gather(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl) {
-    if (bf16) return launch_k(tree_gather_kernel<uint16_t>, dim3(a.B * a.w), dim3(256), 0, s, pdl, a);
-    return launch_k(tree_gather_kernel<float>, dim3(a.B * a.w), dim3(256), 0, s, pdl, a);
+    const int vec = bf16 ? 8 : 4;
+    const dim3 grid(a.B * a.w, (a.d / vec + kGatherThreads - 1) / kGatherThreads);
+    if (bf16) return launch_k(tree_gather_kernel<uint16_t>, grid, dim3(kGatherThreads), 0, s, pdl, a);
+    return launch_k(tree_gather_kernel<float>, grid, dim3(kGatherThreads), 0, s, pdl, a);
 }
 
 cudaError_t launch_tree_rope(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl) {
