@@ -367,9 +367,10 @@ prism_status prism_profile_round(prism_ctx *ctx, int32_t batch, const int32_t *t
                                  int32_t *n_kernels);
 
 /* The same instrumentation for a tree round (prism_draft_tree's arguments);
- * kernel kinds add 9 tree gather, 10 tree log-sum-exp, 11 tree selection (the
- * tree steps' RoPE/append and attention report 2 and 3).  Synchronises the
- * stream.  Errors: as prism_draft_tree and prism_profile_round. */
+ * kernel kinds add 9 tree gather and 10 tree log-sum-exp + selection (a tree
+ * step's RoPE, KV append and attention are one kernel, reported as 3).
+ * Synchronises the stream.  Errors: as prism_draft_tree and
+ * prism_profile_round. */
 prism_status prism_profile_tree(prism_ctx *ctx, int32_t batch, const int32_t *tokens, const void *hidden,
                                 const int32_t *n_new, const int32_t *kv_len, void *k_cache, void *v_cache,
                                 int32_t width, int32_t n_nodes, const prism_tree_outputs *out, void *stream,

@@ -19,7 +19,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.environ.get("PRISM_LIB") or os.path.join(_HERE, "libprism.so")
 STEP_TENSORS = ("w_fuse", "g_attn", "w_qkv", "w_o", "g_mlp", "w_gate_up", "w_down", "g_final")
 KERNEL_KINDS = ("fusion", "qkv", "rope_append", "attention", "o_proj", "gate_up", "down", "lm_head", "sample",
-                "tree_gather", "tree_lse", "tree_select")
+                "tree_gather", "tree_lse_select")
 _STATUS = ["OK", "INVALID_ARG", "SHAPE", "CAPACITY", "NOT_LOADED", "CUDA", "OOM", "DEVICE_FLAG", "TIMEOUT"]
 
 

@@ -277,11 +277,11 @@ struct TreeArgs {
     float *lse;                       // [B*w]
     float *lse_part;                  // [B*w, kSampleMaxBlocks, 2]
     int *lse_ctr;                     // [B*w] (left at zero)
+    int *seq_ctr;                     // [B] rows of each sequence with their lse (left at zero)
     int lse_chunk, lse_blocks;
-    // RoPE / append / attention
+    // RoPE / append / attention (one kernel)
     const float *qkv;                 // [B*w, (Hq + 2Hkv) D]
     void *k_cache, *v_cache;          // [B, Hkv, max_ctx, D]
-    float *q;                         // [B*w, Hq, D]
     const float *rope_cos, *rope_sin;
     float *attn_part;                 // [B*w, Hq, splits, D + 4]
     int *attn_ctr;                    // [B, Hkv] (left at zero)
@@ -301,10 +301,8 @@ struct AcceptTreeArgs {
 size_t tree_attention_smem_bytes(bool bf16, int D, int chunk, int G, int w, int splits);
 cudaError_t prepare_tree_kernels(bool bf16, int D, int chunk, int G, int w, int splits);
 cudaError_t launch_tree_gather(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl);
-cudaError_t launch_tree_rope(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl);
 cudaError_t launch_tree_attention(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl);
 cudaError_t launch_tree_lse(const TreeArgs &a, cudaStream_t s, bool pdl);
-cudaError_t launch_tree_select(const TreeArgs &a, cudaStream_t s, bool pdl);
 cudaError_t launch_accept_tree(const AcceptTreeArgs &a, cudaStream_t s);
 
 // Host launchers (return cudaGetLastError of the launch).

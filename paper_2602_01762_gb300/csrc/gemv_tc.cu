@@ -490,7 +490,7 @@ __device__ __forceinline__ void chunk_to_lists(const float (&acc)[16], int row, 
 // marks an empty slot), thread q the entries q, q + P, ...
 template <int P>
 __device__ __forceinline__ void lists_publish(const GemvArgs &a, Key (&l)[kTopK], int T) {
-#pragma unroll
+#pragma unroll 1
     for (int m = 1; m < P; m <<= 1) key_merge_xor(l, m);
     const int e = threadIdx.x - 64, t = e / P, q = e % P;
     if (t < T) {
@@ -507,7 +507,10 @@ __device__ __forceinline__ void lists_publish(const GemvArgs &a, Key (&l)[kTopK]
 }
 
 // This thread's share (candidates first, first + stride, ...) of row t's
-// partial lists, as a sorted list.  Loads are issued 16 at a time.
+// partial lists, as a sorted list.  Loads are issued 16 at a time; ROLLED
+// inserts them through one copy of the insertion network (code that runs once
+// per launch executes at instruction-cache-miss speed), otherwise unrolled.
+template <bool ROLLED>
 __device__ __forceinline__ void gather_keys(const GemvArgs &a, int t, int grid, int first, int stride, Key (&l)[kTopK]) {
     constexpr int kBatch = 16;
     const int ncand = grid * kTopK;
@@ -524,9 +527,15 @@ __device__ __forceinline__ void gather_keys(const GemvArgs &a, int t, int grid, 
             v[b] = cc < ncand ? __ldcg(pv + cc) : 0.f;
             id[b] = cc < ncand ? __ldcg(pi + cc) : -1;
         }
+        if constexpr (ROLLED) {
+#pragma unroll 1
+            for (int b = 0; b < kBatch; ++b)
+                if (id[b] >= 0) key_insert(l, pack_best(v[b], id[b]));
+        } else {
 #pragma unroll
-        for (int b = 0; b < kBatch; ++b)
-            if (id[b] >= 0) key_insert(l, pack_best(v[b], id[b]));
+            for (int b = 0; b < kBatch; ++b)
+                if (id[b] >= 0) key_insert(l, pack_best(v[b], id[b]));
+        }
     }
 }
 
@@ -826,8 +835,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     } else {
                         // one warp per row over every CTA's list
                         for (int t = ew; t < T; t += 4) {
-                            gather_keys(a, t, gridDim.x, lane, 32, lst);
-#pragma unroll
+                            gather_keys<true>(a, t, gridDim.x, lane, 32, lst);
+#pragma unroll 1
                             for (int m = 1; m < 32; m <<= 1) key_merge_xor(lst, m);
                             write_row(a, t, lst);
                         }
@@ -1139,7 +1148,7 @@ __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int g
     pdl_wait();
     const int t = blockIdx.x, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     Key l[kTopK];
-    gather_keys(a, t, grid, threadIdx.x, 128, l);
+    gather_keys<false>(a, t, grid, threadIdx.x, 128, l);
 #pragma unroll
     for (int m = 1; m < 32; m <<= 1) key_merge_xor(l, m);
     if (lane == 0) {

@@ -222,11 +222,12 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
 
     // a projection on the tensor-core kernel when enabled and it fits, else on
     // the CUDA-core ring kernel
-    // (gate/up + SwiGLU stays on the CUDA-core kernel unless gemv_tcgen05 = 2:
-    // with 112 unit tiles it needs split-K on the tensor-core kernel, and
-    // measured slower there)
+    // (gate/up + SwiGLU with one activation row stays on the CUDA-core kernel
+    // unless gemv_tcgen05 = 2: with 112 unit tiles it needs split-K on the
+    // tensor-core kernel, and measured slower there; from two rows on the
+    // CUDA-core kernel's issue cost doubles and the tensor cores win)
     auto proj = [&](const GemvArgs &g, const CUtensorMap *tm, int grid, bool pdl_here) -> cudaError_t {
-        const bool want = c->gemv_tcgen05 == 2 || (c->gemv_tcgen05 == 1 && (g.epi != kEpiSwiGLU || g.T > 2));
+        const bool want = c->gemv_tcgen05 == 2 || (c->gemv_tcgen05 == 1 && (g.epi != kEpiSwiGLU || g.T > 1));
         if (tm && want && c->tc_ready && c->bf16 && g.T >= c->tc_stream_rows && gemv_tcs_supported(g, c->sms)) {
             const size_t ws = gemv_tcs_workspace_floats(g, c->sms);
             if (ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n))
@@ -283,10 +284,10 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         ta.lse = c->tree_lse;
         ta.lse_part = c->tree_lse_part;
         ta.lse_ctr = c->tree_lse_ctr;
+        ta.seq_ctr = c->tree_lse_ctr + c->tree_rows;
         ta.qkv = c->qkv;
         ta.k_cache = r.k_cache;
         ta.v_cache = r.v_cache;
-        ta.q = c->q;
         ta.rope_cos = c->rope_cos;
         ta.rope_sin = c->rope_sin;
         ta.attn_part = c->attn_part;
@@ -357,11 +358,8 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         if (e != cudaSuccess) break;
 
         if (tstep) {
-            // RoPE at the node's depth, K/V at its own slot; attention over the
-            // committed rows and the node's ancestors
-            e = launch_tree_rope(ta, c->bf16, s, pdl);
-            after(2);
-            if (e != cudaSuccess) break;
+            // RoPE at the node's depth, K/V appended at its own slot, attention
+            // over the committed rows and the node's ancestors: one kernel
             e = launch_tree_attention(ta, c->bf16, s, pdl);
             after(3);
             if (e != cudaSuccess) break;
@@ -533,12 +531,10 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         if (e != cudaSuccess) break;
 
         if (tree) {
-            // draft log-probabilities, candidate scores, next frontier (and the tree after step K)
+            // draft log-probabilities; the last row of each sequence then scores
+            // the candidates and picks the next frontier (and the tree after step K)
             e = launch_tree_lse(ta, s, pdl);
             after(10);
-            if (e != cudaSuccess) break;
-            e = launch_tree_select(ta, s, pdl);
-            after(11);
             if (e != cudaSuccess) break;
             continue;
         }
@@ -674,7 +670,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         tree_on * Bw * 4,                                          // tree LM-head top-1 (unused)
         tree_on * Bw * 4,                                          // tree row lse
         tree_on * Bw * kSampleMaxBlocks * 2 * 4,                   // tree lse partials
-        tree_on * Bw * 4,                                          // tree lse tickets
+        tree_on * (Bw + Bseq) * 4,                                 // tree lse tickets, sequence tickets
         tree_on * Bw * 4 * 4,                                      // frontier token, row, pool index, score
         tree_on * Bw * 8,                                          // frontier ancestor masks
         tree_on * Bseq * P_max * 4 * 3,                            // pool tokens, parents, scores

@@ -12,15 +12,16 @@
 // of the round.  The kernels this file adds:
 //   tree_gather_kernel     fusion input row [E(token); round(h^ of the row
 //                          that emitted the token)];
-//   tree_rope_kernel       rotary embedding at the node's depth, K/V stored at
-//                          the node's own cache slot L + n + (k - 2) w + j;
-//   tree_attention_kernel  split-KV attention over the committed rows [0, L+n)
-//                          plus the draft slots in the row's 64-bit ancestor
-//                          mask, all w rows of a sequence against one staged
-//                          chunk of keys, last-CTA merge in split order;
-//   tree_lse_kernel        log-sum-exp of every row's logits;
-//   tree_select_kernel     candidate scores, the next frontier, and after the
-//                          last step the verified tree (one CTA per sequence);
+//   tree_attention_kernel  rotary embedding at the node's depth, K/V appended
+//                          at the node's own cache slot L + n + (k - 2) w + j,
+//                          and split-KV attention over the committed rows
+//                          [0, L+n) plus the draft slots in the row's 64-bit
+//                          ancestor mask, all w rows of a sequence against one
+//                          staged chunk of keys, last-CTA merge in split order;
+//   tree_lse_kernel        log-sum-exp of every row's logits; the last row of
+//                          each sequence to finish then scores the candidates,
+//                          picks the next frontier and, after the last step,
+//                          the verified tree;
 //   accept_tree_kernel     greedy acceptance along the tree (Sec. 2's
 //                          temperature-0 rule applied from the root).
 #include "common.cuh"
@@ -88,50 +89,6 @@ __global__ void __launch_bounds__(kGatherThreads) tree_gather_kernel(const TreeA
 #pragma unroll
     for (int q = 0; q < VEC; ++q) Elem<WT>::store(r, q, hv[q]);   // the fusion input's operand rounding
     *(uint4 *)(u + a.d + i0) = *(const uint4 *)r;
-}
-
-// ------------------------------------------------------------------ RoPE + append
-
-template <typename WT>
-__global__ void __launch_bounds__(128) tree_rope_kernel(const TreeArgs a) {
-    pdl_trigger();
-    pdl_wait();
-    const int lane = threadIdx.x & 31;
-    const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    const int H = a.Hq + 2 * a.Hkv;
-    if (gw >= a.B * a.w * H) return;
-    const int t = gw / H, h = gw % H, b = t / a.w, j = t % a.w;
-    const int n = tree_n(a, b), L = a.kv_len[b];
-    const int pos = L + n + a.step - 2;                  // rotary position: the node's depth
-    const int slot = L + n + (a.step - 2) * a.w + j;     // cache slot: the node's own row (>= pos)
-    const int D = a.D, half = D / 2;
-    const float *x = a.qkv + (size_t)t * H * D + (size_t)h * D;
-    const bool ok = pos >= 0 && slot < a.max_ctx;
-    if (h >= a.Hq && !ok) {
-        if (lane == 0) set_err(a.err, kErrCache);
-        return;
-    }
-    const int pc = ok ? pos : 0;
-    if (h < a.Hq) {
-        float *q = a.q + ((size_t)t * a.Hq + h) * D;
-        for (int i = lane; i < half; i += 32) {
-            const float c = a.rope_cos[(size_t)pc * half + i], s = a.rope_sin[(size_t)pc * half + i];
-            const float x0 = x[i], x1 = x[i + half];
-            q[i] = x0 * c - x1 * s;
-            q[i + half] = x1 * c + x0 * s;
-        }
-    } else if (h < a.Hq + a.Hkv) {
-        WT *k = (WT *)a.k_cache + (((size_t)b * a.Hkv + (h - a.Hq)) * a.max_ctx + slot) * D;
-        for (int i = lane; i < half; i += 32) {
-            const float c = a.rope_cos[(size_t)pos * half + i], s = a.rope_sin[(size_t)pos * half + i];
-            const float x0 = x[i], x1 = x[i + half];
-            Elem<WT>::store(k, i, x0 * c - x1 * s);
-            Elem<WT>::store(k, i + half, x1 * c + x0 * s);
-        }
-    } else {
-        WT *v = (WT *)a.v_cache + (((size_t)b * a.Hkv + (h - a.Hq - a.Hkv)) * a.max_ctx + slot) * D;
-        for (int i = lane; i < D; i += 32) Elem<WT>::store(v, i, x[i]);
-    }
 }
 
 // ------------------------------------------------------------------ attention
@@ -215,19 +172,50 @@ __global__ void __launch_bounds__(kTreeAttnThreads) tree_attention_kernel(const 
     const int j0 = s * C;
     const int nk = PE - j0 < C ? PE - j0 : C;
     const float scale = 1.0f / sqrtf((float)D);
+    // this step's rows: slots new0 + j (j < w), rotary position pos (the depth)
+    const int new0 = base + (a.step - 2) * a.w;
+    const int pos = base + a.step - 2;
+    const int H = a.Hq + 2 * a.Hkv, half = D / 2;
+    if (s == 0 && g == 0 && threadIdx.x == 0 && (L < 0 || new0 + a.w > a.max_ctx)) set_err(a.err, kErrCache);
 
     if (nk > 0 && L >= 0) {
-        const uint4 *kg = (const uint4 *)((const WT *)a.k_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D);
-        const uint4 *vg = (const uint4 *)((const WT *)a.v_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D);
+        // rows written before this step: from the cache
+        const int nold = new0 - j0 < 0 ? 0 : (new0 - j0 < nk ? new0 - j0 : nk);
+        WT *kc = (WT *)a.k_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D;
+        WT *vc = (WT *)a.v_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D;
         constexpr int VPR = D / VEC;
-        for (int e = threadIdx.x; e < nk * VPR; e += blockDim.x) {
+        for (int e = threadIdx.x; e < nold * VPR; e += blockDim.x) {
             const int r = e / VPR, c = e % VPR;
-            cp_async16(Ks + (size_t)r * RS + c * VEC, kg + e);
-            cp_async16(Vs + (size_t)r * RS + c * VEC, vg + e);
+            cp_async16(Ks + (size_t)r * RS + c * VEC, (const uint4 *)kc + e);
+            cp_async16(Vs + (size_t)r * RS + c * VEC, (const uint4 *)vc + e);
         }
-        for (int e = threadIdx.x; e < NQ * D; e += blockDim.x) {
-            const int pr = e / D, c = e % D, j = pr / G, hl = pr % G;
-            qs[e] = a.q[(((size_t)b * a.w + j) * a.Hq + (size_t)g * G + hl) * D + c];
+        // queries of the w rows, rotated at pos
+        const int pc = pos < a.max_ctx ? pos : 0;
+        const float *cs_row = a.rope_cos + (size_t)pc * half, *sn_row = a.rope_sin + (size_t)pc * half;
+        for (int e = threadIdx.x; e < NQ * half; e += blockDim.x) {
+            const int pr = e / half, c = e % half, j = pr / G, hl = pr % G;
+            const float *x = a.qkv + ((size_t)b * a.w + j) * H * D + (size_t)(g * G + hl) * D;
+            const float cs = cs_row[c], sn = sn_row[c], x0 = x[c], x1 = x[c + half];
+            qs[(size_t)pr * D + c] = x0 * cs - x1 * sn;
+            qs[(size_t)pr * D + c + half] = x1 * cs + x0 * sn;
+        }
+        // this step's rows in the chunk (each slot lies in exactly one chunk):
+        // rotate the key, store key and value in the cache and the stage
+        for (int e = threadIdx.x; e < (nk - nold) * half; e += blockDim.x) {
+            const int r = nold + e / half, c = e % half, j = j0 + r - new0;
+            const float *x = a.qkv + ((size_t)b * a.w + j) * H * D + (size_t)(a.Hq + g) * D;
+            const float cs = cs_row[c], sn = sn_row[c], x0 = x[c], x1 = x[c + half];
+            const float k0 = x0 * cs - x1 * sn, k1 = x1 * cs + x0 * sn;
+            Elem<WT>::store(kc + (size_t)r * D, c, k0);
+            Elem<WT>::store(kc + (size_t)r * D, c + half, k1);
+            Elem<WT>::store(Ks + (size_t)r * RS, c, k0);
+            Elem<WT>::store(Ks + (size_t)r * RS, c + half, k1);
+        }
+        for (int e = threadIdx.x; e < (nk - nold) * D; e += blockDim.x) {
+            const int r = nold + e / D, c = e % D, j = j0 + r - new0;
+            const float v = a.qkv[((size_t)b * a.w + j) * H * D + (size_t)(a.Hq + a.Hkv + g) * D + c];
+            Elem<WT>::store(vc + (size_t)r * D, c, v);
+            Elem<WT>::store(Vs + (size_t)r * RS, c, v);
         }
         cp_async_wait_all();
         __syncthreads();
@@ -351,64 +339,6 @@ __global__ void __launch_bounds__(kTreeAttnThreads) tree_attention_kernel(const 
     if (threadIdx.x == 0) *ctr = 0;
 }
 
-// ------------------------------------------------------------------ log-sum-exp
-
-// Grid (blocks per row, B * R): row t = b * w + j of the LM head's logits.
-__global__ void __launch_bounds__(256) tree_lse_kernel(const TreeArgs a) {
-    __shared__ float s_m[8], s_s[8];
-    __shared__ int s_last;
-    pdl_trigger();
-    pdl_wait();
-    const int blk = blockIdx.x, nblk = gridDim.x;
-    const int b = blockIdx.y / a.R, j = blockIdx.y % a.R, t = b * a.w + j;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const float *z = a.logits + (size_t)t * a.V;
-    const int lo = blk * a.lse_chunk, hi = min(a.V, lo + a.lse_chunk);
-    float m = -INFINITY, s = 0.f;
-    for (int i = lo + tid; i < hi; i += blockDim.x) lse_merge(m, s, z[i], 1.f);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, s, o);
-        lse_merge(m, s, m2, s2);
-    }
-    if (lane == 0) { s_m[warp] = m; s_s[warp] = s; }
-    __syncthreads();
-    if (tid == 0) {
-        for (int q = 1; q < (int)(blockDim.x >> 5); ++q) lse_merge(m, s, s_m[q], s_s[q]);
-        float *part = a.lse_part + ((size_t)t * kSampleMaxBlocks + blk) * 2;
-        part[0] = m;
-        part[1] = s;
-        __threadfence();
-        s_last = atomicAdd(a.lse_ctr + t, 1) == nblk - 1;
-    }
-    __syncthreads();
-    if (!s_last || warp != 0) return;
-    // the last CTA of the row: lane l merges partials l, l + 32, ... (all
-    // loads issued first), then the lanes merge in a fixed butterfly order
-    __threadfence();
-    constexpr int kPer = kSampleMaxBlocks / 32;
-    float pm[kPer], ps[kPer];
-#pragma unroll
-    for (int i = 0; i < kPer; ++i) {
-        const int q = lane + 32 * i;
-        const float *pq = a.lse_part + ((size_t)t * kSampleMaxBlocks + q) * 2;
-        pm[i] = q < nblk ? __ldcg(pq) : -INFINITY;
-        ps[i] = q < nblk ? __ldcg(pq + 1) : 0.f;
-    }
-    float M = -INFINITY, S = 0.f;
-#pragma unroll
-    for (int i = 0; i < kPer; ++i) lse_merge(M, S, pm[i], ps[i]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, M, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, S, o);
-        lse_merge(M, S, m2, s2);
-    }
-    if (lane == 0) {
-        a.lse[t] = M + logf(S);
-        a.lse_ctr[t] = 0;
-    }
-}
-
 // ------------------------------------------------------------------ selection
 
 constexpr int kSelectThreads = 256;
@@ -417,17 +347,23 @@ constexpr int kSelectThreads = 256;
 // token) has pool index base + c and score = frontier score of row j +
 // logit - lse.  Frontier and tree orders: score descending, then pool index
 // ascending (a parent always ranks before its children).
-__global__ void __launch_bounds__(kSelectThreads) tree_select_kernel(const TreeArgs a) {
-    __shared__ float s_fscore[kTreeMaxWidth];
-    __shared__ int s_fpool[kTreeMaxWidth];
-    __shared__ unsigned long long s_fmask[kTreeMaxWidth];
-    __shared__ float s_cs[kTreeMaxWidth * kTreeMaxWidth];
-    __shared__ float s_ps[kTreeMaxPool];
-    __shared__ int s_sel[kTreeMaxPool];
-    __shared__ int s_pos[kTreeMaxPool];
-    pdl_trigger();
-    pdl_wait();
-    const int b = blockIdx.x, tid = threadIdx.x, w = a.w, k = a.step, R = a.R;
+struct SelectSmem {
+    unsigned long long fmask[kTreeMaxWidth];
+    float fscore[kTreeMaxWidth];
+    int fpool[kTreeMaxWidth];
+    float cs[kTreeMaxWidth * kTreeMaxWidth];
+    float ps[kTreeMaxPool];
+    int sel[kTreeMaxPool];
+    int pos[kTreeMaxPool];
+};
+
+// Run by all kSelectThreads threads of one CTA for sequence b, once every row
+// of b has its log-sum-exp (read through L2: other CTAs wrote them).
+__device__ void select_sequence(const TreeArgs &a, int b, SelectSmem &sm) {
+    float *s_fscore = sm.fscore, *s_cs = sm.cs, *s_ps = sm.ps;
+    int *s_fpool = sm.fpool, *s_sel = sm.sel, *s_pos = sm.pos;
+    unsigned long long *s_fmask = sm.fmask;
+    const int tid = threadIdx.x, w = a.w, k = a.step, R = a.R;
     const int base = k == 1 ? 0 : w + (k - 2) * w * w;
     const int nc = R * w;
     if (tid < R) {
@@ -441,7 +377,7 @@ __global__ void __launch_bounds__(kSelectThreads) tree_select_kernel(const TreeA
     if (tid < nc) {
         const int j = tid / w, r = tid % w, t = b * w + j;
         tok = a.top_ids[(size_t)t * w + r];
-        sc = s_fscore[j] + (a.top_vals[(size_t)t * w + r] - a.lse[t]);
+        sc = s_fscore[j] + (a.top_vals[(size_t)t * w + r] - __ldcg(a.lse + t));
         s_cs[tid] = sc;
         const size_t e = (size_t)b * a.P + base + tid;
         a.pool_tok[e] = tok;
@@ -503,6 +439,86 @@ __global__ void __launch_bounds__(kSelectThreads) tree_select_kernel(const TreeA
         a.tree_scores[o] = s_ps[e];
         a.tree_parents[o] = par < 0 ? -1 : s_pos[par];
     }
+}
+
+// ------------------------------------------------------------------ log-sum-exp
+
+// Grid (blocks per row, B * R): row t = b * w + j of the LM head's logits.
+__global__ void __launch_bounds__(256) tree_lse_kernel(const TreeArgs a) {
+    __shared__ float s_m[8], s_s[8];
+    __shared__ int s_last, s_seq;
+    __shared__ SelectSmem sm;
+    pdl_trigger();
+    pdl_wait();
+    const int blk = blockIdx.x, nblk = gridDim.x;
+    const int b = blockIdx.y / a.R, j = blockIdx.y % a.R, t = b * a.w + j;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const float *z = a.logits + (size_t)t * a.V;
+    const int lo = blk * a.lse_chunk, hi = min(a.V, lo + a.lse_chunk);
+    float m = -INFINITY, s = 0.f;
+    constexpr int kBatch = 8;                  // loads in flight per thread before any use
+    for (int i0 = lo + tid; i0 < hi; i0 += kBatch * 256) {
+        float v[kBatch];
+#pragma unroll
+        for (int q = 0; q < kBatch; ++q) {
+            const int i = i0 + q * 256;
+            v[q] = i < hi ? z[i] : -INFINITY;
+        }
+#pragma unroll
+        for (int q = 0; q < kBatch; ++q)
+            if (v[q] != -INFINITY) lse_merge(m, s, v[q], 1.f);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, s, o);
+        lse_merge(m, s, m2, s2);
+    }
+    if (lane == 0) { s_m[warp] = m; s_s[warp] = s; }
+    __syncthreads();
+    if (tid == 0) {
+        for (int q = 1; q < (int)(blockDim.x >> 5); ++q) lse_merge(m, s, s_m[q], s_s[q]);
+        float *part = a.lse_part + ((size_t)t * kSampleMaxBlocks + blk) * 2;
+        part[0] = m;
+        part[1] = s;
+        __threadfence();
+        s_last = atomicAdd(a.lse_ctr + t, 1) == nblk - 1;
+    }
+    __syncthreads();
+    if (!s_last) return;                       // uniform over the CTA
+    // the last CTA of the row: lane l of warp 0 merges partials l, l + 32, ...
+    // (all loads issued first), then the lanes merge in a fixed butterfly order
+    __threadfence();
+    if (warp == 0) {
+    constexpr int kPer = kSampleMaxBlocks / 32;
+    float pm[kPer], ps[kPer];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        const int q = lane + 32 * i;
+        const float *pq = a.lse_part + ((size_t)t * kSampleMaxBlocks + q) * 2;
+        pm[i] = q < nblk ? __ldcg(pq) : -INFINITY;
+        ps[i] = q < nblk ? __ldcg(pq + 1) : 0.f;
+    }
+    float M = -INFINITY, S = 0.f;
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) lse_merge(M, S, pm[i], ps[i]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, M, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, S, o);
+        lse_merge(M, S, m2, s2);
+    }
+    if (lane == 0) {
+        a.lse[t] = M + logf(S);
+        a.lse_ctr[t] = 0;
+        __threadfence();
+        s_seq = atomicAdd(a.seq_ctr + b, 1) == a.R - 1;
+    }
+    }
+    __syncthreads();
+    if (!s_seq) return;                        // uniform over the CTA
+    // the last row of sequence b to finish: candidates, frontier (and the tree)
+    __threadfence();
+    if (threadIdx.x == 0) a.seq_ctr[b] = 0;
+    select_sequence(a, b, sm);
 }
 
 // ------------------------------------------------------------------ acceptance
@@ -572,13 +588,6 @@ cudaError_t launch_tree_gather(const TreeArgs &a, bool bf16, cudaStream_t s, boo
     return launch_k(tree_gather_kernel<float>, grid, dim3(kGatherThreads), 0, s, pdl, a);
 }
 
-cudaError_t launch_tree_rope(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl) {
-    const int warps = a.B * a.w * (a.Hq + 2 * a.Hkv);
-    const dim3 grid((warps + 3) / 4);
-    if (bf16) return launch_k(tree_rope_kernel<uint16_t>, grid, dim3(128), 0, s, pdl, a);
-    return launch_k(tree_rope_kernel<float>, grid, dim3(128), 0, s, pdl, a);
-}
-
 cudaError_t launch_tree_attention(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl) {
     if (bf16) return a.D == 64 ? launch_tree_attn_t<uint16_t, 64>(a, s, pdl) : launch_tree_attn_t<uint16_t, 128>(a, s, pdl);
     return a.D == 64 ? launch_tree_attn_t<float, 64>(a, s, pdl) : launch_tree_attn_t<float, 128>(a, s, pdl);
@@ -588,10 +597,6 @@ cudaError_t launch_tree_lse(const TreeArgs &args, cudaStream_t s, bool pdl) {
     TreeArgs a = args;
     a.lse_blocks = sample_blocks(a.V, &a.lse_chunk);
     return launch_k(tree_lse_kernel, dim3(a.lse_blocks, a.B * a.R), dim3(256), 0, s, pdl, a);
-}
-
-cudaError_t launch_tree_select(const TreeArgs &a, cudaStream_t s, bool pdl) {
-    return launch_k(tree_select_kernel, dim3(a.B), dim3(kSelectThreads), 0, s, pdl, a);
 }
 
 cudaError_t launch_accept_tree(const AcceptTreeArgs &a, cudaStream_t s) {
