@@ -299,7 +299,7 @@ struct AcceptTreeArgs {
     int B, n_nodes, K;
 };
 size_t tree_attention_smem_bytes(bool bf16, int D, int chunk, int G, int w, int splits);
-cudaError_t prepare_tree_kernels(bool bf16, int D, int chunk, int G, int w, int splits);
+cudaError_t prepare_tree_kernels(bool bf16, int D, int chunk, int G, int w, int splits, int max_ctx);
 cudaError_t launch_tree_gather(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl);
 cudaError_t launch_tree_attention(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl);
 cudaError_t launch_tree_lse(const TreeArgs &a, cudaStream_t s, bool pdl);

@@ -554,16 +554,20 @@ __device__ __forceinline__ void write_row(const GemvArgs &a, int t, const Key (&
     }
 }
 
-template <int NB, int RPW, bool TOPK, int PRO>
+// TK: 0 no selection; 1 top-1 through the packed 64-bit atomic maximum; 2 top-k
+// through the register lists (separate instances, so neither carries the
+// other's code).
+template <int NB, int RPW, int TK, int PRO>
 __global__ void __launch_bounds__(kTcThreads, 1)
     gemv_tc_kernel(const GemvArgs a, const TcPlan p, const __grid_constant__ CUtensorMap tmW) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full[kTcMaxStages], empty[kTcMaxStages], acc_full[2], acc_empty[2], mma_done;
     __shared__ uint32_t s_tmem;
     __shared__ float red[kStageThreads / 32];
-    __shared__ float s_val[TOPK ? 4 : 1][TOPK ? NB : 1];   // top-1: each epilogue warp's best per row
-    __shared__ int s_id[TOPK ? 4 : 1][TOPK ? NB : 1];
-    __shared__ float s_tr[TOPK ? 16 : 1][TOPK ? kTrMax : 1];
+    constexpr bool TOPK = TK != 0;
+    __shared__ float s_val[TK == 1 ? 4 : 1][TK == 1 ? NB : 1];   // top-1: each epilogue warp's best per row
+    __shared__ int s_id[TK == 1 ? 4 : 1][TK == 1 ? NB : 1];
+    __shared__ float s_tr[TK == 2 ? 16 : 1][TK == 2 ? kTrMax : 1];
     __shared__ int s_last;
     constexpr uint32_t kCols = RPW == 1 ? 32 : 64;   // two accumulator buffers x RPW x 16 columns
 
@@ -698,14 +702,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int T = a.T;
             // top-1 with the 64-bit atomic maximum: per warp and row the best so
             // far (thr, cached in registers); otherwise the register lists
-            const bool top1 = a.topk == 1 && a.best != nullptr;
+            constexpr bool top1 = TK == 1;
             float thr_v[NB];
             int thr_i[NB];
             Key lst[kTopK];
             if constexpr (TOPK) {
 #pragma unroll
                 for (int t = 0; t < NB; ++t) { thr_v[t] = -INFINITY; thr_i[t] = 0x7FFFFFFF; }
-                if (lane < NB) { s_val[ew][lane] = -INFINITY; s_id[ew][lane] = 0x7FFFFFFF; }
+                if constexpr (TK == 1) {
+                    if (lane < NB) { s_val[ew][lane] = -INFINITY; s_id[ew][lane] = 0x7FFFFFFF; }
+                }
                 key_clear(lst);
                 __syncwarp();
             }
@@ -742,7 +748,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         for (int t = 0; t < NB; ++t)
                             if (t < T) a.logits[((size_t)t * a.K + a.step - 1) * a.vocab + u] = acc[0][t];
                     }
-                    if (top1) {
+                    if constexpr (top1) {
 #pragma unroll
                         for (int t = 0; t < NB; ++t) {
                             if (t >= T) break;
@@ -800,7 +806,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
             }
             if constexpr (TOPK) {
-                if (top1) {
+                if constexpr (top1) {
                     // this CTA's best of each row joins a 64-bit atomic maximum;
                     // the last CTA to finish reads and clears it
                     epi_sync();
@@ -821,7 +827,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 epi_sync();
                 if (s_last) {
                     __threadfence();
-                    if (top1) {
+                    if constexpr (top1) {
                         if (ew == 0 && lane < T) {
                             const Key key = atomicExch(a.best + lane, 0ull);
                             float v;
@@ -1221,16 +1227,19 @@ template <int NB>
 cudaError_t dispatch_tc(const GemvArgs &a, const TcPlan &p, const CUtensorMap &m, int grid, size_t smem,
                         cudaStream_t s, bool pdl) {
     const dim3 g(grid), b(kTcThreads);
-    if (a.epi == kEpiTopK && a.pro == kProNorm)
-        return launch_k(gemv_tc_kernel<NB, 1, true, kProNorm>, g, b, smem, s, pdl, a, p, m);
+    if (a.epi == kEpiTopK && a.pro == kProNorm) {
+        if (a.topk == 1 && a.best != nullptr)
+            return launch_k(gemv_tc_kernel<NB, 1, 1, kProNorm>, g, b, smem, s, pdl, a, p, m);
+        return launch_k(gemv_tc_kernel<NB, 1, 2, kProNorm>, g, b, smem, s, pdl, a, p, m);
+    }
     if (a.epi == kEpiSwiGLU && a.pro == kProNorm)
-        return launch_k(gemv_tc_kernel<NB, 2, false, kProNorm>, g, b, smem, s, pdl, a, p, m);
+        return launch_k(gemv_tc_kernel<NB, 2, 0, kProNorm>, g, b, smem, s, pdl, a, p, m);
     if (a.epi == kEpiStore || a.epi == kEpiResid) {
         switch (a.pro) {
-            case kProFusePrefill: return launch_k(gemv_tc_kernel<NB, 1, false, kProFusePrefill>, g, b, smem, s, pdl, a, p, m);
-            case kProFuseDecode: return launch_k(gemv_tc_kernel<NB, 1, false, kProFuseDecode>, g, b, smem, s, pdl, a, p, m);
-            case kProNorm: return launch_k(gemv_tc_kernel<NB, 1, false, kProNorm>, g, b, smem, s, pdl, a, p, m);
-            case kProCopy: return launch_k(gemv_tc_kernel<NB, 1, false, kProCopy>, g, b, smem, s, pdl, a, p, m);
+            case kProFusePrefill: return launch_k(gemv_tc_kernel<NB, 1, 0, kProFusePrefill>, g, b, smem, s, pdl, a, p, m);
+            case kProFuseDecode: return launch_k(gemv_tc_kernel<NB, 1, 0, kProFuseDecode>, g, b, smem, s, pdl, a, p, m);
+            case kProNorm: return launch_k(gemv_tc_kernel<NB, 1, 0, kProNorm>, g, b, smem, s, pdl, a, p, m);
+            case kProCopy: return launch_k(gemv_tc_kernel<NB, 1, 0, kProCopy>, g, b, smem, s, pdl, a, p, m);
         }
     }
     return cudaErrorInvalidValue;
@@ -1242,12 +1251,13 @@ cudaError_t set_tc_attrs(int bytes) {
 #define PRISM_TC_ATTR(RPW, TK, PRO)                                                                      \
     if (e == cudaSuccess)                                                                                \
         e = cudaFuncSetAttribute(gemv_tc_kernel<NB, RPW, TK, PRO>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    PRISM_TC_ATTR(1, true, kProNorm)
-    PRISM_TC_ATTR(2, false, kProNorm)
-    PRISM_TC_ATTR(1, false, kProFusePrefill)
-    PRISM_TC_ATTR(1, false, kProFuseDecode)
-    PRISM_TC_ATTR(1, false, kProNorm)
-    PRISM_TC_ATTR(1, false, kProCopy)
+    PRISM_TC_ATTR(1, 1, kProNorm)
+    PRISM_TC_ATTR(1, 2, kProNorm)
+    PRISM_TC_ATTR(2, 0, kProNorm)
+    PRISM_TC_ATTR(1, 0, kProFusePrefill)
+    PRISM_TC_ATTR(1, 0, kProFuseDecode)
+    PRISM_TC_ATTR(1, 0, kProNorm)
+    PRISM_TC_ATTR(1, 0, kProCopy)
 #undef PRISM_TC_ATTR
     return e;
 }

@@ -774,7 +774,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
             delete c;
             return fail(nullptr, PRISM_ERR_INVALID_ARG, "max_ctx too large for the tree attention combine");
         }
-        e = prepare_tree_kernels(c->bf16, D, c->attn_chunk, Hq / Hkv, (int)TW, c->attn_splits);
+        e = prepare_tree_kernels(c->bf16, D, c->attn_chunk, Hq / Hkv, (int)TW, c->attn_splits, f.max_ctx);
     }
     if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking);
     if (e != cudaSuccess) {

@@ -139,12 +139,143 @@ __device__ __forceinline__ void load_run(const WT *p, float (&out)[DPL]) {
     }
 }
 
+// Stage keys [j0, j0 + nk) of KV head g of sequence b and the queries of its
+// G heads in all w rows.  Rows written before this step come from the cache
+// (cp.async); this step's rows (slots new0 + j) are rotated at the node's
+// depth and written to the cache and the stage; queries are rotated,
+// multiplied by q_scale and stored QS floats apart.  Callers wait for the
+// copies and synchronise.
+template <typename WT, int D, int RS, int QS>
+__device__ __forceinline__ void tree_stage(const TreeArgs &a, int b, int g, int j0, int nk, int base, WT *Ks,
+                                           WT *Vs, float *qs, float q_scale) {
+    constexpr int VEC = Elem<WT>::kPerVec;
+    const int G = a.Hq / a.Hkv, NQ = a.w * G;
+    const int new0 = base + (a.step - 2) * a.w;
+    const int pos = base + a.step - 2;
+    const int H = a.Hq + 2 * a.Hkv, half = D / 2;
+    const int nold = new0 - j0 < 0 ? 0 : (new0 - j0 < nk ? new0 - j0 : nk);
+    WT *kc = (WT *)a.k_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D;
+    WT *vc = (WT *)a.v_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D;
+    constexpr int VPR = D / VEC;
+    for (int e = threadIdx.x; e < nold * VPR; e += blockDim.x) {
+        const int r = e / VPR, c = e % VPR;
+        cp_async16(Ks + (size_t)r * RS + c * VEC, (const uint4 *)kc + e);
+        cp_async16(Vs + (size_t)r * RS + c * VEC, (const uint4 *)vc + e);
+    }
+    const int pc = pos < a.max_ctx ? pos : 0;
+    const float *cs_row = a.rope_cos + (size_t)pc * half, *sn_row = a.rope_sin + (size_t)pc * half;
+    for (int e = threadIdx.x; e < NQ * half; e += blockDim.x) {
+        const int pr = e / half, c = e % half, j = pr / G, hl = pr % G;
+        const float *x = a.qkv + ((size_t)b * a.w + j) * H * D + (size_t)(g * G + hl) * D;
+        const float cs = cs_row[c], sn = sn_row[c], x0 = x[c], x1 = x[c + half];
+        qs[(size_t)pr * QS + c] = (x0 * cs - x1 * sn) * q_scale;
+        qs[(size_t)pr * QS + c + half] = (x1 * cs + x0 * sn) * q_scale;
+    }
+    // this step's rows in the chunk (each slot lies in exactly one chunk)
+    for (int e = threadIdx.x; e < (nk - nold) * half; e += blockDim.x) {
+        const int r = nold + e / half, c = e % half, j = j0 + r - new0;
+        const float *x = a.qkv + ((size_t)b * a.w + j) * H * D + (size_t)(a.Hq + g) * D;
+        const float cs = cs_row[c], sn = sn_row[c], x0 = x[c], x1 = x[c + half];
+        const float k0 = x0 * cs - x1 * sn, k1 = x1 * cs + x0 * sn;
+        Elem<WT>::store(kc + (size_t)r * D, c, k0);
+        Elem<WT>::store(kc + (size_t)r * D, c + half, k1);
+        Elem<WT>::store(Ks + (size_t)r * RS, c, k0);
+        Elem<WT>::store(Ks + (size_t)r * RS, c + half, k1);
+    }
+    for (int e = threadIdx.x; e < (nk - nold) * D; e += blockDim.x) {
+        const int r = nold + e / D, c = e % D, j = j0 + r - new0;
+        const float v = a.qkv[((size_t)b * a.w + j) * H * D + (size_t)(a.Hq + a.Hkv + g) * D + c];
+        Elem<WT>::store(vc + (size_t)r * D, c, v);
+        Elem<WT>::store(Vs + (size_t)r * RS, c, v);
+    }
+}
+
+// The last CTA of (b, g) to finish merges every pair's split partials in
+// split order (log-sum-exp rule, eight splits' loads in flight at a time) and
+// writes the rounded attention output.  ws: [NQ][splits] shared floats.
+template <typename WT, int D>
+__device__ __forceinline__ void tree_merge_splits(const TreeArgs &a, int b, int g, float *ws, int *s_last) {
+    constexpr int DPL = D / 32;
+    constexpr int PS = D + 4;
+    const int G = a.Hq / a.Hkv, NQ = a.w * G;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
+    __threadfence();
+    __syncthreads();
+    int *ctr = a.attn_ctr + (size_t)b * a.Hkv + g;
+    if (threadIdx.x == 0) *s_last = (atomicAdd(ctr, 1) == a.splits - 1);
+    __syncthreads();
+    if (!*s_last) return;
+    __threadfence();
+    for (int pr = warp; pr < NQ; pr += nwarp) {
+        const int j = pr / G, hl = pr % G, t = b * a.w + j, h = g * G + hl;
+        const float *part = a.attn_part + ((size_t)t * a.Hq + h) * a.splits * PS;
+        float *wh = ws + (size_t)pr * a.splits;
+        constexpr int kMaxPerLane = 8;           // splits <= 256
+        float mv[kMaxPerLane], lv[kMaxPerLane];
+#pragma unroll
+        for (int k = 0; k < kMaxPerLane; ++k) {
+            const int sp = lane + 32 * k;
+            const bool in = sp < a.splits;
+            mv[k] = in ? __ldcg(part + (size_t)sp * PS + D) : -INFINITY;
+            lv[k] = in ? __ldcg(part + (size_t)sp * PS + D + 1) : 0.f;
+        }
+        float M = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < kMaxPerLane; ++k) M = fmaxf(M, mv[k]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xFFFFFFFFu, M, o));
+        float den = 0.f;
+#pragma unroll
+        for (int k = 0; k < kMaxPerLane; ++k) {
+            const int sp = lane + 32 * k;
+            const float wgt = lv[k] > 0.f ? expf(mv[k] - M) : 0.f;
+            if (sp < a.splits) wh[sp] = wgt;
+            den = fmaf(wgt, lv[k], den);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) den += __shfl_xor_sync(0xFFFFFFFFu, den, o);
+        __syncwarp();
+        float acc[DPL];
+#pragma unroll
+        for (int u = 0; u < DPL; ++u) acc[u] = 0.f;
+        // a split with no visible key has weight 0 and zero sums
+        constexpr int kBatch = 8;
+        for (int sp0 = 0; sp0 < a.splits; sp0 += kBatch) {
+            float v[kBatch][DPL], wv[kBatch];
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i) {
+                const int sp = sp0 + i;
+                const bool in = sp < a.splits;
+                wv[i] = in ? wh[sp] : 0.f;
+                const float *src = part + (size_t)(in ? sp : 0) * PS + lane * DPL;
+#pragma unroll
+                for (int u = 0; u < DPL; ++u) v[i][u] = in ? __ldcg(src + u) : 0.f;
+            }
+#pragma unroll
+            for (int i = 0; i < kBatch; ++i)
+#pragma unroll
+                for (int u = 0; u < DPL; ++u) acc[u] = fmaf(wv[i], v[i][u], acc[u]);
+        }
+        WT *o = (WT *)a.o_out + ((size_t)t * a.Hq + h) * D;
+        const float inv = den > 0.f ? 1.0f / den : 0.f;
+#pragma unroll
+        for (int u = 0; u < DPL; ++u) Elem<WT>::store(o, lane * DPL + u, acc[u] * inv);
+    }
+    if (threadIdx.x == 0) *ctr = 0;
+}
+
+// Key slot p of sequence b is visible to a row with ancestor mask msk when it
+// is committed or a step-1 row (p < base) or its draft-slot bit is set.
+__device__ __forceinline__ bool tree_visible(int p, int base, unsigned long long msk) {
+    const int off = p - base;
+    return off < 0 || (off < kTreeMaskBits && ((msk >> off) & 1ull));
+}
+
 constexpr int kTreeAttnThreads = 512;   // 16 warps: one (row, query head) pair each when w * G = 16
 
-// Grid (splits, Hkv, B); CTA (s, g, b) stages keys [s C, s C + C) of KV head g
-// once and scores them against the G query heads of g in each of the w rows
-// of sequence b.  Key slot p is visible to row j when p < L + n (committed and
-// step-1 rows) or bit p - (L + n) of the row's ancestor mask is set.
+// CUDA-core kernel (fp32 caches, or more than 16 row-head pairs).  Grid
+// (splits, Hkv, B); CTA (s, g, b) stages keys [s C, s C + C) of KV head g once
+// and each warp scores them against one (row, query head) pair at a time.
 template <typename WT, int D>
 __global__ void __launch_bounds__(kTreeAttnThreads) tree_attention_kernel(const TreeArgs a) {
     extern __shared__ __align__(16) uint8_t smem_raw[];
@@ -172,54 +303,13 @@ __global__ void __launch_bounds__(kTreeAttnThreads) tree_attention_kernel(const 
     const int j0 = s * C;
     const int nk = PE - j0 < C ? PE - j0 : C;
     const float scale = 1.0f / sqrtf((float)D);
-    // this step's rows: slots new0 + j (j < w), rotary position pos (the depth)
-    const int new0 = base + (a.step - 2) * a.w;
-    const int pos = base + a.step - 2;
-    const int H = a.Hq + 2 * a.Hkv, half = D / 2;
-    if (s == 0 && g == 0 && threadIdx.x == 0 && (L < 0 || new0 + a.w > a.max_ctx)) set_err(a.err, kErrCache);
+    if (s == 0 && g == 0 && threadIdx.x == 0 && (L < 0 || base + (a.step - 1) * a.w > a.max_ctx))
+        set_err(a.err, kErrCache);
 
     if (nk > 0 && L >= 0) {
-        // rows written before this step: from the cache
-        const int nold = new0 - j0 < 0 ? 0 : (new0 - j0 < nk ? new0 - j0 : nk);
-        WT *kc = (WT *)a.k_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D;
-        WT *vc = (WT *)a.v_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D;
-        constexpr int VPR = D / VEC;
-        for (int e = threadIdx.x; e < nold * VPR; e += blockDim.x) {
-            const int r = e / VPR, c = e % VPR;
-            cp_async16(Ks + (size_t)r * RS + c * VEC, (const uint4 *)kc + e);
-            cp_async16(Vs + (size_t)r * RS + c * VEC, (const uint4 *)vc + e);
-        }
-        // queries of the w rows, rotated at pos
-        const int pc = pos < a.max_ctx ? pos : 0;
-        const float *cs_row = a.rope_cos + (size_t)pc * half, *sn_row = a.rope_sin + (size_t)pc * half;
-        for (int e = threadIdx.x; e < NQ * half; e += blockDim.x) {
-            const int pr = e / half, c = e % half, j = pr / G, hl = pr % G;
-            const float *x = a.qkv + ((size_t)b * a.w + j) * H * D + (size_t)(g * G + hl) * D;
-            const float cs = cs_row[c], sn = sn_row[c], x0 = x[c], x1 = x[c + half];
-            qs[(size_t)pr * D + c] = x0 * cs - x1 * sn;
-            qs[(size_t)pr * D + c + half] = x1 * cs + x0 * sn;
-        }
-        // this step's rows in the chunk (each slot lies in exactly one chunk):
-        // rotate the key, store key and value in the cache and the stage
-        for (int e = threadIdx.x; e < (nk - nold) * half; e += blockDim.x) {
-            const int r = nold + e / half, c = e % half, j = j0 + r - new0;
-            const float *x = a.qkv + ((size_t)b * a.w + j) * H * D + (size_t)(a.Hq + g) * D;
-            const float cs = cs_row[c], sn = sn_row[c], x0 = x[c], x1 = x[c + half];
-            const float k0 = x0 * cs - x1 * sn, k1 = x1 * cs + x0 * sn;
-            Elem<WT>::store(kc + (size_t)r * D, c, k0);
-            Elem<WT>::store(kc + (size_t)r * D, c + half, k1);
-            Elem<WT>::store(Ks + (size_t)r * RS, c, k0);
-            Elem<WT>::store(Ks + (size_t)r * RS, c + half, k1);
-        }
-        for (int e = threadIdx.x; e < (nk - nold) * D; e += blockDim.x) {
-            const int r = nold + e / D, c = e % D, j = j0 + r - new0;
-            const float v = a.qkv[((size_t)b * a.w + j) * H * D + (size_t)(a.Hq + a.Hkv + g) * D + c];
-            Elem<WT>::store(vc + (size_t)r * D, c, v);
-            Elem<WT>::store(Vs + (size_t)r * RS, c, v);
-        }
+        tree_stage<WT, D, RS, D>(a, b, g, j0, nk, base, Ks, Vs, qs, 1.0f);
         cp_async_wait_all();
         __syncthreads();
-
         for (int pr = warp; pr < NQ; pr += nwarp) {
             const int j = pr / G, hl = pr % G, t = b * a.w + j;
             const unsigned long long msk = a.front_mask[t];
@@ -227,11 +317,8 @@ __global__ void __launch_bounds__(kTreeAttnThreads) tree_attention_kernel(const 
             float *pp = ps + (size_t)pr * C;
             float mloc = -INFINITY;
             for (int jj = lane; jj < nk; jj += 32) {
-                const int p = j0 + jj;
-                const int off = p - base;
-                const bool vis = off < 0 || (off < kTreeMaskBits && ((msk >> off) & 1ull));
                 float sc = -INFINITY;
-                if (vis) sc = dot_row<WT, D>(q, Ks + (size_t)jj * RS) * scale;
+                if (tree_visible(j0 + jj, base, msk)) sc = dot_row<WT, D>(q, Ks + (size_t)jj * RS) * scale;
                 pp[jj] = sc;
                 mloc = fmaxf(mloc, sc);
             }
@@ -271,72 +358,226 @@ __global__ void __launch_bounds__(kTreeAttnThreads) tree_attention_kernel(const 
             if (lane == 0) { part[D] = -INFINITY; part[D + 1] = 0.f; }
         }
     }
+    tree_merge_splits<WT, D>(a, b, g, ws, &s_last);
+}
 
-    // last CTA of (b, g): log-sum-exp merge of the splits in split order
-    __threadfence();
-    __syncthreads();
-    int *ctr = a.attn_ctr + (size_t)b * a.Hkv + g;
-    if (threadIdx.x == 0) s_last = (atomicAdd(ctr, 1) == a.splits - 1);
-    __syncthreads();
-    if (!s_last) return;
-    __threadfence();
-    for (int pr = warp; pr < NQ; pr += nwarp) {
-        const int j = pr / G, hl = pr % G, t = b * a.w + j, h = g * G + hl;
-        const float *part = a.attn_part + ((size_t)t * a.Hq + h) * a.splits * PS;
-        float *wh = ws + (size_t)pr * a.splits;
-        constexpr int kMaxPerLane = 8;           // splits <= 256
-        float mv[kMaxPerLane], lv[kMaxPerLane];
-#pragma unroll
-        for (int k = 0; k < kMaxPerLane; ++k) {
-            const int sp = lane + 32 * k;
-            const bool in = sp < a.splits;
-            mv[k] = in ? __ldcg(part + (size_t)sp * PS + D) : -INFINITY;
-            lv[k] = in ? __ldcg(part + (size_t)sp * PS + D + 1) : 0.f;
+// ------------------------------------------------------------------ attention on tensor cores
+
+// bf16 caches with at most 16 row-head pairs (w * G <= 16).  CTA (s, g, b)
+// stages kTcChunk keys as above; compute warp w takes keys 16w .. 16w + 15 in
+// the M dimension of mma.sync.m16n8k16 with the pairs in N (one or two n8
+// tiles).  S^T = K q^T with each query (rotated, times 1/sqrt(D)) split into a
+// bf16 hi + lo pair (two MMAs: operand error near 2^-17, K exact); the warp's
+// softmax per pair over its 16 keys; P^T from the S^T tile by movmatrix (the
+// accumulator layout of S^T is the B-fragment layout of P^T, transposed), also
+// split hi + lo; O^T += V^T P^T with V^T read by a transposing ldmatrix.  The
+// warps' (max, sum, O) merge in shared memory into the CTA's split partial;
+// the splits then merge as in the CUDA-core kernel.
+constexpr int kTcWarps = 8;
+constexpr int kTcChunk = kTcWarps * 16;
+constexpr int kTcMaxPairs = 16;
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t (&r)[4]) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(addr));
+}
+__device__ __forceinline__ uint32_t movm_t(uint32_t x) {
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
+}
+__device__ __forceinline__ void mma16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+                 "{%8, %9}, {%0, %1, %2, %3};"
+                 : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// bf16 hi / lo parts of two floats, packed (low half = first element).
+__device__ __forceinline__ void split2(float x, float y, uint32_t &hi, uint32_t &lo) {
+    const uint16_t hx = f32_to_bf16(x), hy = f32_to_bf16(y);
+    hi = (uint32_t)hx | ((uint32_t)hy << 16);
+    lo = (uint32_t)f32_to_bf16(x - bf16_to_f32(hx)) | ((uint32_t)f32_to_bf16(y - bf16_to_f32(hy)) << 16);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kTcWarps * 32) tree_attention_tc_kernel(const TreeArgs a) {
+    constexpr int RS = D + 8;                 // bf16 row stride: 16-byte rows, conflict-free ldmatrix
+    constexpr int NT = D / 16;                // 16-dim tiles
+    constexpr int PS = D + 4;
+    constexpr int QS = D + 8;                 // query row stride: at most 2-way bank conflicts in the B loads
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    __shared__ int s_last;
+    __shared__ unsigned long long s_mask[kTreeMaxWidth];
+    uint16_t *Ks = (uint16_t *)smem_raw;
+    uint16_t *Vs = Ks + (size_t)kTcChunk * RS;
+    float *qs = (float *)(Vs + (size_t)kTcChunk * RS);  // [16][QS] scaled queries, pairs >= NQ zero
+    float *wm = qs + kTcMaxPairs * QS;                  // [warp][16]
+    float *wl = wm + kTcWarps * kTcMaxPairs;            // [warp][16]
+    float *ws = wl + kTcWarps * kTcMaxPairs;            // [16][splits]
+    float *wo = (float *)smem_raw;                      // [warp][16][D], after the keys are consumed
+    const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int G = a.Hq / a.Hkv, NQ = a.w * G;
+
+    pdl_trigger();
+    pdl_wait();
+
+    const int n = tree_n(a, b), L = a.kv_len[b];
+    const int base = L + n;
+    int PE = base + (a.step - 1) * a.w;
+    if (PE > a.max_ctx) PE = a.max_ctx;
+    const int j0 = s * kTcChunk;
+    int nk = PE - j0 < kTcChunk ? PE - j0 : kTcChunk;
+    if (L < 0) nk = 0;
+    if (s == 0 && g == 0 && tid == 0 && (L < 0 || base + (a.step - 1) * a.w > a.max_ctx)) set_err(a.err, kErrCache);
+    if (tid < a.w) s_mask[tid] = a.front_mask[b * a.w + tid];
+    for (int e = tid; e < (kTcMaxPairs - NQ) * QS; e += blockDim.x) qs[NQ * QS + e] = 0.f;
+    if (nk > 0) {
+        tree_stage<uint16_t, D, RS, QS>(a, b, g, j0, nk, base, Ks, Vs, qs, 1.0f / sqrtf((float)D));
+        // rows past the chunk's keys: zero (their probabilities are 0, and 0 * NaN would not be)
+        for (int e = tid; e < (kTcChunk - nk) * (D / 8); e += blockDim.x) {
+            const int r = nk + e / (D / 8), c = e % (D / 8);
+            *(uint4 *)(Ks + (size_t)r * RS + c * 8) = make_uint4(0, 0, 0, 0);
+            *(uint4 *)(Vs + (size_t)r * RS + c * 8) = make_uint4(0, 0, 0, 0);
         }
+    }
+    cp_async_wait_all();
+    __syncthreads();
+
+    // warp state: pairs nt * 8 + 2 (lane % 4) + {0, 1}; O^T dims 16 t + lane / 4 (+ 8)
+    const int kr = 16 * warp;
+    const int cnt = nk - kr;                  // keys of this warp (may be <= 0)
+    const int ntn = (NQ + 7) / 8;
+    float mx[2][2], sm[2][2], o[2][NT][4];
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt) {
+        mx[nt][0] = mx[nt][1] = -INFINITY;
+        sm[nt][0] = sm[nt][1] = 0.f;
+#pragma unroll
+        for (int t = 0; t < NT; ++t) o[nt][t][0] = o[nt][t][1] = o[nt][t][2] = o[nt][t][3] = 0.f;
+    }
+    if (cnt > 0) {
+        const uint32_t kb = (uint32_t)__cvta_generic_to_shared(Ks), vb = (uint32_t)__cvta_generic_to_shared(Vs);
+        const int mi = lane >> 3;
+        float sh[2][4], sl[2][4];
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) sh[nt][q] = sl[nt][q] = 0.f;
+#pragma unroll
+        for (int ks = 0; ks < NT; ++ks) {
+            uint32_t ka[4];
+            ldsm_x4(kb + (uint32_t)(((kr + (mi & 1) * 8 + (lane & 7)) * RS + 16 * ks + (mi >> 1) * 8) * 2), ka);
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                if (nt >= ntn) break;
+                uint32_t qh[2], ql[2];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const float *src = qs + (nt * 8 + (lane >> 2)) * QS + 16 * ks + 2 * (lane & 3) + 8 * u;
+                    split2(src[0], src[1], qh[u], ql[u]);
+                }
+                mma16816(sh[nt], ka, qh[0], qh[1]);
+                mma16816(sl[nt], ka, ql[0], ql[1]);
+            }
+        }
+        uint32_t pbh[2][2], pbl[2][2];
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt) {
+            float sv[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int key = (lane >> 2) + (q >> 1) * 8, pr = nt * 8 + 2 * (lane & 3) + (q & 1);
+                const bool vis = key < cnt && pr < NQ && tree_visible(j0 + kr + key, base, s_mask[pr / G]);
+                sv[q] = vis ? sh[nt][q] + sl[nt][q] : -INFINITY;
+            }
+            // softmax per pair over the warp's 16 keys: lanes with equal lane % 4 share pairs
+            float c0 = fmaxf(sv[0], sv[2]), c1 = fmaxf(sv[1], sv[3]);
+#pragma unroll
+            for (int off = 4; off < 32; off <<= 1) {
+                c0 = fmaxf(c0, __shfl_xor_sync(0xFFFFFFFFu, c0, off));
+                c1 = fmaxf(c1, __shfl_xor_sync(0xFFFFFFFFu, c1, off));
+            }
+            mx[nt][0] = c0;
+            mx[nt][1] = c1;
+            float p[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float mq = (q & 1) ? c1 : c0;
+                p[q] = sv[q] == -INFINITY ? 0.f : expf(sv[q] - mq);
+            }
+            sm[nt][0] = p[0] + p[2];
+            sm[nt][1] = p[1] + p[3];
+            uint32_t h01, l01, h23, l23;
+            split2(p[0], p[1], h01, l01);
+            split2(p[2], p[3], h23, l23);
+            pbh[nt][0] = movm_t(h01);
+            pbh[nt][1] = movm_t(h23);
+            pbl[nt][0] = movm_t(l01);
+            pbl[nt][1] = movm_t(l23);
+        }
+#pragma unroll
+        for (int t = 0; t < NT; ++t) {
+            uint32_t va[4];
+            ldsm_x4_t(vb + (uint32_t)(((kr + (mi >> 1) * 8 + (lane & 7)) * RS + 16 * t + (mi & 1) * 8) * 2), va);
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                if (nt >= ntn) break;
+                mma16816(o[nt][t], va, pbh[nt][0], pbh[nt][1]);
+                mma16816(o[nt][t], va, pbl[nt][0], pbl[nt][1]);
+            }
+        }
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+            for (int off = 4; off < 32; off <<= 1) {
+                sm[nt][0] += __shfl_xor_sync(0xFFFFFFFFu, sm[nt][0], off);
+                sm[nt][1] += __shfl_xor_sync(0xFFFFFFFFu, sm[nt][1], off);
+            }
+    }
+    __syncthreads();                          // every warp is done with K and V: wo may overwrite them
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt) {
+        const int p0 = nt * 8 + 2 * (lane & 3);
+        if (lane < 4) {
+            wm[warp * kTcMaxPairs + p0] = mx[nt][0];
+            wm[warp * kTcMaxPairs + p0 + 1] = mx[nt][1];
+            wl[warp * kTcMaxPairs + p0] = sm[nt][0];
+            wl[warp * kTcMaxPairs + p0 + 1] = sm[nt][1];
+        }
+#pragma unroll
+        for (int t = 0; t < NT; ++t)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int d = 16 * t + (lane >> 2) + (q >> 1) * 8, pr = p0 + (q & 1);
+                wo[((size_t)warp * kTcMaxPairs + pr) * D + d] = o[nt][t][q];
+            }
+    }
+    __syncthreads();
+    // the CTA's partial of each pair: warps merged in warp order
+    for (int e = tid; e < NQ * D; e += blockDim.x) {
+        const int pr = e / D, d = e % D;
         float M = -INFINITY;
 #pragma unroll
-        for (int k = 0; k < kMaxPerLane; ++k) M = fmaxf(M, mv[k]);
+        for (int w = 0; w < kTcWarps; ++w) M = fmaxf(M, wm[w * kTcMaxPairs + pr]);
+        float acc = 0.f, den = 0.f;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xFFFFFFFFu, M, o));
-        float den = 0.f;
-#pragma unroll
-        for (int k = 0; k < kMaxPerLane; ++k) {
-            const int sp = lane + 32 * k;
-            const float wgt = lv[k] > 0.f ? expf(mv[k] - M) : 0.f;
-            if (sp < a.splits) wh[sp] = wgt;
-            den = fmaf(wgt, lv[k], den);
+        for (int w = 0; w < kTcWarps; ++w) {
+            const float lw = wl[w * kTcMaxPairs + pr];
+            const float wt = lw > 0.f ? expf(wm[w * kTcMaxPairs + pr] - M) : 0.f;
+            acc = fmaf(wt, wo[((size_t)w * kTcMaxPairs + pr) * D + d], acc);
+            den = fmaf(wt, lw, den);
         }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) den += __shfl_xor_sync(0xFFFFFFFFu, den, o);
-        __syncwarp();
-        float acc[DPL];
-#pragma unroll
-        for (int u = 0; u < DPL; ++u) acc[u] = 0.f;
-        // weighted sum in split order, eight splits' loads in flight at a time
-        // (a split with no visible key has weight 0 and zero sums)
-        constexpr int kBatch = 8;
-        for (int sp0 = 0; sp0 < a.splits; sp0 += kBatch) {
-            float v[kBatch][DPL], wv[kBatch];
-#pragma unroll
-            for (int i = 0; i < kBatch; ++i) {
-                const int sp = sp0 + i;
-                const bool in = sp < a.splits;
-                wv[i] = in ? wh[sp] : 0.f;
-                const float *src = part + (size_t)(in ? sp : 0) * PS + lane * DPL;
-#pragma unroll
-                for (int u = 0; u < DPL; ++u) v[i][u] = in ? __ldcg(src + u) : 0.f;
-            }
-#pragma unroll
-            for (int i = 0; i < kBatch; ++i)
-#pragma unroll
-                for (int u = 0; u < DPL; ++u) acc[u] = fmaf(wv[i], v[i][u], acc[u]);
-        }
-        WT *o = (WT *)a.o_out + ((size_t)t * a.Hq + h) * D;
-        const float inv = den > 0.f ? 1.0f / den : 0.f;
-#pragma unroll
-        for (int u = 0; u < DPL; ++u) Elem<WT>::store(o, lane * DPL + u, acc[u] * inv);
+        const int j = pr / G, hl = pr % G, t = b * a.w + j;
+        float *part = a.attn_part + (((size_t)t * a.Hq + (size_t)g * G + hl) * a.splits + s) * PS;
+        part[d] = acc;
+        if (d == 0) { part[D] = M; part[D + 1] = den; }
     }
-    if (threadIdx.x == 0) *ctr = 0;
+    tree_merge_splits<uint16_t, D>(a, b, g, ws, &s_last);
 }
 
 // ------------------------------------------------------------------ selection
@@ -555,15 +796,36 @@ size_t tree_attn_smem(int chunk, int G, int w, int splits) {
     return 2 * (size_t)chunk * RS * sizeof(WT) + ((size_t)NQ * D + (size_t)NQ * chunk + (size_t)NQ * splits) * 4;
 }
 
+template <int D>
+size_t tree_attn_tc_smem(int splits) {
+    return 2 * (size_t)kTcChunk * (D + 8) * 2 + ((size_t)kTcMaxPairs * (D + 8) + 2 * kTcWarps * kTcMaxPairs +
+                                                 (size_t)kTcMaxPairs * splits) * 4;
+}
+
+// the tensor-core kernel's split count (kTcChunk keys per CTA)
+int tc_splits(int max_ctx) { return (max_ctx + kTcChunk - 1) / kTcChunk; }
+
 template <typename WT, int D>
-cudaError_t launch_tree_attn_t(const TreeArgs &a, cudaStream_t s, bool pdl) {
-    const size_t smem = tree_attn_smem<WT, D>(a.chunk, a.Hq / a.Hkv, a.w, a.splits);
-    return launch_k(tree_attention_kernel<WT, D>, dim3(a.splits, a.Hkv, a.B), dim3(kTreeAttnThreads), smem, s, pdl,
-                    a);
+cudaError_t launch_tree_attn_t(const TreeArgs &args, cudaStream_t s, bool pdl) {
+    if (sizeof(WT) == 2 && args.w * (args.Hq / args.Hkv) <= kTcMaxPairs && tc_splits(args.max_ctx) <= 256) {
+        TreeArgs a = args;
+        a.chunk = kTcChunk;
+        a.splits = tc_splits(a.max_ctx);
+        return launch_k(tree_attention_tc_kernel<D>, dim3(a.splits, a.Hkv, a.B), dim3(kTcWarps * 32),
+                        tree_attn_tc_smem<D>(a.splits), s, pdl, a);
+    }
+    const size_t smem = tree_attn_smem<WT, D>(args.chunk, args.Hq / args.Hkv, args.w, args.splits);
+    return launch_k(tree_attention_kernel<WT, D>, dim3(args.splits, args.Hkv, args.B), dim3(kTreeAttnThreads), smem,
+                    s, pdl, args);
 }
 
 template <typename WT, int D>
-cudaError_t prepare_tree_attn_t(int chunk, int G, int w, int splits) {
+cudaError_t prepare_tree_attn_t(int chunk, int G, int w, int splits, int max_ctx) {
+    if (sizeof(WT) == 2 && tc_splits(max_ctx) <= 256) {
+        cudaError_t e = cudaFuncSetAttribute(tree_attention_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)tree_attn_tc_smem<D>(tc_splits(max_ctx)));
+        if (e != cudaSuccess) return e;
+    }
     const size_t smem = tree_attn_smem<WT, D>(chunk, G, w, splits);
     return cudaFuncSetAttribute(tree_attention_kernel<WT, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 }
@@ -575,10 +837,11 @@ size_t tree_attention_smem_bytes(bool bf16, int D, int chunk, int G, int w, int 
     return D == 64 ? tree_attn_smem<float, 64>(chunk, G, w, splits) : tree_attn_smem<float, 128>(chunk, G, w, splits);
 }
 
-cudaError_t prepare_tree_kernels(bool bf16, int D, int chunk, int G, int w, int splits) {
-    if (bf16) return D == 64 ? prepare_tree_attn_t<uint16_t, 64>(chunk, G, w, splits)
-                             : prepare_tree_attn_t<uint16_t, 128>(chunk, G, w, splits);
-    return D == 64 ? prepare_tree_attn_t<float, 64>(chunk, G, w, splits) : prepare_tree_attn_t<float, 128>(chunk, G, w, splits);
+cudaError_t prepare_tree_kernels(bool bf16, int D, int chunk, int G, int w, int splits, int max_ctx) {
+    if (bf16) return D == 64 ? prepare_tree_attn_t<uint16_t, 64>(chunk, G, w, splits, max_ctx)
+                             : prepare_tree_attn_t<uint16_t, 128>(chunk, G, w, splits, max_ctx);
+    return D == 64 ? prepare_tree_attn_t<float, 64>(chunk, G, w, splits, max_ctx)
+                   : prepare_tree_attn_t<float, 128>(chunk, G, w, splits, max_ctx);
 }
 
 cudaError_t launch_tree_gather(const TreeArgs &a, bool bf16, cudaStream_t s, bool pdl) {
