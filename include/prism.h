@@ -157,6 +157,32 @@ prism_status prism_accept_greedy(prism_ctx *ctx, int32_t batch, const int32_t *d
                                  const int32_t *target, const int32_t *n_new, int32_t *kv_len,
                                  int32_t *accept_len, int32_t *out_tokens, void *stream);
 
+/* Steady-state draft loop: `rounds` greedy rounds back to back on the device,
+ * each one prism_draft_round followed by prism_accept_greedy, where the
+ * acceptance also writes the next round's input: the a accepted drafts and
+ * the target's token at position a go to tokens[b, 0..a] and n_new[b] =
+ * a + 1, and kv_len[b] += n_new[b] commits the rows the round prefilled
+ * (Sec. 2 and Sec. 3.2: the next round re-fuses the accepted tokens with the
+ * target's hidden states of its verification pass).  Nothing returns to the
+ * host between rounds; the whole loop is one CUDA graph (cached per argument
+ * set, like a round).
+ *   tokens     int32 [batch, max_new] in/out (round 0's tokens; afterwards
+ *              the next round's); max_new >= K + 1 is required
+ *   hidden     wtype [rounds, batch, max_new, d]: the target hidden states
+ *              paired with each round's tokens (row i of round r pairs with
+ *              token i of that round)
+ *   n_new      int32 [batch] in/out; kv_len int32 [batch] in/out
+ *   k_cache, v_cache as prism_draft_round
+ *   target     int32 [rounds, batch, K + 1]: the target's tokens per round
+ *   draft_ids  int32 [rounds, batch, K] out; accept_len int32 [rounds, batch]
+ *   out; out_tokens int32 [rounds, batch, K + 1] out (as prism_accept_greedy)
+ * Errors: INVALID_ARG, SHAPE (rounds < 1), CAPACITY (batch > max_batch, or
+ * max_new < K + 1), NOT_LOADED, CUDA. */
+prism_status prism_draft_loop(prism_ctx *ctx, int32_t batch, int32_t rounds, int32_t *tokens, const void *hidden,
+                              int32_t *n_new, int32_t *kv_len, void *k_cache, void *v_cache,
+                              const int32_t *target, int32_t *draft_ids, int32_t *accept_len,
+                              int32_t *out_tokens, void *stream);
+
 /* Random numbers of the sampled calls below: the n-th output x of SplitMix64
  * (Steele, Lea and Flood, OOPSLA 2014) started from state *seed, with
  * n = (stream << 60) | (b << 40) | (k << 32) | i, taken as

@@ -78,6 +78,7 @@ def library() -> ctypes.CDLL:
         lib.prism_accept_sampled.argtypes = [vp, i32, vp, vp, vp, flt] + [vp] * 7
         lib.prism_draft_tree.argtypes = [vp, i32] + [vp] * 6 + [i32, i32, P(_TreeOutputs), vp]
         lib.prism_accept_tree.argtypes = [vp, i32, i32] + [vp] * 9
+        lib.prism_draft_loop.argtypes = [vp, i32, i32] + [vp] * 11
         lib.prism_profile_tree.argtypes = [vp, i32] + [vp] * 6 + [i32, i32, P(_TreeOutputs), vp,
                                                                 P(ctypes.c_float), P(i32), i32, P(i32)]
         lib.prism_get_error.restype = ctypes.c_char_p
@@ -86,7 +87,7 @@ def library() -> ctypes.CDLL:
                   "prism_draft_round", "prism_accept_greedy", "prism_sync_status", "prism_set_option",
                   "prism_profile_round", "prism_lm_head_topk_static", "prism_round_launches",
                   "prism_draft_round_sampled", "prism_accept_sampled", "prism_draft_tree", "prism_accept_tree",
-                  "prism_profile_tree"):
+                  "prism_profile_tree", "prism_draft_loop"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -249,6 +250,25 @@ class Drafter:
         self._check(self.lib.prism_accept_sampled(
             self.h, B, _ptr(draft), _ptr(logits), _ptr(draft_lse), float(temperature), _ptr(target_probs),
             _ptr(seed), _ptr(n_new), _ptr(kv_len), _ptr(accept_len), _ptr(out_tokens), _stream(stream)))
+
+    def draft_loop(self, tokens, hidden, n_new, kv_len, k_cache, v_cache, target, draft_ids, accept_len, out_tokens,
+                   stream=None):
+        """``prism_draft_loop``: R greedy rounds on the device, each followed by
+        acceptance that writes the next round's tokens and n_new.  hidden
+        [R, B, max_new, d]; target [R, B, K + 1]; draft_ids [R, B, K];
+        accept_len [R, B]; out_tokens [R, B, K + 1]; tokens, n_new and kv_len
+        are updated in place."""
+        R, B = hidden.shape[0], tokens.shape[0]
+        K = self.n_steps
+        i32 = torch.int32
+        self._round_args(tokens, hidden[0], n_new, kv_len, k_cache, v_cache, None, None, None)
+        self._tensor(hidden, (R, B, self.max_new, self.hidden), self.tdtype, "hidden")
+        for t, shp, name in ((target, (R, B, K + 1), "target"), (draft_ids, (R, B, K), "draft_ids"),
+                             (accept_len, (R, B), "accept_len"), (out_tokens, (R, B, K + 1), "out_tokens")):
+            self._tensor(t, shp, i32, name)
+        self._check(self.lib.prism_draft_loop(
+            self.h, B, R, _ptr(tokens), _ptr(hidden), _ptr(n_new), _ptr(kv_len), _ptr(k_cache), _ptr(v_cache),
+            _ptr(target), _ptr(draft_ids), _ptr(accept_len), _ptr(out_tokens), _stream(stream)))
 
     def tree_pool_size(self, width: int) -> int:
         """Candidates of one tree round of this width: w + (K - 1) w^2."""

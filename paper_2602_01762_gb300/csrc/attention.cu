@@ -315,6 +315,11 @@ __global__ void accept_kernel(const AcceptArgs a) {
         a.out_tokens[b * (K + 1) + j] = v;
     }
     a.kv_len[b] += a.n_new[b];
+    if (a.next_tokens) {
+        // the next round prefills the accepted drafts and the target's token
+        for (int j = 0; j <= acc; ++j) a.next_tokens[b * a.max_new + j] = a.out_tokens[b * (K + 1) + j];
+        a.next_n[b] = acc + 1;
+    }
 }
 
 // ------------------------------------------------------------------ fused

@@ -219,6 +219,10 @@ struct AcceptArgs {
     const int32_t *draft, *target, *n_new;
     int32_t *kv_len, *accept_len, *out_tokens;
     int B, K;
+    // multi-round loop (optional): the next round's accepted tokens
+    // [B, max_new] and their count (a + 1); next_n may alias n_new
+    int32_t *next_tokens, *next_n;
+    int max_new;
 };
 
 // Sampled drafting (Sec. 2 at a temperature T > 0): the draw of step `step`

@@ -55,6 +55,22 @@ RoundArgs round_args(int B, const int32_t *tokens, const void *hidden, const int
     return r;
 }
 
+// A multi-round loop: round 0's arguments, the round count and the
+// acceptance arrays (per-round strides follow from the configuration).
+struct LoopArgs {
+    RoundArgs r0;
+    int rounds;
+    const int32_t *target;
+    int32_t *accept_len, *out_tokens;
+    bool operator==(const LoopArgs &o) const { return std::memcmp(this, &o, sizeof(LoopArgs)) == 0; }
+};
+
+struct LoopGraph {
+    LoopArgs key;
+    bool pdl;
+    cudaGraphExec_t exec;
+};
+
 struct GraphEntry {
     RoundArgs key;
     bool pdl;
@@ -132,6 +148,7 @@ struct prism_ctx {
     int tc_ctr_n = 0;
     uint16_t *xbuf = nullptr;                             // bf16 activation rows of the streamed kernel
     std::vector<GraphEntry> graphs;
+    std::vector<LoopGraph> loop_graphs;
     int last_round_kernels = -1;                          // kernel launches of the last replayed round
     unsigned long long tick = 0;
     std::string error;
@@ -157,6 +174,8 @@ bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
 void drop_graphs(prism_ctx *c) {
     for (auto &g : c->graphs) cudaGraphExecDestroy(g.exec);
     c->graphs.clear();
+    for (auto &g : c->loop_graphs) cudaGraphExecDestroy(g.exec);
+    c->loop_graphs.clear();
 }
 
 // Persistent projection grid: one CTA per SM (never more CTAs than units).
@@ -983,6 +1002,90 @@ prism_status prism_accept_tree(prism_ctx *c, int32_t batch, int32_t n_nodes, con
     return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "tree accept kernel launch");
 }
 
+}  // extern "C"
+
+namespace {
+
+// rounds x (draft round, acceptance that also writes the next round's tokens
+// and n_new), all on the device
+cudaError_t enqueue_loop(prism_ctx *c, const LoopArgs &L, cudaStream_t s, bool pdl) {
+    const prism_config &f = c->cfg;
+    const int B = L.r0.B, K = f.n_steps;
+    const size_t es = c->bf16 ? 2 : 4;
+    const size_t hid_stride = (size_t)B * f.max_new * f.hidden * es;
+    cudaError_t e = cudaSuccess;
+    for (int i = 0; i < L.rounds && e == cudaSuccess; ++i) {
+        RoundArgs r = L.r0;
+        r.hidden = (const uint8_t *)L.r0.hidden + i * hid_stride;
+        r.draft = L.r0.draft + (size_t)i * B * K;
+        e = enqueue_round(c, r, s, pdl, nullptr, nullptr, nullptr);
+        if (e != cudaSuccess) break;
+        AcceptArgs a{r.draft, L.target + (size_t)i * B * (K + 1), r.n_new, const_cast<int32_t *>(r.kv_len),
+                     L.accept_len + (size_t)i * B, L.out_tokens + (size_t)i * B * (K + 1), B, K,
+                     const_cast<int32_t *>(r.tokens), const_cast<int32_t *>(r.n_new), f.max_new};
+        e = launch_accept(a, s);
+    }
+    return e;
+}
+
+}  // namespace
+
+extern "C" {
+
+prism_status prism_draft_loop(prism_ctx *c, int32_t batch, int32_t rounds, int32_t *tokens, const void *hidden,
+                              int32_t *n_new, int32_t *kv_len, void *k_cache, void *v_cache, const int32_t *target,
+                              int32_t *draft_ids, int32_t *accept_len, int32_t *out_tokens, void *stream) {
+    if (!c) return fail(c, PRISM_ERR_INVALID_ARG, "null context");
+    if (rounds < 1) return fail(c, PRISM_ERR_SHAPE, "rounds must be >= 1");
+    if (!target || !accept_len || !out_tokens) return fail(c, PRISM_ERR_INVALID_ARG, "null tensor argument");
+    if (c->cfg.max_new < c->cfg.n_steps + 1)
+        return fail(c, PRISM_ERR_CAPACITY, "a loop needs max_new >= K + 1 (the next round prefills up to K + 1 tokens)");
+    LoopArgs L;
+    std::memset(&L, 0, sizeof L);
+    L.r0 = round_args(batch, tokens, hidden, n_new, kv_len, k_cache, v_cache, draft_ids, nullptr, nullptr, nullptr,
+                      nullptr);
+    L.rounds = rounds;
+    L.target = target;
+    L.accept_len = accept_len;
+    L.out_tokens = out_tokens;
+    prism_status st = check_round_args(c, L.r0);
+    if (st != PRISM_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e = cudaSetDevice(c->device);
+    if (e != cudaSuccess) return cuda_fail(c, e, "cudaSetDevice");
+    if (!c->use_graph) {
+        e = enqueue_loop(c, L, s, c->use_pdl);
+        return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "kernel launch");
+    }
+    LoopGraph *hit = nullptr;
+    for (auto &g : c->loop_graphs)
+        if (g.key == L && g.pdl == c->use_pdl) hit = &g;
+    if (!hit) {
+        if ((int)c->loop_graphs.size() >= kGraphCache) {
+            cudaGraphExecDestroy(c->loop_graphs.front().exec);
+            c->loop_graphs.erase(c->loop_graphs.begin());
+        }
+        cudaGraph_t graph = nullptr;
+        e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
+        if (e != cudaSuccess) return cuda_fail(c, e, "cudaStreamBeginCapture");
+        cudaError_t le = enqueue_loop(c, L, c->cap_stream, c->use_pdl);
+        e = cudaStreamEndCapture(c->cap_stream, &graph);
+        if (le != cudaSuccess) {
+            if (graph) cudaGraphDestroy(graph);
+            return cuda_fail(c, le, "kernel launch during capture");
+        }
+        if (e != cudaSuccess) return cuda_fail(c, e, "cudaStreamEndCapture");
+        cudaGraphExec_t exec = nullptr;
+        e = cudaGraphInstantiate(&exec, graph, 0);
+        cudaGraphDestroy(graph);
+        if (e != cudaSuccess) return cuda_fail(c, e, "cudaGraphInstantiate");
+        c->loop_graphs.push_back(LoopGraph{L, c->use_pdl, exec});
+        hit = &c->loop_graphs.back();
+    }
+    e = cudaGraphLaunch(hit->exec, s);
+    return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "cudaGraphLaunch");
+}
+
 prism_status prism_round_launches(prism_ctx *c, int32_t *n_launches) {
     if (!c || !n_launches) return fail(c, PRISM_ERR_INVALID_ARG, "null argument");
     if (c->last_round_kernels < 0) return fail(c, PRISM_ERR_INVALID_ARG, "no round has been replayed from a graph");
@@ -1065,7 +1168,7 @@ prism_status prism_accept_greedy(prism_ctx *c, int32_t batch, const int32_t *dra
     if (batch < 1) return fail(c, PRISM_ERR_SHAPE, "batch must be >= 1");
     if (batch > c->cfg.max_batch) return fail(c, PRISM_ERR_CAPACITY, "batch exceeds max_batch");
     cudaSetDevice(c->device);
-    AcceptArgs a{draft, target, n_new, kv_len, accept_len, out_tokens, batch, c->cfg.n_steps};
+    AcceptArgs a{draft, target, n_new, kv_len, accept_len, out_tokens, batch, c->cfg.n_steps, nullptr, nullptr, 0};
     cudaError_t e = launch_accept(a, (cudaStream_t)stream);
     return e == cudaSuccess ? PRISM_OK : cuda_fail(c, e, "accept kernel launch");
 }

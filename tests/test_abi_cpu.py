@@ -91,3 +91,10 @@ def test_create_rejects_tree_width_above_eight(lib):
     out = ctypes.c_void_p()
     lib.prism_create.argtypes = [ctypes.POINTER(_Config), ctypes.c_int32, ctypes.POINTER(ctypes.c_void_p)]
     assert lib.prism_create(ctypes.byref(bad), 0, ctypes.byref(out)) == 1
+
+
+def test_loop_entry_point_rejects_null_context(lib):
+    vp, i32 = ctypes.c_void_p, ctypes.c_int32
+    f = lib.prism_draft_loop
+    f.argtypes = [vp, i32, i32] + [vp] * 11
+    assert f(None, 1, 2, *([None] * 11)) == 1
