@@ -225,6 +225,10 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--temperature", type=float, default=0.0,
+                    help="> 0: sampled drafting (prism_draft_round_sampled) at this temperature")
+    ap.add_argument("--loop", type=int, default=0, metavar="R",
+                    help="> 0: time prism_draft_loop, R rounds with acceptance per step")
     ap.add_argument("--opt", action="append", default=[], metavar="NAME=VALUE",
                     help="drafter option (prism_set_option), repeatable")
     args = ap.parse_args()
@@ -241,6 +245,8 @@ def main():
     world, rank, local = dist_setup()
     if w.tree_width > 0:
         run_tree(args, w, world, rank, local)
+    elif args.loop > 0:
+        run_loop(args, w, world, rank, local)
     else:
         run_ours(args, w, world, rank, local)
     if world > 1:
@@ -332,10 +338,20 @@ def run_ours(args, w, world, rank, local):
     tk_ids = torch.empty((B, K, w.topk), dtype=torch.int32, device=dev)
     tk_val = torch.empty((B, K, w.topk), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
+    sampled = args.temperature > 0
+    if sampled:
+        logits_buf = torch.empty((B, K, s.vocab), dtype=torch.float32, device=dev)
+        lse_buf = torch.empty((B, K), dtype=torch.float32, device=dev)
+        seed_buf = torch.tensor([12345], dtype=torch.int64, device=dev)
 
     def one_round():
-        dr.draft_round(t["tokens"], t["hidden"], t["n_new"], t["kv_len"], t["k_cache"], t["v_cache"],
-                       ids, tk_ids, tk_val, stream=stream)
+        if sampled:
+            dr.draft_round_sampled(t["tokens"], t["hidden"], t["n_new"], t["kv_len"], t["k_cache"], t["v_cache"],
+                                   args.temperature, seed_buf, ids, logits_buf, lse_buf, tk_ids, tk_val,
+                                   stream=stream)
+        else:
+            dr.draft_round(t["tokens"], t["hidden"], t["n_new"], t["kv_len"], t["k_cache"], t["v_cache"],
+                           ids, tk_ids, tk_val, stream=stream)
 
     # ---- device-resident timing (graph replay) ---------------------------------
     for _ in range(args.warmup):
@@ -422,7 +438,8 @@ def run_ours(args, w, world, rank, local):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": per_round_ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if s.dtype == "bf16" else "f32",
-            "data": "synthetic", "config": dict(config_of(w), options=options),
+            "data": "synthetic", "config": dict(config_of(w), options=options,
+                                                **({"temperature": args.temperature} if sampled else {})),
             "round_latency_us": per_round_ms * 1e3,
             "hbm": {"bytes_per_round": total_bytes,
                     "achieved_gbs": total_bytes / (per_round_ms / 1e3) / 1e9,
@@ -433,6 +450,8 @@ def run_ours(args, w, world, rank, local):
                          "traffic": traffic_from_profile(kernel_src, w.name), "bytes_per_launch": lm_b,
                          "avg_launch_ms": lm_ms},
             "kernel_time_share": shares,
+            **({"kernel_time_share_note": "from the greedy round: the sampled draws are not in it"}
+               if sampled else {}),
             "kernel_ms_per_round": kind_total,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
@@ -582,6 +601,94 @@ def run_tree(args, w, world, rank, local):
             "gpu_launches": launches_per_round * args.steps,
             "clocks": clk,
             "device_error_word": flags,
+        }), flush=True)
+    dr.close()
+    del weights_dev
+
+def run_loop(args, w, world, rank, local):
+    """prism_draft_loop: a step is one call of R greedy rounds with acceptance
+    on the device.  Targets agree with the drafts of a first pass per position
+    with probability 1/2 (round 0's agreement is exact; later rounds' inputs
+    follow the acceptances, so their agreement is incidental); every step
+    starts from the same tokens, n_new and kv_len."""
+    import numpy as np
+    import torch
+
+    import synth
+    from paper_2602_01762_gb300 import Drafter
+    from paper_2602_01762_gb300.host import bind_weights, to_device, to_numpy
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    s = w.shape
+    B, K, R = w.batch, s.n_steps, args.loop
+    W = synth.make_weights(w)
+    I = synth.make_round_inputs(w, max_new=K + 1)
+    mc = (w.ctx_hi + (R + 1) * (K + 1) + K + 15) // 16 * 16
+    for key in ("k_cache", "v_cache"):
+        a = I[key]
+        pad = np.zeros(a.shape[:2] + (mc,) + a.shape[3:], a.dtype)
+        pad[:, :, :a.shape[2]] = a
+        I[key] = pad
+    hid = np.stack([synth.normal(w.seed, f"loop_hidden_{r}", I["hidden"].shape, 1.0, s.dtype) for r in range(R)])
+    dr = Drafter.from_shape(s, max_batch=B, max_ctx=mc, max_new=K + 1, topk=1, device=local)
+    weights_dev = bind_weights(dr, W, device=dev)
+    t0 = {n: to_device(I[n], dev) for n in ("tokens", "n_new", "kv_len")}
+    t = {n: to_device(I[n], dev) for n in ("tokens", "n_new", "kv_len", "k_cache", "v_cache")}
+    hd = to_device(hid, dev)
+    i32 = torch.int32
+    draft = torch.empty((R, B, K), dtype=i32, device=dev)
+    acc = torch.empty((R, B), dtype=i32, device=dev)
+    out = torch.empty((R, B, K + 1), dtype=i32, device=dev)
+    rnd = synth.uniform_int(w.seed, "loop_target_tok", (R, B, K + 1), 0, s.vocab - 1)
+    target = to_device(rnd, dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def one_step():
+        for n in ("tokens", "n_new", "kv_len"):
+            t[n].copy_(t0[n], non_blocking=True)
+        dr.draft_loop(t["tokens"], hd, t["n_new"], t["kv_len"], t["k_cache"], t["v_cache"], target, draft, acc,
+                      out, stream=stream)
+
+    one_step()
+    torch.cuda.synchronize(dev)
+    u = synth.uniform01(w.seed, "loop_target_u", (R, B, K))
+    tg = rnd.copy()
+    tg[:, :, :K] = np.where(u < 0.5, to_numpy(draft), rnd[:, :, :K])
+    target.copy_(to_device(tg.astype(np.int32), dev))
+    for _ in range(args.warmup):
+        one_step()
+    assert dr.sync_status(stream) == 0
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.2)
+    dist_barrier(world)
+    torch.cuda.synchronize(dev)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        one_step()
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    dist_barrier(world)
+    clk = clocks.stop()
+    ms = dist_reduce(ev0.elapsed_time(ev1), "max", world, dev if world > 1 else None)
+    flags = dr.sync_status(stream)
+    accepted = to_numpy(acc)
+    value = B * K * R * args.steps * world / (ms / 1e3)
+    per_round_ms = ms / args.steps / R
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16" if s.dtype == "bf16" else "f32", "data": "synthetic",
+            "config": dict(config_of(w), loop_rounds=R, max_new=K + 1),
+            "round_latency_us": per_round_ms * 1e3,
+            "loop": {"rounds_per_step": R, "mean_accept_len": float(accepted.mean()),
+                     "accepted_tokens_per_s": float((accepted + 1).sum()) * args.steps * world / (ms / 1e3)},
+            "cpu_baseline": None, "e2e": None,
+            "gpu_launches": None,
+            "clocks": clk, "device_error_word": flags,
         }), flush=True)
     dr.close()
     del weights_dev

@@ -98,22 +98,45 @@ __global__ void __launch_bounds__(kSampleThreads) sample_kernel(const SampleArgs
         part[3] = __int_as_float(bi);
         __threadfence();
         s_last = atomicAdd(a.counter + b, 1) == nblk - 1;
-        if (s_last) {
-            __threadfence();
-            float M = -INFINITY, S = 0.f, BV = -INFINITY;
-            int BI = 0x7FFFFFFF;
-            for (int q = 0; q < nblk; ++q) {
-                const float *pq = a.part + ((size_t)b * a.max_blocks + q) * 4;
-                lse_merge(M, S, __ldcg(pq), __ldcg(pq + 1));
-                const float v2 = __ldcg(pq + 2);
-                const int i2 = __float_as_int(__ldcg(pq + 3));
-                if (score_better(v2, i2, BV, BI)) { BV = v2; BI = i2; }
-            }
-            const size_t o = (size_t)b * a.K + a.step - 1;
-            a.draft[o] = BI;
-            a.lse[o] = M + logf(S);
-            a.counter[b] = 0;
-        }
+    }
+    __syncthreads();
+    if (!s_last || warp != 0) return;
+    // the row's last CTA: lane l merges partials l, l + 32, ... (loads first),
+    // then the lanes merge in a fixed butterfly order
+    __threadfence();
+    constexpr int kPer = kSampleMaxBlocks / 32;
+    float pm[kPer], ps[kPer], pv[kPer];
+    int pi[kPer];
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        const int q = lane + 32 * i;
+        const float4 v = q < nblk ? __ldcg((const float4 *)(a.part + ((size_t)b * a.max_blocks + q) * 4))
+                                  : make_float4(-INFINITY, 0.f, -INFINITY, __int_as_float(0x7FFFFFFF));
+        pm[i] = v.x;
+        ps[i] = v.y;
+        pv[i] = v.z;
+        pi[i] = __float_as_int(v.w);
+    }
+    float M = -INFINITY, S = 0.f, BV = -INFINITY;
+    int BI = 0x7FFFFFFF;
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        lse_merge(M, S, pm[i], ps[i]);
+        if (score_better(pv[i], pi[i], BV, BI)) { BV = pv[i]; BI = pi[i]; }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, M, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, S, o);
+        const float v2 = __shfl_xor_sync(0xFFFFFFFFu, BV, o);
+        const int i2 = __shfl_xor_sync(0xFFFFFFFFu, BI, o);
+        lse_merge(M, S, m2, s2);
+        if (score_better(v2, i2, BV, BI)) { BV = v2; BI = i2; }
+    }
+    if (lane == 0) {
+        const size_t o = (size_t)b * a.K + a.step - 1;
+        a.draft[o] = BI;
+        a.lse[o] = M + logf(S);
+        a.counter[b] = 0;
     }
 }
 
