@@ -94,6 +94,11 @@ WORKLOADS = {
     # the tree the paper evaluates (Sec. 4): 6 steps, 4 branches, 16 verified tokens, batch 1
     "l3-8b-b1-tree": Workload("l3-8b-b1-tree", replace(L3_8B, name="llama3-8b-k6", n_steps=6), 1, 2048, 2048, 1,
                               1, 1, tree_width=4, tree_nodes=16),
+    # the module layout of the paper's experiments (Sec. 4): two modules, the first for the prefill
+    # step and the second for every decoding step
+    "l3-8b-b1-m2": Workload("l3-8b-b1-m2", L3_8B, 1, 2048, 2048, 1, 1, 1, f_map=(0, 1, 1, 1, 1)),
+    "l3-8b-b1-tree-m2": Workload("l3-8b-b1-tree-m2", replace(L3_8B, name="llama3-8b-k6", n_steps=6), 1, 2048, 2048,
+                                 1, 1, 1, f_map=(0, 1, 1, 1, 1, 1), tree_width=4, tree_nodes=16),
 }
 
 

@@ -79,7 +79,7 @@ def test_mid_ragged_batch_round():
 
 
 @pytest.mark.slow
-@pytest.mark.parametrize("name,n_sample", [("l3-8b-b1", 1), ("l3-8b-b16", 3), ("l3-8b-b64", 3),
+@pytest.mark.parametrize("name,n_sample", [("l3-8b-b1", 1), ("l3-8b-b1-m2", 1), ("l3-8b-b16", 3), ("l3-8b-b64", 3),
                                            ("l2-7b-b8", 3), ("l3-70b-b32", 2)])
 def test_full_size_round(name, n_sample):
     w = synth.WORKLOADS[name]

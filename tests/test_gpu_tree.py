@@ -255,10 +255,12 @@ def test_tree_widths(width, n_nodes):
     assert rep["rows"] >= 2
 
 
-def test_full_size_tree_l3_8b_b1():
+@pytest.mark.parametrize("name", ["l3-8b-b1-tree", "l3-8b-b1-tree-m2"])
+def test_full_size_tree_l3_8b_b1(name):
     """The paper's tree (6 steps, 4 branches, 16 verified) on the Llama-3-8B
-    shape at batch 1, in the launch configuration the benchmark times."""
-    w = synth.WORKLOADS["l3-8b-b1-tree"]
+    shape at batch 1, in the launch configuration the benchmark times; with a
+    module per step and with the paper's two modules."""
+    w = synth.WORKLOADS[name]
     W, I = synth.make_weights(w), synth.make_round_inputs(w)
     _, _, rep = run_case(w, W, I, [0])
     print(rep)
