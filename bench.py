@@ -374,6 +374,18 @@ def run_ours(args, w, world, rank, local):
     ms = dist_reduce(ms_local, "max", world, dev if world > 1 else None)
     flags = dr.sync_status(stream)
     launches_per_round = dr.round_launches()
+
+    # per-replay latency distribution (after the timed region: an event pair around each replay)
+    n_pct = min(200, args.steps)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_pct)]
+    for e0, e1 in evs:
+        e0.record(stream)
+        one_round()
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    lat = sorted(e0.elapsed_time(e1) * 1e3 for e0, e1 in evs)
+    pct = {"p10": lat[len(lat) // 10], "p50": lat[len(lat) // 2], "p90": lat[(len(lat) * 9) // 10],
+           "replays": n_pct}
     tokens_total = B * K * args.steps * world
     value = tokens_total / (ms / 1e3)
     per_round_ms = ms / args.steps
@@ -441,6 +453,7 @@ def run_ours(args, w, world, rank, local):
             "data": "synthetic", "config": dict(config_of(w), options=options,
                                                 **({"temperature": args.temperature} if sampled else {})),
             "round_latency_us": per_round_ms * 1e3,
+            "round_latency_percentiles_us": pct,
             "hbm": {"bytes_per_round": total_bytes,
                     "achieved_gbs": total_bytes / (per_round_ms / 1e3) / 1e9,
                     "frac_of_8tbs": total_bytes / (per_round_ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,
