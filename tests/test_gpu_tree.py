@@ -351,3 +351,15 @@ def test_tree_rejects_bad_arguments():
                       big[0], big[1], big[2], torch.zeros((B, 1000), dtype=torch.float32, device="cuda"))
     dr.close()
     model.close()
+
+
+@pytest.mark.parametrize("K,width,n_nodes", [(1, 4, 3), (9, 8, 40)])
+def test_tree_step_count_edges(K, width, n_nodes):
+    """One step (the tree is the best candidates of the prefill row alone) and
+    (K - 1) * width = 64, every bit of the ancestor mask in use."""
+    base = synth.WORKLOADS["tiny-bf16-tree"]
+    w = base.with_(shape=replace(base.shape, name=f"tiny-bf16-k{K}", n_steps=K), tree_width=width, tree_nodes=n_nodes)
+    W = synth.make_weights(w)
+    I = ragged(w, synth.make_round_inputs(w))
+    _, _, rep = run_case(w, W, I, list(range(w.batch)))
+    assert rep["rows"] == w.batch * (1 + (K - 1) * width)
