@@ -45,7 +45,11 @@ constexpr uint32_t kBoxBytes = kTileM * 128;  // 16 KB
 constexpr int kMmaN = 16;
 constexpr int kTcMaxStages = 8;
 constexpr int kMaxSplits = 8;
-constexpr size_t kTcSmem = 212 * 1024;      // dynamic shared memory budget
+constexpr size_t kTcSmem = 212 * 1024;      // dynamic shared memory budget of the top-k list instances
+// the other staged instances keep about 1 KB of static shared memory, so their
+// rings can grow to what the 227 KB per-CTA limit leaves (more bytes in flight
+// per SM: HBM reads scale with them up to tens of MB in flight device-wide)
+constexpr size_t kTcSmemLarge = 225 * 1024;
 constexpr size_t kXBudget = 128 * 1024;     // largest X slice
 constexpr long kTcWaitLimit = 1L << 22;
 
@@ -1251,8 +1255,9 @@ cudaError_t set_tc_attrs(int bytes) {
 #define PRISM_TC_ATTR(RPW, TK, PRO)                                                                      \
     if (e == cudaSuccess)                                                                                \
         e = cudaFuncSetAttribute(gemv_tc_kernel<NB, RPW, TK, PRO>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    PRISM_TC_ATTR(1, 1, kProNorm)
     PRISM_TC_ATTR(1, 2, kProNorm)
+    bytes = (int)kTcSmemLarge;
+    PRISM_TC_ATTR(1, 1, kProNorm)
     PRISM_TC_ATTR(2, 0, kProNorm)
     PRISM_TC_ATTR(1, 0, kProFusePrefill)
     PRISM_TC_ATTR(1, 0, kProFuseDecode)
@@ -1288,7 +1293,8 @@ bool tc_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem) {
     p.nkb = nkb;
     p.splits = best_s;
     p.x_bytes = (uint32_t)(NB * 128 * ((nkb + best_s - 1) / best_s));
-    const size_t room = kTcSmem - 1024 - p.x_bytes;
+    const bool lists = a.epi == kEpiTopK && !(a.topk == 1 && a.best != nullptr);
+    const size_t room = (lists ? kTcSmem : kTcSmemLarge) - 1024 - p.x_bytes;
     // 32 KB stages, or 16 KB ones when fewer than four 32 KB stages fit
     p.kb_per_stage = (RPW == 1 && room >= 4 * 2 * (size_t)kBoxBytes) ? 2 : 1;
     p.stage_bytes = (uint32_t)p.kb_per_stage * RPW * kBoxBytes;
