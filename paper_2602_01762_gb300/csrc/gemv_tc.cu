@@ -1295,8 +1295,8 @@ bool tc_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem) {
     p.x_bytes = (uint32_t)(NB * 128 * ((nkb + best_s - 1) / best_s));
     const bool lists = a.epi == kEpiTopK && !(a.topk == 1 && a.best != nullptr);
     const size_t room = (lists ? kTcSmem : kTcSmemLarge) - 1024 - p.x_bytes;
-    // 32 KB stages, or 16 KB ones when fewer than four 32 KB stages fit
-    p.kb_per_stage = (RPW == 1 && room >= 4 * 2 * (size_t)kBoxBytes) ? 2 : 1;
+    // 48 KB stages when three fit, 32 KB ones when four fit, else 16 KB
+    p.kb_per_stage = RPW != 1 ? 1 : room >= 3 * 3 * (size_t)kBoxBytes ? 3 : room >= 4 * 2 * (size_t)kBoxBytes ? 2 : 1;
     p.stage_bytes = (uint32_t)p.kb_per_stage * RPW * kBoxBytes;
     p.stages = (int)(room / p.stage_bytes);
     if (p.stages > kTcMaxStages) p.stages = kTcMaxStages;
