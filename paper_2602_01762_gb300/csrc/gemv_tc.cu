@@ -1350,7 +1350,11 @@ bool tcs_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem, in
     p.n_tiles = n_tiles;
     p.nkb = nkb;
     p.splits = best_s;
-    p.kb_per_stage = kb_bytes <= 20 * 1024 && room >= 4 * 2 * kb_bytes ? 2 : 1;
+    // the largest stage of up to 64 KB of which four still fit (larger
+    // stages stream faster than more, smaller ones)
+    p.kb_per_stage = 1;
+    for (int k = 3; k >= 2; --k)
+        if (k * kb_bytes <= 64 * 1024 && room >= 4 * (size_t)k * kb_bytes) { p.kb_per_stage = k; break; }
     p.stage_bytes = (uint32_t)(p.kb_per_stage * kb_bytes);
     p.x_bytes = 0;
     p.stages = (int)(room / p.stage_bytes);
