@@ -12,12 +12,15 @@
 // of the round.  The kernels this file adds:
 //   tree_gather_kernel     fusion input row [E(token); round(h^ of the row
 //                          that emitted the token)];
-//   tree_attention_kernel  rotary embedding at the node's depth, K/V appended
+//   tree_attention_tc_kernel / tree_attention_kernel
+//                          rotary embedding at the node's depth, K/V appended
 //                          at the node's own cache slot L + n + (k - 2) w + j,
 //                          and split-KV attention over the committed rows
 //                          [0, L+n) plus the draft slots in the row's 64-bit
 //                          ancestor mask, all w rows of a sequence against one
-//                          staged chunk of keys, last-CTA merge in split order;
+//                          staged chunk of keys, last-CTA merge in split order
+//                          (tensor cores for bf16 caches with w * G <= 16
+//                          row-head pairs, CUDA cores otherwise);
 //   tree_lse_kernel        log-sum-exp of every row's logits; the last row of
 //                          each sequence to finish then scores the candidates,
 //                          picks the next frontier and, after the last step,
