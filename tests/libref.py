@@ -28,7 +28,13 @@ def _t(a) -> torch.Tensor:
 
 
 def _bf16(t: torch.Tensor) -> torch.Tensor:
-    return t.to(torch.bfloat16).to(f64)
+    """Round to the nearest bf16 value, ties to even, directly from fp64:
+    x = m * 2^e with 0.5 <= |m| < 1, and bf16 keeps 8 significant bits, so the
+    result is rint(m * 2^8) / 2^8 * 2^e (numpy's rint rounds half to even).
+    (torch's own conversion goes through float32 and can round twice.)"""
+    x = t.detach().numpy()
+    m, e = np.frexp(x)
+    return torch.from_numpy(np.ldexp(np.rint(m * 256.0) / 256.0, e))
 
 
 def _rope(x: torch.Tensor, pos: torch.Tensor, theta: float) -> torch.Tensor:

@@ -34,12 +34,21 @@ MUTANTS = [
     ("argmax-tie", "return (a > b) - (a < b);", "return (a < b) - (a > b);"),
     ("accept-commit", "kv_len[b] += n_new[b];", "kv_len[b] += n_new[b] + a;"),
     ("accept-bonus", "else if (j == a) v = target[b * (K + 1) + a];", "else if (j == a) v = draft[b * K + (a < K ? a : K - 1)];"),
+    # the bf16 contract: each projection operand is rounded right before its product
+    ("round-n1", "round_vec(w->n1, d, ra);", "(void)0;"),
+    ("round-o", "round_vec(w->o, Hq * D, ra);", "(void)0;"),
+    ("round-n2", "round_vec(w->n2, d, ra);", "(void)0;"),
+    ("round-m", "round_vec(w->mm, F, ra);", "(void)0;"),
+    ("round-final", "round_vec(nf, d, c->round_acts);", "(void)0;"),
+    ("round-decode-input", "round_vec(u, 2 * d, c->round_acts);\n                layer_row(c, m, u, L + n + k - 2,",
+     "layer_row(c, m, u, L + n + k - 2,"),
 ]
 
 PINS = [
     lambda: pins.test_round_matches_library_reference((0, 1, 2)),
     lambda: pins.test_round_matches_library_reference((0, 1, 1)),
     pins.test_round_without_final_norm_matches_reference,
+    pins.test_bf16_contract_matches_reference,
     pins.test_prefill_equals_sequential_decode,
     pins.test_closed_form_draft_repeats_last_token,
     pins.test_closed_form_hidden_passthrough,

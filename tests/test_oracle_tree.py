@@ -76,6 +76,25 @@ def test_tree_rows_equal_the_reference_chain_forced_down_their_path():
                 assert pins.max_rel(o["v_cache"][b, :, slot], ref["v_cache"][b, :, pos]) < 1e-6
 
 
+def test_tree_rows_under_the_bf16_contract_equal_the_reference_chain():
+    """The same, with bf16 weights, caches and operand rounding: the reference
+    rounds fp64 to bf16 by another route, so every rounding point must agree."""
+    shape = replace(TREE_SHAPE, name="pin-tree-bf16", dtype="bf16")
+    w = TREE.with_(shape=shape)
+    W, I = pins.pin_case(w)
+    K, wd = shape.n_steps, w.tree_width
+    o = oracle.draft_tree(shape, W, I, width=wd, n_nodes=w.tree_nodes, want_hidden=True)
+    B = I["tokens"].shape[0]
+    for b in range(B):
+        for k, j in _rows(K, wd):
+            path = [] if k == 1 else _path(o, b, int(o["frontier"][b, k - 2, j]))
+            forced = np.zeros((B, K - 1), np.int32)
+            forced[b, :k - 1] = path
+            ref = reference_round(shape, W, I, forced=forced, round_acts=True)
+            assert pins.max_rel(o["row_logits"][b, k - 1, j], ref["logits"][b, k - 1]) < 1e-9, (b, k, j)
+            assert pins.max_rel(o["row_hidden"][b, k - 1, j], ref["hidden_out"][b, k - 1]) < 1e-9, (b, k, j)
+
+
 def test_committed_rows_untouched_and_step1_rows_as_chain():
     W, I = tree_case()
     o = oracle.draft_tree(TREE_SHAPE, W, I, width=TREE.tree_width, n_nodes=TREE.tree_nodes)
@@ -276,12 +295,14 @@ TREE_MUTANTS = [
     ("tree-final-size", "for (int64_t i = 0; i < n_nodes; ++i) pos_in_tree[idx[i]] = 0;",
      "for (int64_t i = 0; i < n_nodes; ++i) pos_in_tree[idx[i + (i + 1 < n_nodes ? 0 : 1)]] = 0;"),
     ("accept-tree-wrong-target", "const int32_t want = tn[cur + 1];", "const int32_t want = tn[a];"),
+    ("tree-round-input", "round_vec(u, 2 * d, c->round_acts);\n                    int64_t nv = 0;", "int64_t nv = 0;"),
     ("accept-tree-commit", "kv_len[b] = kv_len[b] + n_new[b];   /* only", "kv_len[b] = kv_len[b] + n_new[b] + a;   /* only"),
     ("accept-tree-bonus", "out_tokens[b * (K + 1) + a] = tn[cur + 1];", "out_tokens[b * (K + 1) + a] = tn[a];"),
 ]
 
 TREE_PINS = [
     test_tree_rows_equal_the_reference_chain_forced_down_their_path,
+    test_tree_rows_under_the_bf16_contract_equal_the_reference_chain,
     test_scores_candidates_frontiers_and_tree_by_brute_force,
     test_tree_acceptance_matches_brute_force,
 ]
