@@ -7,6 +7,8 @@ What fixes these functions, other than the oracle itself:
     is the argmax;
   * speculative sampling is lossless: with drafts drawn from p_draft, the first
     output token is distributed as p_target (chi-square), whatever p_draft is;
+  * the same at a later position (its own draft and target distributions),
+    and the extra token after K accepted drafts follows p_target at K;
   * special cases: p_target = p_draft accepts everything; a draft token the
     target gives probability 0 is always rejected and replaced by a token where
     p_target > p_draft;
@@ -92,6 +94,46 @@ def test_speculative_sampling_is_lossless():
     assert 0.2 < r["accept_len"].mean() < 0.9
 
 
+def test_lossless_at_every_position():
+    """Two draft positions with their own draft and target distributions: the
+    first output token follows p_target[0]; where the first draft is accepted,
+    the second output token follows p_target[1] (the rule applied at that
+    position, with its own random numbers)."""
+    V, K, n, tau, seed = 5, 2, 40000, 1.0, 777
+    zd = np.array([[1.2, -0.5, 0.3, 0.0, -1.0],
+                   [-0.8, 0.9, 0.1, 1.4, -0.2]])
+    pt = np.array([[0.10, 0.35, 0.25, 0.20, 0.10],
+                   [0.40, 0.05, 0.30, 0.05, 0.20],
+                   [0.20, 0.20, 0.20, 0.20, 0.20]])
+    draft = np.stack([_draws(zd[k], tau, seed, n, k) for k in range(K)], axis=1)
+    z = np.broadcast_to(zd, (n, K, V))
+    lse = np.broadcast_to(special.logsumexp(zd / tau, axis=-1), (n, K))
+    target = np.broadcast_to(pt, (n, K + 1, V))
+    r = oracle.accept_sampled(draft, z, lse, tau, target, seed, np.ones(n, np.int32), np.zeros(n, np.int32))
+    out, a = r["out_tokens"], r["accept_len"]
+    assert stats.chisquare(np.bincount(out[:, 0], minlength=V), pt[0] * n).pvalue > P_MIN
+    sel = a >= 1
+    m = int(sel.sum())
+    assert m > n // 4
+    assert stats.chisquare(np.bincount(out[sel, 1], minlength=V), pt[1] * m).pvalue > P_MIN
+
+
+def test_bonus_token_follows_the_targets_last_distribution():
+    """When every draft is accepted, the extra token is drawn from p_target at
+    position K."""
+    V, K, n, tau = 5, 2, 20000, 1.0
+    zd = np.array([0.5, -0.2, 0.1, 0.8, -1.0])
+    pd = special.softmax(zd / tau)
+    last = np.array([0.70, 0.05, 0.05, 0.15, 0.05])
+    target = np.broadcast_to(np.stack([pd, pd, last]), (n, K + 1, V))
+    draft = np.stack([_draws(zd, tau, 9, n, k) for k in range(K)], axis=1)
+    z = np.broadcast_to(zd, (n, K, V))
+    lse = np.full((n, K), special.logsumexp(zd / tau))
+    r = oracle.accept_sampled(draft, z, lse, tau, target, 9, np.ones(n, np.int32), np.zeros(n, np.int32))
+    assert (r["accept_len"] == K).all()
+    assert stats.chisquare(np.bincount(r["out_tokens"][:, K], minlength=V), last * n).pvalue > P_MIN
+
+
 def test_equal_distributions_accept_everything():
     V, K, n, tau = 5, 3, 500, 0.7
     rng = np.random.default_rng(8)
@@ -162,6 +204,8 @@ SAMPLING_PINS = [
     test_gumbel_draws_follow_softmax,
     test_gumbel_draw_at_tiny_temperature_is_the_argmax,
     test_speculative_sampling_is_lossless,
+    test_lossless_at_every_position,
+    test_bonus_token_follows_the_targets_last_distribution,
     test_equal_distributions_accept_everything,
     test_a_token_the_target_excludes_is_replaced_where_target_exceeds_draft,
     test_sampled_round_draws_from_its_own_logits,
@@ -175,6 +219,12 @@ MUTANTS = [
     ("residual-direction", "w[i] = fmax(0.0, pk[i] - exp(", "w[i] = fmax(0.0, -pk[i] + 2.0 * exp("),
     ("replacement-stream", "const double u = orc_uniform(seed, 3, sb, a, 0);", "const double u = orc_uniform(seed, 2, sb, a, 0);"),
     ("round-stream-index", "seq_index ? seq_index[b] : b, k - 1, &prev", "b, k - 1, &prev"),
+    ("bonus-position", "+ K) * V, V, orc_uniform(seed, 3, sb, K, 0)", "+ K - 1) * V, V, orc_uniform(seed, 3, sb, K, 0)"),
+    ("target-position", "*pk = pt + ((int64_t)b * (K + 1) + a) * V;", "*pk = pt + ((int64_t)b * (K + 1)) * V;"),
+    ("draft-lse-position", "const double pd = exp(zk[x] / tau - lse[b * K + a]);",
+     "const double pd = exp(zk[x] / tau - lse[b * K]);"),
+    ("replacement-not-residual", "extra = tot > 0.0 ? draw_cdf(w, V, u) : draw_cdf(pk, V, u);", "extra = draw_cdf(pk, V, u);"),
+    ("accept-stream-position", "const double r = orc_uniform(seed, 2, sb, a, 0);", "const double r = orc_uniform(seed, 2, sb, 0, 0);"),
 ]
 
 
