@@ -34,6 +34,18 @@ MUTANTS = [
     ("argmax-tie", "return (a > b) - (a < b);", "return (a < b) - (a > b);"),
     ("accept-commit", "kv_len[b] += n_new[b];", "kv_len[b] += n_new[b] + a;"),
     ("accept-bonus", "else if (j == a) v = target[b * (K + 1) + a];", "else if (j == a) v = draft[b * K + (a < K ? a : K - 1)];"),
+    ("silu-sign", "return t / (1.0 + exp(-t));", "return t / (1.0 + exp(t));"),
+    ("rmsnorm-eps-outside", "double inv = 1.0 / sqrt(ss / (double)n + eps);", "double inv = 1.0 / (sqrt(ss / (double)n) + eps);"),
+    ("value-split", "*v = w->qkv + (Hq + Hkv) * D;", "*v = w->qkv + Hq * D;"),
+    ("cache-store-swap", "store_el(kc_b, idx, bf, k[g * D + t]);", "store_el(kc_b, idx, bf, v[g * D + t]);"),
+    ("attend-with-keys", "o[t] += s[j] * load_el(vc, j * row_stride + t, bf16);",
+     "o[t] += s[j] * load_el(kc, j * row_stride + t, bf16);"),
+    ("key-rope-position", "orc_rope(k + g * D, (int32_t)D, pos, c->rope_theta);",
+     "orc_rope(k + g * D, (int32_t)D, pos + 1, c->rope_theta);"),
+    ("prefill-hidden-shift", "\n                        u[d + t] = load_el(hidden, ((int64_t)b * max_new + i) * d + t, bf);",
+     "\n                        u[d + t] = i > 0 ? load_el(hidden, ((int64_t)b * max_new + i - 1) * d + t, bf) : 0.0;"),
+    ("hhat-normed", "prev = tid[0];\n            if (tau > 0.0) {", "prev = tid[0];\n            memcpy(hhat, w.n1, sizeof(double) * (size_t)d);\n            if (tau > 0.0) {"),
+    ("topk-order", "top_vals[r] = z[order[r]];", "top_vals[r] = z[order[c->topk - 1 - r]];"),
     # the bf16 contract: each projection operand is rounded right before its product
     ("round-n1", "round_vec(w->n1, d, ra);", "(void)0;"),
     ("round-o", "round_vec(w->o, Hq * D, ra);", "(void)0;"),
@@ -55,6 +67,7 @@ PINS = [
     pins.test_closed_form_uniform_attention,
     pins.test_accept_exhaustive_patterns,
     pins.test_greedy_acceptance_is_the_zero_temperature_rule,
+    pins.test_topk_lists_are_the_sorted_logits,
 ]
 
 

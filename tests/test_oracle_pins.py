@@ -222,6 +222,20 @@ def test_argmax_ties_go_to_lowest_id():
     assert (r["topk_ids"] == np.arange(3)).all()
 
 
+def test_topk_lists_are_the_sorted_logits():
+    """The top-k list of every step is numpy's stable sort of that step's
+    logits (descending value, ascending id), and the greedy chain takes its
+    first entry."""
+    W, I = pin_case()
+    k = 7
+    r = oracle.draft_round(PIN_SHAPE, W, I, topk=k, want_logits=True)
+    z = r["logits"]
+    order = np.argsort(-z, axis=-1, kind="stable")[..., :k]
+    assert np.array_equal(r["topk_ids"], order)
+    assert np.array_equal(r["topk_logits"], np.take_along_axis(z, order, axis=-1))
+    assert np.array_equal(r["draft_ids"], order[..., 0])
+
+
 # ------------------------------------------------------------------ closed forms
 
 def _structured(shape, fuse_half, n_new=3, seed=5):

@@ -295,6 +295,8 @@ TREE_MUTANTS = [
     ("tree-final-size", "for (int64_t i = 0; i < n_nodes; ++i) pos_in_tree[idx[i]] = 0;",
      "for (int64_t i = 0; i < n_nodes; ++i) pos_in_tree[idx[i + (i + 1 < n_nodes ? 0 : 1)]] = 0;"),
     ("accept-tree-wrong-target", "const int32_t want = tn[cur + 1];", "const int32_t want = tn[a];"),
+    ("tree-prefill-hidden-shift", "\n                            u[d + t] = load_el(hidden, ((int64_t)b * max_new + i) * d + t, bf);",
+     "\n                            u[d + t] = i > 0 ? load_el(hidden, ((int64_t)b * max_new + i - 1) * d + t, bf) : 0.0;"),
     ("tree-round-input", "round_vec(u, 2 * d, c->round_acts);\n                    int64_t nv = 0;", "int64_t nv = 0;"),
     ("accept-tree-commit", "kv_len[b] = kv_len[b] + n_new[b];   /* only", "kv_len[b] = kv_len[b] + n_new[b] + a;   /* only"),
     ("accept-tree-bonus", "out_tokens[b * (K + 1) + a] = tn[cur + 1];", "out_tokens[b * (K + 1) + a] = tn[a];"),
