@@ -98,3 +98,29 @@ def test_loop_entry_point_rejects_null_context(lib):
     f = lib.prism_draft_loop
     f.argtypes = [vp, i32, i32] + [vp] * 11
     assert f(None, 1, 2, *([None] * 11)) == 1
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """No fallback: without the built library every entry of the binding raises."""
+    import paper_2602_01762_gb300 as pkg
+    monkeypatch.setattr(pkg, "LIB_PATH", str(tmp_path / "libprism.so"))
+    monkeypatch.setattr(pkg, "_lib", None)
+    with pytest.raises(RuntimeError, match="missing"):
+        pkg.library()
+    with pytest.raises(RuntimeError, match="missing"):
+        pkg.Drafter(hidden=64, n_q_heads=4, n_kv_heads=2, head_dim=16, ffn=96, vocab=300, n_steps=3)
+
+
+def test_product_path_does_not_reach_the_oracle():
+    """The package and its CUDA sources name neither the oracle nor the test
+    helpers; only the tests, the smoke check and the benchmark's CPU legs may."""
+    pkg = os.path.join(ROOT, "paper_2602_01762_gb300")
+    offenders = []
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if not f.endswith((".py", ".cu", ".cuh", ".h", ".cpp")):
+                continue
+            text = open(os.path.join(dirpath, f)).read()
+            if re.search(r"^\s*(import|from)\s+(oracle|tests|synth)\b", text, flags=re.M) or "orc_" in text:
+                offenders.append(f)
+    assert not offenders, offenders
