@@ -124,3 +124,18 @@ def test_product_path_does_not_reach_the_oracle():
             if re.search(r"^\s*(import|from)\s+(oracle|tests|synth)\b", text, flags=re.M) or "orc_" in text:
                 offenders.append(f)
     assert not offenders, offenders
+
+
+def test_oracle_is_independent_of_the_product():
+    """The oracle includes only system headers and imports nothing of the
+    package: the two sides share no code."""
+    odir = os.path.join(ROOT, "oracle")
+    for f in os.listdir(odir):
+        path = os.path.join(odir, f)
+        if f.endswith((".c", ".h")):
+            incs = re.findall(r'^\s*#\s*include\s*([<"][^>"]+[>"])', open(path).read(), flags=re.M)
+            assert all(i.startswith("<") for i in incs), (f, incs)
+        elif f.endswith(".py"):
+            text = open(path).read()
+            assert not re.search(r"^\s*(import|from)\s+paper_2602_01762_gb300\b", text, flags=re.M), f
+            assert "libprism" not in text and "csrc" not in text, f
