@@ -19,10 +19,13 @@ random times) and check at every step that
 
 The models restate the control flow of ``gemv_kernel`` (csrc/gemv.cu: one
 producer lane, 16 consumer warps in G groups, group g taking stages s = g mod
-G) and of ``gemv_tc_kernel`` / ``gemv_tcs_kernel`` (csrc/gemv_tc.cu: producer
+G), of ``gemv_tc_kernel`` / ``gemv_tcs_kernel`` (csrc/gemv_tc.cu: producer
 lane, MMA lane committing to the stage and accumulator barriers, four
-epilogue warps over two accumulator buffers), with the plans the host code
-can choose (S stages a multiple of G, 2 <= S <= 16; 1..8 stages; splits)."""
+epilogue warps over two accumulator buffers) and of
+``fused_attention_tc_kernel`` (csrc/attention.cu: stages of committed rows
+requested before the block-wide barrier, eight compute warps releasing every
+stage), with the plans the host code can choose (S stages a multiple of G,
+2 <= S <= 16; 1..8 stages; any stage and tile counts)."""
 from __future__ import annotations
 
 import random
@@ -346,6 +349,84 @@ def test_tcgen05_ring_and_accumulator_handoff(S, tiles, kst):
                     event_bias=[0.15, 0.5, 0.85][trial % 3], mma_lag=trial % 4)
 
 
+# ------------------------------------------------- fused_attention_tc_kernel
+
+def run_attention_ring(S, nst, pre, seed, event_bias, empty_count=8):
+    """fused_attention_tc_kernel: the producer requests stages [0, pre)
+    (committed rows only) before the block-wide barrier, then stages
+    [pre, nst), each i >= S after waiting empty[i % S] for the release of
+    stage i - S (parity (i / S - 1) & 1); eight compute warps wait full[i % S]
+    (parity (i / S) & 1) for every stage and arrive on empty[i % S] (count 8)."""
+    warps = 8
+    rng = random.Random(seed)
+    sim = Sim(rng, event_bias)
+    full = [Barrier(1) for _ in range(S)]
+    empty = [Barrier(empty_count) for _ in range(S)]
+    content = [None] * S
+    readers = [set() for _ in range(S)]
+    block = Group(warps + 1)
+    read = {}
+
+    def load(i):
+        s = i % S
+        assert not readers[s], f"slot {s} overwritten while stage {content[s]} is read"
+        full[s].arrive_expect_tx(1)
+        content[s] = None
+
+        def land(s=s, i=i):
+            content[s] = i
+            readers[s] = set(range(warps))
+            full[s].complete_tx(1)
+        sim.post(land)
+
+    def producer():
+        for i in range(pre):
+            load(i)
+            yield ("step",)
+        yield from block.sync()
+        issued = pre
+        for i in range(pre, nst):
+            if i >= S:
+                par = (i // S - 1) & 1
+                yield ("wait", lambda i=i, par=par: empty[i % S].ready(par))
+                check_wait(empty[i % S], par, i // S - 1, "attention producer empty")
+            load(i)
+            issued = i + 1
+            yield ("step",)
+        for i in range(max(0, issued - S), issued):
+            yield ("wait", lambda i=i: full[i % S].ready((i // S) & 1))
+            check_wait(full[i % S], (i // S) & 1, i // S, "attention producer drain")
+
+    def compute(w):
+        yield from block.sync()
+        for i in range(nst):
+            s = i % S
+            yield ("wait", lambda s=s, i=i: full[s].ready((i // S) & 1))
+            check_wait(full[s], (i // S) & 1, i // S, f"attention warp {w} full")
+            assert content[s] == i, f"warp {w} reads slot {s}: stage {content[s]} instead of {i}"
+            read.setdefault(i, set()).add(w)
+            yield ("step",)
+            assert content[s] == i
+            readers[s].discard(w)
+            empty[s].arrive()
+
+    sim.add("producer", producer())
+    for w in range(warps):
+        sim.add(f"warp{w}", compute(w))
+    sim.run()
+    assert all(read.get(i) == set(range(warps)) for i in range(nst))
+
+
+ATTN_CASES = [(S, nst, pre) for S in (2, 3, 4) for nst in (1, 2, 3, 4, 7, 12) for pre in range(0, min(S, nst) + 1)]
+
+
+@pytest.mark.parametrize("S,nst,pre", ATTN_CASES)
+def test_attention_ring_parity_waits_are_unambiguous(S, nst, pre):
+    for trial in range(12):
+        run_attention_ring(S, nst, pre, seed=104729 * S + 101 * nst + 7 * pre + trial,
+                           event_bias=[0.1, 0.5, 0.9][trial % 3])
+
+
 def _fails(run, n=40):
     bad = 0
     for seed in range(n):
@@ -367,3 +448,7 @@ def test_the_checks_catch_an_early_accumulator_release():
     """Likewise for the accumulator: released after the first epilogue warp
     instead of all four, the MMA lane overwrites a buffer still being read."""
     assert _fails(lambda seed: run_tc_ring(2, 5, 2, seed=seed, event_bias=0.5, mma_lag=0, acc_empty_count=1)) > 0
+
+
+def test_the_checks_catch_an_early_attention_stage_release():
+    assert _fails(lambda seed: run_attention_ring(3, 9, 2, seed=seed, event_bias=0.5, empty_count=1)) > 0
