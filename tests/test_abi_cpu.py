@@ -139,3 +139,17 @@ def test_oracle_is_independent_of_the_product():
             text = open(path).read()
             assert not re.search(r"^\s*(import|from)\s+paper_2602_01762_gb300\b", text, flags=re.M), f
             assert "libprism" not in text and "csrc" not in text, f
+
+
+def test_host_marshalling_round_trips_bit_patterns():
+    """bf16 tensors travel as their uint16 bit patterns (NaN and -0 included);
+    other dtypes unchanged."""
+    import numpy as np
+    from paper_2602_01762_gb300.host import to_device, to_numpy
+    bits = np.array([0x0000, 0x8000, 0x3F80, 0xBF80, 0x7F80, 0xFF80, 0x7FC1, 0x0001, 0xFFFF], np.uint16)
+    t = to_device(bits.reshape(3, 3), device="cpu")
+    assert str(t.dtype) == "torch.bfloat16" and tuple(t.shape) == (3, 3)
+    assert np.array_equal(to_numpy(t), bits.reshape(3, 3))
+    assert float(t[0, 2]) == 1.0 and float(t[1, 0]) == -1.0 and float(t[1, 1]) == float("inf")
+    for a in (np.arange(12, dtype=np.int32).reshape(3, 4), np.linspace(-2, 2, 7, dtype=np.float32)):
+        assert np.array_equal(to_numpy(to_device(a, device="cpu")), a)
