@@ -22,6 +22,11 @@
  *     argmax; a draft token x is accepted when r < min(1, p_target(x) /
  *     p_draft(x)), and the first rejected position draws its replacement from
  *     max(0, p_target - p_draft) normalised.
+ *   tree drafting (the tree of Sec. 3.2 and Sec. 4, read as a dynamic top-w
+ *     expansion; see orc_draft_tree): each step expands the w best frontier
+ *     rows by their w best tokens, scores candidates by summed draft
+ *     log-probabilities, and the verified tree is the best n_nodes of the
+ *     pool; its greedy acceptance follows the target's tokens from the root.
  *
  * Readings where the paper is silent (each is a reading, not a quote):
  *   fusion F = one bias-free linear map W_fuse [d, 2d] applied to the
