@@ -97,6 +97,26 @@ def lm_head_bytes(w):
 kTOP = 8
 
 
+def smi_index(local: int, uuid: str | None = None) -> str:
+    """nvidia-smi's index of CUDA device `local`, matched by the device's UUID
+    (CUDA's device numbering need not be nvidia-smi's when only some GPUs are
+    visible); `local` itself when the UUID or nvidia-smi is unavailable."""
+    try:
+        if uuid is None:
+            import torch
+            uuid = str(torch.cuda.get_device_properties(local).uuid)
+        if not uuid.startswith("GPU-"):
+            uuid = "GPU-" + uuid
+        r = subprocess.run(["nvidia-smi", f"--id={uuid}", "--query-gpu=index", "--format=csv,noheader"],
+                           capture_output=True, text=True, timeout=20)
+        out = r.stdout.strip()
+        if r.returncode == 0 and out.isdigit():
+            return out
+    except Exception:
+        pass
+    return str(local)
+
+
 class ClockSampler:
     """nvidia-smi clock/throttle samples while the timed region runs."""
 
@@ -104,12 +124,14 @@ class ClockSampler:
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, uuid: str | None = None):
         self.idx = gpu_index
+        self.uuid = uuid
         self.proc = None
 
     def start(self):
         try:
+            self.idx = smi_index(self.idx, self.uuid)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
                  "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)

@@ -146,3 +146,26 @@ def test_config_names_the_workload_and_its_l2_policy(name):
     c = bench.config_of(WORKLOADS[name])
     assert c["workload"] == name and "larger than L2" in c["l2"]
     assert ("tree_width" in c) == name.endswith("tree")
+
+
+def _fake_smi(tmp_path, monkeypatch, script: str):
+    exe = tmp_path / "nvidia-smi"
+    exe.write_text("#!/bin/sh\n" + script)
+    exe.chmod(0o755)
+    monkeypatch.setenv("PATH", f"{tmp_path}:{os.environ.get('PATH', '')}")
+
+
+def test_clock_sampler_finds_the_device_by_uuid(tmp_path, monkeypatch):
+    """CUDA device 0 may be nvidia-smi's GPU 5 when only some GPUs are visible:
+    the sampler asks nvidia-smi for the index of the device's UUID."""
+    _fake_smi(tmp_path, monkeypatch, 'case "$1" in --id=GPU-abc) echo 5 ;; *) exit 6 ;; esac\n')
+    assert bench.smi_index(0, "abc") == "5"
+    assert bench.smi_index(0, "GPU-abc") == "5"
+    assert bench.smi_index(2, "GPU-other") == "2"          # unknown UUID: CUDA's index
+    _fake_smi(tmp_path, monkeypatch, "echo 'No devices were found'\n")
+    assert bench.smi_index(1, "abc") == "1"
+
+
+def test_clock_sampler_without_nvidia_smi_keeps_the_index(tmp_path, monkeypatch):
+    monkeypatch.setenv("PATH", str(tmp_path))
+    assert bench.smi_index(3, "abc") == "3"
