@@ -322,7 +322,9 @@ prism_status prism_accept_tree(prism_ctx *ctx, int32_t batch, int32_t n_nodes, c
  *   draft int32 [batch] out; topk_ids int32 [batch, topk], topk_logits fp32
  *   [batch, topk], logits fp32 [batch, vocab]: outputs, each may be NULL;
  *   dev_flags int32 [1] or NULL: receives the device error word of this call.
- * All pointers are device pointers; h, lm_head and g_final 16-byte aligned.
+ * All pointers are device (or managed) memory of the current device; h,
+ * lm_head and g_final 16-byte aligned.  A pointer to host memory or to
+ * another device's memory returns PRISM_ERR_INVALID_ARG before any launch.
  * Limits: batch <= 64 rows; larger batches return PRISM_ERR_CAPACITY with a
  * message from prism_get_error(NULL): split them into several calls.
  * The first call on a device (the current one) does that device's set-up:

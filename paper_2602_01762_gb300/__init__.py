@@ -97,9 +97,9 @@ def _ptr(t):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
 
-def _stream(stream):
+def _stream(stream, device=None):
     if stream is None:
-        stream = torch.cuda.current_stream()
+        stream = torch.cuda.current_stream(device)
     return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
 
 
@@ -423,8 +423,12 @@ def lm_head_topk_static(h, g_final, lm_head, draft, topk_ids=None, topk_logits=N
     for t, shape, dtype, name in want:
         if tuple(t.shape) != shape or t.dtype != dtype or not t.is_cuda or not t.is_contiguous():
             raise ValueError(f"{name}: expected contiguous CUDA {dtype} {shape}, got {t.dtype} {tuple(t.shape)}")
-    st = lib.prism_lm_head_topk_static(dt, d, V, B, topk, float(rms_eps), _ptr(h), _ptr(g_final),
-                                       _ptr(lm_head), _ptr(draft), _ptr(topk_ids), _ptr(topk_logits),
-                                       _ptr(logits), _ptr(dev_flags), _stream(stream))
+        if t.device != h.device:
+            raise ValueError(f"{name} is on {t.device}, h on {h.device}: every tensor must be on one device")
+    # the library launches on the current device: make it the tensors' device
+    with torch.cuda.device(h.device):
+        st = lib.prism_lm_head_topk_static(dt, d, V, B, topk, float(rms_eps), _ptr(h), _ptr(g_final),
+                                           _ptr(lm_head), _ptr(draft), _ptr(topk_ids), _ptr(topk_logits),
+                                           _ptr(logits), _ptr(dev_flags), _stream(stream, h.device))
     if st != 0:
         raise PrismError(st, (lib.prism_get_error(None) or b"").decode())

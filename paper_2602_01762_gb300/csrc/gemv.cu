@@ -589,7 +589,8 @@ cudaError_t prepare_gemv_kernels() {
 }
 
 bool gemv_supported(const GemvArgs &a, bool bf16) {
-    if (bf16 && gemv_mma_supported(a)) return true;
+    // launch_gemv takes the mma.sync kernel only when the CUDA-core one is not forced
+    if (bf16 && !a.force_cuda_core && gemv_mma_supported(a)) return true;
     int tc;
     RingPlan pl;
     size_t smem;

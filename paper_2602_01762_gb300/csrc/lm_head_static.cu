@@ -74,6 +74,20 @@ prism_status reject(prism_status s, const std::string &msg) {
 
 bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
 
+// True when p is memory the current device dev can address as its own:
+// device memory of dev, or managed memory.  Host pointers and other devices'
+// memory are refused before any launch.
+bool on_device(const void *p, int dev) {
+    if (!p) return true;
+    cudaPointerAttributes at{};
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    if (at.type == cudaMemoryTypeManaged) return true;
+    return at.type == cudaMemoryTypeDevice && at.device == dev;
+}
+
 }  // namespace
 
 extern "C" prism_status prism_lm_head_topk_static(int32_t dtype, int32_t hidden, int32_t vocab,
@@ -97,6 +111,14 @@ extern "C" prism_status prism_lm_head_topk_static(int32_t dtype, int32_t hidden,
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return reject(PRISM_ERR_CUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));
     if (dev < 0 || dev >= kMaxDevices) return reject(PRISM_ERR_CAPACITY, "device ordinal beyond the static setup table");
+    {
+        const void *ptrs[] = {h, g_final, lm_head, draft, topk_ids, topk_logits, logits, dev_flags};
+        const char *names[] = {"h", "g_final", "lm_head", "draft", "topk_ids", "topk_logits", "logits", "dev_flags"};
+        for (int i = 0; i < 8; ++i)
+            if (!on_device(ptrs[i], dev))
+                return reject(PRISM_ERR_INVALID_ARG, std::string(names[i]) + " is not device memory of the current device " +
+                                                         std::to_string(dev));
+    }
     DeviceState st;
     prism_status ps = setup_device(dev, st);
     if (ps != PRISM_OK) return ps;
