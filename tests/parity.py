@@ -8,14 +8,19 @@ How it is applied:
   * per step from a common state (teacher forcing: step k recomputed from the
     oracle's state after step k-1) and on step 1 of every round: the full
     bar, strictly;
-  * along the free-running K-step chain: relative L2 on every step, and draft
-    ids equal wherever the margin exceeds both MARGIN and twice the measured
-    max-abs logit deviation of that step.  The chain re-rounds h^ to bf16 at
-    every step, so fp32-vs-fp64 differences of ~1e-7 flip occasional bf16
-    roundings and grow step by step; on the Llama-shaped drafters a single
-    one-ulp change of one input element moves the oracle's OWN logits by more
-    than ATOL after a few steps, so no fp32 implementation can promise ATOL
-    there;
+  * along the free-running K-step chain: relative L2 on every step; max-abs
+    within ENVELOPE_FACTOR times the oracle's own sensitivity envelope (below),
+    and never held above that; draft ids equal wherever the margin exceeds
+    both MARGIN and twice the measured max-abs logit deviation of that step.
+    The chain rounds every activation operand to bf16, so fp32-vs-fp64
+    differences of ~1e-7 flip occasional bf16 roundings, and each flip
+    cascades through the later steps.  ``one_ulp_envelope`` measures this on
+    the oracle itself, on the same weights and inputs: it moves one element of
+    the last input hidden row by one ulp of its storage type and records how
+    far the oracle's own logits move at every step.  On the Llama-3-8B shape
+    that move is already 0.011-0.016 at step 1 and 0.038-0.043 at step 5
+    (above ATOL), so no fp32 implementation can promise ATOL along the chain;
+    the GPU is held to the same order as the oracle's distance from itself;
   * after a (margin-exempt) id difference the two chains legitimately
     diverge, so later steps of that sequence are not compared;
   * KV rows the round must not touch are bit-identical; written rows and h^
@@ -28,11 +33,50 @@ import numpy as np
 MARGIN = 1e-2
 ATOL = 3e-2
 REL_L2 = 1e-2
+# Free-running bar: the GPU's max-abs deviation at step k may be at most this
+# many times the oracle's own largest move under a one-ulp input change.  Two
+# realisations of the chain's rounding decisions (the GPU's and the oracle's)
+# each sit about one envelope away from a third, so their distance is bounded
+# by about two envelopes.
+ENVELOPE_FACTOR = 2.0
 
 
 def rel_l2(a, b):
     a, b = np.asarray(a, np.float64), np.asarray(b, np.float64)
     return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
+
+
+def one_ulp_envelope(shape, W, I, seqs, base, *, trials: int = 3, round_acts: bool | None = None):
+    """The oracle's own sensitivity along the chain: for each sequence of
+    ``seqs``, ``trials`` oracle rounds each with ONE element of the last input
+    hidden row moved by one ulp of its storage type (bf16 or fp32), compared
+    with the unperturbed oracle round ``base`` (same seqs, with logits).
+    Returns [len(seqs), K]: per step the largest max-abs logit move over the
+    trials, made non-decreasing along the steps.  A trial stops counting at
+    the first step where its draft id differs from ``base`` (after that the
+    two chains draft different tokens, which is not a rounding effect).
+    ``round_acts`` is passed to the oracle (False: fp32 activations; ``base``
+    must then be computed the same way)."""
+    import oracle
+    K, d = shape.n_steps, shape.hidden
+    env = np.zeros((len(seqs), K))
+    for t in range(trials):
+        hid = I["hidden"].copy()
+        e = (t + 1) * d // (trials + 1)
+        for b in seqs:
+            i = int(I["n_new"][b]) - 1
+            if hid.dtype == np.uint16:
+                hid[b, i, e] = np.uint16(hid[b, i, e] + 1)
+            else:
+                hid[b, i, e] = np.nextafter(hid[b, i, e], np.float32(np.inf))
+        o = oracle.draft_round(shape, W, dict(I, hidden=hid), topk=1, want_logits=True, want_hidden=False,
+                               seqs=seqs, round_acts=round_acts)
+        for j in range(len(seqs)):
+            for k in range(K):
+                env[j, k] = max(env[j, k], float(np.max(np.abs(o["logits"][j, k] - base["logits"][j, k]))))
+                if o["draft_ids"][j, k] != base["draft_ids"][j, k]:
+                    break
+    return np.maximum.accumulate(env, axis=1)
 
 
 def _as_f64(cache):
@@ -43,16 +87,19 @@ def _as_f64(cache):
 
 
 def compare_round(gpu: dict, orc: dict, inputs: dict, seqs, K: int, topk: int, *,
-                  chain: bool = False, report: dict | None = None):
+                  chain: bool = False, envelope=None, report: dict | None = None):
     """gpu: device outputs as numpy over the full batch; orc: oracle outputs
-    over the sequences `seqs` (in that order).  Raises AssertionError."""
+    over the sequences `seqs` (in that order); envelope: for a free-running
+    chain, ``one_ulp_envelope`` of the same round.  Raises AssertionError."""
     rep = report if report is not None else {}
     for key in ("ids_compared", "ids_exempt"):
         rep.setdefault(key, 0)
-    for key in ("max_abs_logit", "max_rel_l2_logit", "max_rel_l2_hidden", "max_abs_logit_step1"):
+    for key in ("max_abs_logit", "max_rel_l2_logit", "max_rel_l2_hidden", "max_abs_logit_step1",
+                "max_envelope", "max_abs_over_envelope"):
         rep.setdefault(key, 0.0)
     have_logits = gpu.get("logits") is not None and orc.get("logits") is not None
     assert have_logits or not chain, "the chain comparison needs logits"
+    assert envelope is not None or not chain, "the chain comparison needs the oracle's one-ulp envelope"
     for j, b in enumerate(seqs):
         for k in range(K):
             o_top = orc["topk_logits"][j, k]
@@ -69,6 +116,13 @@ def compare_round(gpu: dict, orc: dict, inputs: dict, seqs, K: int, topk: int, *
                     rep["max_abs_logit_step1"] = max(rep["max_abs_logit_step1"], ma)
                 if not chain or k == 0:
                     assert ma <= ATOL, f"seq {b} step {k + 1}: logit max-abs {ma:.3e} > {ATOL}"
+                else:
+                    env = float(envelope[j, k])
+                    rep["max_envelope"] = max(rep["max_envelope"], env)
+                    rep["max_abs_over_envelope"] = max(rep["max_abs_over_envelope"], ma / max(env, 1e-30))
+                    bar = max(ATOL, ENVELOPE_FACTOR * env)
+                    assert ma <= bar, (f"seq {b} step {k + 1}: logit max-abs {ma:.3e} > {bar:.3e} "
+                                       f"({ENVELOPE_FACTOR} x the oracle's one-ulp envelope {env:.3e})")
                 assert rl <= REL_L2, f"seq {b} step {k + 1}: logit rel-L2 {rl:.3e} > {REL_L2}"
             if gpu.get("hidden_out") is not None and orc.get("hidden_out") is not None:
                 rh = rel_l2(gpu["hidden_out"][b, k], orc["hidden_out"][j, k])

@@ -16,7 +16,7 @@ import synth
 from synth.workloads import Shape, Workload
 from tests.gpu_harness import (GpuModel, forced_step_inputs, gpu_round, oracle_step, run_round,
                                sample_seqs)
-from tests.parity import compare_cache, compare_round
+from tests.parity import compare_cache, compare_round, one_ulp_envelope
 
 pytestmark = pytest.mark.gpu
 
@@ -45,7 +45,8 @@ def _check(w, W, I, seqs, *, topk, options=None):
         # one candidate more than is compared: the margin of the last compared
         # rank is its gap to the next one
         o = oracle.draft_round(w.shape, W, I, topk=topk + 1, want_logits=True, seqs=seqs)
-        rep = compare_round(g, o, I, seqs, K, topk, chain=True)
+        env = one_ulp_envelope(w.shape, W, I, seqs, o)
+        rep = compare_round(g, o, I, seqs, K, topk, chain=True, envelope=env)
         compare_cache(g["k_cache"], g["v_cache"], o["k_cache"], o["v_cache"], I, seqs, K)
         forced = {}
         for k in range(2, K + 1):
@@ -111,7 +112,8 @@ def test_fallback_projection_kernels_match_oracle(options):
     g = gpu_round(MID_W, W, I, topk=8, options=options)
     assert g["flags"] == 0
     o = oracle.draft_round(MID_W.shape, W, I, topk=8, want_logits=True, seqs=[0, 1, 2])
-    compare_round(g, o, I, [0, 1, 2], MID_W.shape.n_steps, 8, chain=True)
+    env = one_ulp_envelope(MID_W.shape, W, I, [0, 1, 2], o)
+    compare_round(g, o, I, [0, 1, 2], MID_W.shape.n_steps, 8, chain=True, envelope=env)
     compare_cache(g["k_cache"], g["v_cache"], o["k_cache"], o["v_cache"], I, [0, 1, 2], MID_W.shape.n_steps)
 
 
@@ -237,7 +239,7 @@ def test_round_then_accept_then_next_round():
     W, I = synth.make_weights(w), synth.make_round_inputs(w, max_new=K + 1)
     g = gpu_round(w, W, I, topk=2, keep=True)
     o = oracle.draft_round(w.shape, W, I, topk=2, want_logits=True)
-    compare_round(g, o, I, [0, 1], K, 2, chain=True)
+    compare_round(g, o, I, [0, 1], K, 2, chain=True, envelope=one_ulp_envelope(w.shape, W, I, [0, 1], o))
     assert np.array_equal(g["draft_ids"], o["draft_ids"])
     target = synth.make_targets(w, o["draft_ids"])
     exp = oracle.accept_greedy(o["draft_ids"], target, I["n_new"], I["kv_len"])
@@ -264,7 +266,8 @@ def test_round_then_accept_then_next_round():
     I2_orc = next_inputs(exp["accept_len"], exp["out_tokens"], exp["kv_len"], o["k_cache"], o["v_cache"])
     g2 = gpu_round(w, W, I2_gpu, topk=2)
     o2 = oracle.draft_round(w.shape, W, I2_orc, topk=2, want_logits=True)
-    compare_round(g2, o2, I2_gpu, [0, 1], K, 2, chain=True)
+    compare_round(g2, o2, I2_gpu, [0, 1], K, 2, chain=True,
+                  envelope=one_ulp_envelope(w.shape, W, I2_orc, [0, 1], o2))
     compare_cache(g2["k_cache"], g2["v_cache"], o2["k_cache"], o2["v_cache"], I2_gpu, [0, 1], K)
 
 

@@ -4,9 +4,17 @@ through the C ABI.
 The oracle recomputes the GPU's own tree (``follow``: the GPU's candidate
 tokens and frontier choices), so every processed row can be compared.  Along
 the tree the hidden state is re-rounded to bf16 at every step, exactly as in
-the chain, so the bar is the chain's: step 1 strictly (max-abs and relative
-L2), later steps by relative L2 with id and order decisions compared where
-the oracle's gaps exceed max(MARGIN, twice the measured max-abs deviation).
+the chain, so the bar is the chain's:
+  * step 1 strictly (max-abs and relative L2);
+  * later steps of the free-running tree by relative L2, and max-abs within
+    ENVELOPE_FACTOR times the oracle's own one-ulp envelope of the same tree
+    (``tree_envelope``); id and order decisions compared where the oracle's
+    gaps exceed max(MARGIN, twice the measured max-abs deviation);
+  * every row of steps 2..K once more from the oracle's own state (teacher
+    forcing, ``forced_tree_rows``): the row's token, its emitting row's h^ and
+    a cache holding the oracle's committed rows and the row's ancestors, run
+    on the GPU as a one-step round, strictly: max-abs, relative L2 and the
+    row's candidates wherever the oracle's gaps exceed MARGIN.
 Decisions the GPU takes from its own numbers (frontiers, the verified tree,
 its structure) are checked exactly against a re-sort of those numbers.
 """
@@ -21,7 +29,7 @@ import oracle
 import synth
 from synth.workloads import Shape, Workload
 from tests.gpu_harness import GpuModel
-from tests.parity import ATOL, MARGIN, REL_L2, _as_f64, rel_l2
+from tests.parity import ATOL, ENVELOPE_FACTOR, MARGIN, REL_L2, _as_f64, rel_l2
 
 pytestmark = pytest.mark.gpu
 
@@ -117,14 +125,128 @@ def check_self_consistent(g, K, w, m):
             assert g["tree_scores"][b, i] == g["pool_scores"][b, e]
 
 
-def compare_tree(g, o, I, seqs, K, w, m, report):
-    """g: GPU outputs over the full batch; o: the oracle following g's tree on `seqs`."""
+def tree_envelope(shape, W, I, seqs, follow, base, *, width, n_nodes, trials: int = 3):
+    """The oracle's own sensitivity along the tree: ``trials`` oracle tree
+    rounds following the same tree (``follow``), each with ONE element of the
+    last input hidden row of every sequence moved by one ulp of its storage
+    type, against the unperturbed oracle tree ``base``.  Returns [len(seqs),
+    K]: per step the largest max-abs move of any row's logits over the
+    trials, made non-decreasing along the steps."""
+    K, d = shape.n_steps, shape.hidden
+    env = np.zeros((len(seqs), K))
+    for t in range(trials):
+        hid = I["hidden"].copy()
+        e = (t + 1) * d // (trials + 1)
+        for b in seqs:
+            i = int(I["n_new"][b]) - 1
+            if hid.dtype == np.uint16:
+                hid[b, i, e] = np.uint16(hid[b, i, e] + 1)
+            else:
+                hid[b, i, e] = np.nextafter(hid[b, i, e], np.float32(np.inf))
+        o = oracle.draft_tree(shape, W, dict(I, hidden=hid), width=width, n_nodes=n_nodes, follow=follow,
+                              seqs=seqs)
+        move = np.abs(o["row_logits"] - base["row_logits"]).max(axis=(2, 3))      # [seqs, K]
+        env = np.maximum(env, move)
+    return np.maximum.accumulate(env, axis=1)
+
+
+def _tree_row_path(g, b, k, j, w):
+    """(emitting step, emitting row) of row j of step k >= 2 of sequence b in
+    the GPU's tree, and the rows (step, row) of its ancestors at steps
+    2..k-1, nearest first."""
+    def emitter(kk, jj):
+        parent = int(g["frontier"][b, kk - 2, jj])
+        if parent < w:
+            return 1, 0
+        return kk - 1, (parent - (w + (kk - 3) * w * w)) // w
+    em = emitter(k, j)
+    anc = []
+    cur = em
+    while cur[0] >= 2:
+        anc.append(cur)
+        cur = emitter(*cur)
+    return em, anc
+
+
+def forced_tree_rows(w, W, I, g, o, seqs, width, model, report):
+    """Every row of steps 2..K recomputed on the GPU from the oracle's state.
+
+    A tree row at step k is the chain's row at position L + n + k - 2 whose
+    visible keys are the committed and prefill rows plus its ancestors'
+    rows (Sec. 3.2's recurrence along one path of the tree; the oracle pins
+    show the two equal).  So each row runs as a one-step round of step k's
+    module: token = the row's candidate token, hidden = the oracle's h^ of
+    the emitting row (rounded to the storage type, as the fusion input is),
+    cache = the oracle's rows [0, L + n) followed by the oracle's ancestor
+    rows at the positions L + n + i - 2 of their steps i, and kv_len =
+    L + n + k - 2.  ``o`` must hold ``row_hidden`` and the oracle's caches.
+    Returns the number of rows compared."""
+    from tests.gpu_harness import run_round
+    K, V = w.shape.n_steps, w.shape.vocab
+    bf16 = I["hidden"].dtype == np.uint16
+    rows = 0
+    for k in range(2, K + 1):
+        items = [(jj, b, j) for jj, b in enumerate(seqs) for j in range(width)]
+        Bf = len(items)
+        hsh = I["k_cache"].shape
+        kc = np.zeros((Bf,) + hsh[1:], I["k_cache"].dtype)
+        vc = np.zeros_like(kc)
+        tokens = np.zeros((Bf, 1), np.int32)
+        hidden = np.zeros((Bf, 1, w.shape.hidden), I["hidden"].dtype)
+        kv = np.zeros(Bf, np.int32)
+        for f, (jj, b, j) in enumerate(items):
+            L, n = int(I["kv_len"][b]), int(I["n_new"][b])
+            (ek, ej), anc = _tree_row_path(g, b, k, j, width)
+            parent = int(g["frontier"][b, k - 2, j])
+            tokens[f, 0] = g["pool_tokens"][b, parent]
+            h = o["row_hidden"][jj, ek - 1, ej]
+            hidden[f, 0] = oracle.to_bf16_bits(h) if bf16 else h.astype(np.float32)
+            kc[f, :, :L + n] = o["k_cache"][jj, :, :L + n]
+            vc[f, :, :L + n] = o["v_cache"][jj, :, :L + n]
+            for (ak, aj) in anc:
+                slot, pos = L + n + (ak - 2) * width + aj, L + n + ak - 2
+                kc[f, :, pos] = o["k_cache"][jj, :, slot]
+                vc[f, :, pos] = o["v_cache"][jj, :, slot]
+            kv[f] = L + n + k - 2
+        Ik = {"tokens": tokens, "hidden": hidden, "n_new": np.ones(Bf, np.int32), "kv_len": kv,
+              "k_cache": kc, "v_cache": vc, "max_ctx": I["max_ctx"]}
+        dr = model.drafter(w.shape, [W["f_map"][k - 1]], max_batch=Bf, max_ctx=int(I["max_ctx"]), max_new=1,
+                           topk=width)
+        gk = run_round(dr, Ik, n_steps=1, topk=width)
+        dr.close()
+        assert gk["flags"] == 0, f"device error word {gk['flags']}"
+        for f, (jj, b, j) in enumerate(items):
+            zg, zo = gk["logits"][f, 0].astype(np.float64), o["row_logits"][jj, k - 1, j]
+            ma, rl = float(np.max(np.abs(zg - zo))), rel_l2(zg, zo)
+            report["forced_max_abs_logit"] = max(report.get("forced_max_abs_logit", 0.0), ma)
+            assert ma <= ATOL, f"seq {b} step {k} row {j} (forced): logit max-abs {ma:.3e}"
+            assert rl <= REL_L2, f"seq {b} step {k} row {j} (forced): logit rel-L2 {rl:.3e}"
+            order = np.lexsort((np.arange(V), -zo))
+            top = zo[order[:width + 1]]
+            for r in range(width):
+                lo = top[r - 1] - top[r] if r > 0 else np.inf
+                if min(lo, top[r] - top[r + 1]) > MARGIN:
+                    report["forced_ids_compared"] = report.get("forced_ids_compared", 0) + 1
+                    assert gk["topk_ids"][f, 0, r] == order[r], f"seq {b} step {k} row {j} (forced): candidate {r}"
+            # the row's own key and value, at its chain position and at its tree slot
+            L, n = int(I["kv_len"][b]), int(I["n_new"][b])
+            pos, slot = L + n + k - 2, L + n + (k - 2) * width + j
+            for gc, oc in ((gk["k_cache"], o["k_cache"]), (gk["v_cache"], o["v_cache"])):
+                assert rel_l2(_as_f64(gc[f, :, pos]), _as_f64(oc[jj, :, slot])) <= REL_L2
+            rows += 1
+    return rows
+
+
+def compare_tree(g, o, I, seqs, K, w, m, report, envelope):
+    """g: GPU outputs over the full batch; o: the oracle following g's tree on
+    `seqs`; envelope: ``tree_envelope`` of the same tree."""
     rep = report
     for key in ("rows", "ids_compared", "frontier_compared", "tree_compared"):
         rep.setdefault(key, 0)
     rep.setdefault("max_abs_logit", 0.0)
     rep.setdefault("max_rel_l2_logit", 0.0)
     rep.setdefault("max_score_err", 0.0)
+    rep.setdefault("max_abs_over_envelope", 0.0)
     for jj, b in enumerate(seqs):
         ma_row = {}
         for k in range(1, K + 1):
@@ -142,6 +264,12 @@ def compare_tree(g, o, I, seqs, K, w, m, report):
                 ma_row[(k, j)] = ma
                 if k == 1:
                     assert ma <= ATOL, f"seq {b} step 1: logit max-abs {ma:.3e}"
+                else:
+                    env = float(envelope[jj, k - 1])
+                    rep["max_abs_over_envelope"] = max(rep["max_abs_over_envelope"], ma / max(env, 1e-30))
+                    bar = max(ATOL, ENVELOPE_FACTOR * env)
+                    assert ma <= bar, (f"seq {b} step {k} row {j}: logit max-abs {ma:.3e} > {bar:.3e} "
+                                       f"({ENVELOPE_FACTOR} x the oracle's one-ulp envelope {env:.3e})")
                 assert rl <= REL_L2, f"seq {b} step {k} row {j}: logit rel-L2 {rl:.3e}"
                 thr = max(MARGIN, 2 * ma) if k > 1 else MARGIN
                 # the row's w candidates: the oracle's best w where its gaps allow
@@ -206,17 +334,26 @@ def compare_tree_cache(g, o, I, seqs, K, w):
             assert rel_l2(got, exp) <= REL_L2, f"seq {b}: tree KV rows rel-L2 {rel_l2(got, exp):.3e}"
 
 
-def run_case(w, W, I, seqs, *, width=None, n_nodes=None, options=None):
+def run_case(w, W, I, seqs, *, width=None, n_nodes=None, options=None, forced=True):
     width = width or w.tree_width
     n_nodes = n_nodes or w.tree_nodes
     K = w.shape.n_steps
-    g = gpu_tree(w, W, I, width=width, n_nodes=n_nodes, options=options)
-    assert g["flags"] == 0, f"device error word {g['flags']}"
-    check_self_consistent(g, K, width, n_nodes)
-    follow = {"pool_tokens": g["pool_tokens"][seqs], "frontier": g["frontier"][seqs]}
-    o = oracle.draft_tree(w.shape, W, I, width=width, n_nodes=n_nodes, follow=follow, seqs=seqs)
-    rep = compare_tree(g, o, I, seqs, K, width, n_nodes, {})
-    compare_tree_cache(g, o, I, seqs, K, width)
+    model = GpuModel(W)
+    try:
+        g = gpu_tree(w, W, I, width=width, n_nodes=n_nodes, options=options, model=model)
+        assert g["flags"] == 0, f"device error word {g['flags']}"
+        check_self_consistent(g, K, width, n_nodes)
+        follow = {"pool_tokens": g["pool_tokens"][seqs], "frontier": g["frontier"][seqs]}
+        o = oracle.draft_tree(w.shape, W, I, width=width, n_nodes=n_nodes, follow=follow, seqs=seqs,
+                              want_hidden=forced)
+        env = tree_envelope(w.shape, W, I, seqs, follow, o, width=width, n_nodes=n_nodes)
+        rep = compare_tree(g, o, I, seqs, K, width, n_nodes, {}, env)
+        compare_tree_cache(g, o, I, seqs, K, width)
+        if forced and K > 1:
+            rep["forced_rows"] = forced_tree_rows(w, W, I, g, o, seqs, width, model, rep)
+            assert rep["forced_rows"] == len(seqs) * (K - 1) * width
+    finally:
+        model.close()
     return g, o, rep
 
 
