@@ -367,7 +367,12 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * 0: the warp-level mma.sync kernel), "attn_fused" (1, the default: RoPE,
  * KV append and attention run as one kernel, a cluster of up to 8 CTAs per
  * sequence and KV head merging through distributed shared memory; 0: a
- * RoPE/append kernel, then split-KV attention with a last-CTA merge).
+ * RoPE/append kernel, then split-KV attention with a last-CTA merge),
+ * "fuse_rows" (1, the default: a streamed projection's last kernel, the
+ * split-K finish or the LM head's top-k merge, also writes the next
+ * projection's bf16 activation rows, its RMSNorm or the next step's fusion
+ * input, so that the next projection needs no row-preparation kernel; 0:
+ * a preparation kernel before each projection).
  * Changing an option drops cached graphs.  Errors: INVALID_ARG (unknown name
  * or value out of range). */
 prism_status prism_set_option(prism_ctx *ctx, const char *name, int32_t value);

@@ -33,12 +33,6 @@ __device__ __forceinline__ void pdl_wait() {
     asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
-// Bulk (TMA-engine) prefetch of a contiguous byte range into L2.  Address and
-// size must be multiples of 16 bytes.
-__device__ __forceinline__ void prefetch_l2_bulk(const void *p, uint32_t bytes) {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
-
 // 128-bit streaming load of read-only data: not kept in L1.
 __device__ __forceinline__ uint4 ldg_stream(const uint4 *p) {
     uint4 r;
@@ -59,6 +53,10 @@ __device__ __forceinline__ uint16_t f32_to_bf16(float f) {
     uint32_t u = __float_as_uint(f);
     u += 0x7FFFu + ((u >> 16) & 1u);
     return (uint16_t)(u >> 16);
+}
+// Two floats as adjacent bf16 values in one word (the first at the lower address).
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    return (uint32_t)f32_to_bf16(lo) | ((uint32_t)f32_to_bf16(hi) << 16);
 }
 __device__ __forceinline__ float round_bf16(float f) {
     return __uint_as_float((uint32_t)f32_to_bf16(f) << 16);
@@ -179,6 +177,15 @@ struct GemvArgs {
     // ring plan knobs: target stage bytes, smem budget bytes, consumer groups;
     // force_cuda_core selects the CUDA-core kernel for bf16 too
     int chunk_target, smem_budget, groups, force_cuda_core;
+    // streamed projections: the next projection's bf16 activation rows
+    // [T][kin of the next projection], written by this projection's last
+    // kernel so that the next one needs no row preparation.  next_norm: the
+    // split-K finish writes RMSNorm(out row) * next_gain (next_gain null: the
+    // row as it is), rounded.  next_fuse: the LM head's top-k merge writes the
+    // next decode step's fusion row [E(chosen token); round(src row)].
+    uint16_t *next_x;
+    const void *next_gain;
+    int next_norm, next_fuse;
 };
 
 struct RopeArgs {
@@ -343,8 +350,10 @@ cudaError_t launch_gemv_tc(const GemvArgs &a, const CUtensorMap &m, int sms, flo
 // the cross-CTA merge kernel.
 bool gemv_tcs_supported(const GemvArgs &a, int sms);
 size_t gemv_tcs_workspace_floats(const GemvArgs &a, int sms);
+// *next_done (may be null) reports whether the launch also wrote the next
+// projection's rows (a.next_norm or a.next_fuse) into a.next_x.
 cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, float *part, int *tile_ctr,
-                            uint16_t *xbuf, cudaStream_t s, bool pdl);
+                            uint16_t *xbuf, cudaStream_t s, bool pdl, bool *next_done = nullptr);
 cudaError_t prepare_attention_kernel(bool bf16, int D, int chunk, int G, int splits);
 // Sets kernel attributes; *max_cs receives the largest cluster size (8 or 16)
 // for which `need` clusters can be resident at once.

@@ -933,34 +933,62 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             int s = 0, issued = 0;
             uint32_t ph = 0;
             bool dead = false;
-            bool x_ready = false;      // X is the previous kernel's output: wait before the first X box
-            for (int i = 0; i < my_tiles && !dead; ++i) {
-                const int tile = blockIdx.x / p.splits + i * tiles_step;
-                for (int q = 0; q < n_kst; ++q) {
-                    if (!mbar_wait(&empty[s], ph ^ 1)) {
-                        set_err(a.err, kErrTimeout);
-                        dead = true;
-                        break;
-                    }
-                    if (!x_ready) {
-                        pdl_wait();
-                        x_ready = true;
-                    }
-                    const int kbs = kb0 + q * p.kb_per_stage;
-                    const int nkb = kb1 - kbs < p.kb_per_stage ? kb1 - kbs : p.kb_per_stage;
-                    mbar_arrive_tx(&full[s], (uint32_t)nkb * kb_bytes);
-                    const uint32_t st = saddr(ring) + (uint32_t)s * p.stage_bytes;
-                    for (int j = 0; j < nkb; ++j) {
+            const int total = my_tiles * n_kst;
+            // item f of this CTA: tile, first K block and K blocks of its stage
+            auto item = [&](int f, int &tile, int &kbs, int &nkb) {
+                tile = blockIdx.x / p.splits + (f / n_kst) * tiles_step;
+                kbs = kb0 + (f % n_kst) * p.kb_per_stage;
+                nkb = kb1 - kbs < p.kb_per_stage ? kb1 - kbs : p.kb_per_stage;
+            };
+            auto load_w = [&](int f, int stage) {
+                int tile, kbs, nkb;
+                item(f, tile, kbs, nkb);
+                const uint32_t st = saddr(ring) + (uint32_t)stage * p.stage_bytes;
+                for (int j = 0; j < nkb; ++j)
 #pragma unroll
-                        for (int r = 0; r < RPW; ++r)
-                            tma_load_2d(st + (uint32_t)j * kb_bytes + (uint32_t)r * kBoxBytes, &tmW, (kbs + j) * kBoxK,
-                                        tile * kTileM + r * a.pair_offset, &full[s]);
-                        tma_load_2d(st + (uint32_t)j * kb_bytes + RPW * kBoxBytes, &tmX, (kbs + j) * kBoxK, 0,
-                                    &full[s]);
-                    }
-                    ++issued;
-                    if (++s == S) { s = 0; ph ^= 1; }
+                    for (int r = 0; r < RPW; ++r)
+                        tma_load_2d(st + (uint32_t)j * kb_bytes + (uint32_t)r * kBoxBytes, &tmW, (kbs + j) * kBoxK,
+                                    tile * kTileM + r * a.pair_offset, &full[stage]);
+            };
+            auto load_x = [&](int f, int stage) {
+                int tile, kbs, nkb;
+                item(f, tile, kbs, nkb);
+                const uint32_t st = saddr(ring) + (uint32_t)stage * p.stage_bytes;
+                for (int j = 0; j < nkb; ++j)
+                    tma_load_2d(st + (uint32_t)j * kb_bytes + RPW * kBoxBytes, &tmX, (kbs + j) * kBoxK, 0, &full[stage]);
+            };
+            auto arm = [&](int f, int stage) {
+                int tile, kbs, nkb;
+                item(f, tile, kbs, nkb);
+                mbar_arrive_tx(&full[stage], (uint32_t)nkb * kb_bytes);
+            };
+            // The first ring pass: the stages are free (fresh barriers), and the
+            // weight boxes do not depend on the previous kernel, so they are
+            // requested before the dependency wait; X is the previous kernel's
+            // output, so its boxes of those stages follow the wait.  Each stage's
+            // barrier expects both from the start, so it completes only when both
+            // have landed.
+            const int pre = total < S ? total : S;
+            for (int f = 0; f < pre; ++f) {
+                arm(f, f);
+                load_w(f, f);
+            }
+            pdl_wait();
+            for (int f = 0; f < pre; ++f) load_x(f, f);
+            issued = pre;
+            s = pre % S;
+            ph = pre == S ? 1u : 0u;
+            for (int f = pre; f < total; ++f) {
+                if (!mbar_wait(&empty[s], ph ^ 1)) {
+                    set_err(a.err, kErrTimeout);
+                    dead = true;
+                    break;
                 }
+                arm(f, s);
+                load_w(f, s);
+                load_x(f, s);
+                ++issued;
+                if (++s == S) { s = 0; ph ^= 1; }
             }
             const int first = issued > S ? issued - S : 0;
             for (int i = first; i < issued; ++i)
@@ -1166,6 +1194,7 @@ __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int g
         for (int i = 0; i < kTopK; ++i) s_k[w][i] = l[i];
     }
     __syncthreads();
+    __shared__ int s_tok;
     if (w == 0) {
 #pragma unroll
         for (int i = 0; i < kTopK; ++i) l[i] = lane < 4 ? s_k[lane][i] : 0ull;
@@ -1173,6 +1202,108 @@ __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int g
 #pragma unroll
         for (int m = 1; m < 32; m <<= 1) key_merge_xor(l, m);
         write_row(a, t, l);
+        if (lane == 0) {
+            float v;
+            int id;
+            unpack_best(l[0], v, id);
+            s_tok = id;
+        }
+    }
+    if (a.next_fuse) {
+        // the next decode step's fusion row: [E(token); round(h^ row t)]
+        __syncthreads();
+        const int d = a.d;
+        const uint4 *e = (const uint4 *)((const uint16_t *)a.embed + (size_t)token_ok(a, s_tok) * d);
+        const float4 *h = (const float4 *)(a.src + (size_t)t * d);
+        uint4 *x = (uint4 *)(a.next_x + (size_t)t * 2 * d);
+        for (int c = threadIdx.x; c < d / 8; c += 128) {
+            const uint4 ev = __ldg(e + c);
+            const float4 h0 = __ldcg(h + 2 * c), h1 = __ldcg(h + 2 * c + 1);
+            x[c] = ev;
+            x[d / 8 + c] = make_uint4(pack_bf16x2(h0.x, h0.y), pack_bf16x2(h0.z, h0.w), pack_bf16x2(h1.x, h1.y),
+                                      pack_bf16x2(h1.z, h1.w));
+        }
+    }
+}
+
+// Split-K sums of one activation row per CTA (Store and Resid epilogues of a
+// streamed projection), in slice order like splitk_finish_kernel, and the
+// next projection's activation row: RMSNorm of the finished row with
+// next_gain (or the row as it is when next_gain is null), rounded to bf16,
+// into next_x.  One kernel instead of the finish and the next row
+// preparation.  Dynamic shared memory: the row, n_units floats.
+constexpr int kRowThreads = 512;
+__global__ void __launch_bounds__(kRowThreads) splitk_finish_row_kernel(const GemvArgs a, const float *part,
+                                                                      int splits) {
+    extern __shared__ float rowv[];
+    __shared__ float red[kRowThreads / 32];
+    pdl_trigger();
+    pdl_wait();
+    const int t = blockIdx.x, n = a.n_units, tid = threadIdx.x;
+    const int rrow = a.epi == kEpiResid && a.resid_prefill_rows ? t * a.max_new + clamp_n(a, t) - 1 : t;
+    float ss = 0.f;
+    for (int u = tid * 4; u < n; u += kRowThreads * 4) {
+        float4 v[kMaxSplits];
+#pragma unroll
+        for (int k = 0; k < kMaxSplits; ++k)
+            if (k < splits) v[k] = __ldcg((const float4 *)&part[((size_t)k * a.T + t) * n + u]);
+        float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int k = 0; k < kMaxSplits; ++k)
+            if (k < splits) {
+                r.x += v[k].x;
+                r.y += v[k].y;
+                r.z += v[k].z;
+                r.w += v[k].w;
+            }
+        if (a.epi == kEpiResid) {
+            const float4 q = __ldcg((const float4 *)&a.resid[(size_t)rrow * a.out_ld + u]);
+            r.x += q.x;
+            r.y += q.y;
+            r.z += q.z;
+            r.w += q.w;
+            if (a.hidden_out) {
+                float *ho = a.hidden_out + ((size_t)t * a.K + a.step - 1) * a.d + u;
+                ho[0] = r.x;
+                ho[1] = r.y;
+                ho[2] = r.z;
+                ho[3] = r.w;
+            }
+        }
+        *(float4 *)&a.out[(size_t)t * a.out_ld + u] = r;
+        *(float4 *)&rowv[u] = r;
+        ss = fmaf(r.x, r.x, ss);
+        ss = fmaf(r.y, r.y, ss);
+        ss = fmaf(r.z, r.z, ss);
+        ss = fmaf(r.w, r.w, ss);
+    }
+    if (!a.next_norm) return;
+    float inv = 1.f;
+    if (a.next_gain) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
+        if ((tid & 31) == 0) red[tid >> 5] = ss;
+    }
+    __syncthreads();
+    if (a.next_gain) {
+        float tot = 0.f;
+#pragma unroll
+        for (int i = 0; i < kRowThreads / 32; ++i) tot += red[i];
+        inv = 1.0f / sqrtf(tot / (float)n + a.eps);
+    }
+    const uint16_t *g = (const uint16_t *)a.next_gain;
+    uint2 *x = (uint2 *)(a.next_x + (size_t)t * n);
+    for (int u = tid * 4; u < n; u += kRowThreads * 4) {
+        const float4 r = *(const float4 *)&rowv[u];
+        float y[4] = {r.x, r.y, r.z, r.w};
+        if (g) {
+            const uint2 gw = __ldg((const uint2 *)(g + u));
+            y[0] = y[0] * inv * bf16lo(gw.x);
+            y[1] = y[1] * inv * bf16hi(gw.x);
+            y[2] = y[2] * inv * bf16lo(gw.y);
+            y[3] = y[3] * inv * bf16hi(gw.y);
+        }
+        x[u / 4] = make_uint2(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]));
     }
 }
 
@@ -1183,16 +1314,24 @@ __global__ void __launch_bounds__(256) prep_x_kernel(const GemvArgs a, uint16_t 
     __shared__ float red[8];
     pdl_trigger();
     pdl_wait();
+    // 16-byte vectors (d is a multiple of 8): a thread issues its loads of a
+    // row before using any
     const int t = blockIdx.x, tid = threadIdx.x;
     const int d = a.d, kin = a.kin;
-    uint16_t *xr = X + (size_t)t * kin;
+    uint4 *xr = (uint4 *)(X + (size_t)t * kin);
     if (a.pro == kProNorm) {
         const int sr = a.src_prefill_rows ? (t * a.max_new + clamp_n(a, t) - 1) : t;
-        const float *src = a.src + (size_t)sr * d;
+        const float4 *src = (const float4 *)(a.src + (size_t)sr * d);
         float inv = 1.f;
         if (a.gain) {
             float ss = 0.f;
-            for (int c = tid; c < d; c += 256) ss = fmaf(src[c], src[c], ss);
+            for (int c = tid; c < d / 4; c += 256) {
+                const float4 v = __ldcg(src + c);
+                ss = fmaf(v.x, v.x, ss);
+                ss = fmaf(v.y, v.y, ss);
+                ss = fmaf(v.z, v.z, ss);
+                ss = fmaf(v.w, v.w, ss);
+            }
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
             if ((tid & 31) == 0) red[tid >> 5] = ss;
@@ -1202,25 +1341,43 @@ __global__ void __launch_bounds__(256) prep_x_kernel(const GemvArgs a, uint16_t 
             for (int i = 0; i < 8; ++i) tot += red[i];
             inv = 1.0f / sqrtf(tot / (float)d + a.eps);
         }
-        const uint16_t *g = (const uint16_t *)a.gain;
-        for (int c = tid; c < d; c += 256) xr[c] = f32_to_bf16(a.gain ? src[c] * inv * bf16_to_f32(g[c]) : src[c]);
+        const uint4 *g = (const uint4 *)a.gain;
+        for (int c = tid; c < d / 8; c += 256) {
+            const float4 v0 = __ldcg(src + 2 * c), v1 = __ldcg(src + 2 * c + 1);
+            float y[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+            if (g) {
+                const uint4 gw = __ldg(g + c);
+                const uint32_t gg[4] = {gw.x, gw.y, gw.z, gw.w};
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    y[2 * i] = y[2 * i] * inv * bf16lo(gg[i]);
+                    y[2 * i + 1] = y[2 * i + 1] * inv * bf16hi(gg[i]);
+                }
+            }
+            xr[c] = make_uint4(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]), pack_bf16x2(y[4], y[5]),
+                               pack_bf16x2(y[6], y[7]));
+        }
     } else if (a.pro == kProFuseDecode) {
         const int tok = token_ok(a, a.draft[t * a.K + a.step - 2]);
-        const uint16_t *e = (const uint16_t *)a.embed + (size_t)tok * d;
-        const float *h = a.src + (size_t)t * d;
-        for (int c = tid; c < d; c += 256) {
-            xr[c] = e[c];
-            xr[d + c] = f32_to_bf16(h[c]);
+        const uint4 *e = (const uint4 *)((const uint16_t *)a.embed + (size_t)tok * d);
+        const float4 *h = (const float4 *)(a.src + (size_t)t * d);
+        for (int c = tid; c < d / 8; c += 256) {
+            const uint4 ev = __ldg(e + c);
+            const float4 h0 = __ldcg(h + 2 * c), h1 = __ldcg(h + 2 * c + 1);
+            xr[c] = ev;
+            xr[d / 8 + c] = make_uint4(pack_bf16x2(h0.x, h0.y), pack_bf16x2(h0.z, h0.w), pack_bf16x2(h1.x, h1.y),
+                                       pack_bf16x2(h1.z, h1.w));
         }
     } else if (a.pro == kProFusePrefill) {
         const int b = t / a.max_new, r = t % a.max_new;
         const bool valid = r < clamp_n(a, b);
         const int tok = valid ? token_ok(a, a.tokens[b * a.max_new + r]) : 0;
-        const uint16_t *e = (const uint16_t *)a.embed + (size_t)tok * d;
-        const uint16_t *h = (const uint16_t *)a.hidden_in + ((size_t)b * a.max_new + r) * d;
-        for (int c = tid; c < d; c += 256) {
-            xr[c] = valid ? e[c] : (uint16_t)0;
-            xr[d + c] = valid ? h[c] : (uint16_t)0;
+        const uint4 *e = (const uint4 *)((const uint16_t *)a.embed + (size_t)tok * d);
+        const uint4 *h = (const uint4 *)((const uint16_t *)a.hidden_in + ((size_t)b * a.max_new + r) * d);
+        const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+        for (int c = tid; c < d / 8; c += 256) {
+            xr[c] = valid ? __ldg(e + c) : z;
+            xr[d / 8 + c] = valid ? __ldg(h + c) : z;
         }
     }
 }
@@ -1455,7 +1612,8 @@ size_t gemv_tcs_workspace_floats(const GemvArgs &a, int sms) {
 }
 
 cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, float *part, int *tile_ctr,
-                            uint16_t *xbuf, cudaStream_t s, bool pdl) {
+                            uint16_t *xbuf, cudaStream_t s, bool pdl, bool *next_done) {
+    if (next_done) *next_done = false;
     TcPlan p{};
     int grid, NB;
     size_t smem;
@@ -1495,12 +1653,25 @@ cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, f
         case 128: e = dispatch_tcs<128>(a, p, mw, mx, grid, smem, s, pdl); break;
         default: e = dispatch_tcs<256>(a, p, mw, mx, grid, smem, s, pdl); break;
     }
-    if (e == cudaSuccess && a.epi == kEpiTopK)
-        e = launch_k(topk_merge_kernel, dim3(a.T), dim3(128), 0, s, true, a, grid);
+    if (e == cudaSuccess && a.epi == kEpiTopK) {
+        GemvArgs m = a;
+        m.next_fuse = a.next_fuse && a.next_x && a.d % 8 == 0;
+        e = launch_k(topk_merge_kernel, dim3(a.T), dim3(128), 0, s, true, m, grid);
+        if (e == cudaSuccess && next_done) *next_done = m.next_fuse != 0;
+    }
     if (e == cudaSuccess && p.defer) {
-        const dim3 fg((unsigned)(((long)a.T * a.n_units + 255) / 256));
-        e = a.epi == kEpiSwiGLU ? launch_k(splitk_finish_kernel<2>, fg, dim3(256), 0, s, true, a, (const float *)part, p.splits)
-                                : launch_k(splitk_finish_kernel<1>, fg, dim3(256), 0, s, true, a, (const float *)part, p.splits);
+        const size_t row_smem = (size_t)a.n_units * sizeof(float);
+        if (a.epi != kEpiSwiGLU && a.next_norm && a.next_x && a.n_units % 4 == 0 && row_smem <= 48 * 1024) {
+            // one CTA per row: the sums, then the next projection's normalised row
+            e = launch_k(splitk_finish_row_kernel, dim3(a.T), dim3(kRowThreads), row_smem, s, true, a,
+                         (const float *)part, p.splits);
+            if (e == cudaSuccess && next_done) *next_done = true;
+        } else {
+            const dim3 fg((unsigned)(((long)a.T * a.n_units + 255) / 256));
+            e = a.epi == kEpiSwiGLU
+                    ? launch_k(splitk_finish_kernel<2>, fg, dim3(256), 0, s, true, a, (const float *)part, p.splits)
+                    : launch_k(splitk_finish_kernel<1>, fg, dim3(256), 0, s, true, a, (const float *)part, p.splits);
+        }
     }
     return e;
 }

@@ -136,6 +136,7 @@ struct prism_ctx {
     int attn_ctas_per_sm = 2;                             // fused attention: clusters shrink until B*Hkv*cs <= this * SMs
     int tc_stream_rows = 8;                               // tcgen05 projections with this many rows or more stream X
     int attn_max_cs = 8;                                  // largest cluster the device co-schedules
+    int fuse_rows = 1;                                    // streamed projections write the next one's activation rows
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
     bool tc_ready = false;
     CUtensorMap tm_lm;
@@ -168,7 +169,7 @@ prism_status cuda_fail(prism_ctx *c, cudaError_t e, const char *what) {
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-// 16-byte vector loads and bulk prefetches need 16-byte aligned bases.
+// 16-byte vector loads need 16-byte aligned bases.
 bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
 
 void drop_graphs(prism_ctx *c) {
@@ -245,14 +246,45 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
     // unless gemv_tcgen05 = 2: with 112 unit tiles it needs split-K on the
     // tensor-core kernel, and measured slower there; from two rows on the
     // CUDA-core kernel's issue cost doubles and the tensor cores win)
-    auto proj = [&](const GemvArgs &g, const CUtensorMap *tm, int grid, bool pdl_here) -> cudaError_t {
-        const bool want = c->gemv_tcgen05 == 2 || (c->gemv_tcgen05 == 1 && (g.epi != kEpiSwiGLU || g.T > 1));
-        if (tm && want && c->tc_ready && c->bf16 && g.T >= c->tc_stream_rows && gemv_tcs_supported(g, c->sms)) {
-            const size_t ws = gemv_tcs_workspace_floats(g, c->sms);
-            if (ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n))
-                return launch_gemv_tcs(g, *tm, c->sms, c->tc_part, c->tc_ctr, c->xbuf, s, pdl_here);
+    auto want_tc = [&](const GemvArgs &g) {
+        return c->gemv_tcgen05 == 2 || (c->gemv_tcgen05 == 1 && (g.epi != kEpiSwiGLU || g.T > 1));
+    };
+    // the streamed tcgen05 kernel takes g (its activation rows in the bf16 buffer)
+    auto on_tcs = [&](const GemvArgs &g, const CUtensorMap *tm) -> bool {
+        if (!(tm && want_tc(g) && c->tc_ready && c->bf16 && g.T >= c->tc_stream_rows && gemv_tcs_supported(g, c->sms)))
+            return false;
+        const size_t ws = gemv_tcs_workspace_floats(g, c->sms);
+        return ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n);
+    };
+    // x_ready: the bf16 buffer already holds the rows of the next projection,
+    // written by the previous projection's last kernel
+    bool x_ready = false;
+    auto proj = [&](GemvArgs g, const CUtensorMap *tm, int grid, bool pdl_here, const GemvArgs *next = nullptr,
+                    const CUtensorMap *ntm = nullptr) -> cudaError_t {
+        if (on_tcs(g, tm)) {
+            if (x_ready) {
+                g.pro = kProCopy;
+                g.act = c->xbuf;
+            }
+            x_ready = false;
+            if (c->fuse_rows && next && next->T == g.T && on_tcs(*next, ntm)) {
+                if (g.epi == kEpiTopK && next->pro == kProFuseDecode) {
+                    g.next_fuse = 1;
+                    g.next_x = c->xbuf;
+                } else if ((g.epi == kEpiStore || g.epi == kEpiResid) && next->pro == kProNorm &&
+                           next->kin == g.n_units) {
+                    g.next_norm = 1;
+                    g.next_gain = next->gain;
+                    g.next_x = c->xbuf;
+                }
+            }
+            bool done = false;
+            const cudaError_t le = launch_gemv_tcs(g, *tm, c->sms, c->tc_part, c->tc_ctr, c->xbuf, s, pdl_here, &done);
+            x_ready = le == cudaSuccess && done;
+            return le;
         }
-        if (tm && want && c->tc_ready && c->bf16 && gemv_tc_supported(g, c->sms)) {
+        x_ready = false;
+        if (tm && want_tc(g) && c->tc_ready && c->bf16 && gemv_tc_supported(g, c->sms)) {
             // split-K launches need the partial-sum workspace and one ticket per tile
             const size_t ws = gemv_tc_workspace_floats(g, c->sms);
             if (ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n))
@@ -324,9 +356,127 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         ta.out_frontier = r.tree.frontier;
     }
 
+    // the projections of step k (rows: T1 for the fusion and QKV, which see
+    // every prefill row at step 1; Trow from the O projection on)
+    auto step_tm = [&](int k, int i) -> const CUtensorMap * {
+        return c->tm_step_ok[k - 1] ? &c->tm_step[k - 1][i] : nullptr;
+    };
+    auto rows_trow = [&](int k) { return tree && k > 1 ? r.B * tw : r.B; };
+    auto rows_t1 = [&](int k) { return k == 1 ? r.B * f.max_new : rows_trow(k); };
+    auto fusion_args = [&](int k) {
+        GemvArgs g = base;
+        g.step = k;
+        g.W = c->steps[k - 1].w_fuse;
+        g.n_units = d;
+        g.kin = 2 * d;
+        g.T = rows_t1(k);
+        g.pro = k == 1 ? kProFusePrefill : (tree ? kProCopy : kProFuseDecode);
+        g.src = c->hhat;
+        g.act = c->tree_u;
+        g.epi = kEpiStore;
+        g.out = c->x0;
+        g.out_ld = d;
+        return g;
+    };
+    auto qkv_args = [&](int k) {
+        GemvArgs g = base;
+        g.step = k;
+        g.W = c->steps[k - 1].w_qkv;
+        g.n_units = c->qkv_rows;
+        g.kin = d;
+        g.T = rows_t1(k);
+        g.pro = kProNorm;
+        g.src = c->x0;
+        g.gain = c->steps[k - 1].g_attn;
+        g.epi = kEpiStore;
+        g.out = c->qkv;
+        g.out_ld = c->qkv_rows;
+        return g;
+    };
+    auto o_args = [&](int k) {
+        GemvArgs g = base;
+        g.step = k;
+        g.W = c->steps[k - 1].w_o;
+        g.n_units = d;
+        g.kin = Hq * D;
+        g.T = rows_trow(k);
+        g.pro = kProCopy;
+        g.act = c->o_buf;
+        g.epi = kEpiResid;
+        g.resid = c->x0;
+        g.resid_prefill_rows = k == 1;
+        g.out = c->a;
+        g.out_ld = d;
+        return g;
+    };
+    auto gate_up_args = [&](int k) {
+        GemvArgs g = base;
+        g.step = k;
+        g.W = c->steps[k - 1].w_gate_up;
+        g.n_units = F;
+        g.pair_offset = F;
+        g.kin = d;
+        g.T = rows_trow(k);
+        g.pro = kProNorm;
+        g.src = c->a;
+        g.gain = c->steps[k - 1].g_mlp;
+        g.epi = kEpiSwiGLU;
+        g.out_act = c->m_buf;
+        g.out_ld = F;
+        return g;
+    };
+    auto down_args = [&](int k) {
+        GemvArgs g = base;
+        g.step = k;
+        g.W = c->steps[k - 1].w_down;
+        g.n_units = d;
+        g.kin = F;
+        g.T = rows_trow(k);
+        g.pro = kProCopy;
+        g.act = c->m_buf;
+        g.epi = kEpiResid;
+        g.resid = c->a;
+        g.out = c->hhat;
+        g.out_ld = d;
+        g.hidden_out = tree ? nullptr : r.hidden_out;
+        return g;
+    };
+    auto lm_args = [&](int k) {
+        GemvArgs g = base;
+        g.step = k;
+        g.W = c->lm_head;
+        g.n_units = V;
+        g.kin = d;
+        g.T = rows_trow(k);
+        g.pro = kProNorm;
+        g.src = c->hhat;
+        g.gain = f.final_norm ? c->steps[k - 1].g_final : nullptr;
+        g.epi = kEpiTopK;
+        g.logits = r.logits;
+        g.lm_part = c->lm_val;
+        g.lm_part_id = c->lm_id;
+        g.counter = c->counters + (size_t)f.max_batch * Hkv;
+        g.best = c->lm_best;
+        g.draft_out = r.draft;
+        g.topk_ids = r.topk_ids;
+        g.topk_logits = r.topk_logits;
+        if (tree) {
+            // rows b * w + j of [B * w, .] buffers: at step 1 (one row per
+            // sequence) K = w puts row b at b * w; later steps index by row
+            float *lg = r.tree.row_logits ? r.tree.row_logits + (size_t)(k - 1) * r.B * tw * V : c->tree_logits;
+            g.K = k == 1 ? tw : 1;
+            g.step = 1;
+            g.topk = tw;
+            g.logits = lg;
+            g.draft_out = c->tree_draft;
+            g.topk_ids = c->tree_top_ids;
+            g.topk_logits = c->tree_top_vals;
+        }
+        return g;
+    };
+    const CUtensorMap *lm_tm = c->tm_lm_ok ? &c->tm_lm : nullptr;
+
     for (int k = 1; k <= K && e == cudaSuccess; ++k) {
-        const prism_step_weights &w = c->steps[k - 1];
-        const CUtensorMap *tms = c->tm_step_ok[k - 1] ? c->tm_step[k - 1] : nullptr;
         const bool prefill = k == 1;
         const bool tstep = tree && !prefill;       // a tree step: w rows per sequence
         const int Trow = tstep ? r.B * tw : r.B;   // rows from attention on
@@ -342,37 +492,13 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
             if (e != cudaSuccess) break;
         }
 
-        // fusion F(E(x), h)
-        GemvArgs g = base;
-        g.step = k;
-        g.W = w.w_fuse;
-        g.n_units = d;
-        g.kin = 2 * d;
-        g.T = T1;
-        g.pro = prefill ? kProFusePrefill : (tstep ? kProCopy : kProFuseDecode);
-        g.src = c->hhat;
-        g.act = c->tree_u;
-        g.epi = kEpiStore;
-        g.out = c->x0;
-        g.out_ld = d;
-        e = proj(g, tms ? &tms[0] : nullptr, gemv_grid(c, d), tstep ? pdl : p);
+        // fusion F(E(x), h), then the attention pre-norm + QKV, whose rows the
+        // fusion's last kernel can write
+        const GemvArgs gq = qkv_args(k);
+        e = proj(fusion_args(k), step_tm(k, 0), gemv_grid(c, d), tstep ? pdl : p, &gq, step_tm(k, 1));
         after(0);
         if (e != cudaSuccess) break;
-
-        // attention pre-norm + QKV
-        g = base;
-        g.step = k;
-        g.W = w.w_qkv;
-        g.n_units = c->qkv_rows;
-        g.kin = d;
-        g.T = T1;
-        g.pro = kProNorm;
-        g.src = c->x0;
-        g.gain = w.g_attn;
-        g.epi = kEpiStore;
-        g.out = c->qkv;
-        g.out_ld = c->qkv_rows;
-        e = proj(g, tms ? &tms[1] : nullptr, gemv_grid(c, c->qkv_rows), pdl);
+        e = proj(gq, step_tm(k, 1), gemv_grid(c, c->qkv_rows), pdl);
         after(1);
         if (e != cudaSuccess) break;
 
@@ -459,93 +585,24 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         if (e != cudaSuccess) break;
         }
 
-        // O projection + residual
-        g = base;
-        g.step = k;
-        g.W = w.w_o;
-        g.n_units = d;
-        g.kin = Hq * D;
-        g.T = Trow;
-        g.pro = kProCopy;
-        g.act = c->o_buf;
-        g.epi = kEpiResid;
-        g.resid = c->x0;
-        g.resid_prefill_rows = prefill;
-        g.out = c->a;
-        g.out_ld = d;
-        e = proj(g, tms ? &tms[2] : nullptr, gemv_grid(c, d), pdl);
+        // O projection + residual; MLP pre-norm + gate/up + SwiGLU; down
+        // projection + residual -> h^_{k-1}; final norm + LM head + top-8
+        // selection -> x^_k.  Each hands its rows to the next where it can;
+        // the LM head to the next step's fusion in a greedy chain.
+        const GemvArgs gg = gate_up_args(k), gl = lm_args(k);
+        e = proj(o_args(k), step_tm(k, 2), gemv_grid(c, d), pdl, &gg, step_tm(k, 3));
         after(4);
         if (e != cudaSuccess) break;
-
-        // MLP pre-norm + gate/up + SwiGLU
-        g = base;
-        g.step = k;
-        g.W = w.w_gate_up;
-        g.n_units = F;
-        g.pair_offset = F;
-        g.kin = d;
-        g.T = Trow;
-        g.pro = kProNorm;
-        g.src = c->a;
-        g.gain = w.g_mlp;
-        g.epi = kEpiSwiGLU;
-        g.out_act = c->m_buf;
-        g.out_ld = F;
-        e = proj(g, tms ? &tms[3] : nullptr, gemv_grid(c, F), pdl);
+        e = proj(gg, step_tm(k, 3), gemv_grid(c, F), pdl);
         after(5);
         if (e != cudaSuccess) break;
-
-        // down projection + residual -> h^_{k-1}
-        g = base;
-        g.step = k;
-        g.W = w.w_down;
-        g.n_units = d;
-        g.kin = F;
-        g.T = Trow;
-        g.pro = kProCopy;
-        g.act = c->m_buf;
-        g.epi = kEpiResid;
-        g.resid = c->a;
-        g.out = c->hhat;
-        g.out_ld = d;
-        g.hidden_out = tree ? nullptr : r.hidden_out;
-        e = proj(g, tms ? &tms[4] : nullptr, gemv_grid(c, d), pdl);
+        e = proj(down_args(k), step_tm(k, 4), gemv_grid(c, d), pdl, &gl, lm_tm);
         after(6);
         if (e != cudaSuccess) break;
-
-        // final norm + LM head + top-8 selection -> x^_k
-        g = base;
-        g.step = k;
-        g.W = c->lm_head;
-        g.n_units = V;
-        g.kin = d;
-        g.T = Trow;
-        g.pro = kProNorm;
-        g.src = c->hhat;
-        g.gain = f.final_norm ? w.g_final : nullptr;
-        g.epi = kEpiTopK;
-        g.logits = r.logits;
-        g.lm_part = c->lm_val;
-        g.lm_part_id = c->lm_id;
-        g.counter = c->counters + (size_t)f.max_batch * Hkv;
-        g.best = c->lm_best;
-        g.draft_out = r.draft;
-        g.topk_ids = r.topk_ids;
-        g.topk_logits = r.topk_logits;
-        if (tree) {
-            // rows b * w + j of [B * w, .] buffers: at step 1 (one row per
-            // sequence) K = w puts row b at b * w; later steps index by row
-            float *lg = r.tree.row_logits ? r.tree.row_logits + (size_t)(k - 1) * r.B * tw * V : c->tree_logits;
-            g.K = prefill ? tw : 1;
-            g.step = 1;
-            g.topk = tw;
-            g.logits = lg;
-            g.draft_out = c->tree_draft;
-            g.topk_ids = c->tree_top_ids;
-            g.topk_logits = c->tree_top_vals;
-            ta.logits = lg;
-        }
-        e = proj(g, c->tm_lm_ok ? &c->tm_lm : nullptr, c->lm_grid, pdl);
+        const bool chain_next = k < K && !tree && !(r.temperature > 0.f);
+        const GemvArgs gn = chain_next ? fusion_args(k + 1) : GemvArgs{};
+        e = proj(gl, lm_tm, c->lm_grid, pdl, chain_next ? &gn : nullptr, chain_next ? step_tm(k + 1, 0) : nullptr);
+        if (tree) ta.logits = gl.logits;
         after(7);
         if (e != cudaSuccess) break;
 
@@ -865,6 +922,7 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "attn_fused")) c->attn_fused = value != 0;
     else if (!std::strcmp(name, "tc_stream_rows") && value >= 1) c->tc_stream_rows = value;
     else if (!std::strcmp(name, "attn_ctas_per_sm") && value >= 1 && value <= 64) c->attn_ctas_per_sm = value;
+    else if (!std::strcmp(name, "fuse_rows")) c->fuse_rows = value != 0;
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);
     return PRISM_OK;

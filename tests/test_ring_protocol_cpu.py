@@ -223,16 +223,29 @@ def test_cuda_core_ring_parity_waits_are_unambiguous(S, G):
 
 # ------------------------------------------------------------ gemv_tc_kernel
 
-def run_tc_ring(S, my_tiles, n_kst, seed, event_bias, mma_lag, acc_empty_count=4):
+def run_tc_ring(S, my_tiles, n_kst, seed, event_bias, mma_lag, acc_empty_count=4, streamed=False,
+                early_x=False):
     """gemv_tc_kernel: producer as above (empty[s] has one arrival: the MMA
     lane's tcgen05.commit); the MMA lane waits acc_empty[ab] (parity
     ((i >> 1) & 1) ^ 1), then full[s] per stage, issues MMAs into accumulator
     buffer ab = i & 1 and commits them to empty[s], then commits the tile to
     acc_full[ab]; four epilogue warps wait acc_full[ab] (parity (i >> 1) & 1),
     read the buffer and arrive on acc_empty[ab] (count 4).  Commits arrive
-    when every MMA issued before them has completed (in issue order)."""
+    when every MMA issued before them has completed (in issue order).
+
+    streamed=True: gemv_tcs_kernel, whose stages hold weight boxes and
+    activation (X) boxes, X being the previous kernel's output.  The producer
+    arms each of the first min(total, S) stages for both parts and requests
+    their weight boxes, waits for the previous kernel (griddepcontrol.wait,
+    here a gate that opens at a random time), then requests those stages' X
+    boxes; later stages get both parts together.  A stage's data is complete
+    only when both parts have landed.  early_x=True requests the first X boxes
+    before the gate (a planted mistake the checks must catch)."""
     rng = random.Random(seed)
     sim = Sim(rng, event_bias)
+    gate = {"open": not streamed}
+    if streamed:
+        sim.post(lambda: gate.update(open=True))
     full = [Barrier(1) for _ in range(S)]
     empty = [Barrier(1) for _ in range(S)]
     acc_full = [Barrier(1), Barrier(1)]
@@ -258,20 +271,51 @@ def run_tc_ring(S, my_tiles, n_kst, seed, event_bias, mma_lag, acc_empty_count=4
         if len(queue) == 1:
             sim.post(pump)
 
+    parts = [set() for _ in range(S)]
+
+    def request(s, j, part):
+        if part == "x":
+            assert gate["open"], f"X box of item {j} requested before the previous kernel completed"
+
+        def land(s=s, j=j, part=part):
+            parts[s].add((j, part))
+            if {(j, "w"), (j, "x")} <= parts[s] or not streamed:
+                content[s] = j
+            full[s].complete_tx(1)
+        sim.post(land)
+
     def producer():
         s, ph, issued = 0, 0, 0
-        for j in range(total):
+        nparts = 2 if streamed else 1
+        pre = min(total, S) if streamed else 0
+        for j in range(pre):                  # first pass: arm, weight boxes only
+            assert stage_readers[j] == 0
+            full[j].arrive_expect_tx(nparts)
+            content[j] = None
+            parts[j] = set()
+            request(j, j, "w")
+            if early_x:
+                request(j, j, "x")
+            yield ("step",)
+        if streamed:
+            yield ("wait", lambda: gate["open"])        # griddepcontrol.wait
+            for j in range(pre):
+                if not early_x:
+                    request(j, j, "x")
+                yield ("step",)
+            issued = pre
+            s, ph = pre % S, 1 if pre == S else 0
+        for j in range(pre, total):
             yield ("wait", lambda s=s, ph=ph: empty[s].ready(ph ^ 1))
             if j >= S:
                 check_wait(empty[s], ph ^ 1, j // S - 1, "producer empty")
             assert stage_readers[s] == 0, f"stage {s} overwritten while MMAs read it"
-            full[s].arrive_expect_tx(1)
+            full[s].arrive_expect_tx(nparts)
             content[s] = None
-
-            def land(s=s, j=j):
-                content[s] = j
-                full[s].complete_tx(1)
-            sim.post(land)
+            parts[s] = set()
+            request(s, j, "w")
+            if streamed:
+                request(s, j, "x")
             issued += 1
             s += 1
             if s == S:
@@ -283,6 +327,8 @@ def run_tc_ring(S, my_tiles, n_kst, seed, event_bias, mma_lag, acc_empty_count=4
 
     def mma():
         s, ph, j = 0, 0, 0
+        if streamed:
+            yield ("wait", lambda: gate["open"])        # griddepcontrol.wait
         for i in range(my_tiles):
             ab = i & 1
             par = ((i >> 1) & 1) ^ 1
@@ -343,10 +389,11 @@ TC_PLANS = [(S, tiles, kst) for S in (1, 2, 3, 4, 5, 8) for tiles in (1, 2, 3, 7
 
 
 @pytest.mark.parametrize("S,tiles,kst", TC_PLANS)
-def test_tcgen05_ring_and_accumulator_handoff(S, tiles, kst):
+@pytest.mark.parametrize("streamed", [False, True], ids=["staged", "streamed"])
+def test_tcgen05_ring_and_accumulator_handoff(S, tiles, kst, streamed):
     for trial in range(12):
         run_tc_ring(S, tiles, kst, seed=7919 * S + 31 * tiles + kst + trial,
-                    event_bias=[0.15, 0.5, 0.85][trial % 3], mma_lag=trial % 4)
+                    event_bias=[0.15, 0.5, 0.85][trial % 3], mma_lag=trial % 4, streamed=streamed)
 
 
 # ------------------------------------------------- fused_attention_tc_kernel
@@ -448,6 +495,13 @@ def test_the_checks_catch_an_early_accumulator_release():
     """Likewise for the accumulator: released after the first epilogue warp
     instead of all four, the MMA lane overwrites a buffer still being read."""
     assert _fails(lambda seed: run_tc_ring(2, 5, 2, seed=seed, event_bias=0.5, mma_lag=0, acc_empty_count=1)) > 0
+
+
+def test_the_checks_catch_x_boxes_requested_before_the_dependency_wait():
+    """The streamed producer requests its first weight boxes early; its X
+    boxes (the previous kernel's output) must wait, and the checks see it."""
+    assert _fails(lambda seed: run_tc_ring(3, 2, 4, seed=seed, event_bias=0.5, mma_lag=1, streamed=True,
+                                           early_x=True)) > 0
 
 
 def test_the_checks_catch_an_early_attention_stage_release():
