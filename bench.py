@@ -333,6 +333,29 @@ def config_of(w):
             **({"tree_width": w.tree_width, "tree_nodes": w.tree_nodes} if w.tree_width else {})}
 
 
+def eager_round_us(dr, one_round, stream, steps, dev):
+    """Round latency with the graph off: every kernel launched from the host,
+    one event pair around the rounds (after 3 untimed rounds).  Reported next
+    to the replayed round as evidence of what the graph saves; the option is
+    restored afterwards (the graph is captured again on the next call)."""
+    import torch
+    n = max(3, min(20, steps))
+    dr.set_option("use_graph", 0)
+    try:
+        for _ in range(3):
+            one_round()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(dev)
+        e0.record(stream)
+        for _ in range(n):
+            one_round()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+    finally:
+        dr.set_option("use_graph", 1)
+    return e0.elapsed_time(e1) * 1e3 / n
+
+
 def run_ours(args, w, world, rank, local):
     import numpy as np
     import torch
@@ -412,6 +435,9 @@ def run_ours(args, w, world, rank, local):
     value = tokens_total / (ms / 1e3)
     per_round_ms = ms / args.steps
 
+    # ---- the same round without the graph (eager launches, evidence only) -------
+    eager_us = eager_round_us(dr, one_round, stream, args.steps, dev)
+
     # ---- per-kernel durations (eager launches, an event around each kernel) -----
     prof = []
     for _ in range(max(3, min(20, args.steps))):
@@ -476,6 +502,7 @@ def run_ours(args, w, world, rank, local):
                                                 **({"temperature": args.temperature} if sampled else {})),
             "round_latency_us": per_round_ms * 1e3,
             "round_latency_percentiles_us": pct,
+            "round_latency_eager_us": eager_us,
             "hbm": {"bytes_per_round": total_bytes,
                     "achieved_gbs": total_bytes / (per_round_ms / 1e3) / 1e9,
                     "frac_of_8tbs": total_bytes / (per_round_ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,
@@ -555,6 +582,7 @@ def run_tree(args, w, world, rank, local):
     tokens_total = B * m * args.steps * world
     value = tokens_total / (ms / 1e3)
     per_round_ms = ms / args.steps
+    eager_us = eager_round_us(dr, one_round, stream, args.steps, dev)
 
     prof = [dr.profile_tree(t["tokens"], t["hidden"], t["n_new"], t["kv_len"], t["k_cache"], t["v_cache"], tw,
                             tt, tp, td, ts, stream=stream) for _ in range(max(3, min(20, args.steps)))]
@@ -621,6 +649,7 @@ def run_tree(args, w, world, rank, local):
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if s.dtype == "bf16" else "f32",
             "data": "synthetic", "config": dict(config_of(w), options=options),
             "round_latency_us": per_round_ms * 1e3,
+            "round_latency_eager_us": eager_us,
             "hbm": {"bytes_per_round": total_bytes,
                     "achieved_gbs": total_bytes / (per_round_ms / 1e3) / 1e9,
                     "frac_of_8tbs": total_bytes / (per_round_ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,

@@ -343,8 +343,12 @@ prism_status prism_lm_head_topk_static(int32_t dtype, int32_t hidden, int32_t vo
                                        int32_t *dev_flags, void *stream);
 
 /* Synchronise `stream`, read and clear the device error word.  Returns
- * PRISM_ERR_DEVICE_FLAG (bits in *flags if non-NULL) when it was set,
- * PRISM_ERR_CUDA when the stream reports an error, PRISM_OK otherwise. */
+ * PRISM_ERR_TIMEOUT when its timeout bit is set (a bounded device-side wait
+ * gave up: the kernel wound down, every copy it had in flight landed, and
+ * the outputs of the calls since the last check are not to be used),
+ * PRISM_ERR_DEVICE_FLAG when only other bits are set (bits in *flags if
+ * non-NULL in both cases), PRISM_ERR_CUDA when the stream reports an
+ * error, PRISM_OK otherwise.  The context stays usable after either flag. */
 prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
 
 /* Options (name, value): "use_graph" (1: capture and replay, default 1),
@@ -368,6 +372,15 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * KV append and attention run as one kernel, a cluster of up to 8 CTAs per
  * sequence and KV head merging through distributed shared memory; 0: a
  * RoPE/append kernel, then split-KV attention with a last-CTA merge),
+ * "wait_polls" (0, the default: every wait between two roles of a kernel,
+ * a consumer for a filled ring stage or accumulator, a producer for a
+ * released one, gives up after a built-in bound of 2^22 polls; N > 0: after
+ * N polls; N < 0: at once, so that every such wait fails: a setting for
+ * testing the error path.  A wait that gives up sets the timeout bit and
+ * the kernel winds down: it issues no more copies or MMAs, still waits
+ * (with the built-in bound) for the copies and MMAs it has in flight, and
+ * frees its tensor memory.  Covers the projection kernels and the fused
+ * attention kernel),
  * "fuse_rows" (1, the default: a streamed projection's last kernel, the
  * split-K finish or the LM head's top-k merge, also writes the next
  * projection's bf16 activation rows, its RMSNorm or the next step's fusion

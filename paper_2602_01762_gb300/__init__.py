@@ -373,10 +373,13 @@ class Drafter:
 
     def sync_status(self, stream=None) -> int:
         """Synchronise and return the device error word (0 when clean); raises
-        on CUDA errors.  A set word is returned, not raised."""
+        on CUDA errors.  A set word is returned, not raised (the C status,
+        PRISM_ERR_DEVICE_FLAG or PRISM_ERR_TIMEOUT, is kept in
+        ``last_status``)."""
         flags = ctypes.c_int32(0)
         st = self.lib.prism_sync_status(self.h, _stream(stream), ctypes.byref(flags))
-        if st not in (0, 7):
+        self.last_status = st
+        if st not in (0, 7, 8):
             self._check(st)
         return int(flags.value)
 

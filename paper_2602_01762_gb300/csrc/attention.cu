@@ -686,11 +686,11 @@ __device__ __forceinline__ void split2(float x, float y, uint32_t &hi, uint32_t 
 }
 // Whole-warp bounded wait on an mbarrier phase: lane 0 polls, every lane then
 // observes the completed phase itself.  Warp-uniform result.
-__device__ __forceinline__ bool ta_wait_warp(uint64_t *bar, uint32_t parity) {
+__device__ __forceinline__ bool ta_wait_warp(uint64_t *bar, uint32_t parity, long limit) {
     bool ok = true;
     if ((threadIdx.x & 31) == 0) {
         ok = false;
-        for (long it = 0; it < kAttnWaitLimit && !ok; ++it) ok = fa_try(bar, parity);
+        for (long it = 0; it < limit && !ok; ++it) ok = fa_try(bar, parity);
     }
     ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
     if (ok) fa_try(bar, parity);
@@ -726,6 +726,7 @@ __global__ void __launch_bounds__(kTaThreads, 1)
     const int r = blockIdx.x, g = blockIdx.y, b = blockIdx.z, CS = a.cs;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int half = D / 2, H = a.Hq + 2 * a.Hkv, G = a.Hq / a.Hkv;
+    const long lim = wait_bound(a.wait_polls, kAttnWaitLimit);
     pdl_trigger();
 
     const int n = clamp_n(a.n_new, b, a.max_new, a.err);
@@ -838,7 +839,7 @@ __global__ void __launch_bounds__(kTaThreads, 1)
                     // slot i % S is free once every warp has released stage i - S
                     bool ok = false;
                     const uint32_t par = (uint32_t)((i / kTaStages - 1) & 1);
-                    for (long it = 0; it < kAttnWaitLimit && !ok; ++it) ok = fa_try(&empty[i % kTaStages], par);
+                    for (long it = 0; it < lim && !ok; ++it) ok = fa_try(&empty[i % kTaStages], par);
                     if (!ok) {
                         set_err(a.err, kErrTimeout);
                         dead = true;
@@ -870,7 +871,7 @@ __global__ void __launch_bounds__(kTaThreads, 1)
         const int kr = 16 * warp;                     // this warp's first row in a stage
         for (int i = 0; i < nst; ++i) {
             const int s = i % kTaStages;
-            if (!dead && !ta_wait_warp(&full[s], (uint32_t)((i / kTaStages) & 1))) {
+            if (!dead && !ta_wait_warp(&full[s], (uint32_t)((i / kTaStages) & 1), lim)) {
                 if (lane == 0) set_err(a.err, kErrTimeout);
                 dead = true;
             }
@@ -948,7 +949,10 @@ __global__ void __launch_bounds__(kTaThreads, 1)
                 if (cnt < 16) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             }
             __syncwarp();
-            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(sa(&empty[s])) : "memory");
+            // a warp that gave up on this stage does not release it (its copy may
+            // still be in flight); the producer's wait for the slot then gives up
+            if (lane == 0 && !dead)
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(sa(&empty[s])) : "memory");
         }
         // the warp's sums over its lanes' keys
 #pragma unroll

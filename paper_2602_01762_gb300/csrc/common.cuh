@@ -81,6 +81,17 @@ __device__ __forceinline__ void set_err(int *err, int bit) {
     if (err) atomicOr(err, bit);
 }
 
+// Polls a wait between two roles of a kernel (a consumer for a filled stage
+// or accumulator, a producer for a released one) makes before it gives up,
+// sets the timeout bit and lets the kernel wind down: wait_polls > 0 is that
+// count, 0 the built-in bound `dflt`, < 0 none (every such wait gives up at
+// once; used to test the error path).  The drain waits (a producer for its
+// own copies in flight, the MMA lane for its own MMAs) always use `dflt`,
+// so that nothing is in flight when a CTA exits.
+__device__ __forceinline__ long wait_bound(int wait_polls, long dflt) {
+    return wait_polls > 0 ? (long)wait_polls : (wait_polls < 0 ? 0L : dflt);
+}
+
 // Checked builds (-DPRISM_CHECKED): record the first failed bounds or
 // alignment check (code, block, two values) in the four words after the
 // device error word, and skip the access.  Compiled out otherwise.
@@ -186,6 +197,7 @@ struct GemvArgs {
     uint16_t *next_x;
     const void *next_gain;
     int next_norm, next_fuse;
+    int wait_polls;          // see wait_bound
 };
 
 struct RopeArgs {
@@ -220,6 +232,7 @@ struct FusedAttnArgs {
     const int32_t *n_new, *kv_len;
     int B, max_new, prefill, step, Hq, Hkv, D, max_ctx, cs;
     int *err;
+    int wait_polls;                    // see wait_bound
 };
 
 struct AcceptArgs {

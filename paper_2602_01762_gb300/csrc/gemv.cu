@@ -58,8 +58,8 @@ __device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity) {
     return ok != 0;
 }
 // Bounded wait for the completion of the phase with the given parity.
-__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity) {
-    for (long i = 0; i < kWaitLimit; ++i)
+__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity, long limit = kWaitLimit) {
+    for (long i = 0; i < limit; ++i)
         if (mbar_try(b, parity)) return true;
     return false;
 }
@@ -273,7 +273,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
         int s = 0, c = 0;
         uint32_t ph = 0;                                      // phase parity of stage s
         for (int i = 0; i < total; ++i) {
-            if (!mbar_wait(&empty[s], ph ^ 1)) {
+            if (!mbar_wait(&empty[s], ph ^ 1, wait_bound(a.wait_polls, kWaitLimit))) {
                 set_err(a.err, kErrTimeout);
                 break;
             }
@@ -338,7 +338,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
 
         for (; item < (p + 1) * n_chunks; item += G, ++lc) {
             const int c = item - p * n_chunks;
-            if (!dead && !mbar_wait(&full[s], ph)) {
+            if (!dead && !mbar_wait(&full[s], ph, wait_bound(a.wait_polls, kWaitLimit))) {
                 set_err(a.err, kErrTimeout);
                 dead = true;
             }
@@ -450,7 +450,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
                 }
             }
             __syncwarp();
-            if (lane == 0) mbar_arrive(&empty[s]);
+            // a warp that gave up on this stage does not release it: its copy
+            // may still be in flight, and the producer must not reuse the slot
+            // (the producer's own wait then gives up and it drains)
+            if (lane == 0 && !dead) mbar_arrive(&empty[s]);
             s += G;
             if (s >= S) { s -= S; ph ^= 1; }
         }

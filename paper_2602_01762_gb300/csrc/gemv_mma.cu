@@ -47,8 +47,8 @@ __device__ __forceinline__ void bar_arrive(uint64_t *b) {
 __device__ __forceinline__ void bar_arrive_tx(uint64_t *b, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(sa(b)), "r"(bytes) : "memory");
 }
-__device__ __forceinline__ bool bar_wait(uint64_t *b, uint32_t parity) {
-    for (long i = 0; i < kWaitLimitM; ++i) {
+__device__ __forceinline__ bool bar_wait(uint64_t *b, uint32_t parity, long limit = kWaitLimitM) {
+    for (long i = 0; i < limit; ++i) {
         uint32_t ok;
         asm volatile("{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
                      : "=r"(ok) : "r"(sa(b)), "r"(parity) : "memory");
@@ -236,7 +236,7 @@ __global__ void __launch_bounds__(kThreadsM, 1) gemv_mma_kernel(const GemvArgs a
         uint32_t ph = 0;
         for (long i = 0; i < total; ++i) {
             int ok = 1;
-            if (lane == 0) ok = bar_wait(&empty[s], ph ^ 1u);
+            if (lane == 0) ok = bar_wait(&empty[s], ph ^ 1u, wait_bound(a.wait_polls, kWaitLimitM));
             ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
             if (!ok) {
                 if (lane == 0) set_err(a.err, kErrTimeout);
@@ -305,7 +305,7 @@ __global__ void __launch_bounds__(kThreadsM, 1) gemv_mma_kernel(const GemvArgs a
 #pragma unroll
                 for (int q = 0; q < 4; ++q) acc4[r][q][0] = acc4[r][q][1] = acc4[r][q][2] = acc4[r][q][3] = 0.f;
             for (int j = 0; j < KS; ++j) {
-                if (!dead && !bar_wait(&full[s], ph)) {
+                if (!dead && !bar_wait(&full[s], ph, wait_bound(a.wait_polls, kWaitLimitM))) {
                     set_err(a.err, kErrTimeout);
                     dead = true;
                 }
@@ -334,7 +334,9 @@ __global__ void __launch_bounds__(kThreadsM, 1) gemv_mma_kernel(const GemvArgs a
                     }
                 }
                 __syncwarp();
-                if (lane == 0) bar_arrive(&empty[s]);
+                // a warp that gave up on this stage does not release it (its copy
+                // may still be in flight); the producer's wait then gives up
+                if (lane == 0 && !dead) bar_arrive(&empty[s]);
                 if (++s == S) { s = 0; ph ^= 1u; }
             }
             float acc[RPW][4];

@@ -70,8 +70,8 @@ __device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity) {
                  : "=r"(ok) : "r"(saddr(b)), "r"(parity) : "memory");
     return ok != 0;
 }
-__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity) {
-    for (long i = 0; i < kTcWaitLimit; ++i)
+__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity, long limit = kTcWaitLimit) {
+    for (long i = 0; i < limit; ++i)
         if (mbar_try(b, parity)) return true;
     return false;
 }
@@ -79,11 +79,11 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity) {
 // Whole-warp wait: lane 0 polls with a short back-off (a warp of spinning
 // lanes would compete with the TMA and MMA traffic on shared memory), then
 // every lane observes the completed phase.  Warp-uniform result.
-__device__ __forceinline__ bool mbar_wait_warp(uint64_t *b, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t *b, uint32_t parity, long limit) {
     bool ok = true;
     if ((threadIdx.x & 31) == 0) {
         ok = false;
-        for (long i = 0; i < kTcWaitLimit; ++i) {
+        for (long i = 0; i < limit; ++i) {
             if (mbar_try(b, parity)) { ok = true; break; }
             __nanosleep(64);
         }
@@ -470,6 +470,7 @@ __device__ __forceinline__ Key key_at(const Key (&l)[kTopK], int r) {
 // (tr[j][row]: column j becomes a row of 128 logits), then the threads of
 // those columns' rows scan them.  A transposed row is 128 + P floats long, so
 // the 32 lanes of a scanning warp read 32 distinct banks.
+// With P = 8 every epilogue thread scans: thread e takes row c0 + e / 8.
 template <int P>
 __device__ __forceinline__ void chunk_to_lists(const float (&acc)[16], int row, float *tr, int tile, int c0, int T,
                                                int n_units, bool dead, Key (&l)[kTopK]) {
@@ -477,7 +478,7 @@ __device__ __forceinline__ void chunk_to_lists(const float (&acc)[16], int row, 
 #pragma unroll
     for (int j = 0; j < 16; ++j) tr[j * S + row] = acc[j];
     epi_sync();
-    const int e = threadIdx.x - 64, t = e / P, q = e % P;
+    const int e = threadIdx.x - 64, t = (P == 8 ? c0 : 0) + e / P, q = e % P;
     if (!dead && t >= c0 && t < c0 + 16 && t < T) {
         const float *src = tr + (t - c0) * S;
 #pragma unroll 4
@@ -493,10 +494,10 @@ __device__ __forceinline__ void chunk_to_lists(const float (&acc)[16], int row, 
 // it to the per-CTA partial lists ([row][CTA][kTopK] values and ids; id -1
 // marks an empty slot), thread q the entries q, q + P, ...
 template <int P>
-__device__ __forceinline__ void lists_publish(const GemvArgs &a, Key (&l)[kTopK], int T) {
+__device__ __forceinline__ void lists_publish(const GemvArgs &a, Key (&l)[kTopK], int T, int t0 = 0) {
 #pragma unroll 1
     for (int m = 1; m < P; m <<= 1) key_merge_xor(l, m);
-    const int e = threadIdx.x - 64, t = e / P, q = e % P;
+    const int e = threadIdx.x - 64, t = t0 + e / P, q = e % P;
     if (t < T) {
 #pragma unroll
         for (int r0 = 0; r0 < kTopK; r0 += P) {
@@ -576,6 +577,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     constexpr uint32_t kCols = RPW == 1 ? 32 : 64;   // two accumulator buffers x RPW x 16 columns
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const long lim = wait_bound(a.wait_polls, kTcWaitLimit);
     uint8_t *base = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *ring = base;
     uint8_t *X = base + (size_t)p.stages * p.stage_bytes;
@@ -620,7 +622,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             for (int i = 0; i < my_tiles && !dead; ++i) {
                 const int tile = blockIdx.x / p.splits + i * tiles_step;
                 for (int q = 0; q < n_kst; ++q) {
-                    if (!mbar_wait(&empty[s], ph ^ 1)) {
+                    if (!mbar_wait(&empty[s], ph ^ 1, lim)) {
                         set_err(a.err, kErrTimeout);
                         dead = true;
                         break;
@@ -659,14 +661,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 const uint32_t sbo_b = NB == 16 ? 1024u : 0u;
                 for (int i = 0; i < my_tiles && !dead; ++i) {
                     const int ab = i & 1;
-                    if (!mbar_wait(&acc_empty[ab], ((i >> 1) & 1) ^ 1)) {
+                    if (!mbar_wait(&acc_empty[ab], ((i >> 1) & 1) ^ 1, lim)) {
                         set_err(a.err, kErrTimeout);
                         dead = true;
                         break;
                     }
                     tc_fence_after();
                     for (int q = 0; q < n_kst; ++q) {
-                        if (!mbar_wait(&full[s], ph)) {
+                        if (!mbar_wait(&full[s], ph, lim)) {
                             set_err(a.err, kErrTimeout);
                             dead = true;
                             break;
@@ -723,7 +725,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             for (int i = 0; i < my_tiles; ++i) {
                 const int tile = blockIdx.x / p.splits + i * tiles_step;
                 const int ab = i & 1;
-                if (!dead && !mbar_wait_warp(&acc_full[ab], (i >> 1) & 1)) {
+                if (!dead && !mbar_wait_warp(&acc_full[ab], (i >> 1) & 1, lim)) {
                     if (lane == 0) set_err(a.err, kErrTimeout);
                     dead = true;
                 }
@@ -892,6 +894,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                  ((uint32_t)(kTileM >> 4) << 24);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const long lim = wait_bound(a.wait_polls, kTcWaitLimit);
     uint8_t *ring = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const int S = p.stages;
     const uint32_t kb_bytes = RPW * kBoxBytes + kXBox;                // one K block in a stage
@@ -979,7 +982,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             s = pre % S;
             ph = pre == S ? 1u : 0u;
             for (int f = pre; f < total; ++f) {
-                if (!mbar_wait(&empty[s], ph ^ 1)) {
+                if (!mbar_wait(&empty[s], ph ^ 1, lim)) {
                     set_err(a.err, kErrTimeout);
                     dead = true;
                     break;
@@ -1004,14 +1007,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 bool dead = false;
                 for (int i = 0; i < my_tiles && !dead; ++i) {
                     const int ab = i & 1;
-                    if (!mbar_wait(&acc_empty[ab], ((i >> 1) & 1) ^ 1)) {
+                    if (!mbar_wait(&acc_empty[ab], ((i >> 1) & 1) ^ 1, lim)) {
                         set_err(a.err, kErrTimeout);
                         dead = true;
                         break;
                     }
                     tc_fence_after();
                     for (int q = 0; q < n_kst; ++q) {
-                        if (!mbar_wait(&full[s], ph)) {
+                        if (!mbar_wait(&full[s], ph, lim)) {
                             set_err(a.err, kErrTimeout);
                             dead = true;
                             break;
@@ -1053,22 +1056,29 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int quarter = warp & 3;
             const int row = quarter * 32 + lane;
             const int T = a.T;
-            constexpr int kP = NB <= 128 ? kTileM / NB : 1;     // threads per activation row
-            Key lst[kTopK];
-            if constexpr (TOPK) key_clear(lst);
+            // top-k: every 16-row chunk of a tile is scanned by all 128 epilogue
+            // threads, 8 per row (each thread keeps one list per chunk position)
+            constexpr int kNL = TOPK ? NB / 16 : 1;
+            Key lst[kNL][kTopK];
+            if constexpr (TOPK) {
+#pragma unroll
+                for (int cc = 0; cc < kNL; ++cc) key_clear(lst[cc]);
+            }
             bool dead = false;
             for (int i = 0; i < my_tiles; ++i) {
                 const int tile = blockIdx.x / p.splits + i * tiles_step;
                 const int ab = i & 1;
-                if (!dead && !mbar_wait_warp(&acc_full[ab], (i >> 1) & 1)) {
+                if (!dead && !mbar_wait_warp(&acc_full[ab], (i >> 1) & 1, lim)) {
                     if (lane == 0) set_err(a.err, kErrTimeout);
                     dead = true;
                 }
                 const int u = tile * kTileM + row;
                 const bool valid = !dead && u < a.n_units;
                 if constexpr (TOPK) {
-#pragma unroll 1
-                    for (int c0 = 0; c0 < NB && c0 < T; c0 += 16) {
+#pragma unroll
+                    for (int cc = 0; cc < kNL; ++cc) {
+                        const int c0 = 16 * cc;
+                        if (c0 >= T) break;
                         float acc[16];
                         if (!dead) {
                             tc_fence_after();
@@ -1082,7 +1092,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             for (int tt = 0; tt < 16; ++tt)
                                 if (c0 + tt < T) a.logits[((size_t)(c0 + tt) * a.K + a.step - 1) * a.vocab + u] = acc[tt];
                         }
-                        chunk_to_lists<kP>(acc, row, &s_tr[0][0], tile, c0, T, a.n_units, dead, lst);
+                        chunk_to_lists<8>(acc, row, &s_tr[0][0], tile, c0, T, a.n_units, dead, lst[cc]);
                     }
                 }
                 // accumulator columns 16 at a time (all RPW sets of one chunk together)
@@ -1136,7 +1146,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             if constexpr (TOPK) {
                 // this CTA's list of every row; the cross-CTA merge is a separate kernel
-                lists_publish<kP>(a, lst, T);
+#pragma unroll
+                for (int cc = 0; cc < kNL; ++cc) lists_publish<8>(a, lst[cc], T, 16 * cc);
             }
         }
     }
@@ -1154,40 +1165,48 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // (the same sums as the last-CTA path), and finishes the unit.  Inline in the
 // projection, the last CTA of a tile would read T x 128 x splits partial sums
 // through L2 while the tile's other work waits behind it.
+// The grid is at most a few CTAs per SM, all resident at once (a grid of
+// one CTA per output element came to many waves, which the next projection's
+// early-started CTAs delayed further): each thread strides over the outputs.
+constexpr int kFinishCtasPerSm = 4;
 template <int RPW>
 __global__ void __launch_bounds__(256) splitk_finish_kernel(const GemvArgs a, const float *part, int splits) {
     pdl_trigger();
     pdl_wait();
     const long total = (long)a.T * a.n_units;
-    const long e = (long)blockIdx.x * 256 + threadIdx.x;
-    if (e >= total) return;
-    const int t = (int)(e / a.n_units), u = (int)(e % a.n_units);
-    float v[kMaxSplits][RPW];
+    for (long e = (long)blockIdx.x * 256 + threadIdx.x; e < total; e += (long)gridDim.x * 256) {
+        const int t = (int)(e / a.n_units), u = (int)(e % a.n_units);
+        float v[kMaxSplits][RPW];
 #pragma unroll
-    for (int k = 0; k < kMaxSplits; ++k)
+        for (int k = 0; k < kMaxSplits; ++k)
 #pragma unroll
-        for (int r = 0; r < RPW; ++r)
-            v[k][r] = k < splits ? __ldcg(&part[(((size_t)k * RPW + r) * a.T + t) * a.n_units + u]) : 0.f;
-    float s0 = 0.f, s1 = 0.f;
+            for (int r = 0; r < RPW; ++r)
+                v[k][r] = k < splits ? __ldcg(&part[(((size_t)k * RPW + r) * a.T + t) * a.n_units + u]) : 0.f;
+        float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-    for (int k = 0; k < kMaxSplits; ++k)
-        if (k < splits) {
-            s0 += v[k][0];
-            s1 += v[k][RPW - 1];
-        }
-    finish_unit<RPW>(a, t, u, s0, s1);
+        for (int k = 0; k < kMaxSplits; ++k)
+            if (k < splits) {
+                s0 += v[k][0];
+                s1 += v[k][RPW - 1];
+            }
+        finish_unit<RPW>(a, t, u, s0, s1);
+    }
 }
 
 // Cross-CTA top-k merge of the streamed LM head: one CTA (4 warps) per row;
 // each warp merges a quarter of the row's candidates, warp 0 the four lists.
+// This kernel runs once per row and step, right after the LM head, with
+// HBM busy streaming the next step's weights: its instructions arrive at
+// cache-miss speed, so it is written with rolled loops (one copy of the
+// insertion and merge networks).
 __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int grid) {
     __shared__ Key s_k[4][kTopK];
     pdl_trigger();
     pdl_wait();
     const int t = blockIdx.x, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     Key l[kTopK];
-    gather_keys<false>(a, t, grid, threadIdx.x, 128, l);
-#pragma unroll
+    gather_keys<true>(a, t, grid, threadIdx.x, 128, l);
+#pragma unroll 1
     for (int m = 1; m < 32; m <<= 1) key_merge_xor(l, m);
     if (lane == 0) {
 #pragma unroll
@@ -1199,7 +1218,7 @@ __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int g
 #pragma unroll
         for (int i = 0; i < kTopK; ++i) l[i] = lane < 4 ? s_k[lane][i] : 0ull;
         // every lane ends with the merged list (write_row reads rank r from lane r)
-#pragma unroll
+#pragma unroll 1
         for (int m = 1; m < 32; m <<= 1) key_merge_xor(l, m);
         write_row(a, t, l);
         if (lane == 0) {
@@ -1488,7 +1507,12 @@ bool tcs_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem, in
     if (!NB) return false;
     const int nkb = (a.kin + kBoxK - 1) / kBoxK;
     const int n_tiles = (a.n_units + kTileM - 1) / kTileM;
-    const int max_s = topk ? 1 : kMaxSplits;
+    // No split when the tiles alone already occupy most SMs in one wave: a
+    // split then buys little streaming time and costs a finish pass over
+    // every partial sum (gate/up at 112 tiles: 2440 -> 2197 us per round at
+    // batch 64, 1663 -> 1615 us at batch 16)
+    const bool one_wave = n_tiles <= sms && 10 * n_tiles >= 7 * sms;
+    const int max_s = topk || one_wave ? 1 : kMaxSplits;
     long best = -1;
     int best_s = 0, best_ctas = 0;
     for (int sp = 1; sp <= max_s && sp <= nkb; ++sp) {
@@ -1667,7 +1691,9 @@ cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, f
                          (const float *)part, p.splits);
             if (e == cudaSuccess && next_done) *next_done = true;
         } else {
-            const dim3 fg((unsigned)(((long)a.T * a.n_units + 255) / 256));
+            long nb = ((long)a.T * a.n_units + 255) / 256;
+            if (nb > (long)kFinishCtasPerSm * sms) nb = (long)kFinishCtasPerSm * sms;
+            const dim3 fg((unsigned)nb);
             e = a.epi == kEpiSwiGLU
                     ? launch_k(splitk_finish_kernel<2>, fg, dim3(256), 0, s, true, a, (const float *)part, p.splits)
                     : launch_k(splitk_finish_kernel<1>, fg, dim3(256), 0, s, true, a, (const float *)part, p.splits);

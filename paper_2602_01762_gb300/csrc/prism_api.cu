@@ -137,6 +137,7 @@ struct prism_ctx {
     int tc_stream_rows = 8;                               // tcgen05 projections with this many rows or more stream X
     int attn_max_cs = 8;                                  // largest cluster the device co-schedules
     int fuse_rows = 1;                                    // streamed projections write the next one's activation rows
+    int wait_polls = 0;                                   // role-to-role wait bound (0: built in, < 0: none)
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
     bool tc_ready = false;
     CUtensorMap tm_lm;
@@ -239,6 +240,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
     base.smem_budget = c->gemv_smem;
     base.groups = c->gemv_groups;
     base.force_cuda_core = c->gemv_cuda_core;
+    base.wait_polls = c->wait_polls;
 
     // a projection on the tensor-core kernel when enabled and it fits, else on
     // the CUDA-core ring kernel
@@ -530,6 +532,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
             fa.cs = c->attn_max_cs;
             while (fa.cs > 1 && (long long)r.B * Hkv * fa.cs > (long long)c->attn_ctas_per_sm * c->sms) fa.cs /= 2;
             fa.err = c->err;
+            fa.wait_polls = c->wait_polls;
             e = launch_fused_attention(fa, c->bf16, s, pdl, cache_maps ? &tmk : nullptr, cache_maps ? &tmv : nullptr);
             after(3);
             if (e != cudaSuccess) break;
@@ -923,6 +926,7 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "tc_stream_rows") && value >= 1) c->tc_stream_rows = value;
     else if (!std::strcmp(name, "attn_ctas_per_sm") && value >= 1 && value <= 64) c->attn_ctas_per_sm = value;
     else if (!std::strcmp(name, "fuse_rows")) c->fuse_rows = value != 0;
+    else if (!std::strcmp(name, "wait_polls")) c->wait_polls = value;
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);
     return PRISM_OK;
@@ -1278,7 +1282,8 @@ prism_status prism_sync_status(prism_ctx *c, void *stream, int32_t *flags) {
         char buf[160];
         std::snprintf(buf, sizeof(buf), "device error word 0x%x (token range %d, cache range %d, n_new range %d, timeout %d)",
                       w, !!(w & 1), !!(w & 2), !!(w & 4), !!(w & 8));
-        return fail(c, PRISM_ERR_DEVICE_FLAG, buf);
+        // a wait that gave up means the results are not to be trusted at all
+        return fail(c, (w & kErrTimeout) ? PRISM_ERR_TIMEOUT : PRISM_ERR_DEVICE_FLAG, buf);
     }
     return PRISM_OK;
 }
