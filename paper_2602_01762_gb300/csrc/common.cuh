@@ -88,6 +88,23 @@ __device__ __forceinline__ void set_err(int *err, int bit) {
 // once; used to test the error path).  The drain waits (a producer for its
 // own copies in flight, the MMA lane for its own MMAs) always use `dflt`,
 // so that nothing is in flight when a CTA exits.
+// Running log-sum-exp as (max m, sum s of exp(z - m)): add one logit, and
+// combine two partial pairs.
+__device__ __forceinline__ void lse_add(float &m, float &s, float z) {
+    if (z > m) {
+        s = s * expf(m - z) + 1.f;
+        m = z;
+    } else {
+        s += expf(z - m);
+    }
+}
+__device__ __forceinline__ void lse_combine(float &m, float &s, float m2, float s2) {
+    if (m2 == -INFINITY) return;
+    if (m == -INFINITY) { m = m2; s = s2; return; }
+    if (m2 > m) { s = s * expf(m - m2) + s2; m = m2; }
+    else s += s2 * expf(m2 - m);
+}
+
 __device__ __forceinline__ long wait_bound(int wait_polls, long dflt) {
     return wait_polls > 0 ? (long)wait_polls : (wait_polls < 0 ? 0L : dflt);
 }
@@ -198,6 +215,9 @@ struct GemvArgs {
     const void *next_gain;
     int next_norm, next_fuse;
     int wait_polls;          // see wait_bound
+    // LM head with top-k lists: per row and CTA, (max, sum of exp(z - max))
+    // of the logits the CTA produced, [T][gridDim.x][2]; null: not computed
+    float *lse_part;
 };
 
 struct RopeArgs {
@@ -303,6 +323,9 @@ struct TreeArgs {
     int *lse_ctr;                     // [B*w] (left at zero)
     int *seq_ctr;                     // [B] rows of each sequence with their lse (left at zero)
     int lse_chunk, lse_blocks;
+    // > 0: the LM head wrote per-CTA (max, sum exp) partials of every row,
+    // lm_lse_grid of them, into lse_part ([LM-head row][lm_lse_grid][2])
+    int lm_lse_grid;
     // RoPE / append / attention (one kernel)
     const float *qkv;                 // [B*w, (Hq + 2Hkv) D]
     void *k_cache, *v_cache;          // [B, Hkv, max_ctx, D]

@@ -471,9 +471,12 @@ __device__ __forceinline__ Key key_at(const Key (&l)[kTopK], int r) {
 // those columns' rows scan them.  A transposed row is 128 + P floats long, so
 // the 32 lanes of a scanning warp read 32 distinct banks.
 // With P = 8 every epilogue thread scans: thread e takes row c0 + e / 8.
+// With want_lse the scanning thread also adds each logit to its running
+// log-sum-exp (lm, ls) of that row.
 template <int P>
 __device__ __forceinline__ void chunk_to_lists(const float (&acc)[16], int row, float *tr, int tile, int c0, int T,
-                                               int n_units, bool dead, Key (&l)[kTopK]) {
+                                               int n_units, bool dead, Key (&l)[kTopK], bool want_lse, float &lm,
+                                               float &ls) {
     constexpr int S = kTileM + P;
 #pragma unroll
     for (int j = 0; j < 16; ++j) tr[j * S + row] = acc[j];
@@ -484,10 +487,29 @@ __device__ __forceinline__ void chunk_to_lists(const float (&acc)[16], int row, 
 #pragma unroll 4
         for (int i = 0; i < kTileM / P; ++i) {
             const int r = i * P + q, u = tile * kTileM + r;
-            if (u < n_units) key_insert(l, pack_best(src[r], u));
+            if (u < n_units) {
+                key_insert(l, pack_best(src[r], u));
+                if (want_lse) lse_add(lm, ls, src[r]);
+            }
         }
     }
     epi_sync();
+}
+
+// The CTA's (max, sum exp) of each row: the 8 threads of a row combine
+// theirs (fixed butterfly order), the first writes the CTA's partial.
+__device__ __forceinline__ void lse_publish(const GemvArgs &a, float m, float s, int T, int t0) {
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1) {
+        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, s, o);
+        lse_combine(m, s, m2, s2);
+    }
+    const int e = threadIdx.x - 64, t = t0 + e / 8;
+    if ((e & 7) == 0 && t < T) {
+        float *pp = a.lse_part + ((size_t)t * gridDim.x + blockIdx.x) * 2;
+        pp[0] = m;
+        pp[1] = s;
+    }
 }
 
 // The CTA's list of each row: the P threads of a row merge theirs and write
@@ -721,6 +743,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 key_clear(lst);
                 __syncwarp();
             }
+            float lse_m = -INFINITY, lse_s = 0.f;     // this thread's row, with a.lse_part
             bool dead = false;
             for (int i = 0; i < my_tiles; ++i) {
                 const int tile = blockIdx.x / p.splits + i * tiles_step;
@@ -778,7 +801,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             }
                         }
                     } else {
-                        chunk_to_lists<8>(acc[0], row, &s_tr[0][0], tile, 0, T, a.n_units, dead, lst);
+                        chunk_to_lists<8>(acc[0], row, &s_tr[0][0], tile, 0, T, a.n_units, dead, lst,
+                                          a.lse_part != nullptr, lse_m, lse_s);
                     }
                 } else if (p.splits == 1) {
                     if (valid) {
@@ -826,6 +850,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                 } else {
                     lists_publish<8>(a, lst, T);
+                    if (a.lse_part) lse_publish(a, lse_m, lse_s, T, 0);
                 }
                 __threadfence();
                 epi_sync();
@@ -1060,9 +1085,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             // threads, 8 per row (each thread keeps one list per chunk position)
             constexpr int kNL = TOPK ? NB / 16 : 1;
             Key lst[kNL][kTopK];
+            float lse_m[kNL], lse_s[kNL];         // per chunk position, with a.lse_part
             if constexpr (TOPK) {
 #pragma unroll
-                for (int cc = 0; cc < kNL; ++cc) key_clear(lst[cc]);
+                for (int cc = 0; cc < kNL; ++cc) {
+                    key_clear(lst[cc]);
+                    lse_m[cc] = -INFINITY;
+                    lse_s[cc] = 0.f;
+                }
             }
             bool dead = false;
             for (int i = 0; i < my_tiles; ++i) {
@@ -1092,7 +1122,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             for (int tt = 0; tt < 16; ++tt)
                                 if (c0 + tt < T) a.logits[((size_t)(c0 + tt) * a.K + a.step - 1) * a.vocab + u] = acc[tt];
                         }
-                        chunk_to_lists<8>(acc, row, &s_tr[0][0], tile, c0, T, a.n_units, dead, lst[cc]);
+                        chunk_to_lists<8>(acc, row, &s_tr[0][0], tile, c0, T, a.n_units, dead, lst[cc],
+                                          a.lse_part != nullptr, lse_m[cc], lse_s[cc]);
                     }
                 }
                 // accumulator columns 16 at a time (all RPW sets of one chunk together)
@@ -1147,7 +1178,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if constexpr (TOPK) {
                 // this CTA's list of every row; the cross-CTA merge is a separate kernel
 #pragma unroll
-                for (int cc = 0; cc < kNL; ++cc) lists_publish<8>(a, lst[cc], T, 16 * cc);
+                for (int cc = 0; cc < kNL; ++cc) {
+                    lists_publish<8>(a, lst[cc], T, 16 * cc);
+                    if (a.lse_part) lse_publish(a, lse_m[cc], lse_s[cc], T, 16 * cc);
+                }
             }
         }
     }

@@ -258,6 +258,10 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         const size_t ws = gemv_tcs_workspace_floats(g, c->sms);
         return ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n);
     };
+    // the staged tcgen05 kernel takes g (when the streamed one does not)
+    auto on_tc_staged = [&](const GemvArgs &g, const CUtensorMap *tm) -> bool {
+        return tm && want_tc(g) && c->tc_ready && c->bf16 && gemv_tc_supported(g, c->sms);
+    };
     // x_ready: the bf16 buffer already holds the rows of the next projection,
     // written by the previous projection's last kernel
     bool x_ready = false;
@@ -286,7 +290,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
             return le;
         }
         x_ready = false;
-        if (tm && want_tc(g) && c->tc_ready && c->bf16 && gemv_tc_supported(g, c->sms)) {
+        if (on_tc_staged(g, tm)) {
             // split-K launches need the partial-sum workspace and one ticket per tile
             const size_t ws = gemv_tc_workspace_floats(g, c->sms);
             if (ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n))
@@ -473,6 +477,14 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
             g.draft_out = c->tree_draft;
             g.topk_ids = c->tree_top_ids;
             g.topk_logits = c->tree_top_vals;
+            g.best = nullptr;           // the list path, which also yields the log-sum-exp partials
+            // on a tcgen05 kernel the LM head also writes each row's per-CTA
+            // log-sum-exp partials, and the logits only when the caller wants them
+            const CUtensorMap *ltm = c->tm_lm_ok ? &c->tm_lm : nullptr;
+            if (on_tcs(g, ltm) || on_tc_staged(g, ltm)) {
+                g.lse_part = c->tree_lse_part;
+                if (!r.tree.row_logits) g.logits = nullptr;
+            }
         }
         return g;
     };
@@ -605,7 +617,10 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         const bool chain_next = k < K && !tree && !(r.temperature > 0.f);
         const GemvArgs gn = chain_next ? fusion_args(k + 1) : GemvArgs{};
         e = proj(gl, lm_tm, c->lm_grid, pdl, chain_next ? &gn : nullptr, chain_next ? step_tm(k + 1, 0) : nullptr);
-        if (tree) ta.logits = gl.logits;
+        if (tree) {
+            ta.logits = gl.logits;
+            ta.lm_lse_grid = gl.lse_part ? (V + 127) / 128 < c->sms ? (V + 127) / 128 : c->sms : 0;
+        }
         after(7);
         if (e != cudaSuccess) break;
 
@@ -748,7 +763,7 @@ prism_status prism_create(const prism_config *cfg, int32_t device, prism_ctx **o
         tree_on * Bw * kTopK * 4,                                  // tree top-w logits
         tree_on * Bw * 4,                                          // tree LM-head top-1 (unused)
         tree_on * Bw * 4,                                          // tree row lse
-        tree_on * Bw * kSampleMaxBlocks * 2 * 4,                   // tree lse partials
+        tree_on * Bw * (size_t)(c->lm_grid > kSampleMaxBlocks ? c->lm_grid : kSampleMaxBlocks) * 2 * 4,  // tree lse partials
         tree_on * (Bw + Bseq) * 4,                                 // tree lse tickets, sequence tickets
         tree_on * Bw * 4 * 4,                                      // frontier token, row, pool index, score
         tree_on * Bw * 8,                                          // frontier ancestor masks

@@ -687,7 +687,12 @@ __device__ void select_sequence(const TreeArgs &a, int b, SelectSmem &sm) {
 
 // ------------------------------------------------------------------ log-sum-exp
 
-// Grid (blocks per row, B * R): row t = b * w + j of the LM head's logits.
+// Grid (blocks per row, B * R): row t = b * w + j.  Its log-sum-exp comes
+// either from the LM head's per-CTA partials (lm_lse_grid > 0: one CTA per
+// row merges them) or from the logits the LM head wrote (chunks of the row
+// per CTA, the row's last CTA merging the chunks' partials).  The last row
+// of a sequence to finish then scores the candidates and picks the frontier.
+constexpr int kLseMaxParts = 256;
 __global__ void __launch_bounds__(256) tree_lse_kernel(const TreeArgs a) {
     __shared__ float s_m[8], s_s[8];
     __shared__ int s_last, s_seq;
@@ -697,65 +702,75 @@ __global__ void __launch_bounds__(256) tree_lse_kernel(const TreeArgs a) {
     const int blk = blockIdx.x, nblk = gridDim.x;
     const int b = blockIdx.y / a.R, j = blockIdx.y % a.R, t = b * a.w + j;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const float *z = a.logits + (size_t)t * a.V;
-    const int lo = blk * a.lse_chunk, hi = min(a.V, lo + a.lse_chunk);
-    float m = -INFINITY, s = 0.f;
-    constexpr int kBatch = 8;                  // loads in flight per thread before any use
-    for (int i0 = lo + tid; i0 < hi; i0 += kBatch * 256) {
-        float v[kBatch];
+    const float *parts;
+    int nparts;
+    if (a.lm_lse_grid > 0) {
+        // the LM head's row of this tree row: b at step 1 (one row per sequence), t after
+        const int lm_row = a.step == 1 ? b : t;
+        parts = a.lse_part + (size_t)lm_row * a.lm_lse_grid * 2;
+        nparts = a.lm_lse_grid;
+    } else {
+        const float *z = a.logits + (size_t)t * a.V;
+        const int lo = blk * a.lse_chunk, hi = min(a.V, lo + a.lse_chunk);
+        float m = -INFINITY, s = 0.f;
+        constexpr int kBatch = 8;                  // loads in flight per thread before any use
+        for (int i0 = lo + tid; i0 < hi; i0 += kBatch * 256) {
+            float v[kBatch];
 #pragma unroll
-        for (int q = 0; q < kBatch; ++q) {
-            const int i = i0 + q * 256;
-            v[q] = i < hi ? z[i] : -INFINITY;
+            for (int q = 0; q < kBatch; ++q) {
+                const int i = i0 + q * 256;
+                v[q] = i < hi ? z[i] : -INFINITY;
+            }
+#pragma unroll
+            for (int q = 0; q < kBatch; ++q)
+                if (v[q] != -INFINITY) lse_merge(m, s, v[q], 1.f);
         }
 #pragma unroll
-        for (int q = 0; q < kBatch; ++q)
-            if (v[q] != -INFINITY) lse_merge(m, s, v[q], 1.f);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, s, o);
-        lse_merge(m, s, m2, s2);
-    }
-    if (lane == 0) { s_m[warp] = m; s_s[warp] = s; }
-    __syncthreads();
-    if (tid == 0) {
-        for (int q = 1; q < (int)(blockDim.x >> 5); ++q) lse_merge(m, s, s_m[q], s_s[q]);
-        float *part = a.lse_part + ((size_t)t * kSampleMaxBlocks + blk) * 2;
-        part[0] = m;
-        part[1] = s;
+        for (int o = 16; o > 0; o >>= 1) {
+            const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, s, o);
+            lse_merge(m, s, m2, s2);
+        }
+        if (lane == 0) { s_m[warp] = m; s_s[warp] = s; }
+        __syncthreads();
+        if (tid == 0) {
+            for (int q = 1; q < (int)(blockDim.x >> 5); ++q) lse_merge(m, s, s_m[q], s_s[q]);
+            float *part = a.lse_part + ((size_t)t * kSampleMaxBlocks + blk) * 2;
+            part[0] = m;
+            part[1] = s;
+            __threadfence();
+            s_last = atomicAdd(a.lse_ctr + t, 1) == nblk - 1;
+        }
+        __syncthreads();
+        if (!s_last) return;                       // uniform over the CTA
         __threadfence();
-        s_last = atomicAdd(a.lse_ctr + t, 1) == nblk - 1;
+        if (tid == 0) a.lse_ctr[t] = 0;
+        parts = a.lse_part + (size_t)t * kSampleMaxBlocks * 2;
+        nparts = nblk;
     }
-    __syncthreads();
-    if (!s_last) return;                       // uniform over the CTA
-    // the last CTA of the row: lane l of warp 0 merges partials l, l + 32, ...
-    // (all loads issued first), then the lanes merge in a fixed butterfly order
-    __threadfence();
+    // lane l of warp 0 merges partials l, l + 32, ... (all loads issued
+    // first), then the lanes merge in a fixed butterfly order
     if (warp == 0) {
-    constexpr int kPer = kSampleMaxBlocks / 32;
-    float pm[kPer], ps[kPer];
+        constexpr int kPer = kLseMaxParts / 32;
+        float pm[kPer], ps[kPer];
 #pragma unroll
-    for (int i = 0; i < kPer; ++i) {
-        const int q = lane + 32 * i;
-        const float *pq = a.lse_part + ((size_t)t * kSampleMaxBlocks + q) * 2;
-        pm[i] = q < nblk ? __ldcg(pq) : -INFINITY;
-        ps[i] = q < nblk ? __ldcg(pq + 1) : 0.f;
-    }
-    float M = -INFINITY, S = 0.f;
+        for (int i = 0; i < kPer; ++i) {
+            const int q = lane + 32 * i;
+            pm[i] = q < nparts ? __ldcg(parts + 2 * q) : -INFINITY;
+            ps[i] = q < nparts ? __ldcg(parts + 2 * q + 1) : 0.f;
+        }
+        float M = -INFINITY, S = 0.f;
 #pragma unroll
-    for (int i = 0; i < kPer; ++i) lse_merge(M, S, pm[i], ps[i]);
+        for (int i = 0; i < kPer; ++i) lse_merge(M, S, pm[i], ps[i]);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, M, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, S, o);
-        lse_merge(M, S, m2, s2);
-    }
-    if (lane == 0) {
-        a.lse[t] = M + logf(S);
-        a.lse_ctr[t] = 0;
-        __threadfence();
-        s_seq = atomicAdd(a.seq_ctr + b, 1) == a.R - 1;
-    }
+        for (int o = 16; o > 0; o >>= 1) {
+            const float m2 = __shfl_xor_sync(0xFFFFFFFFu, M, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, S, o);
+            lse_merge(M, S, m2, s2);
+        }
+        if (lane == 0) {
+            a.lse[t] = M + logf(S);
+            __threadfence();
+            s_seq = atomicAdd(a.seq_ctr + b, 1) == a.R - 1;
+        }
     }
     __syncthreads();
     if (!s_seq) return;                        // uniform over the CTA
@@ -861,7 +876,8 @@ cudaError_t launch_tree_attention(const TreeArgs &a, bool bf16, cudaStream_t s, 
 
 cudaError_t launch_tree_lse(const TreeArgs &args, cudaStream_t s, bool pdl) {
     TreeArgs a = args;
-    a.lse_blocks = sample_blocks(a.V, &a.lse_chunk);
+    a.lse_blocks = a.lm_lse_grid > 0 ? 1 : sample_blocks(a.V, &a.lse_chunk);
+    if (a.lm_lse_grid > kLseMaxParts) return cudaErrorInvalidValue;
     return launch_k(tree_lse_kernel, dim3(a.lse_blocks, a.B * a.R), dim3(256), 0, s, pdl, a);
 }
 
