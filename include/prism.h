@@ -381,6 +381,10 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * (with the built-in bound) for the copies and MMAs it has in flight, and
  * frees its tensor memory.  Covers the projection kernels and the fused
  * attention kernel),
+ * "w_evict_first" (1, the default: the projection kernels load weight boxes
+ * with an L2 evict-first cache policy, since each weight byte is read once
+ * per step, so that the KV cache and the activations stay in L2; 0: the
+ * default policy),
  * "fuse_rows" (1, the default: a streamed projection's last kernel, the
  * split-K finish or the LM head's top-k merge, also writes the next
  * projection's bf16 activation rows, its RMSNorm or the next step's fusion

@@ -88,6 +88,14 @@ __device__ __forceinline__ void set_err(int *err, int bit) {
 // once; used to test the error path).  The drain waits (a producer for its
 // own copies in flight, the MMA lane for its own MMAs) always use `dflt`,
 // so that nothing is in flight when a CTA exits.
+// An L2 cache policy under which the lines a load brings in are evicted
+// first (for data read once, such as a weight stream).
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
 // Running log-sum-exp as (max m, sum s of exp(z - m)): add one logit, and
 // combine two partial pairs.
 __device__ __forceinline__ void lse_add(float &m, float &s, float z) {
@@ -215,6 +223,9 @@ struct GemvArgs {
     const void *next_gain;
     int next_norm, next_fuse;
     int wait_polls;          // see wait_bound
+    // 1: weight boxes are loaded with an L2 evict-first policy (each weight
+    // byte is read once per step; other data then stays in L2)
+    int w_evict_first;
     // LM head with top-k lists: per row and CTA, (max, sum of exp(z - max))
     // of the logits the CTA produced, [T][gridDim.x][2]; null: not computed
     float *lse_part;

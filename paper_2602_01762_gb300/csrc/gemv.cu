@@ -64,9 +64,14 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity, long lim
     return false;
 }
 // 1-D TMA bulk copy global -> shared, completing on mbarrier b.
-__device__ __forceinline__ void tma_load(void *dst, const void *src, uint32_t bytes, uint64_t *b) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-                 ::"r"(saddr(dst)), "l"(src), "r"(bytes), "r"(saddr(b)) : "memory");
+__device__ __forceinline__ void tma_load(void *dst, const void *src, uint32_t bytes, uint64_t *b, uint64_t pol = 0) {
+    if (pol == 0) {
+        asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                     ::"r"(saddr(dst)), "l"(src), "r"(bytes), "r"(saddr(b)) : "memory");
+        return;
+    }
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
+                 ::"r"(saddr(dst)), "l"(src), "r"(bytes), "r"(saddr(b)), "l"(pol) : "memory");
 }
 // Barrier among the consumer warps only (the producer warp never joins).
 __device__ __forceinline__ void consumers_sync() {
@@ -269,6 +274,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
         // ------------------------------------------------------------ producer
         if (lane != 0) return;
         const int total = n_pass * n_chunks;
+        const uint64_t wpol = a.w_evict_first ? l2_evict_first_policy() : 0ull;
         int issued = 0;
         int s = 0, c = 0;
         uint32_t ph = 0;                                      // phase parity of stage s
@@ -291,7 +297,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
             for (int r = 0; r < RPW; ++r)
                 tma_load(st + (size_t)r * R * row_bytes,
                          (const uint8_t *)a.W + ((size_t)first + (size_t)r * a.pair_offset) * row_bytes, bytes,
-                         &full[s]);
+                         &full[s], wpol);
             issued = i + 1;
             if (++c == n_chunks) c = 0;
             if (++s == S) { s = 0; ph ^= 1; }

@@ -99,6 +99,17 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
         ::"r"(dst), "l"((uint64_t)map), "r"(x), "r"(y), "r"(saddr(bar)) : "memory");
 }
+// The same with an L2 cache policy (pol != 0), else without.
+__device__ __forceinline__ void tma_load_2d_pol(uint32_t dst, const CUtensorMap *map, int x, int y, uint64_t *bar,
+                                                uint64_t pol) {
+    if (pol == 0) {
+        tma_load_2d(dst, map, x, y, bar);
+        return;
+    }
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%2, "
+        "%3}], [%4], %5;" ::"r"(dst), "l"((uint64_t)map), "r"(x), "r"(y), "r"(saddr(bar)), "l"(pol) : "memory");
+}
 
 // tcgen05 shared-memory matrix descriptor: K-major operand in the 128-byte
 // swizzle layout (8-row x 128-byte atoms, `sbo` bytes between 8-row groups).
@@ -638,6 +649,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
+            const uint64_t wpol = a.w_evict_first ? l2_evict_first_policy() : 0ull;
             int s = 0, issued = 0;
             uint32_t ph = 0;
             bool dead = false;
@@ -656,8 +668,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     for (int j = 0; j < nkb; ++j)
 #pragma unroll
                         for (int r = 0; r < RPW; ++r)
-                            tma_load_2d(st + (uint32_t)(j * RPW + r) * kBoxBytes, &tmW, (kbs + j) * kBoxK,
-                                        tile * kTileM + r * a.pair_offset, &full[s]);
+                            tma_load_2d_pol(st + (uint32_t)(j * RPW + r) * kBoxBytes, &tmW, (kbs + j) * kBoxK,
+                                        tile * kTileM + r * a.pair_offset, &full[s], wpol);
                     ++issued;
                     if (++s == S) { s = 0; ph ^= 1; }
                 }
@@ -958,6 +970,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
+            const uint64_t wpol = a.w_evict_first ? l2_evict_first_policy() : 0ull;
             int s = 0, issued = 0;
             uint32_t ph = 0;
             bool dead = false;
@@ -975,8 +988,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 for (int j = 0; j < nkb; ++j)
 #pragma unroll
                     for (int r = 0; r < RPW; ++r)
-                        tma_load_2d(st + (uint32_t)j * kb_bytes + (uint32_t)r * kBoxBytes, &tmW, (kbs + j) * kBoxK,
-                                    tile * kTileM + r * a.pair_offset, &full[stage]);
+                        tma_load_2d_pol(st + (uint32_t)j * kb_bytes + (uint32_t)r * kBoxBytes, &tmW, (kbs + j) * kBoxK,
+                                        tile * kTileM + r * a.pair_offset, &full[stage], wpol);
             };
             auto load_x = [&](int f, int stage) {
                 int tile, kbs, nkb;

@@ -138,6 +138,7 @@ struct prism_ctx {
     int attn_max_cs = 8;                                  // largest cluster the device co-schedules
     int fuse_rows = 1;                                    // streamed projections write the next one's activation rows
     int wait_polls = 0;                                   // role-to-role wait bound (0: built in, < 0: none)
+    int w_evict_first = 1;                                // weight streams with an L2 evict-first policy
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
     bool tc_ready = false;
     CUtensorMap tm_lm;
@@ -241,6 +242,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
     base.groups = c->gemv_groups;
     base.force_cuda_core = c->gemv_cuda_core;
     base.wait_polls = c->wait_polls;
+    base.w_evict_first = c->w_evict_first;
 
     // a projection on the tensor-core kernel when enabled and it fits, else on
     // the CUDA-core ring kernel
@@ -942,6 +944,7 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "attn_ctas_per_sm") && value >= 1 && value <= 64) c->attn_ctas_per_sm = value;
     else if (!std::strcmp(name, "fuse_rows")) c->fuse_rows = value != 0;
     else if (!std::strcmp(name, "wait_polls")) c->wait_polls = value;
+    else if (!std::strcmp(name, "w_evict_first")) c->w_evict_first = value != 0;
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);
     return PRISM_OK;
