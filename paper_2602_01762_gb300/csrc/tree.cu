@@ -148,9 +148,10 @@ __device__ __forceinline__ void load_run(const WT *p, float (&out)[DPL]) {
 // depth and written to the cache and the stage; queries are rotated,
 // multiplied by q_scale and stored QS floats apart.  Callers wait for the
 // copies and synchronise.
+// Rows [j0, j0 + done) were requested earlier (tree_stage_committed).
 template <typename WT, int D, int RS, int QS>
 __device__ __forceinline__ void tree_stage(const TreeArgs &a, int b, int g, int j0, int nk, int base, WT *Ks,
-                                           WT *Vs, float *qs, float q_scale) {
+                                           WT *Vs, float *qs, float q_scale, int done) {
     constexpr int VEC = Elem<WT>::kPerVec;
     const int G = a.Hq / a.Hkv, NQ = a.w * G;
     const int new0 = base + (a.step - 2) * a.w;
@@ -160,7 +161,7 @@ __device__ __forceinline__ void tree_stage(const TreeArgs &a, int b, int g, int 
     WT *kc = (WT *)a.k_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D;
     WT *vc = (WT *)a.v_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D;
     constexpr int VPR = D / VEC;
-    for (int e = threadIdx.x; e < nold * VPR; e += blockDim.x) {
+    for (int e = threadIdx.x + done * VPR; e < nold * VPR; e += blockDim.x) {
         const int r = e / VPR, c = e % VPR;
         cp_async16(Ks + (size_t)r * RS + c * VEC, (const uint4 *)kc + e);
         cp_async16(Vs + (size_t)r * RS + c * VEC, (const uint4 *)vc + e);
@@ -191,6 +192,25 @@ __device__ __forceinline__ void tree_stage(const TreeArgs &a, int b, int g, int 
         Elem<WT>::store(vc + (size_t)r * D, c, v);
         Elem<WT>::store(Vs + (size_t)r * RS, c, v);
     }
+}
+
+// The chunk's rows that were committed before the round (below kv_len): they
+// do not depend on any kernel of this round, so they are requested before
+// the dependency wait.  Returns how many rows that is.
+template <typename WT, int D, int RS>
+__device__ __forceinline__ int tree_stage_committed(const TreeArgs &a, int b, int g, int j0, int nk, int L, WT *Ks,
+                                                    WT *Vs) {
+    constexpr int VEC = Elem<WT>::kPerVec;
+    constexpr int VPR = D / VEC;
+    const int ncom = L - j0 < 0 ? 0 : (L - j0 < nk ? L - j0 : nk);
+    const WT *kc = (const WT *)a.k_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D;
+    const WT *vc = (const WT *)a.v_cache + (((size_t)b * a.Hkv + g) * a.max_ctx + j0) * D;
+    for (int e = threadIdx.x; e < ncom * VPR; e += blockDim.x) {
+        const int r = e / VPR, c = e % VPR;
+        cp_async16(Ks + (size_t)r * RS + c * VEC, (const uint4 *)kc + e);
+        cp_async16(Vs + (size_t)r * RS + c * VEC, (const uint4 *)vc + e);
+    }
+    return ncom;
 }
 
 // The last CTA of (b, g) to finish merges every pair's split partials in
@@ -297,7 +317,6 @@ __global__ void __launch_bounds__(kTreeAttnThreads) tree_attention_kernel(const 
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
 
     pdl_trigger();
-    pdl_wait();
 
     const int n = tree_n(a, b), L = a.kv_len[b];
     const int base = L + n;
@@ -306,11 +325,13 @@ __global__ void __launch_bounds__(kTreeAttnThreads) tree_attention_kernel(const 
     const int j0 = s * C;
     const int nk = PE - j0 < C ? PE - j0 : C;
     const float scale = 1.0f / sqrtf((float)D);
+    const int ncom = nk > 0 && L >= 0 ? tree_stage_committed<WT, D, RS>(a, b, g, j0, nk, L, Ks, Vs) : 0;
+    pdl_wait();
     if (s == 0 && g == 0 && threadIdx.x == 0 && (L < 0 || base + (a.step - 1) * a.w > a.max_ctx))
         set_err(a.err, kErrCache);
 
     if (nk > 0 && L >= 0) {
-        tree_stage<WT, D, RS, D>(a, b, g, j0, nk, base, Ks, Vs, qs, 1.0f);
+        tree_stage<WT, D, RS, D>(a, b, g, j0, nk, base, Ks, Vs, qs, 1.0f, ncom);
         cp_async_wait_all();
         __syncthreads();
         for (int pr = warp; pr < NQ; pr += nwarp) {
@@ -427,7 +448,6 @@ __global__ void __launch_bounds__(kTcWarps * 32) tree_attention_tc_kernel(const 
     const int G = a.Hq / a.Hkv, NQ = a.w * G;
 
     pdl_trigger();
-    pdl_wait();
 
     const int n = tree_n(a, b), L = a.kv_len[b];
     const int base = L + n;
@@ -436,11 +456,13 @@ __global__ void __launch_bounds__(kTcWarps * 32) tree_attention_tc_kernel(const 
     const int j0 = s * kTcChunk;
     int nk = PE - j0 < kTcChunk ? PE - j0 : kTcChunk;
     if (L < 0) nk = 0;
+    const int ncom = nk > 0 ? tree_stage_committed<uint16_t, D, RS>(a, b, g, j0, nk, L, Ks, Vs) : 0;
+    pdl_wait();
     if (s == 0 && g == 0 && tid == 0 && (L < 0 || base + (a.step - 1) * a.w > a.max_ctx)) set_err(a.err, kErrCache);
     if (tid < a.w) s_mask[tid] = a.front_mask[b * a.w + tid];
     for (int e = tid; e < (kTcMaxPairs - NQ) * QS; e += blockDim.x) qs[NQ * QS + e] = 0.f;
     if (nk > 0) {
-        tree_stage<uint16_t, D, RS, QS>(a, b, g, j0, nk, base, Ks, Vs, qs, 1.0f / sqrtf((float)D));
+        tree_stage<uint16_t, D, RS, QS>(a, b, g, j0, nk, base, Ks, Vs, qs, 1.0f / sqrtf((float)D), ncom);
         // rows past the chunk's keys: zero (their probabilities are 0, and 0 * NaN would not be)
         for (int e = tid; e < (kTcChunk - nk) * (D / 8); e += blockDim.x) {
             const int r = nk + e / (D / 8), c = e % (D / 8);
