@@ -1251,6 +1251,17 @@ __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int g
     pdl_trigger();
     pdl_wait();
     const int t = blockIdx.x, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (a.next_fuse) {
+        // the h^ half of the next decode step's fusion row does not depend on the token
+        const int d = a.d;
+        const float4 *h = (const float4 *)(a.src + (size_t)t * d);
+        uint4 *x = (uint4 *)(a.next_x + (size_t)t * 2 * d);
+        for (int c = threadIdx.x; c < d / 8; c += 128) {
+            const float4 h0 = __ldcg(h + 2 * c), h1 = __ldcg(h + 2 * c + 1);
+            x[d / 8 + c] = make_uint4(pack_bf16x2(h0.x, h0.y), pack_bf16x2(h0.z, h0.w), pack_bf16x2(h1.x, h1.y),
+                                      pack_bf16x2(h1.z, h1.w));
+        }
+    }
     Key l[kTopK];
     gather_keys<true>(a, t, grid, threadIdx.x, 128, l);
 #pragma unroll 1
@@ -1276,19 +1287,12 @@ __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int g
         }
     }
     if (a.next_fuse) {
-        // the next decode step's fusion row: [E(token); round(h^ row t)]
+        // the token's half of the next decode step's fusion row: E(token)
         __syncthreads();
         const int d = a.d;
         const uint4 *e = (const uint4 *)((const uint16_t *)a.embed + (size_t)token_ok(a, s_tok) * d);
-        const float4 *h = (const float4 *)(a.src + (size_t)t * d);
         uint4 *x = (uint4 *)(a.next_x + (size_t)t * 2 * d);
-        for (int c = threadIdx.x; c < d / 8; c += 128) {
-            const uint4 ev = __ldg(e + c);
-            const float4 h0 = __ldcg(h + 2 * c), h1 = __ldcg(h + 2 * c + 1);
-            x[c] = ev;
-            x[d / 8 + c] = make_uint4(pack_bf16x2(h0.x, h0.y), pack_bf16x2(h0.z, h0.w), pack_bf16x2(h1.x, h1.y),
-                                      pack_bf16x2(h1.z, h1.w));
-        }
+        for (int c = threadIdx.x; c < d / 8; c += 128) x[c] = __ldg(e + c);
     }
 }
 
@@ -1297,77 +1301,97 @@ __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int g
 // next projection's activation row: RMSNorm of the finished row with
 // next_gain (or the row as it is when next_gain is null), rounded to bf16,
 // into next_x.  One kernel instead of the finish and the next row
-// preparation.  Dynamic shared memory: the row, n_units floats.
-constexpr int kRowThreads = 512;
+// preparation.  It sits on the critical path between two projections, so a
+// thread holds its values in registers and issues all its loads at once (the
+// gain, a weight, before the dependency wait).  n_units <= kRowMaxUnits.
+// VEC float4 groups per thread, at most SPL slices (instances keep the
+// loads in flight within the register budget of 1024 threads).
+constexpr int kRowThreads = 1024;
+constexpr int kRowMaxUnits = kRowThreads * 4 * 2;           // 8192
+template <int kRowVec, int SPL>
 __global__ void __launch_bounds__(kRowThreads) splitk_finish_row_kernel(const GemvArgs a, const float *part,
                                                                       int splits) {
-    extern __shared__ float rowv[];
     __shared__ float red[kRowThreads / 32];
     pdl_trigger();
-    pdl_wait();
     const int t = blockIdx.x, n = a.n_units, tid = threadIdx.x;
+    const uint16_t *g = a.next_norm ? (const uint16_t *)a.next_gain : nullptr;
+    uint2 gw[kRowVec];
+#pragma unroll
+    for (int i = 0; i < kRowVec; ++i) {
+        const int u = (tid + i * kRowThreads) * 4;
+        gw[i] = g && u < n ? __ldg((const uint2 *)(g + u)) : make_uint2(0u, 0u);
+    }
+    pdl_wait();
     const int rrow = a.epi == kEpiResid && a.resid_prefill_rows ? t * a.max_new + clamp_n(a, t) - 1 : t;
+    float4 v[kRowVec][SPL], q[kRowVec];
+#pragma unroll
+    for (int i = 0; i < kRowVec; ++i) {
+        const int u = (tid + i * kRowThreads) * 4;
+        if (u >= n) continue;
+#pragma unroll
+        for (int k = 0; k < SPL; ++k)
+            if (k < splits) v[i][k] = __ldcg((const float4 *)&part[((size_t)k * a.T + t) * n + u]);
+        if (a.epi == kEpiResid) q[i] = __ldcg((const float4 *)&a.resid[(size_t)rrow * a.out_ld + u]);
+    }
+    float4 r[kRowVec];
     float ss = 0.f;
-    for (int u = tid * 4; u < n; u += kRowThreads * 4) {
-        float4 v[kMaxSplits];
 #pragma unroll
-        for (int k = 0; k < kMaxSplits; ++k)
-            if (k < splits) v[k] = __ldcg((const float4 *)&part[((size_t)k * a.T + t) * n + u]);
-        float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int i = 0; i < kRowVec; ++i) {
+        const int u = (tid + i * kRowThreads) * 4;
+        r[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (u >= n) continue;
 #pragma unroll
-        for (int k = 0; k < kMaxSplits; ++k)
+        for (int k = 0; k < SPL; ++k)
             if (k < splits) {
-                r.x += v[k].x;
-                r.y += v[k].y;
-                r.z += v[k].z;
-                r.w += v[k].w;
+                r[i].x += v[i][k].x;
+                r[i].y += v[i][k].y;
+                r[i].z += v[i][k].z;
+                r[i].w += v[i][k].w;
             }
         if (a.epi == kEpiResid) {
-            const float4 q = __ldcg((const float4 *)&a.resid[(size_t)rrow * a.out_ld + u]);
-            r.x += q.x;
-            r.y += q.y;
-            r.z += q.z;
-            r.w += q.w;
+            r[i].x += q[i].x;
+            r[i].y += q[i].y;
+            r[i].z += q[i].z;
+            r[i].w += q[i].w;
             if (a.hidden_out) {
                 float *ho = a.hidden_out + ((size_t)t * a.K + a.step - 1) * a.d + u;
-                ho[0] = r.x;
-                ho[1] = r.y;
-                ho[2] = r.z;
-                ho[3] = r.w;
+                ho[0] = r[i].x;
+                ho[1] = r[i].y;
+                ho[2] = r[i].z;
+                ho[3] = r[i].w;
             }
         }
-        *(float4 *)&a.out[(size_t)t * a.out_ld + u] = r;
-        *(float4 *)&rowv[u] = r;
-        ss = fmaf(r.x, r.x, ss);
-        ss = fmaf(r.y, r.y, ss);
-        ss = fmaf(r.z, r.z, ss);
-        ss = fmaf(r.w, r.w, ss);
+        *(float4 *)&a.out[(size_t)t * a.out_ld + u] = r[i];
+        ss = fmaf(r[i].x, r[i].x, ss);
+        ss = fmaf(r[i].y, r[i].y, ss);
+        ss = fmaf(r[i].z, r[i].z, ss);
+        ss = fmaf(r[i].w, r[i].w, ss);
     }
     if (!a.next_norm) return;
     float inv = 1.f;
-    if (a.next_gain) {
+    if (g) {
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
         if ((tid & 31) == 0) red[tid >> 5] = ss;
     }
     __syncthreads();
-    if (a.next_gain) {
+    if (g) {
         float tot = 0.f;
 #pragma unroll
         for (int i = 0; i < kRowThreads / 32; ++i) tot += red[i];
         inv = 1.0f / sqrtf(tot / (float)n + a.eps);
     }
-    const uint16_t *g = (const uint16_t *)a.next_gain;
     uint2 *x = (uint2 *)(a.next_x + (size_t)t * n);
-    for (int u = tid * 4; u < n; u += kRowThreads * 4) {
-        const float4 r = *(const float4 *)&rowv[u];
-        float y[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+    for (int i = 0; i < kRowVec; ++i) {
+        const int u = (tid + i * kRowThreads) * 4;
+        if (u >= n) continue;
+        float y[4] = {r[i].x, r[i].y, r[i].z, r[i].w};
         if (g) {
-            const uint2 gw = __ldg((const uint2 *)(g + u));
-            y[0] = y[0] * inv * bf16lo(gw.x);
-            y[1] = y[1] * inv * bf16hi(gw.x);
-            y[2] = y[2] * inv * bf16lo(gw.y);
-            y[3] = y[3] * inv * bf16hi(gw.y);
+            y[0] = y[0] * inv * bf16lo(gw[i].x);
+            y[1] = y[1] * inv * bf16hi(gw[i].x);
+            y[2] = y[2] * inv * bf16lo(gw[i].y);
+            y[3] = y[3] * inv * bf16hi(gw[i].y);
         }
         x[u / 4] = make_uint2(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]));
     }
@@ -1731,11 +1755,18 @@ cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, f
         if (e == cudaSuccess && next_done) *next_done = m.next_fuse != 0;
     }
     if (e == cudaSuccess && p.defer) {
-        const size_t row_smem = (size_t)a.n_units * sizeof(float);
-        if (a.epi != kEpiSwiGLU && a.next_norm && a.next_x && a.n_units % 4 == 0 && row_smem <= 48 * 1024) {
+        if (a.epi != kEpiSwiGLU && a.next_norm && a.next_x && a.n_units % 4 == 0 && a.n_units <= kRowMaxUnits) {
             // one CTA per row: the sums, then the next projection's normalised row
-            e = launch_k(splitk_finish_row_kernel, dim3(a.T), dim3(kRowThreads), row_smem, s, true, a,
-                         (const float *)part, p.splits);
+            const float *pp = (const float *)part;
+            const dim3 rg(a.T), rb(kRowThreads);
+            if (a.n_units <= kRowThreads * 4)
+                e = p.splits <= 2   ? launch_k(splitk_finish_row_kernel<1, 2>, rg, rb, 0, s, true, a, pp, p.splits)
+                    : p.splits <= 4 ? launch_k(splitk_finish_row_kernel<1, 4>, rg, rb, 0, s, true, a, pp, p.splits)
+                                    : launch_k(splitk_finish_row_kernel<1, 8>, rg, rb, 0, s, true, a, pp, p.splits);
+            else
+                e = p.splits <= 2   ? launch_k(splitk_finish_row_kernel<2, 2>, rg, rb, 0, s, true, a, pp, p.splits)
+                    : p.splits <= 4 ? launch_k(splitk_finish_row_kernel<2, 4>, rg, rb, 0, s, true, a, pp, p.splits)
+                                    : launch_k(splitk_finish_row_kernel<2, 8>, rg, rb, 0, s, true, a, pp, p.splits);
             if (e == cudaSuccess && next_done) *next_done = true;
         } else {
             long nb = ((long)a.T * a.n_units + 255) / 256;
