@@ -372,6 +372,10 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * KV append and attention run as one kernel, a cluster of up to 8 CTAs per
  * sequence and KV head merging through distributed shared memory; 0: a
  * RoPE/append kernel, then split-KV attention with a last-CTA merge),
+ * "attn_tc" (1, the default: the fused attention kernel of a bf16 context
+ * with the tcgen05 projections loads cache chunks with TMA and computes QK^T
+ * and PV with warp-level tensor-core MMAs; 0: the same fused computation on
+ * CUDA cores),
  * "wait_polls" (0, the default: every wait between two roles of a kernel,
  * a consumer for a filled ring stage or accumulator, a producer for a
  * released one, gives up after a built-in bound of 2^22 polls; N > 0: after

@@ -139,6 +139,7 @@ struct prism_ctx {
     int fuse_rows = 1;                                    // streamed projections write the next one's activation rows
     int wait_polls = 0;                                   // role-to-role wait bound (0: built in, < 0: none)
     int w_evict_first = 1;                                // weight streams with an L2 evict-first policy
+    int attn_tc = 1;                                      // fused attention on tensor cores (0: CUDA cores)
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
     bool tc_ready = false;
     CUtensorMap tm_lm;
@@ -303,7 +304,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
 
     // the caches as TMA tensor maps for the tensor-core attention kernel
     CUtensorMap tmk, tmv;
-    const bool cache_maps = c->attn_fused && c->bf16 && c->tc_ready &&
+    const bool cache_maps = c->attn_fused && c->attn_tc && c->bf16 && c->tc_ready &&
                             make_cache_map(&tmk, r.k_cache, r.B * Hkv, f.max_ctx, D, fused_attention_chunk()) == cudaSuccess &&
                             make_cache_map(&tmv, r.v_cache, r.B * Hkv, f.max_ctx, D, fused_attention_chunk()) == cudaSuccess;
 
@@ -945,6 +946,7 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "fuse_rows")) c->fuse_rows = value != 0;
     else if (!std::strcmp(name, "wait_polls")) c->wait_polls = value;
     else if (!std::strcmp(name, "w_evict_first")) c->w_evict_first = value != 0;
+    else if (!std::strcmp(name, "attn_tc")) c->attn_tc = value != 0;
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);
     return PRISM_OK;

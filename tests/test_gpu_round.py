@@ -154,6 +154,14 @@ def test_split_attention_path_matches_oracle(case):
     assert rep["ids_compared"] >= 1
 
 
+def test_fused_attention_on_cuda_cores_matches_oracle():
+    """The fused RoPE/append/attention kernel with QK^T and PV on CUDA cores
+    instead of tensor-core MMAs, at a size whose context spans several chunks."""
+    W, I = mid_case()
+    _, _, rep = _check(MID_W, W, I, [0, 1, 2], topk=4, options={"attn_tc": 0})
+    assert rep["ids_compared"] >= 1
+
+
 def test_tcgen05_modes_bit_identical():
     """Graph replay, eager launches, with and without programmatic dependent
     launch: identical outputs on the tcgen05 path (split-K sums in fixed order)."""
