@@ -375,7 +375,10 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * "attn_tc" (1, the default: the fused attention kernel of a bf16 context
  * with the tcgen05 projections loads cache chunks with TMA and computes QK^T
  * and PV with warp-level tensor-core MMAs; 0: the same fused computation on
- * CUDA cores),
+ * CUDA cores), "attn_warps" (compute warps per CTA of that tensor-core
+ * kernel: 8, stages of 128 keys, one CTA per SM; or 4, stages of 64 keys,
+ * two CTAs per SM; 0, the default: 4 where one CTA per (sequence, KV head)
+ * makes more CTAs than SMs but at most two per SM, else 8),
  * "wait_polls" (0, the default: every wait between two roles of a kernel,
  * a consumer for a filled ring stage or accumulator, a producer for a
  * released one, gives up after a built-in bound of 2^22 polls; N > 0: after
@@ -389,6 +392,10 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * with an L2 evict-first cache policy, since each weight byte is read once
  * per step, so that the KV cache and the activations stay in L2; 0: the
  * default policy),
+ * "prefetch_next_kb" (16384, the default: once a kernel's CTAs have
+ * requested their last weight boxes, they request the first this many KB of
+ * the next kernel's weights into L2, each CTA an even share, so that HBM
+ * keeps streaming across the kernel boundary; 0: none),
  * "fuse_rows" (1, the default: a streamed projection's last kernel, the
  * split-K finish or the LM head's top-k merge, also writes the next
  * projection's bf16 activation rows, its RMSNorm or the next step's fusion

@@ -645,7 +645,7 @@ __global__ void __launch_bounds__(kFusedThreads, 1) fused_attention_kernel(const
 // an error near 2^-17 of the operand, with K and V exact.  Shared memory holds
 // only K and V as TMA wrote them (128-byte swizzle), and each of their bytes is
 // read once.
-//   * Keys stream through a ring of kTaStages stages of kTaC rows, filled by
+//   * Keys stream through a ring of kTaStages stages of 16 W rows, filled by
 //     one producer warp with TMA tensor loads; stages made only of rows
 //     committed before the round are requested before griddepcontrol.wait;
 //   * compute warp w owns keys 16w .. 16w + 15 of every stage and keeps its own
@@ -654,10 +654,16 @@ __global__ void __launch_bounds__(kFusedThreads, 1) fused_attention_kernel(const
 //   * at the end the warps' states merge in shared memory (log-sum-exp rule,
 //     warp order), then the cluster's ranks merge through distributed shared
 //     memory as in the CUDA-core kernel.
-constexpr int kTaWarps = 8;                           // compute warps; one more warp issues loads
-constexpr int kTaThreads = (kTaWarps + 1) * 32;
-constexpr int kTaC = kTaWarps * 16;                   // keys per stage
 constexpr int kTaStages = 3;
+constexpr int kTaBoxRows = 64;                        // rows of one TMA box of the caches
+// W compute warps (one more warp issues loads), 16 W keys per stage; with 4
+// warps two CTAs share an SM
+template <int W> struct TaCfg {
+    static constexpr int kThreads = (W + 1) * 32;
+    static constexpr int kC = 16 * W;
+    static constexpr int kMinBlocks = W <= 4 ? 2 : 1;
+    static_assert(W == 4 || W == 8, "4 or 8 compute warps");
+};
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
@@ -697,16 +703,126 @@ __device__ __forceinline__ bool ta_wait_warp(uint64_t *bar, uint32_t parity, lon
     return ok;
 }
 // Shared-memory address of 16-byte piece `chunk` (8 dims) of row `row` of a
-// stage buffer: D / 64 boxes of kTaC rows x 128 bytes, pieces XOR-swizzled by
-// row (the TMA 128-byte swizzle).
+// stage buffer of C rows: D / 64 column blocks of C rows x 128 bytes (each
+// loaded as C / 64 boxes), pieces XOR-swizzled by row (the TMA 128-byte
+// swizzle).
+template <int C>
 __device__ __forceinline__ uint32_t ta_piece(uint32_t buf, int row, int chunk) {
-    return buf + (uint32_t)(chunk >> 3) * (kTaC * 128) + (uint32_t)row * 128 + ((uint32_t)((chunk & 7) ^ (row & 7)) << 4);
+    return buf + (uint32_t)(chunk >> 3) * (C * 128) + (uint32_t)row * 128 + ((uint32_t)((chunk & 7) ^ (row & 7)) << 4);
 }
 
-template <int D>
-__global__ void __launch_bounds__(kTaThreads, 1)
+// A compute warp's online-softmax state: entries for keys lane / 4 (+ 8) of
+// the warp's 16 and heads h0 = 2 (lane % 4), h1 = h0 + 1; O^T for dims
+// 16 t + lane / 4 (+ 8) of those heads.
+template <int NT> struct TaWarpState {
+    float m0, m1, l0, l1;
+    float o[NT][4];
+    __device__ __forceinline__ void reset() {
+        m0 = m1 = -INFINITY;
+        l0 = l1 = 0.f;
+#pragma unroll
+        for (int t = 0; t < NT; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
+    }
+};
+
+// q^T as B fragments from the rotated, scaled queries qs ([8][D], heads past
+// G zero): b0 = q[h][16 ks + 2 (lane % 4) + {0, 1}], b1 the same dims + 8,
+// h = lane / 4, each as a bf16 pair hi + lo.
+template <int NT>
+__device__ __forceinline__ void ta_q_frags(const float *qs, uint32_t (&qh)[NT][2], uint32_t (&ql)[NT][2]) {
+    constexpr int D = NT * 16;
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int ks = 0; ks < NT; ++ks)
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const float *src = qs + (lane >> 2) * D + 16 * ks + 2 * (lane & 3) + 8 * u;
+            split2(src[0], src[1], qh[ks][u], ql[ks][u]);
+        }
+}
+
+// One stage for one compute warp: its keys kr .. kr + 15 of the stage whose
+// K boxes start at kb and V boxes at vb, the first cnt of them valid (cnt in
+// 1 .. 16), folded into the warp's state.
+template <int NT, int C>
+__device__ __forceinline__ void ta_stage(TaWarpState<NT> &st, uint32_t kb, uint32_t vb, int kr, int cnt,
+                                         const uint32_t (&qh)[NT][2], const uint32_t (&ql)[NT][2]) {
+    constexpr int NH = NT / 4;                        // 64-column boxes per row
+    const int lane = threadIdx.x & 31;
+    // value rows past the range hold other positions' data: zero them
+    // (their probabilities are zero, and 0 * NaN would not be)
+    if (cnt < 16) {
+        for (int e = lane; e < (16 - cnt) * NH * 8; e += 32) {
+            const int row = kr + cnt + e / (NH * 8), piece = e % (NH * 8);
+            asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" ::"r"(ta_piece<C>(vb, row, piece)), "r"(0) : "memory");
+        }
+        __syncwarp();
+    }
+    // S^T for 16 keys x 8 heads, hi and lo queries in separate chains
+    float sh[4] = {0.f, 0.f, 0.f, 0.f}, sl[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int ks = 0; ks < NT; ++ks) {
+        uint32_t ka[4];
+        const int mi = lane >> 3;
+        ldsm_x4(ta_piece<C>(kb, kr + (mi & 1) * 8 + (lane & 7), 2 * ks + (mi >> 1)), ka);
+        mma16816(sh, ka, qh[ks][0], qh[ks][1]);
+        mma16816(sl, ka, ql[ks][0], ql[ks][1]);
+    }
+    float sv[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int key = (lane >> 2) + (q >> 1) * 8;
+        sv[q] = key < cnt ? sh[q] + sl[q] : -INFINITY;
+    }
+    // online softmax of this warp: heads h0 = 2 (lane % 4) (entries 0, 2), h1 (1, 3)
+    float c0 = fmaxf(sv[0], sv[2]), c1 = fmaxf(sv[1], sv[3]);
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+        c0 = fmaxf(c0, __shfl_xor_sync(0xFFFFFFFFu, c0, off));
+        c1 = fmaxf(c1, __shfl_xor_sync(0xFFFFFFFFu, c1, off));
+    }
+    const float n0 = fmaxf(st.m0, c0), n1 = fmaxf(st.m1, c1);
+    const float al0 = st.m0 == -INFINITY ? 0.f : expf(st.m0 - n0), al1 = st.m1 == -INFINITY ? 0.f : expf(st.m1 - n1);
+    float p[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const float mq = (q & 1) ? n1 : n0;
+        p[q] = (sv[q] == -INFINITY || mq == -INFINITY) ? 0.f : expf(sv[q] - mq);
+    }
+    st.l0 = st.l0 * al0 + (p[0] + p[2]);
+    st.l1 = st.l1 * al1 + (p[1] + p[3]);
+    st.m0 = n0;
+    st.m1 = n1;
+#pragma unroll
+    for (int t = 0; t < NT; ++t) {
+        st.o[t][0] *= al0;
+        st.o[t][1] *= al1;
+        st.o[t][2] *= al0;
+        st.o[t][3] *= al1;
+    }
+    // P^T as B fragments: the S^T tile's 8 x 8 halves, transposed in registers
+    uint32_t h01, l01, h23, l23;
+    split2(p[0], p[1], h01, l01);
+    split2(p[2], p[3], h23, l23);
+    const uint32_t pb_h0 = movm_t(h01), pb_h1 = movm_t(h23), pb_l0 = movm_t(l01), pb_l1 = movm_t(l23);
+    // O^T += V^T P^T, one 16-dim tile at a time
+#pragma unroll
+    for (int t = 0; t < NT; ++t) {
+        uint32_t va[4];
+        const int mi = lane >> 3;
+        ldsm_x4_t(ta_piece<C>(vb, kr + (mi >> 1) * 8 + (lane & 7), 2 * t + (mi & 1)), va);
+        mma16816(st.o[t], va, pb_h0, pb_h1);
+        mma16816(st.o[t], va, pb_l0, pb_l1);
+    }
+    // zeros written above precede the next TMA write of this slot
+    if (cnt < 16) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+template <int D, int W>
+__global__ void __launch_bounds__(TaCfg<W>::kThreads, TaCfg<W>::kMinBlocks)
     fused_attention_tc_kernel(const FusedAttnArgs a, const __grid_constant__ CUtensorMap tk,
                               const __grid_constant__ CUtensorMap tv) {
+    constexpr int kTaWarps = W, kTaThreads = TaCfg<W>::kThreads, kTaC = TaCfg<W>::kC;
     constexpr int NH = D / 64;                        // 64-column boxes per row
     constexpr uint32_t kBox = kTaC * 128;
     constexpr uint32_t kStage = 2 * NH * kBox;        // K boxes, then V boxes
@@ -748,16 +864,21 @@ __global__ void __launch_bounds__(kTaThreads, 1)
                      : "memory");
         const uint32_t kd = ring_s + (uint32_t)s * kStage, vd = kd + NH * kBox;
 #pragma unroll
-        for (int h = 0; h < NH; ++h) {
-            asm volatile(
-                "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
-                "%4}], [%5];" ::"r"(kd + h * kBox), "l"((uint64_t)&tk), "r"(h * 64), "r"(j), "r"(z), "r"(sa(&full[s]))
-                : "memory");
-            asm volatile(
-                "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
-                "%4}], [%5];" ::"r"(vd + h * kBox), "l"((uint64_t)&tv), "r"(h * 64), "r"(j), "r"(z), "r"(sa(&full[s]))
-                : "memory");
-        }
+        for (int h = 0; h < NH; ++h)
+#pragma unroll
+            for (int q = 0; q < kTaC / kTaBoxRows; ++q) {
+                const uint32_t o = h * kBox + q * kTaBoxRows * 128;
+                asm volatile(
+                    "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+                    "%3, %4}], [%5];" ::"r"(kd + o), "l"((uint64_t)&tk), "r"(h * 64), "r"(j + q * kTaBoxRows), "r"(z),
+                    "r"(sa(&full[s]))
+                    : "memory");
+                asm volatile(
+                    "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+                    "%3, %4}], [%5];" ::"r"(vd + o), "l"((uint64_t)&tv), "r"(h * 64), "r"(j + q * kTaBoxRows), "r"(z),
+                    "r"(sa(&full[s]))
+                    : "memory");
+            }
     };
     const bool producer = tid == kTaWarps * 32;
     if (producer) {
@@ -823,13 +944,8 @@ __global__ void __launch_bounds__(kTaThreads, 1)
     __syncthreads();
 
     bool dead = false;
-    // compute-warp state: entries for keys lane / 4 (+ 8) of the warp's 16 and
-    // heads h0 = 2 (lane % 4), h1 = h0 + 1; O^T for dims 16 t + lane / 4 (+ 8)
-    constexpr int NTO = NT;
-    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-    float o[NTO][4];
-#pragma unroll
-    for (int t = 0; t < NTO; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
+    TaWarpState<NT> st;
+    st.reset();
     if (warp == kTaWarps) {
         // ---------------------------------------------------------------- producer
         if (producer) {
@@ -849,6 +965,7 @@ __global__ void __launch_bounds__(kTaThreads, 1)
                 load(i);
                 issued = i + 1;
             }
+            if (!dead) prefetch_l2_share(a.pf_next, a.pf_next_bytes, r + CS * (g + a.Hkv * b), CS * a.Hkv * a.B);
             // every copy issued lands before the ring is reused or the CTA exits
             for (int i = issued > kTaStages ? issued - kTaStages : 0; i < issued; ++i) {
                 bool ok = false;
@@ -859,15 +976,8 @@ __global__ void __launch_bounds__(kTaThreads, 1)
         }
     } else {
         // ---------------------------------------------------------------- compute warps
-        // q^T as B fragments: b0 = q[h][16 ks + 2 (lane % 4) + {0, 1}], b1 = the same dims + 8, h = lane / 4
         uint32_t qh[NT][2], ql[NT][2];
-#pragma unroll
-        for (int ks = 0; ks < NT; ++ks)
-#pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                const float *src = qs + (lane >> 2) * D + 16 * ks + 2 * (lane & 3) + 8 * u;
-                split2(src[0], src[1], qh[ks][u], ql[ks][u]);
-            }
+        ta_q_frags<NT>(qs, qh, ql);
         const int kr = 16 * warp;                     // this warp's first row in a stage
         for (int i = 0; i < nst; ++i) {
             const int s = i % kTaStages;
@@ -878,75 +988,8 @@ __global__ void __launch_bounds__(kTaThreads, 1)
             const int key0 = j0 + i * kTaC + kr;     // position of the warp's first key
             const int cnt = min(16, j1 - key0);       // valid keys of the warp (may be <= 0)
             if (!dead && cnt > 0) {
-                const uint32_t kb = ring_s + (uint32_t)s * kStage, vb = kb + NH * kBox;
-                // value rows past the range hold other positions' data: zero them
-                // (their probabilities are zero, and 0 * NaN would not be)
-                if (cnt < 16) {
-                    for (int e = lane; e < (16 - cnt) * NH * 8; e += 32) {
-                        const int row = kr + cnt + e / (NH * 8), piece = e % (NH * 8);
-                        asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" ::"r"(ta_piece(vb, row, piece)), "r"(0)
-                                     : "memory");
-                    }
-                    __syncwarp();
-                }
-                // S^T for 16 keys x 8 heads, hi and lo queries in separate chains
-                float sh[4] = {0.f, 0.f, 0.f, 0.f}, sl[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-                for (int ks = 0; ks < NT; ++ks) {
-                    uint32_t ka[4];
-                    const int mi = lane >> 3;
-                    ldsm_x4(ta_piece(kb, kr + (mi & 1) * 8 + (lane & 7), 2 * ks + (mi >> 1)), ka);
-                    mma16816(sh, ka, qh[ks][0], qh[ks][1]);
-                    mma16816(sl, ka, ql[ks][0], ql[ks][1]);
-                }
-                float sv[4];
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const int key = (lane >> 2) + (q >> 1) * 8;
-                    sv[q] = key < cnt ? sh[q] + sl[q] : -INFINITY;
-                }
-                // online softmax of this warp: heads h0 = 2 (lane % 4) (entries 0, 2), h1 (1, 3)
-                float c0 = fmaxf(sv[0], sv[2]), c1 = fmaxf(sv[1], sv[3]);
-#pragma unroll
-                for (int off = 4; off < 32; off <<= 1) {
-                    c0 = fmaxf(c0, __shfl_xor_sync(0xFFFFFFFFu, c0, off));
-                    c1 = fmaxf(c1, __shfl_xor_sync(0xFFFFFFFFu, c1, off));
-                }
-                const float n0 = fmaxf(m0, c0), n1 = fmaxf(m1, c1);
-                const float al0 = m0 == -INFINITY ? 0.f : expf(m0 - n0), al1 = m1 == -INFINITY ? 0.f : expf(m1 - n1);
-                float p[4];
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const float mq = (q & 1) ? n1 : n0;
-                    p[q] = (sv[q] == -INFINITY || mq == -INFINITY) ? 0.f : expf(sv[q] - mq);
-                }
-                l0 = l0 * al0 + (p[0] + p[2]);
-                l1 = l1 * al1 + (p[1] + p[3]);
-                m0 = n0;
-                m1 = n1;
-#pragma unroll
-                for (int t = 0; t < NT; ++t) {
-                    o[t][0] *= al0;
-                    o[t][1] *= al1;
-                    o[t][2] *= al0;
-                    o[t][3] *= al1;
-                }
-                // P^T as B fragments: the S^T tile's 8 x 8 halves, transposed in registers
-                uint32_t h01, l01, h23, l23;
-                split2(p[0], p[1], h01, l01);
-                split2(p[2], p[3], h23, l23);
-                const uint32_t pb_h0 = movm_t(h01), pb_h1 = movm_t(h23), pb_l0 = movm_t(l01), pb_l1 = movm_t(l23);
-                // O^T += V^T P^T, one 16-dim tile at a time
-#pragma unroll
-                for (int t = 0; t < NT; ++t) {
-                    uint32_t va[4];
-                    const int mi = lane >> 3;
-                    ldsm_x4_t(ta_piece(vb, kr + (mi >> 1) * 8 + (lane & 7), 2 * t + (mi & 1)), va);
-                    mma16816(o[t], va, pb_h0, pb_h1);
-                    mma16816(o[t], va, pb_l0, pb_l1);
-                }
-                // zeros written above precede the next TMA write of this slot
-                if (cnt < 16) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                const uint32_t kb = ring_s + (uint32_t)s * kStage;
+                ta_stage<NT, kTaC>(st, kb, kb + NH * kBox, kr, cnt, qh, ql);
             }
             __syncwarp();
             // a warp that gave up on this stage does not release it (its copy may
@@ -957,26 +1000,26 @@ __global__ void __launch_bounds__(kTaThreads, 1)
         // the warp's sums over its lanes' keys
 #pragma unroll
         for (int off = 4; off < 32; off <<= 1) {
-            l0 += __shfl_xor_sync(0xFFFFFFFFu, l0, off);
-            l1 += __shfl_xor_sync(0xFFFFFFFFu, l1, off);
+            st.l0 += __shfl_xor_sync(0xFFFFFFFFu, st.l0, off);
+            st.l1 += __shfl_xor_sync(0xFFFFFFFFu, st.l1, off);
         }
     }
     __syncthreads();                                  // every copy landed, every warp done with the ring
     if (warp < kTaWarps) {
         const int h0 = 2 * (lane & 3), d0 = lane >> 2;
         if (lane < 4) {
-            wm[warp * 8 + h0] = m0;
-            wm[warp * 8 + h0 + 1] = m1;
-            wl[warp * 8 + h0] = l0;
-            wl[warp * 8 + h0 + 1] = l1;
+            wm[warp * 8 + h0] = st.m0;
+            wm[warp * 8 + h0 + 1] = st.m1;
+            wl[warp * 8 + h0] = st.l0;
+            wl[warp * 8 + h0 + 1] = st.l1;
         }
         float *w0 = wo + (size_t)(warp * 8 + h0) * D, *w1 = w0 + D;
 #pragma unroll
-        for (int t = 0; t < NTO; ++t) {
-            w0[16 * t + d0] = o[t][0];
-            w1[16 * t + d0] = o[t][1];
-            w0[16 * t + d0 + 8] = o[t][2];
-            w1[16 * t + d0 + 8] = o[t][3];
+        for (int t = 0; t < NT; ++t) {
+            w0[16 * t + d0] = st.o[t][0];
+            w1[16 * t + d0] = st.o[t][1];
+            w0[16 * t + d0 + 8] = st.o[t][2];
+            w1[16 * t + d0 + 8] = st.o[t][3];
         }
     }
     __syncthreads();
@@ -1036,14 +1079,14 @@ __global__ void __launch_bounds__(kTaThreads, 1)
     cluster_sync_all();
 }
 
-template <int D>
-constexpr size_t fused_tc_smem_bound() {
-    return 1024 + (size_t)kTaStages * 2 * (D / 64) * kTaC * 128 + (size_t)2 * 8 * D * 4 + 16 * 4;
+template <int D, int W>
+constexpr size_t fused_tc_smem() {
+    return 1024 + (size_t)kTaStages * 2 * (D / 64) * TaCfg<W>::kC * 128 + (size_t)2 * 8 * D * 4 + 16 * 4;
 }
-template <int D>
-size_t fused_tc_smem() { return fused_tc_smem_bound<D>(); }
-static_assert((size_t)kTaWarps * 8 * 128 * 4 + 2 * kTaWarps * 8 * 4 <= (size_t)kTaStages * 2 * 2 * kTaC * 128,
+static_assert((size_t)8 * 8 * 128 * 4 + 2 * 8 * 8 * 4 <= (size_t)kTaStages * 2 * 2 * TaCfg<8>::kC * 128 &&
+                  (size_t)4 * 8 * 128 * 4 + 2 * 4 * 8 * 4 <= (size_t)kTaStages * 2 * 2 * TaCfg<4>::kC * 128,
               "the warps' states fit in the ring");
+static_assert(2 * (fused_tc_smem<128, 4>() + 1024 + 64) <= (size_t)228 * 1024, "two 4-warp CTAs per SM");
 
 template <typename WT, int D>
 size_t fused_smem(int G) {
@@ -1076,8 +1119,13 @@ template <typename WT, int D>
 cudaError_t launch_fused_t(const FusedAttnArgs &a, cudaStream_t s, bool pdl, const CUtensorMap *tk,
                            const CUtensorMap *tv) {
     if constexpr (sizeof(WT) == 2) {
-        if (tk && tv && a.Hq / a.Hkv <= 8)
-            return launch_cluster(fused_attention_tc_kernel<D>, fused_tc_smem<D>(), kTaThreads, a, s, pdl, a, *tk, *tv);
+        if (tk && tv && a.Hq / a.Hkv <= 8) {
+            if (a.warps == 4)
+                return launch_cluster(fused_attention_tc_kernel<D, 4>, fused_tc_smem<D, 4>(), TaCfg<4>::kThreads, a, s,
+                                      pdl, a, *tk, *tv);
+            return launch_cluster(fused_attention_tc_kernel<D, 8>, fused_tc_smem<D, 8>(), TaCfg<8>::kThreads, a, s,
+                                  pdl, a, *tk, *tv);
+        }
     }
     return launch_cluster(fused_attention_kernel<WT, D>, fused_smem<WT, D>(a.Hq / a.Hkv), kFusedThreads, a, s, pdl, a);
 }
@@ -1120,11 +1168,15 @@ cudaError_t prepare_fused_t(int G, int need, int *max_cs) {
         *max_cs = max_cluster_for(fused_attention_kernel<WT, D>, fused_smem<WT, D>(G), kFusedThreads, need);
     if constexpr (sizeof(WT) == 2) {
         if (e == cudaSuccess && G <= 8) {
-            static_assert(fused_tc_smem_bound<D>() <= (size_t)227 * 1024, "tensor-core attention shared memory");
-            e = cudaFuncSetAttribute(fused_attention_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)fused_tc_smem<D>());
+            static_assert(fused_tc_smem<D, 8>() <= (size_t)227 * 1024, "tensor-core attention shared memory");
+            e = cudaFuncSetAttribute(fused_attention_tc_kernel<D, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)fused_tc_smem<D, 8>());
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(fused_attention_tc_kernel<D, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)fused_tc_smem<D, 4>());
             if (e == cudaSuccess && max_cs)
-                *max_cs = max_cluster_for(fused_attention_tc_kernel<D>, fused_tc_smem<D>(), kTaThreads, need);
+                *max_cs = max_cluster_for(fused_attention_tc_kernel<D, 8>, fused_tc_smem<D, 8>(), TaCfg<8>::kThreads,
+                                          need);
         }
     }
     return e;
@@ -1175,7 +1227,7 @@ size_t attention_smem_bytes(bool bf16, int D, int chunk, int G, int splits) {
     return D == 64 ? attn_smem<float, 64>(chunk, G, splits) : attn_smem<float, 128>(chunk, G, splits);
 }
 
-int fused_attention_chunk() { return kTaC; }
+int fused_attention_chunk() { return kTaBoxRows; }
 
 cudaError_t launch_fused_attention(const FusedAttnArgs &a, bool bf16, cudaStream_t s, bool pdl,
                                    const CUtensorMap *tk, const CUtensorMap *tv) {
@@ -1193,7 +1245,7 @@ cudaError_t prepare_fused_attention(bool bf16, int D, int G, int need, int *max_
 }
 
 size_t fused_attention_smem_bytes(bool bf16, int D, int G) {
-    if (bf16 && G <= 8) return D == 64 ? fused_tc_smem<64>() : fused_tc_smem<128>();
+    if (bf16 && G <= 8) return D == 64 ? fused_tc_smem<64, 8>() : fused_tc_smem<128, 8>();
     if (bf16) return D == 64 ? fused_smem<uint16_t, 64>(G) : fused_smem<uint16_t, 128>(G);
     return D == 64 ? fused_smem<float, 64>(G) : fused_smem<float, 128>(G);
 }

@@ -96,6 +96,19 @@ __device__ __forceinline__ uint64_t l2_evict_first_policy() {
     return p;
 }
 
+// Share `part` of `parts` of the byte range [base, base + bytes), cut at
+// 16-byte boundaries, requested into L2 with bulk prefetches of up to 32 KB.
+// A prefetch changes no data; base must be 16-byte aligned.
+__device__ __forceinline__ void prefetch_l2_share(const void *base, long long bytes, int part, int parts) {
+    if (!base || bytes < 16 || parts < 1) return;
+    const long long lo = (bytes * part / parts) & ~15LL;
+    const long long hi = part + 1 == parts ? (bytes & ~15LL) : (bytes * (part + 1) / parts) & ~15LL;
+    for (long long o = lo; o < hi; o += 32768) {
+        const uint32_t n = (uint32_t)(hi - o < 32768 ? hi - o : 32768);
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"((const char *)base + o), "r"(n) : "memory");
+    }
+}
+
 // Running log-sum-exp as (max m, sum s of exp(z - m)): add one logit, and
 // combine two partial pairs.
 __device__ __forceinline__ void lse_add(float &m, float &s, float z) {
@@ -229,6 +242,10 @@ struct GemvArgs {
     // LM head with top-k lists: per row and CTA, (max, sum of exp(z - max))
     // of the logits the CTA produced, [T][gridDim.x][2]; null: not computed
     float *lse_part;
+    // the next kernel's weights: once a CTA has requested its last weight
+    // box it requests its share of these bytes into L2; null / 0: none
+    const void *pf_next;
+    long long pf_next_bytes;
 };
 
 struct RopeArgs {
@@ -264,6 +281,10 @@ struct FusedAttnArgs {
     int B, max_new, prefill, step, Hq, Hkv, D, max_ctx, cs;
     int *err;
     int wait_polls;                    // see wait_bound
+    int warps;                         // tensor-core kernel: compute warps per CTA, 8 (0) or 4 (two CTAs per SM)
+    // the next kernel's weights, requested into L2 as in GemvArgs
+    const void *pf_next;
+    long long pf_next_bytes;
 };
 
 struct AcceptArgs {

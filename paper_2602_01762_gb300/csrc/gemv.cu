@@ -302,6 +302,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvArgs a, con
             if (++c == n_chunks) c = 0;
             if (++s == S) { s = 0; ph ^= 1; }
         }
+        if (issued == total) prefetch_l2_share(a.pf_next, a.pf_next_bytes, blockIdx.x, gridDim.x);
         // drain: the last stages' copies land before this CTA may exit
         for (int i = issued > S ? issued - S : 0; i < issued; ++i)
             if (!mbar_wait(&full[i % S], (uint32_t)((i / S) & 1))) set_err(a.err, kErrTimeout);

@@ -674,6 +674,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     if (++s == S) { s = 0; ph ^= 1; }
                 }
             }
+            if (!dead) prefetch_l2_share(a.pf_next, a.pf_next_bytes, blockIdx.x, gridDim.x);
             // drain: the copies in flight land before this CTA may exit
             const int first = issued > S ? issued - S : 0;
             for (int i = first; i < issued; ++i)
@@ -1031,6 +1032,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 ++issued;
                 if (++s == S) { s = 0; ph ^= 1; }
             }
+            if (!dead) prefetch_l2_share(a.pf_next, a.pf_next_bytes, blockIdx.x, gridDim.x);
             const int first = issued > S ? issued - S : 0;
             for (int i = first; i < issued; ++i)
                 if (!mbar_wait(&full[i % S], (uint32_t)((i / S) & 1))) set_err(a.err, kErrTimeout);
@@ -1247,23 +1249,57 @@ __global__ void __launch_bounds__(256) splitk_finish_kernel(const GemvArgs a, co
 // cache-miss speed, so it is written with rolled loops (one copy of the
 // insertion and merge networks).
 __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int grid) {
+    // It runs once per row while HBM streams the next weights, so each load
+    // round trip waits behind full queues: the candidates and the h^ half of
+    // the next fusion row are all requested before any is used, and the
+    // E(token) half in one more batch once the token is known.
+    constexpr int kB = 16;                          // candidates per thread in the first batch
+    constexpr int kG = 4;                           // 8-element groups of a row per thread and batch
     __shared__ Key s_k[4][kTopK];
+    __shared__ int s_tok;
     pdl_trigger();
     pdl_wait();
-    const int t = blockIdx.x, w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (a.next_fuse) {
+    const int t = blockIdx.x, w = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
+    const int ncand = grid * kTopK, d = a.d, ng = d / 8;
+    const float *pv = a.lm_part + (size_t)t * ncand;
+    const int *pi = a.lm_part_id + (size_t)t * ncand;
+    float cv[kB];
+    int ci[kB];
+#pragma unroll
+    for (int b = 0; b < kB; ++b) {
+        const int cc = tid + b * 128;
+        cv[b] = cc < ncand ? __ldcg(pv + cc) : 0.f;
+        ci[b] = cc < ncand ? __ldcg(pi + cc) : -1;
+    }
+    uint4 *x = a.next_fuse ? (uint4 *)(a.next_x + (size_t)t * 2 * d) : nullptr;
+    if (x) {
         // the h^ half of the next decode step's fusion row does not depend on the token
-        const int d = a.d;
         const float4 *h = (const float4 *)(a.src + (size_t)t * d);
-        uint4 *x = (uint4 *)(a.next_x + (size_t)t * 2 * d);
-        for (int c = threadIdx.x; c < d / 8; c += 128) {
-            const float4 h0 = __ldcg(h + 2 * c), h1 = __ldcg(h + 2 * c + 1);
-            x[d / 8 + c] = make_uint4(pack_bf16x2(h0.x, h0.y), pack_bf16x2(h0.z, h0.w), pack_bf16x2(h1.x, h1.y),
-                                      pack_bf16x2(h1.z, h1.w));
+#pragma unroll 1
+        for (int c0 = 0; c0 < ng; c0 += 128 * kG) {
+            float4 v0[kG], v1[kG];
+#pragma unroll
+            for (int q = 0; q < kG; ++q) {
+                const int c = c0 + tid + q * 128;
+                v0[q] = c < ng ? __ldcg(h + 2 * c) : make_float4(0.f, 0.f, 0.f, 0.f);
+                v1[q] = c < ng ? __ldcg(h + 2 * c + 1) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int q = 0; q < kG; ++q) {
+                const int c = c0 + tid + q * 128;
+                if (c < ng)
+                    x[ng + c] = make_uint4(pack_bf16x2(v0[q].x, v0[q].y), pack_bf16x2(v0[q].z, v0[q].w),
+                                           pack_bf16x2(v1[q].x, v1[q].y), pack_bf16x2(v1[q].z, v1[q].w));
+            }
         }
     }
     Key l[kTopK];
-    gather_keys<true>(a, t, grid, threadIdx.x, 128, l);
+    key_clear(l);
+#pragma unroll 1
+    for (int b = 0; b < kB; ++b)
+        if (ci[b] >= 0) key_insert(l, pack_best(cv[b], ci[b]));
+#pragma unroll 1
+    for (int cc = tid + kB * 128; cc < ncand; cc += 128) key_insert(l, pack_best(__ldcg(pv + cc), __ldcg(pi + cc)));
 #pragma unroll 1
     for (int m = 1; m < 32; m <<= 1) key_merge_xor(l, m);
     if (lane == 0) {
@@ -1271,7 +1307,6 @@ __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int g
         for (int i = 0; i < kTopK; ++i) s_k[w][i] = l[i];
     }
     __syncthreads();
-    __shared__ int s_tok;
     if (w == 0) {
 #pragma unroll
         for (int i = 0; i < kTopK; ++i) l[i] = lane < 4 ? s_k[lane][i] : 0ull;
@@ -1286,13 +1321,24 @@ __global__ void __launch_bounds__(128) topk_merge_kernel(const GemvArgs a, int g
             s_tok = id;
         }
     }
-    if (a.next_fuse) {
+    if (x) {
         // the token's half of the next decode step's fusion row: E(token)
         __syncthreads();
-        const int d = a.d;
         const uint4 *e = (const uint4 *)((const uint16_t *)a.embed + (size_t)token_ok(a, s_tok) * d);
-        uint4 *x = (uint4 *)(a.next_x + (size_t)t * 2 * d);
-        for (int c = threadIdx.x; c < d / 8; c += 128) x[c] = __ldg(e + c);
+#pragma unroll 1
+        for (int c0 = 0; c0 < ng; c0 += 128 * kG) {
+            uint4 r[kG];
+#pragma unroll
+            for (int q = 0; q < kG; ++q) {
+                const int c = c0 + tid + q * 128;
+                r[q] = c < ng ? __ldg(e + c) : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int q = 0; q < kG; ++q) {
+                const int c = c0 + tid + q * 128;
+                if (c < ng) x[c] = r[q];
+            }
+        }
     }
 }
 

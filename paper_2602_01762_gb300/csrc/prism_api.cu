@@ -5,6 +5,7 @@
 #include <cstdio>
 #include <cstring>
 #include <string>
+#include <utility>
 #include <vector>
 
 #include "../../include/prism.h"
@@ -140,6 +141,8 @@ struct prism_ctx {
     int wait_polls = 0;                                   // role-to-role wait bound (0: built in, < 0: none)
     int w_evict_first = 1;                                // weight streams with an L2 evict-first policy
     int attn_tc = 1;                                      // fused attention on tensor cores (0: CUDA cores)
+    int prefetch_next_kb = 16384;                         // KB of the next kernel's weights requested into L2
+    int attn_warps = 0;                                   // tensor-core attention warps per CTA: 0 auto, 4 or 8
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
     bool tc_ready = false;
     CUtensorMap tm_lm;
@@ -492,6 +495,19 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         return g;
     };
     const CUtensorMap *lm_tm = c->tm_lm_ok ? &c->tm_lm : nullptr;
+    // a kernel's CTAs, once their own weights are requested, request the next
+    // kernel's first bytes into L2
+    const size_t wes = c->bf16 ? 2 : 4;
+    auto pf = [&](const void *w, size_t elems) -> std::pair<const void *, long long> {
+        const long long cap = (long long)c->prefetch_next_kb * 1024;
+        if (!w || cap <= 0) return {nullptr, 0};
+        return {w, std::min(cap, (long long)(elems * wes))};
+    };
+    auto with_pf = [&](GemvArgs g, std::pair<const void *, long long> n) {
+        g.pf_next = n.first;
+        g.pf_next_bytes = n.second;
+        return g;
+    };
 
     for (int k = 1; k <= K && e == cudaSuccess; ++k) {
         const bool prefill = k == 1;
@@ -512,7 +528,8 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         // fusion F(E(x), h), then the attention pre-norm + QKV, whose rows the
         // fusion's last kernel can write
         const GemvArgs gq = qkv_args(k);
-        e = proj(fusion_args(k), step_tm(k, 0), gemv_grid(c, d), tstep ? pdl : p, &gq, step_tm(k, 1));
+        e = proj(with_pf(fusion_args(k), pf(c->steps[k - 1].w_qkv, (size_t)c->qkv_rows * d)), step_tm(k, 0),
+                 gemv_grid(c, d), tstep ? pdl : p, &gq, step_tm(k, 1));
         after(0);
         if (e != cudaSuccess) break;
         e = proj(gq, step_tm(k, 1), gemv_grid(c, c->qkv_rows), pdl);
@@ -548,6 +565,16 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
             while (fa.cs > 1 && (long long)r.B * Hkv * fa.cs > (long long)c->attn_ctas_per_sm * c->sms) fa.cs /= 2;
             fa.err = c->err;
             fa.wait_polls = c->wait_polls;
+            {
+                const auto n = pf(c->steps[k - 1].w_o, (size_t)d * Hq * D);
+                fa.pf_next = n.first;
+                fa.pf_next_bytes = n.second;
+            }
+            // more CTAs than SMs but no more than two per SM: 4-warp CTAs, two per
+            // SM, run as one wave instead of two
+            const long long ctas = (long long)r.B * Hkv * fa.cs;
+            fa.warps = c->attn_warps ? c->attn_warps : fa.cs == 1 && ctas > c->sms && ctas <= 2LL * c->sms ? 4 : 8;
+            if (fa.warps == 4 && fa.cs > 8) fa.cs = 8;   // clusters of 16 are checked for the 8-warp kernel only
             e = launch_fused_attention(fa, c->bf16, s, pdl, cache_maps ? &tmk : nullptr, cache_maps ? &tmv : nullptr);
             after(3);
             if (e != cudaSuccess) break;
@@ -608,18 +635,21 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         // selection -> x^_k.  Each hands its rows to the next where it can;
         // the LM head to the next step's fusion in a greedy chain.
         const GemvArgs gg = gate_up_args(k), gl = lm_args(k);
-        e = proj(o_args(k), step_tm(k, 2), gemv_grid(c, d), pdl, &gg, step_tm(k, 3));
+        e = proj(with_pf(o_args(k), pf(c->steps[k - 1].w_gate_up, (size_t)2 * F * d)), step_tm(k, 2),
+                 gemv_grid(c, d), pdl, &gg, step_tm(k, 3));
         after(4);
         if (e != cudaSuccess) break;
-        e = proj(gg, step_tm(k, 3), gemv_grid(c, F), pdl);
+        e = proj(with_pf(gg, pf(c->steps[k - 1].w_down, (size_t)d * F)), step_tm(k, 3), gemv_grid(c, F), pdl);
         after(5);
         if (e != cudaSuccess) break;
-        e = proj(down_args(k), step_tm(k, 4), gemv_grid(c, d), pdl, &gl, lm_tm);
+        e = proj(with_pf(down_args(k), pf(c->lm_head, (size_t)V * d)), step_tm(k, 4), gemv_grid(c, d), pdl, &gl,
+                 lm_tm);
         after(6);
         if (e != cudaSuccess) break;
         const bool chain_next = k < K && !tree && !(r.temperature > 0.f);
         const GemvArgs gn = chain_next ? fusion_args(k + 1) : GemvArgs{};
-        e = proj(gl, lm_tm, c->lm_grid, pdl, chain_next ? &gn : nullptr, chain_next ? step_tm(k + 1, 0) : nullptr);
+        e = proj(with_pf(gl, pf(k < K ? c->steps[k].w_fuse : nullptr, (size_t)d * 2 * d)), lm_tm, c->lm_grid, pdl,
+                 chain_next ? &gn : nullptr, chain_next ? step_tm(k + 1, 0) : nullptr);
         if (tree) {
             ta.logits = gl.logits;
             ta.lm_lse_grid = gl.lse_part ? (V + 127) / 128 < c->sms ? (V + 127) / 128 : c->sms : 0;
@@ -947,6 +977,13 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "wait_polls")) c->wait_polls = value;
     else if (!std::strcmp(name, "w_evict_first")) c->w_evict_first = value != 0;
     else if (!std::strcmp(name, "attn_tc")) c->attn_tc = value != 0;
+    else if (!std::strcmp(name, "prefetch_next_kb")) {
+        if (value < 0) return fail(c, PRISM_ERR_INVALID_ARG, "prefetch_next_kb must be >= 0");
+        c->prefetch_next_kb = value;
+    } else if (!std::strcmp(name, "attn_warps")) {
+        if (value != 0 && value != 4 && value != 8) return fail(c, PRISM_ERR_INVALID_ARG, "attn_warps must be 0, 4 or 8");
+        c->attn_warps = value;
+    }
     else return fail(c, PRISM_ERR_INVALID_ARG, std::string("unknown option ") + name);
     drop_graphs(c);
     return PRISM_OK;

@@ -162,6 +162,15 @@ def test_fused_attention_on_cuda_cores_matches_oracle():
     assert rep["ids_compared"] >= 1
 
 
+def test_four_warp_cluster_attention_matches_oracle():
+    """The cluster attention kernel with 4 compute warps (64-key stages, two
+    CTAs per SM) and a cluster of CTAs per (sequence, KV head) merging
+    through distributed shared memory."""
+    W, I = mid_case()
+    _, _, rep = _check(MID_W, W, I, [0, 1, 2], topk=4, options={"attn_warps": 4})
+    assert rep["ids_compared"] >= 1
+
+
 def test_tcgen05_modes_bit_identical():
     """Graph replay, eager launches, with and without programmatic dependent
     launch: identical outputs on the tcgen05 path (split-K sums in fixed order)."""
