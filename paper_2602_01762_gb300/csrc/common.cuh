@@ -366,6 +366,9 @@ struct TreeArgs {
     int *attn_ctr;                    // [B, Hkv] (left at zero)
     void *o_out;                      // [B*w, Hq*D] wtype
     int chunk, splits;
+    // the O projection's weights, requested into L2 as in GemvArgs
+    const void *pf_next;
+    long long pf_next_bytes;
     // caller outputs: the verified tree [B, n_nodes]; optional pool [B, P] and frontier [B, K, w]
     int32_t *tree_tokens, *tree_parents, *tree_depths;
     float *tree_scores;

@@ -539,6 +539,9 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         if (tstep) {
             // RoPE at the node's depth, K/V appended at its own slot, attention
             // over the committed rows and the node's ancestors: one kernel
+            const auto n = pf(c->steps[k - 1].w_o, (size_t)d * Hq * D);
+            ta.pf_next = n.first;
+            ta.pf_next_bytes = n.second;
             e = launch_tree_attention(ta, c->bf16, s, pdl);
             after(3);
             if (e != cudaSuccess) break;

@@ -472,6 +472,9 @@ __global__ void __launch_bounds__(kTcWarps * 32) tree_attention_tc_kernel(const 
     }
     cp_async_wait_all();
     __syncthreads();
+    // this CTA's keys are in: its share of the next kernel's weights into L2
+    if (tid == 0)
+        prefetch_l2_share(a.pf_next, a.pf_next_bytes, s + a.splits * (g + a.Hkv * b), a.splits * a.Hkv * a.B);
 
     // warp state: pairs nt * 8 + 2 (lane % 4) + {0, 1}; O^T dims 16 t + lane / 4 (+ 8)
     const int kr = 16 * warp;
