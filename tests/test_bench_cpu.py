@@ -92,9 +92,11 @@ def test_committed_traffic_figure_is_tied_to_its_kernel_source(tmp_path):
     got = bench.traffic_from_profile(src, rec["workload"])
     if current:
         assert got == rec["dram_bytes_per_launch_full_size"]
-        # DRAM traffic of the capture is the algorithmic bytes plus well under 1 %
+        # DRAM traffic of the capture is the algorithmic bytes, plus the next
+        # step's first 16 MiB of fusion weights that the kernel requests into
+        # L2 (option prefetch_next_kb), plus well under 1 %
         w = WORKLOADS[rec["workload"]]
-        assert 1.0 <= got / bench.lm_head_bytes(w) < 1.01
+        assert 1.0 <= got / (bench.lm_head_bytes(w) + 16 * 1024 * 1024) < 1.01
     else:
         assert got is None
     other = tmp_path / "edited.cu"
