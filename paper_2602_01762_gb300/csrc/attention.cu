@@ -781,25 +781,33 @@ __device__ __forceinline__ void ta_stage(TaWarpState<NT> &st, uint32_t kb, uint3
         c0 = fmaxf(c0, __shfl_xor_sync(0xFFFFFFFFu, c0, off));
         c1 = fmaxf(c1, __shfl_xor_sync(0xFFFFFFFFu, c1, off));
     }
+    // scores are in log2 units (the queries carry log2(e) / sqrt(D)): exp2
     const float n0 = fmaxf(st.m0, c0), n1 = fmaxf(st.m1, c1);
-    const float al0 = st.m0 == -INFINITY ? 0.f : expf(st.m0 - n0), al1 = st.m1 == -INFINITY ? 0.f : expf(st.m1 - n1);
     float p[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
         const float mq = (q & 1) ? n1 : n0;
-        p[q] = (sv[q] == -INFINITY || mq == -INFINITY) ? 0.f : expf(sv[q] - mq);
+        p[q] = (sv[q] == -INFINITY || mq == -INFINITY) ? 0.f : exp2f(sv[q] - mq);
     }
-    st.l0 = st.l0 * al0 + (p[0] + p[2]);
-    st.l1 = st.l1 * al1 + (p[1] + p[3]);
+    // the running sums rescale only where a lane's maximum moved (rarely,
+    // after the first stages)
+    if (__any_sync(0xFFFFFFFFu, n0 != st.m0 || n1 != st.m1)) {
+        const float al0 = st.m0 == -INFINITY ? 0.f : exp2f(st.m0 - n0);
+        const float al1 = st.m1 == -INFINITY ? 0.f : exp2f(st.m1 - n1);
+        st.l0 *= al0;
+        st.l1 *= al1;
+#pragma unroll
+        for (int t = 0; t < NT; ++t) {
+            st.o[t][0] *= al0;
+            st.o[t][1] *= al1;
+            st.o[t][2] *= al0;
+            st.o[t][3] *= al1;
+        }
+    }
+    st.l0 += p[0] + p[2];
+    st.l1 += p[1] + p[3];
     st.m0 = n0;
     st.m1 = n1;
-#pragma unroll
-    for (int t = 0; t < NT; ++t) {
-        st.o[t][0] *= al0;
-        st.o[t][1] *= al1;
-        st.o[t][2] *= al0;
-        st.o[t][3] *= al1;
-    }
     // P^T as B fragments: the S^T tile's 8 x 8 halves, transposed in registers
     uint32_t h01, l01, h23, l23;
     split2(p[0], p[1], h01, l01);
@@ -924,7 +932,8 @@ __global__ void __launch_bounds__(TaCfg<W>::kThreads, TaCfg<W>::kMinBlocks)
     {
         const int row = a.prefill ? b * a.max_new + n - 1 : b;
         const int pc = qp >= 0 && qp < a.max_ctx ? qp : 0;
-        const float scale = 1.0f / sqrtf((float)D);
+        // 1/sqrt(D), times log2(e): the scores come out in log2 units
+        const float scale = 1.4426950408889634f / sqrtf((float)D);
         for (int e = tid; e < 8 * half; e += kTaThreads) {
             const int h = e / half, j = e % half;
             float y0 = 0.f, y1 = 0.f;
@@ -1033,7 +1042,7 @@ __global__ void __launch_bounds__(TaCfg<W>::kThreads, TaCfg<W>::kMinBlocks)
 #pragma unroll
         for (int w = 0; w < kTaWarps; ++w) {
             const float mw = wm[w * 8 + h];
-            const float f = mw == -INFINITY ? 0.f : expf(mw - M);
+            const float f = mw == -INFINITY ? 0.f : exp2f(mw - M);
             den = fmaf(f, wl[w * 8 + h], den);
             num = fmaf(f, wo[(size_t)(w * 8 + h) * D + d], num);
         }
@@ -1068,7 +1077,7 @@ __global__ void __launch_bounds__(TaCfg<W>::kThreads, TaCfg<W>::kMinBlocks)
             float num = 0.f, den = 0.f;
 #pragma unroll
             for (int q = 0; q < kMaxCluster; ++q) {
-                const float w = mq[q] == -INFINITY ? 0.f : expf(mq[q] - M);
+                const float w = mq[q] == -INFINITY ? 0.f : exp2f(mq[q] - M);
                 den = fmaf(w, lq[q], den);
                 num = fmaf(w, oq[q], num);
             }
