@@ -758,21 +758,22 @@ __device__ __forceinline__ void ta_stage(TaWarpState<NT> &st, uint32_t kb, uint3
         }
         __syncwarp();
     }
-    // S^T for 16 keys x 8 heads, hi and lo queries in separate chains
-    float sh[4] = {0.f, 0.f, 0.f, 0.f}, sl[4] = {0.f, 0.f, 0.f, 0.f};
+    // S^T for 16 keys x 8 heads: hi and lo queries, even and odd 16-dim
+    // tiles in four independent accumulation chains (half the dependent depth)
+    float sh[2][4] = {}, sl[2][4] = {};
 #pragma unroll
     for (int ks = 0; ks < NT; ++ks) {
         uint32_t ka[4];
         const int mi = lane >> 3;
         ldsm_x4(ta_piece<C>(kb, kr + (mi & 1) * 8 + (lane & 7), 2 * ks + (mi >> 1)), ka);
-        mma16816(sh, ka, qh[ks][0], qh[ks][1]);
-        mma16816(sl, ka, ql[ks][0], ql[ks][1]);
+        mma16816(sh[ks & 1], ka, qh[ks][0], qh[ks][1]);
+        mma16816(sl[ks & 1], ka, ql[ks][0], ql[ks][1]);
     }
     float sv[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
         const int key = (lane >> 2) + (q >> 1) * 8;
-        sv[q] = key < cnt ? sh[q] + sl[q] : -INFINITY;
+        sv[q] = key < cnt ? (sh[0][q] + sh[1][q]) + (sl[0][q] + sl[1][q]) : -INFINITY;
     }
     // online softmax of this warp: heads h0 = 2 (lane % 4) (entries 0, 2), h1 (1, 3)
     float c0 = fmaxf(sv[0], sv[2]), c1 = fmaxf(sv[1], sv[3]);
