@@ -378,7 +378,10 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * CUDA cores), "attn_warps" (compute warps per CTA of that tensor-core
  * kernel: 8, stages of 128 keys, one CTA per SM; or 4, stages of 64 keys,
  * two CTAs per SM; 0, the default: 4 where one CTA per (sequence, KV head)
- * makes more CTAs than SMs but at most two per SM, else 8),
+ * makes more CTAs than SMs but at most two per SM, else 8), "attn_lpt" (1,
+ * the default: where that kernel's CTAs make more than one wave but at most
+ * two, the CTAs take the sequences in order of decreasing context length;
+ * 0: in index order),
  * "wait_polls" (0, the default: every wait between two roles of a kernel,
  * a consumer for a filled ring stage or accumulator, a producer for a
  * released one, gives up after a built-in bound of 2^22 polls; N > 0: after

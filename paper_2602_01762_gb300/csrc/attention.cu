@@ -827,6 +827,33 @@ __device__ __forceinline__ void ta_stage(TaWarpState<NT> &st, uint32_t kb, uint3
     if (cnt < 16) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// With two waves of CTAs the order in which they start decides the tail:
+// clusters start roughly in the order of their linear index, so the one with
+// sequence index z takes the sequence of rank z in decreasing key count (ties
+// by index), and the longest contexts run first.  Every CTA ranks the
+// sequences itself from the round's inputs (no kernel of the round writes
+// them), before the dependency wait.
+constexpr int kLptMaxB = 256;
+__device__ __forceinline__ int lpt_sequence(const FusedAttnArgs &a, int z) {
+    __shared__ int s_p[kLptMaxB];
+    __shared__ int s_b;
+    const int B = a.B;
+    for (int t = threadIdx.x; t < B; t += blockDim.x) {
+        const int n = clamp_n(a.n_new, t, a.max_new, a.err);
+        s_p[t] = min(query_pos(a.prefill, a.kv_len[t], n, a.step) + 1, a.max_ctx);
+    }
+    if (threadIdx.x == 0) s_b = z;
+    __syncthreads();
+    for (int t = threadIdx.x; t < B; t += blockDim.x) {
+        const int p = s_p[t];
+        int rank = 0;
+        for (int u = 0; u < B; ++u) rank += s_p[u] > p || (s_p[u] == p && u < t);
+        if (rank == z) s_b = t;
+    }
+    __syncthreads();
+    return s_b;
+}
+
 template <int D, int W>
 __global__ void __launch_bounds__(TaCfg<W>::kThreads, TaCfg<W>::kMinBlocks)
     fused_attention_tc_kernel(const FusedAttnArgs a, const __grid_constant__ CUtensorMap tk,
@@ -848,11 +875,12 @@ __global__ void __launch_bounds__(TaCfg<W>::kThreads, TaCfg<W>::kMinBlocks)
     float *wm = wo + kTaWarps * 8 * D;                 // [warp][8]
     float *wl = wm + kTaWarps * 8;                     // [warp][8]
 
-    const int r = blockIdx.x, g = blockIdx.y, b = blockIdx.z, CS = a.cs;
+    const int r = blockIdx.x, g = blockIdx.y, CS = a.cs;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int half = D / 2, H = a.Hq + 2 * a.Hkv, G = a.Hq / a.Hkv;
     const long lim = wait_bound(a.wait_polls, kAttnWaitLimit);
     pdl_trigger();
+    const int b = a.lpt ? lpt_sequence(a, blockIdx.z) : blockIdx.z;
 
     const int n = clamp_n(a.n_new, b, a.max_new, a.err);
     const int L = a.kv_len[b];
@@ -1096,7 +1124,8 @@ constexpr size_t fused_tc_smem() {
 static_assert((size_t)8 * 8 * 128 * 4 + 2 * 8 * 8 * 4 <= (size_t)kTaStages * 2 * 2 * TaCfg<8>::kC * 128 &&
                   (size_t)4 * 8 * 128 * 4 + 2 * 4 * 8 * 4 <= (size_t)kTaStages * 2 * 2 * TaCfg<4>::kC * 128,
               "the warps' states fit in the ring");
-static_assert(2 * (fused_tc_smem<128, 4>() + 1024 + 64) <= (size_t)228 * 1024, "two 4-warp CTAs per SM");
+static_assert(2 * (fused_tc_smem<128, 4>() + 1024 + 64 + (kLptMaxB + 1) * 4) <= (size_t)228 * 1024,
+              "two 4-warp CTAs per SM");
 
 template <typename WT, int D>
 size_t fused_smem(int G) {

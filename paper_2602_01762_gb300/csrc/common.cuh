@@ -282,6 +282,7 @@ struct FusedAttnArgs {
     int *err;
     int wait_polls;                    // see wait_bound
     int warps;                         // tensor-core kernel: compute warps per CTA, 8 (0) or 4 (two CTAs per SM)
+    int lpt;                           // 1: longest sequences first (B <= 256)
     // the next kernel's weights, requested into L2 as in GemvArgs
     const void *pf_next;
     long long pf_next_bytes;
