@@ -395,7 +395,11 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * with an L2 evict-first cache policy, since each weight byte is read once
  * per step, so that the KV cache and the activations stay in L2; 0: the
  * default policy),
- * "prefetch_next_kb" (16384, the default: once a kernel's CTAs have
+ * "lm_even_waves" (1, the default: the LM head launches the fewest CTAs
+ * that stream its 128-row tiles in as many waves as one CTA per SM would, so
+ * that every CTA streams the same number of tiles, e.g. 144 CTAs of 7 tiles
+ * for a vocabulary of 128256 instead of 152 CTAs of 6 or 7; 0: one CTA per
+ * SM), "prefetch_next_kb" (16384, the default: once a kernel's CTAs have
  * requested their last weight boxes, they request the first this many KB of
  * the next kernel's weights into L2, each CTA an even share, so that HBM
  * keeps streaming across the kernel boundary; 0: none),

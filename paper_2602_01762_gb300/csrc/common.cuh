@@ -246,6 +246,9 @@ struct GemvArgs {
     // box it requests its share of these bytes into L2; null / 0: none
     const void *pf_next;
     long long pf_next_bytes;
+    // 1: a selection (LM head) launch takes the fewest CTAs that keep its
+    // number of tile waves, so that every CTA streams as many tiles
+    int even_waves;
 };
 
 struct RopeArgs {

@@ -1594,6 +1594,10 @@ bool tc_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem) {
     p.stages = (int)(room / p.stage_bytes);
     if (p.stages > kTcMaxStages) p.stages = kTcMaxStages;
     if (p.stages < 2) return false;
+    if (a.even_waves && a.epi == kEpiTopK && best_s == 1) {
+        const int waves = (n_tiles + best_ctas - 1) / best_ctas;
+        best_ctas = (n_tiles + waves - 1) / waves;
+    }
     grid = best_ctas * best_s;
     smem = 1024 + (size_t)p.stages * p.stage_bytes + p.x_bytes;
     return true;
@@ -1658,6 +1662,10 @@ bool tcs_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem, in
     p.stages = (int)(room / p.stage_bytes);
     if (p.stages > kTcMaxStages) p.stages = kTcMaxStages;
     if (p.stages < 2) return false;
+    if (a.even_waves && topk && best_s == 1) {
+        const int waves = (n_tiles + best_ctas - 1) / best_ctas;
+        best_ctas = (n_tiles + waves - 1) / waves;
+    }
     grid = best_ctas * best_s;
     smem = 1024 + (size_t)p.stages * p.stage_bytes;
     return true;

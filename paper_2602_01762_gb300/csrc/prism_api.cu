@@ -142,6 +142,7 @@ struct prism_ctx {
     int w_evict_first = 1;                                // weight streams with an L2 evict-first policy
     int attn_tc = 1;                                      // fused attention on tensor cores (0: CUDA cores)
     int prefetch_next_kb = 16384;                         // KB of the next kernel's weights requested into L2
+    int lm_even_waves = 1;                                // LM head: the fewest CTAs with the same tile waves
     int attn_warps = 0;                                   // tensor-core attention warps per CTA: 0 auto, 4 or 8
     int attn_lpt = 1;                                     // several waves of attention CTAs: longest sequences first
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
@@ -458,6 +459,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         GemvArgs g = base;
         g.step = k;
         g.W = c->lm_head;
+        g.even_waves = c->lm_even_waves;
         g.n_units = V;
         g.kin = d;
         g.T = rows_trow(k);
@@ -664,7 +666,12 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
                  chain_next ? &gn : nullptr, chain_next ? step_tm(k + 1, 0) : nullptr);
         if (tree) {
             ta.logits = gl.logits;
-            ta.lm_lse_grid = gl.lse_part ? (V + 127) / 128 < c->sms ? (V + 127) / 128 : c->sms : 0;
+            // the LM head's grid (one log-sum-exp partial per CTA and row): one
+            // CTA per SM, or with even waves the fewest CTAs for as many waves
+            const int lm_tiles = (V + 127) / 128;
+            int lm_ctas = lm_tiles < c->sms ? lm_tiles : c->sms;
+            if (c->lm_even_waves) lm_ctas = (lm_tiles + (lm_tiles + lm_ctas - 1) / lm_ctas - 1) / ((lm_tiles + lm_ctas - 1) / lm_ctas);
+            ta.lm_lse_grid = gl.lse_part ? lm_ctas : 0;
         }
         after(7);
         if (e != cudaSuccess) break;
@@ -992,6 +999,8 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "prefetch_next_kb")) {
         if (value < 0) return fail(c, PRISM_ERR_INVALID_ARG, "prefetch_next_kb must be >= 0");
         c->prefetch_next_kb = value;
+    } else if (!std::strcmp(name, "lm_even_waves")) {
+        c->lm_even_waves = value != 0;
     } else if (!std::strcmp(name, "attn_lpt")) {
         c->attn_lpt = value != 0;
     } else if (!std::strcmp(name, "attn_warps")) {
