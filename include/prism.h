@@ -395,6 +395,9 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * with an L2 evict-first cache policy, since each weight byte is read once
  * per step, so that the KV cache and the activations stay in L2; 0: the
  * default policy),
+ * "tree_defer_merge" (1, the default: in tree rounds the LM head leaves its
+ * per-CTA top-w lists unmerged and the log-sum-exp kernel merges them, one
+ * CTA per row; 0: the LM head's last CTA merges them),
  * "lm_even_waves" (1, the default: the LM head launches the fewest CTAs
  * that stream its 128-row tiles in as many waves as one CTA per SM would, so
  * that every CTA streams the same number of tiles, e.g. 144 CTAs of 7 tiles

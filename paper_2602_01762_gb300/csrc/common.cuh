@@ -171,6 +171,72 @@ __device__ __forceinline__ void top8_init(float (&vals)[kTopK], int (&ids)[kTopK
     for (int i = 0; i < kTopK; ++i) { vals[i] = -INFINITY; ids[i] = 0x7FFFFFFF; }
 }
 
+// Top-1 as one 64-bit key: an order-preserving image of the fp32 logit in
+// the high word and the inverted id in the low word, so that the numeric
+// maximum is the best candidate under `better` (larger logit, then lower id).
+__device__ __forceinline__ unsigned long long pack_best(float v, int id) {
+    const uint32_t b = __float_as_uint(v);
+    const uint32_t k = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+    return ((unsigned long long)k << 32) | (uint32_t)(0xFFFFFFFFu - (uint32_t)id);
+}
+__device__ __forceinline__ void unpack_best(unsigned long long key, float &v, int &id) {
+    const uint32_t k = (uint32_t)(key >> 32);
+    v = __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+    id = (int)(0xFFFFFFFFu - (uint32_t)key);
+}
+
+using Key = unsigned long long;
+
+__device__ __forceinline__ void key_clear(Key (&l)[kTopK]) {
+#pragma unroll
+    for (int i = 0; i < kTopK; ++i) l[i] = 0ull;
+}
+
+// Insert k into the sorted list l (static indices: l stays in registers).
+__device__ __forceinline__ void key_insert(Key (&l)[kTopK], Key k) {
+    if (k <= l[kTopK - 1]) return;
+    l[kTopK - 1] = k;
+#pragma unroll
+    for (int s = kTopK - 1; s > 0; --s) {
+        const Key x = l[s - 1], y = l[s];
+        l[s - 1] = x > y ? x : y;
+        l[s] = x > y ? y : x;
+    }
+}
+
+// Lanes lane and lane ^ m both end with the best kTopK keys of their two
+// lists: the element-wise maximum of one list and the other reversed is that
+// set as a bitonic sequence, sorted by three half-cleaner stages.  Every lane
+// of the warp takes part.
+__device__ __forceinline__ void key_merge_xor(Key (&l)[kTopK], int m) {
+    Key c[kTopK];
+#pragma unroll
+    for (int i = 0; i < kTopK; ++i) {
+        const Key o = __shfl_xor_sync(0xFFFFFFFFu, l[kTopK - 1 - i], m);
+        c[i] = l[i] > o ? l[i] : o;
+    }
+#pragma unroll
+    for (int d = kTopK / 2; d > 0; d >>= 1)
+#pragma unroll
+        for (int i = 0; i < kTopK; ++i)
+            if ((i & d) == 0) {
+                const Key x = c[i], y = c[i + d];
+                c[i] = x > y ? x : y;
+                c[i + d] = x > y ? y : x;
+            }
+#pragma unroll
+    for (int i = 0; i < kTopK; ++i) l[i] = c[i];
+}
+
+// Entry r of a register list without a dynamic index.
+__device__ __forceinline__ Key key_at(const Key (&l)[kTopK], int r) {
+    Key k = l[0];
+#pragma unroll
+    for (int i = 1; i < kTopK; ++i)
+        if (r == i) k = l[i];
+    return k;
+}
+
 // ----------------------------------------------------------------- launches
 
 // Projection kinds (weight-streaming GEMV family).
@@ -249,6 +315,9 @@ struct GemvArgs {
     // 1: a selection (LM head) launch takes the fewest CTAs that keep its
     // number of tile waves, so that every CTA streams as many tiles
     int even_waves;
+    // 1: top-k lists are only published per CTA ([T][grid][8] in lm_part /
+    // lm_part_id); the kernel that reads the selection merges them
+    int defer_merge;
 };
 
 struct RopeArgs {
@@ -352,8 +421,8 @@ struct TreeArgs {
     float *pool_score;
     // this step's LM-head outputs (rows b*w + j)
     const float *logits;              // [B*w, V]
-    const int32_t *top_ids;           // [B*w, w]
-    const float *top_vals;            // [B*w, w]
+    int32_t *top_ids;                 // [B*w, w] (written by the lse kernel when the LM head defers its merge)
+    float *top_vals;                  // [B*w, w]
     float *lse;                       // [B*w]
     float *lse_part;                  // [B*w, kSampleMaxBlocks, 2]
     int *lse_ctr;                     // [B*w] (left at zero)
@@ -362,6 +431,10 @@ struct TreeArgs {
     // > 0: the LM head wrote per-CTA (max, sum exp) partials of every row,
     // lm_lse_grid of them, into lse_part ([LM-head row][lm_lse_grid][2])
     int lm_lse_grid;
+    // non-null: the LM head left its per-CTA top-8 lists unmerged
+    // ([LM-head row][lm_lse_grid][8] values and ids); the lse kernel merges them
+    const float *lm_val;
+    const int *lm_id;
     // RoPE / append / attention (one kernel)
     const float *qkv;                 // [B*w, (Hq + 2Hkv) D]
     void *k_cache, *v_cache;          // [B, Hkv, max_ctx, D]

@@ -346,20 +346,6 @@ __device__ __forceinline__ void finish_unit(const GemvArgs &a, int t, int u, flo
     }
 }
 
-// Top-1 as one 64-bit key: an order-preserving image of the fp32 logit in
-// the high word and the inverted id in the low word, so that the numeric
-// maximum is the best candidate under `better` (larger logit, then lower id).
-__device__ __forceinline__ unsigned long long pack_best(float v, int id) {
-    const uint32_t b = __float_as_uint(v);
-    const uint32_t k = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
-    return ((unsigned long long)k << 32) | (uint32_t)(0xFFFFFFFFu - (uint32_t)id);
-}
-__device__ __forceinline__ void unpack_best(unsigned long long key, float &v, int &id) {
-    const uint32_t k = (uint32_t)(key >> 32);
-    v = __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
-    id = (int)(0xFFFFFFFFu - (uint32_t)key);
-}
-
 // Split-K: the last CTA of a tile adds the K slices of unit u for every
 // activation row, in slice order, and finishes the unit.  The partial sums
 // come from other SMs through L2, so the loads of several rows and all their
@@ -423,58 +409,6 @@ __device__ __forceinline__ void reduce_slices(const GemvArgs &a, const TcPlan &p
 // row are merged pairwise across lanes (bitonic merge), and the per-CTA lists
 // of all CTAs once at the end.
 constexpr int kTrMax = kTileM + 8;   // floats per transposed row, largest P
-
-using Key = unsigned long long;
-
-__device__ __forceinline__ void key_clear(Key (&l)[kTopK]) {
-#pragma unroll
-    for (int i = 0; i < kTopK; ++i) l[i] = 0ull;
-}
-
-// Insert k into the sorted list l (static indices: l stays in registers).
-__device__ __forceinline__ void key_insert(Key (&l)[kTopK], Key k) {
-    if (k <= l[kTopK - 1]) return;
-    l[kTopK - 1] = k;
-#pragma unroll
-    for (int s = kTopK - 1; s > 0; --s) {
-        const Key x = l[s - 1], y = l[s];
-        l[s - 1] = x > y ? x : y;
-        l[s] = x > y ? y : x;
-    }
-}
-
-// Lanes lane and lane ^ m both end with the best kTopK keys of their two
-// lists: the element-wise maximum of one list and the other reversed is that
-// set as a bitonic sequence, sorted by three half-cleaner stages.  Every lane
-// of the warp takes part.
-__device__ __forceinline__ void key_merge_xor(Key (&l)[kTopK], int m) {
-    Key c[kTopK];
-#pragma unroll
-    for (int i = 0; i < kTopK; ++i) {
-        const Key o = __shfl_xor_sync(0xFFFFFFFFu, l[kTopK - 1 - i], m);
-        c[i] = l[i] > o ? l[i] : o;
-    }
-#pragma unroll
-    for (int d = kTopK / 2; d > 0; d >>= 1)
-#pragma unroll
-        for (int i = 0; i < kTopK; ++i)
-            if ((i & d) == 0) {
-                const Key x = c[i], y = c[i + d];
-                c[i] = x > y ? x : y;
-                c[i + d] = x > y ? y : x;
-            }
-#pragma unroll
-    for (int i = 0; i < kTopK; ++i) l[i] = c[i];
-}
-
-// Entry r of a register list without a dynamic index.
-__device__ __forceinline__ Key key_at(const Key (&l)[kTopK], int r) {
-    Key k = l[0];
-#pragma unroll
-    for (int i = 1; i < kTopK; ++i)
-        if (r == i) k = l[i];
-    return k;
-}
 
 // One 16-column accumulator chunk (columns c0 .. c0 + 15) of a finished tile
 // into the lists.  The four epilogue warps write their TMEM rows transposed
@@ -867,7 +801,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
                 __threadfence();
                 epi_sync();
-                if (threadIdx.x == 64) s_last = atomicAdd(a.counter, 1) == (int)gridDim.x - 1;
+                if (threadIdx.x == 64) s_last = (top1 || !a.defer_merge) && atomicAdd(a.counter, 1) == (int)gridDim.x - 1;
                 epi_sync();
                 if (s_last) {
                     __threadfence();
@@ -1805,8 +1739,8 @@ cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, f
     if (e == cudaSuccess && a.epi == kEpiTopK) {
         GemvArgs m = a;
         m.next_fuse = a.next_fuse && a.next_x && a.d % 8 == 0;
-        e = launch_k(topk_merge_kernel, dim3(a.T), dim3(128), 0, s, true, m, grid);
-        if (e == cudaSuccess && next_done) *next_done = m.next_fuse != 0;
+        if (!a.defer_merge) e = launch_k(topk_merge_kernel, dim3(a.T), dim3(128), 0, s, true, m, grid);
+        if (e == cudaSuccess && next_done) *next_done = !a.defer_merge && m.next_fuse != 0;
     }
     if (e == cudaSuccess && p.defer) {
         if (a.epi != kEpiSwiGLU && a.next_norm && a.next_x && a.n_units % 4 == 0 && a.n_units <= kRowMaxUnits) {

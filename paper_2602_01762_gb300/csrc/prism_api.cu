@@ -143,6 +143,7 @@ struct prism_ctx {
     int attn_tc = 1;                                      // fused attention on tensor cores (0: CUDA cores)
     int prefetch_next_kb = 16384;                         // KB of the next kernel's weights requested into L2
     int lm_even_waves = 1;                                // LM head: the fewest CTAs with the same tile waves
+    int tree_defer_merge = 1;                             // tree: the lse kernel merges the LM head's lists
     int attn_warps = 0;                                   // tensor-core attention warps per CTA: 0 auto, 4 or 8
     int attn_lpt = 1;                                     // several waves of attention CTAs: longest sequences first
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
@@ -493,6 +494,8 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
             if (on_tcs(g, ltm) || on_tc_staged(g, ltm)) {
                 g.lse_part = c->tree_lse_part;
                 if (!r.tree.row_logits) g.logits = nullptr;
+                // the per-CTA lists are merged by the tree's lse kernel, one CTA per row
+                g.defer_merge = c->tree_defer_merge;
             }
         }
         return g;
@@ -672,6 +675,8 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
             int lm_ctas = lm_tiles < c->sms ? lm_tiles : c->sms;
             if (c->lm_even_waves) lm_ctas = (lm_tiles + (lm_tiles + lm_ctas - 1) / lm_ctas - 1) / ((lm_tiles + lm_ctas - 1) / lm_ctas);
             ta.lm_lse_grid = gl.lse_part ? lm_ctas : 0;
+            ta.lm_val = gl.defer_merge ? c->lm_val : nullptr;
+            ta.lm_id = gl.defer_merge ? c->lm_id : nullptr;
         }
         after(7);
         if (e != cudaSuccess) break;
@@ -999,6 +1004,8 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "prefetch_next_kb")) {
         if (value < 0) return fail(c, PRISM_ERR_INVALID_ARG, "prefetch_next_kb must be >= 0");
         c->prefetch_next_kb = value;
+    } else if (!std::strcmp(name, "tree_defer_merge")) {
+        c->tree_defer_merge = value != 0;
     } else if (!std::strcmp(name, "lm_even_waves")) {
         c->lm_even_waves = value != 0;
     } else if (!std::strcmp(name, "attn_lpt")) {

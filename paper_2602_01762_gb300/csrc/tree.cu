@@ -721,6 +721,7 @@ constexpr int kLseMaxParts = 256;
 __global__ void __launch_bounds__(256) tree_lse_kernel(const TreeArgs a) {
     __shared__ float s_m[8], s_s[8];
     __shared__ int s_last, s_seq;
+    __shared__ Key s_k[4][kTopK];
     __shared__ SelectSmem sm;
     pdl_trigger();
     pdl_wait();
@@ -791,12 +792,58 @@ __global__ void __launch_bounds__(256) tree_lse_kernel(const TreeArgs a) {
             const float m2 = __shfl_xor_sync(0xFFFFFFFFu, M, o), s2 = __shfl_xor_sync(0xFFFFFFFFu, S, o);
             lse_merge(M, S, m2, s2);
         }
-        if (lane == 0) {
-            a.lse[t] = M + logf(S);
-            __threadfence();
-            s_seq = atomicAdd(a.seq_ctr + b, 1) == a.R - 1;
+        if (lane == 0) a.lse[t] = M + logf(S);
+    } else if (a.lm_val && a.lm_lse_grid > 0 && warp <= 4) {
+        // warps 1-4: the LM head's per-CTA top-8 lists of this row, merged
+        // (every load of a thread's share first, then its insertions, then
+        // each warp's lists across lanes)
+        const int lm_row = a.step == 1 ? b : t;
+        const int nc = a.lm_lse_grid * kTopK, e = tid - 32;
+        const float *pv = a.lm_val + (size_t)lm_row * nc;
+        const int *pi = a.lm_id + (size_t)lm_row * nc;
+        constexpr int kB = 16;
+        float v[kB];
+        int id[kB];
+#pragma unroll
+        for (int q = 0; q < kB; ++q) {
+            const int c = e + q * 128;
+            v[q] = c < nc ? __ldcg(pv + c) : 0.f;
+            id[q] = c < nc ? __ldcg(pi + c) : -1;
+        }
+        Key l[kTopK];
+        key_clear(l);
+#pragma unroll 1
+        for (int q = 0; q < kB; ++q)
+            if (id[q] >= 0) key_insert(l, pack_best(v[q], id[q]));
+#pragma unroll 1
+        for (int c = e + kB * 128; c < nc; c += 128)
+            if (__ldcg(pi + c) >= 0) key_insert(l, pack_best(__ldcg(pv + c), __ldcg(pi + c)));
+#pragma unroll 1
+        for (int m = 1; m < 32; m <<= 1) key_merge_xor(l, m);
+        if (lane == 0)
+#pragma unroll
+            for (int i = 0; i < kTopK; ++i) s_k[warp - 1][i] = l[i];
+    }
+    __syncthreads();
+    if (a.lm_val && a.lm_lse_grid > 0 && warp == 1) {
+        // the row's top-w candidates, ranked (logit descending, then id ascending)
+        Key l[kTopK];
+#pragma unroll
+        for (int i = 0; i < kTopK; ++i) l[i] = lane < 4 ? s_k[lane][i] : 0ull;
+#pragma unroll 1
+        for (int m = 1; m < 32; m <<= 1) key_merge_xor(l, m);
+        if (lane < a.w) {
+            float v;
+            int id;
+            unpack_best(key_at(l, lane), v, id);
+            a.top_ids[(size_t)t * a.w + lane] = id;
+            a.top_vals[(size_t)t * a.w + lane] = v;
         }
     }
+    // the row's results before its ticket
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) s_seq = atomicAdd(a.seq_ctr + b, 1) == a.R - 1;
     __syncthreads();
     if (!s_seq) return;                        // uniform over the CTA
     // the last row of sequence b to finish: candidates, frontier (and the tree)
