@@ -395,6 +395,12 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * with an L2 evict-first cache policy, since each weight byte is read once
  * per step, so that the KV cache and the activations stay in L2; 0: the
  * default policy),
+ * "lm_stream" (1, the default: the top-1 LM head of a greedy round with up
+ * to 16 rows streams them through its ring beside the weights, leaving the
+ * ring the shared memory staged rows would take, and joins the rows' best
+ * through the packed top-1 in the kernel; 0: below tc_stream_rows rows it
+ * stages them, from there on it selects through per-CTA lists and a merge
+ * kernel; sampled rounds always take the latter),
  * "tree_defer_merge" (1, the default: in tree rounds the LM head leaves its
  * per-CTA top-w lists unmerged and the log-sum-exp kernel merges them, one
  * CTA per row; 0: the LM head's last CTA merges them),

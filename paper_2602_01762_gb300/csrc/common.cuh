@@ -318,6 +318,9 @@ struct GemvArgs {
     // 1: top-k lists are only published per CTA ([T][grid][8] in lm_part /
     // lm_part_id); the kernel that reads the selection merges them
     int defer_merge;
+    // 1: a streamed top-1 selection of up to 16 rows joins through the packed
+    // atomic maximum in the kernel itself (no list merge kernel)
+    int stream_top1;
 };
 
 struct RopeArgs {

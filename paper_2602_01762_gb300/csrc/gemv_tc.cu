@@ -526,6 +526,73 @@ __device__ __forceinline__ void write_row(const GemvArgs &a, int t, const Key (&
     }
 }
 
+// Packed top-1 (one row per accumulator column t < T): a warp's candidates
+// of a tile, unit u of this lane with logit acc[t], join the warp's best of
+// each row (thr_*, the same in every lane, mirrored in s_v / s_i for the CTA's
+// join) in turn, lane by lane, where they beat it.
+template <int N>
+__device__ __forceinline__ void top1_scan(const float *acc, int T, bool valid, int u, float (&thr_v)[N],
+                                          int (&thr_i)[N], float (&s_v)[N], int (&s_i)[N]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int t = 0; t < N; ++t) {
+        if (t >= T) break;
+        const float z = acc[t];
+        unsigned m = __ballot_sync(0xFFFFFFFFu, valid && better(z, u, thr_v[t], thr_i[t]));
+        while (m) {
+            const int src = __ffs(m) - 1;
+            m &= m - 1;
+            const float zv = __shfl_sync(0xFFFFFFFFu, z, src);
+            const int uv = __shfl_sync(0xFFFFFFFFu, u, src);
+            if (!better(zv, uv, thr_v[t], thr_i[t])) continue;
+            if (lane == 0) {
+                s_v[t] = zv;
+                s_i[t] = uv;
+            }
+            __syncwarp();
+            thr_v[t] = s_v[t];
+            thr_i[t] = s_i[t];
+            __syncwarp();
+        }
+    }
+}
+
+// The CTA's best of each row (the four epilogue warps' s_v / s_i) joins a
+// 64-bit atomic maximum; the last CTA to finish writes each row's top-1 and
+// clears the maximum.  Epilogue warps only.
+template <int N>
+__device__ __forceinline__ void top1_join(const GemvArgs &a, int T, float (&s_v)[4][N], int (&s_i)[4][N],
+                                          int &s_last) {
+    const int ew = (threadIdx.x >> 5) - 2, lane = threadIdx.x & 31;
+    epi_sync();
+    if (ew == 0 && lane < T) {
+        float bv = s_v[0][lane];
+        int bi = s_i[0][lane];
+#pragma unroll
+        for (int w = 1; w < 4; ++w)
+            if (better(s_v[w][lane], s_i[w][lane], bv, bi)) { bv = s_v[w][lane]; bi = s_i[w][lane]; }
+        if (bi != 0x7FFFFFFF) atomicMax(a.best + lane, pack_best(bv, bi));
+    }
+    __threadfence();
+    epi_sync();
+    if (threadIdx.x == 64) s_last = atomicAdd(a.counter, 1) == (int)gridDim.x - 1;
+    epi_sync();
+    if (s_last) {
+        __threadfence();
+        if (ew == 0 && lane < T) {
+            const Key key = atomicExch(a.best + lane, 0ull);
+            float v;
+            int id;
+            unpack_best(key, v, id);
+            const size_t o = (size_t)lane * a.K + a.step - 1;
+            a.draft_out[o] = id;
+            if (a.topk_ids) a.topk_ids[o] = id;
+            if (a.topk_logits) a.topk_logits[o] = v;
+        }
+        if (threadIdx.x == 64) *a.counter = 0;
+    }
+}
+
 // TK: 0 no selection; 1 top-1 through the packed 64-bit atomic maximum; 2 top-k
 // through the register lists (separate instances, so neither carries the
 // other's code).
@@ -725,28 +792,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             if (t < T) a.logits[((size_t)t * a.K + a.step - 1) * a.vocab + u] = acc[0][t];
                     }
                     if constexpr (top1) {
-#pragma unroll
-                        for (int t = 0; t < NB; ++t) {
-                            if (t >= T) break;
-                            const float z = acc[0][t];
-                            // insert the qualifying lanes in turn
-                            unsigned m = __ballot_sync(0xFFFFFFFFu, valid && better(z, u, thr_v[t], thr_i[t]));
-                            while (m) {
-                                const int src = __ffs(m) - 1;
-                                m &= m - 1;
-                                const float zv = __shfl_sync(0xFFFFFFFFu, z, src);
-                                const int uv = __shfl_sync(0xFFFFFFFFu, u, src);
-                                if (!better(zv, uv, thr_v[t], thr_i[t])) continue;
-                                if (lane == 0) {
-                                    s_val[ew][t] = zv;
-                                    s_id[ew][t] = uv;
-                                }
-                                __syncwarp();
-                                thr_v[t] = s_val[ew][t];
-                                thr_i[t] = s_id[ew][t];
-                                __syncwarp();
-                            }
-                        }
+                        top1_scan<NB>(acc[0], T, valid, u, thr_v, thr_i, s_val[ew], s_id[ew]);
                     } else {
                         chunk_to_lists<8>(acc[0], row, &s_tr[0][0], tile, 0, T, a.n_units, dead, lst,
                                           a.lse_part != nullptr, lse_m, lse_s);
@@ -782,48 +828,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     epi_sync();
                 }
             }
-            if constexpr (TOPK) {
-                if constexpr (top1) {
-                    // this CTA's best of each row joins a 64-bit atomic maximum;
-                    // the last CTA to finish reads and clears it
-                    epi_sync();
-                    if (ew == 0 && lane < T) {
-                        float bv = s_val[0][lane];
-                        int bi = s_id[0][lane];
-#pragma unroll
-                        for (int w = 1; w < 4; ++w)
-                            if (better(s_val[w][lane], s_id[w][lane], bv, bi)) { bv = s_val[w][lane]; bi = s_id[w][lane]; }
-                        if (bi != 0x7FFFFFFF) atomicMax(a.best + lane, pack_best(bv, bi));
-                    }
-                } else {
-                    lists_publish<8>(a, lst, T);
-                    if (a.lse_part) lse_publish(a, lse_m, lse_s, T, 0);
-                }
+            if constexpr (top1) {
+                top1_join<NB>(a, T, s_val, s_id, s_last);
+            } else if constexpr (TOPK) {
+                lists_publish<8>(a, lst, T);
+                if (a.lse_part) lse_publish(a, lse_m, lse_s, T, 0);
                 __threadfence();
                 epi_sync();
-                if (threadIdx.x == 64) s_last = (top1 || !a.defer_merge) && atomicAdd(a.counter, 1) == (int)gridDim.x - 1;
+                if (threadIdx.x == 64) s_last = !a.defer_merge && atomicAdd(a.counter, 1) == (int)gridDim.x - 1;
                 epi_sync();
                 if (s_last) {
                     __threadfence();
-                    if constexpr (top1) {
-                        if (ew == 0 && lane < T) {
-                            const Key key = atomicExch(a.best + lane, 0ull);
-                            float v;
-                            int id;
-                            unpack_best(key, v, id);
-                            const size_t o = (size_t)lane * a.K + a.step - 1;
-                            a.draft_out[o] = id;
-                            if (a.topk_ids) a.topk_ids[o] = id;
-                            if (a.topk_logits) a.topk_logits[o] = v;
-                        }
-                    } else {
-                        // one warp per row over every CTA's list
-                        for (int t = ew; t < T; t += 4) {
-                            gather_keys<true>(a, t, gridDim.x, lane, 32, lst);
+                    // one warp per row over every CTA's list
+                    for (int t = ew; t < T; t += 4) {
+                        gather_keys<true>(a, t, gridDim.x, lane, 32, lst);
 #pragma unroll 1
-                            for (int m = 1; m < 32; m <<= 1) key_merge_xor(lst, m);
-                            write_row(a, t, lst);
-                        }
+                        for (int m = 1; m < 32; m <<= 1) key_merge_xor(lst, m);
+                        write_row(a, t, lst);
                     }
                     if (threadIdx.x == 64) *a.counter = 0;
                 }
@@ -848,14 +869,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // prologue) has written.  MMA N = NB (16 .. 256); rows of X past T arrive as
 // zeros.  The epilogue reads the NB accumulator columns 16 at a time.  With
 // top-k, the per-row merge across CTAs is left to topk_merge_kernel.
-template <int NB, int RPW, bool TOPK>
+template <int NB, int RPW, int TK>
 __global__ void __launch_bounds__(kTcThreads, 1)
     gemv_tcs_kernel(const GemvArgs a, const TcPlan p, const __grid_constant__ CUtensorMap tmW,
                     const __grid_constant__ CUtensorMap tmX) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full[kTcMaxStages], empty[kTcMaxStages], acc_full[2], acc_empty[2], mma_done;
     __shared__ uint32_t s_tmem;
-    __shared__ float s_tr[TOPK ? 16 : 1][TOPK ? kTrMax : 1];
+    constexpr bool TOPK = TK != 0, LISTS = TK == 2;   // TK: 0 none, 1 packed top-1, 2 top-k lists
+    __shared__ float s_tr[LISTS ? 16 : 1][LISTS ? kTrMax : 1];
+    __shared__ float s_val[TK == 1 ? 4 : 1][TK == 1 ? NB : 1];   // top-1: each epilogue warp's best per row
+    __shared__ int s_id[TK == 1 ? 4 : 1][TK == 1 ? NB : 1];
     __shared__ int s_last;
     constexpr uint32_t kXBox = NB * 128;                              // one X box
     constexpr uint32_t kColsNeed = 2 * RPW * NB;
@@ -1032,16 +1056,26 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int T = a.T;
             // top-k: every 16-row chunk of a tile is scanned by all 128 epilogue
             // threads, 8 per row (each thread keeps one list per chunk position)
-            constexpr int kNL = TOPK ? NB / 16 : 1;
+            constexpr int kNL = LISTS ? NB / 16 : 1;
             Key lst[kNL][kTopK];
             float lse_m[kNL], lse_s[kNL];         // per chunk position, with a.lse_part
-            if constexpr (TOPK) {
+            if constexpr (LISTS) {
 #pragma unroll
                 for (int cc = 0; cc < kNL; ++cc) {
                     key_clear(lst[cc]);
                     lse_m[cc] = -INFINITY;
                     lse_s[cc] = 0.f;
                 }
+            }
+            // top-1: per warp and row the best so far (the same in every lane)
+            constexpr int kN1 = TK == 1 ? NB : 1;
+            float thr_v[kN1];
+            int thr_i[kN1];
+            if constexpr (TK == 1) {
+#pragma unroll
+                for (int t = 0; t < NB; ++t) { thr_v[t] = -INFINITY; thr_i[t] = 0x7FFFFFFF; }
+                if (lane < NB) { s_val[ew][lane] = -INFINITY; s_id[ew][lane] = 0x7FFFFFFF; }
+                __syncwarp();
             }
             bool dead = false;
             for (int i = 0; i < my_tiles; ++i) {
@@ -1071,8 +1105,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             for (int tt = 0; tt < 16; ++tt)
                                 if (c0 + tt < T) a.logits[((size_t)(c0 + tt) * a.K + a.step - 1) * a.vocab + u] = acc[tt];
                         }
-                        chunk_to_lists<8>(acc, row, &s_tr[0][0], tile, c0, T, a.n_units, dead, lst[cc],
-                                          a.lse_part != nullptr, lse_m[cc], lse_s[cc]);
+                        if constexpr (LISTS)
+                            chunk_to_lists<8>(acc, row, &s_tr[0][0], tile, c0, T, a.n_units, dead, lst[cc],
+                                              a.lse_part != nullptr, lse_m[cc], lse_s[cc]);
+                        else
+                            top1_scan<kN1>(acc, T, valid, u, thr_v, thr_i, s_val[ew], s_id[ew]);
                     }
                 }
                 // accumulator columns 16 at a time (all RPW sets of one chunk together)
@@ -1124,13 +1161,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                 }
             }
-            if constexpr (TOPK) {
+            if constexpr (LISTS) {
                 // this CTA's list of every row; the cross-CTA merge is a separate kernel
 #pragma unroll
                 for (int cc = 0; cc < kNL; ++cc) {
                     lists_publish<8>(a, lst[cc], T, 16 * cc);
                     if (a.lse_part) lse_publish(a, lse_m[cc], lse_s[cc], T, 16 * cc);
                 }
+            } else if constexpr (TK == 1) {
+                top1_join<kN1>(a, T, s_val, s_id, s_last);
             }
         }
     }
@@ -1539,9 +1578,9 @@ bool tc_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem) {
 
 }  // namespace
 
-template <int NB, int RPW, bool TOPK>
+template <int NB, int RPW, int TK>
 cudaError_t set_tcs_attr(int bytes) {
-    return cudaFuncSetAttribute(gemv_tcs_kernel<NB, RPW, TOPK>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    return cudaFuncSetAttribute(gemv_tcs_kernel<NB, RPW, TK>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
 int tcs_nb(int T, int RPW, bool topk) {
@@ -1551,8 +1590,17 @@ int tcs_nb(int T, int RPW, bool topk) {
     return nb <= cap ? nb : 0;
 }
 
-// static shared memory of a streamed kernel (barriers, top-k lists)
-size_t tcs_static(int NB, bool topk) { return 512 + (topk ? (size_t)16 * kTrMax * 4 : 64); }
+// The selection a streamed launch makes: 0 none, 1 the packed top-1 (one
+// 16-row tile of activation rows), 2 top-k lists.
+int tcs_tk(const GemvArgs &a, int NB) {
+    if (a.epi != kEpiTopK) return 0;
+    return a.stream_top1 && a.topk == 1 && a.best && NB == 16 ? 1 : 2;
+}
+
+// static shared memory of a streamed kernel (barriers, top-1 bests, top-k lists)
+size_t tcs_static(int NB, int tk) {
+    return 512 + (tk == 2 ? (size_t)16 * kTrMax * 4 : tk == 1 ? (size_t)4 * NB * 8 : 64);
+}
 
 bool tcs_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem, int &NB) {
     const bool topk = a.epi == kEpiTopK;
@@ -1580,8 +1628,11 @@ bool tcs_plan(const GemvArgs &a, int sms, TcPlan &p, int &grid, size_t &smem, in
     }
     if (best < 0) return false;
     const size_t kb_bytes = (size_t)RPW * kBoxBytes + (size_t)NB * 128;
-    const size_t budget = (size_t)220 * 1024 - tcs_static(NB, topk);
-    const size_t dyn = budget < kTcSmem ? budget : kTcSmem;
+    // the packed top-1 instance takes the larger budget (its ring is what an
+    // LM head at batch 1 gains by streaming its row); the others 212 KB at most
+    const int tk = tcs_tk(a, NB);
+    const size_t dyn = tk == 1 ? kTcSmemLarge
+                               : std::min((size_t)220 * 1024 - tcs_static(NB, tk), kTcSmem);
     const size_t room = dyn - 1024;
     p.n_tiles = n_tiles;
     p.nkb = nkb;
@@ -1610,14 +1661,16 @@ cudaError_t dispatch_tcs(const GemvArgs &a, const TcPlan &p, const CUtensorMap &
                          size_t smem, cudaStream_t s, bool pdl) {
     const dim3 g(grid), b(kTcThreads);
     if (a.epi == kEpiTopK) {
-        if constexpr (NB <= 64) return launch_k(gemv_tcs_kernel<NB, 1, true>, g, b, smem, s, pdl, a, p, mw, mx);
+        if constexpr (NB == 16)
+            if (tcs_tk(a, NB) == 1) return launch_k(gemv_tcs_kernel<NB, 1, 1>, g, b, smem, s, pdl, a, p, mw, mx);
+        if constexpr (NB <= 64) return launch_k(gemv_tcs_kernel<NB, 1, 2>, g, b, smem, s, pdl, a, p, mw, mx);
         return cudaErrorInvalidValue;
     }
     if (a.epi == kEpiSwiGLU) {
-        if constexpr (NB <= 128) return launch_k(gemv_tcs_kernel<NB, 2, false>, g, b, smem, s, pdl, a, p, mw, mx);
+        if constexpr (NB <= 128) return launch_k(gemv_tcs_kernel<NB, 2, 0>, g, b, smem, s, pdl, a, p, mw, mx);
         return cudaErrorInvalidValue;
     }
-    return launch_k(gemv_tcs_kernel<NB, 1, false>, g, b, smem, s, pdl, a, p, mw, mx);
+    return launch_k(gemv_tcs_kernel<NB, 1, 0>, g, b, smem, s, pdl, a, p, mw, mx);
 }
 
 cudaError_t prepare_gemv_tc_kernels() {
@@ -1636,10 +1689,11 @@ cudaError_t prepare_gemv_tc_kernels() {
 #define PRISM_TCS(NB, RPW, TK)                                                                          \
     if (e == cudaSuccess)                                                                               \
         e = set_tcs_attr<NB, RPW, TK>((int)std::min((size_t)b, (size_t)220 * 1024 - tcs_static(NB, TK)));
-    PRISM_TCS(16, 1, false) PRISM_TCS(32, 1, false) PRISM_TCS(64, 1, false) PRISM_TCS(128, 1, false)
-    PRISM_TCS(256, 1, false) PRISM_TCS(16, 2, false) PRISM_TCS(32, 2, false) PRISM_TCS(64, 2, false)
-    PRISM_TCS(128, 2, false) PRISM_TCS(16, 1, true) PRISM_TCS(32, 1, true) PRISM_TCS(64, 1, true)
+    PRISM_TCS(16, 1, 0) PRISM_TCS(32, 1, 0) PRISM_TCS(64, 1, 0) PRISM_TCS(128, 1, 0)
+    PRISM_TCS(256, 1, 0) PRISM_TCS(16, 2, 0) PRISM_TCS(32, 2, 0) PRISM_TCS(64, 2, 0)
+    PRISM_TCS(128, 2, 0) PRISM_TCS(16, 1, 2) PRISM_TCS(32, 1, 2) PRISM_TCS(64, 1, 2)
 #undef PRISM_TCS
+    if (e == cudaSuccess) e = set_tcs_attr<16, 1, 1>((int)kTcSmemLarge);
     return e;
 }
 
@@ -1736,7 +1790,7 @@ cudaError_t launch_gemv_tcs(const GemvArgs &a, const CUtensorMap &mw, int sms, f
         case 128: e = dispatch_tcs<128>(a, p, mw, mx, grid, smem, s, pdl); break;
         default: e = dispatch_tcs<256>(a, p, mw, mx, grid, smem, s, pdl); break;
     }
-    if (e == cudaSuccess && a.epi == kEpiTopK) {
+    if (e == cudaSuccess && a.epi == kEpiTopK && tcs_tk(a, NB) == 2) {
         GemvArgs m = a;
         m.next_fuse = a.next_fuse && a.next_x && a.d % 8 == 0;
         if (!a.defer_merge) e = launch_k(topk_merge_kernel, dim3(a.T), dim3(128), 0, s, true, m, grid);

@@ -144,6 +144,7 @@ struct prism_ctx {
     int prefetch_next_kb = 16384;                         // KB of the next kernel's weights requested into L2
     int lm_even_waves = 1;                                // LM head: the fewest CTAs with the same tile waves
     int tree_defer_merge = 1;                             // tree: the lse kernel merges the LM head's lists
+    int lm_stream = 1;                                    // top-1 LM head: rows streamed beside the weights
     int attn_warps = 0;                                   // tensor-core attention warps per CTA: 0 auto, 4 or 8
     int attn_lpt = 1;                                     // several waves of attention CTAs: longest sequences first
     // tensor-core path: TMA tensor maps of the weights, split-K workspace
@@ -262,7 +263,11 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
     };
     // the streamed tcgen05 kernel takes g (its activation rows in the bf16 buffer)
     auto on_tcs = [&](const GemvArgs &g, const CUtensorMap *tm) -> bool {
-        if (!(tm && want_tc(g) && c->tc_ready && c->bf16 && g.T >= c->tc_stream_rows && gemv_tcs_supported(g, c->sms)))
+        // the top-1 LM head streams its rows from one row on with lm_stream
+        // (not in sampled rounds, whose draw reads the logits it writes)
+        const bool lm1 = c->lm_stream && g.stream_top1 && g.epi == kEpiTopK && g.topk == 1 && g.best;
+        if (!(tm && want_tc(g) && c->tc_ready && c->bf16 && (g.T >= c->tc_stream_rows || lm1) &&
+              gemv_tcs_supported(g, c->sms)))
             return false;
         const size_t ws = gemv_tcs_workspace_floats(g, c->sms);
         return ws == 0 || (ws <= c->tc_part_floats && gemv_tc_tiles(g) <= c->tc_ctr_n);
@@ -461,6 +466,7 @@ cudaError_t enqueue_round(prism_ctx *c, const RoundArgs &r, cudaStream_t s, bool
         g.step = k;
         g.W = c->lm_head;
         g.even_waves = c->lm_even_waves;
+        g.stream_top1 = c->lm_stream && !(r.temperature > 0.f);
         g.n_units = V;
         g.kin = d;
         g.T = rows_trow(k);
@@ -1004,6 +1010,8 @@ prism_status prism_set_option(prism_ctx *c, const char *name, int32_t value) {
     else if (!std::strcmp(name, "prefetch_next_kb")) {
         if (value < 0) return fail(c, PRISM_ERR_INVALID_ARG, "prefetch_next_kb must be >= 0");
         c->prefetch_next_kb = value;
+    } else if (!std::strcmp(name, "lm_stream")) {
+        c->lm_stream = value != 0;
     } else if (!std::strcmp(name, "tree_defer_merge")) {
         c->tree_defer_merge = value != 0;
     } else if (!std::strcmp(name, "lm_even_waves")) {
