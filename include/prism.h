@@ -308,8 +308,8 @@ prism_status prism_accept_tree(prism_ctx *ctx, int32_t batch, int32_t n_nodes, c
  * this entry point; it serves callers that cannot call cudaMalloc, so cannot
  * own a prism_ctx workspace: an inference server whose caching allocator has
  * already reserved the device memory it may use, a plugin whose host
- * framework forbids allocation outside its own pool, or code enqueued while a
- * stream capture in a mode that treats allocation as an error is under way.
+ * framework forbids allocation outside its own pool, or a process that fixes
+ * its whole device-memory budget at start-up.
  * It computes what the last stage of a draft step computes (final RMSNorm with
  * gain g_final, logits = lm_head . norm(h), top-1 and top-k), using the same
  * kernel, and keeps that kernel's scratch (the per-CTA partial top-8 lists,

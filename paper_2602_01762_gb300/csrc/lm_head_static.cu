@@ -5,10 +5,10 @@
 //
 // Some callers cannot call cudaMalloc: an inference server whose caching
 // allocator has already reserved the device memory it may use, a plugin whose
-// host framework forbids allocation outside its own pool, or code issued while
-// a stream is being captured in a mode where allocation is an error.  They
-// cannot create a prism_ctx (which owns a workspace), so this entry point
-// takes only inputs and outputs and keeps its scratch here.
+// host framework forbids allocation outside its own pool, or a process that
+// fixes its whole device-memory budget at start-up.  They cannot create a
+// prism_ctx (which owns a workspace), so this entry point takes only inputs
+// and outputs and keeps its scratch here.
 #include <cstdio>
 #include <mutex>
 #include <string>

@@ -2,8 +2,8 @@
 
 ``prism_lm_head_topk_static`` is for callers that cannot call cudaMalloc (a
 server whose caching allocator already holds the memory it may use, a plugin
-limited to its host's pool, code enqueued under a capture mode that forbids
-allocation): it keeps its scratch in a static device array inside the library
+limited to its host's pool, a process that fixes its whole device-memory
+budget at start-up): it keeps its scratch in a static device array inside the library
 instead of a context workspace.  Here it must reproduce what the draft round
 itself selects at each step: fed a step's hidden rows (the round's
 ``hidden_out``) and that step's final-norm gain, its logits and its top-k must
