@@ -193,6 +193,18 @@ def test_tcgen05_modes_bit_identical():
         model.close()
 
 
+@pytest.mark.parametrize("lm_stream", [1, 0], ids=["streamed", "staged"])
+def test_mid_top1_round(lm_stream):
+    """The greedy top-1 round at mid size (3 rows, a vocabulary of 32000 in
+    250 tiles of 128 rows, hidden size 1024): the LM head with its rows
+    streamed beside the weights and the packed top-1 joined in the kernel,
+    and with its rows staged in shared memory, both against the oracle,
+    free-running and teacher-forced."""
+    W, I = mid_case()
+    _, _, rep = _check(MID_W, W, I, [0, 1, 2], topk=1, options={"lm_stream": lm_stream})
+    assert rep["ids_compared"] >= 1
+
+
 @pytest.mark.slow
 @pytest.mark.parametrize("name,n_sample", [("l3-8b-b1", 1), ("l3-8b-b16", 3)])
 def test_cuda_core_full_size_round(name, n_sample):
