@@ -361,10 +361,13 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * loads into tensor-memory accumulators, except gate/up + SwiGLU with at
  * most 2 activation rows, which measures faster on the CUDA-core kernel;
  * 2: gate/up as well; 0: every projection on the kernels below),
- * "tc_stream_rows" (>= 1, default 8: a tcgen05 projection with at least
+ * "tc_stream_rows" (>= 1, default 1: a tcgen05 projection with at least
  * this many activation rows streams them through the TMA ring beside the
- * weights instead of staging them whole in shared memory; at most 16 rows
- * can be staged), "attn_ctas_per_sm" (1..64, default 2: the fused attention
+ * weights instead of staging them whole in shared memory, its split-K sums
+ * added by a separate finish kernel that also writes the next projection's
+ * rows; at most 16 rows can be staged, and a staged projection's last CTA
+ * per tile adds the sums itself; an LM head other than that streamed top-1
+ * below (lm_stream) streams from max(this, 8) rows outside tree rounds), "attn_ctas_per_sm" (1..64, default 2: the fused attention
  * kernel's cluster size halves while batch x KV heads x cluster size exceeds
  * this many CTAs per SM), "gemv_cuda_core" (for projections
  * not on the tcgen05 kernel: 1, the default, the CUDA-core TMA-ring kernel;
@@ -398,9 +401,10 @@ prism_status prism_sync_status(prism_ctx *ctx, void *stream, int32_t *flags);
  * "lm_stream" (1, the default: the top-1 LM head of a greedy round with up
  * to 16 rows streams them through its ring beside the weights, leaving the
  * ring the shared memory staged rows would take, and joins the rows' best
- * through the packed top-1 in the kernel; 0: below tc_stream_rows rows it
- * stages them, from there on it selects through per-CTA lists and a merge
- * kernel; sampled rounds always take the latter),
+ * through the packed top-1 in the kernel; 0: as the LM head of a sampled
+ * round, it stages fewer than max(tc_stream_rows, 8) rows (a top-1 then
+ * joins through the packed maximum) and streams more, selecting through
+ * per-CTA lists and a merge kernel),
  * "tree_defer_merge" (1, the default: in tree rounds the LM head leaves its
  * per-CTA top-w lists unmerged and the log-sum-exp kernel merges them, one
  * CTA per row; 0: the LM head's last CTA merges them),

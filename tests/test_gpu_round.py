@@ -193,6 +193,27 @@ def test_tcgen05_modes_bit_identical():
         model.close()
 
 
+STAGED = {"tc_stream_rows": 8}      # fewer than 8 activation rows staged in shared memory
+
+
+@pytest.mark.parametrize("case,topk", [("tiny-bf16", 4), ("mid", 8), ("mid", 1)])
+def test_staged_projection_path_matches_oracle(case, topk):
+    """The tcgen05 projections with their activation rows staged whole in
+    shared memory (built per CTA: embedding gather, RMSNorm, bf16 rounding)
+    and split-K sums added by each tile's last CTA, which the rounds of fewer
+    than tc_stream_rows rows take; by default every row streams."""
+    if case == "mid":
+        w = MID_W
+        W, I = mid_case()
+        seqs = [0, 1, 2]
+    else:
+        w = synth.WORKLOADS[case]
+        W, I = synth.make_weights(w), synth.make_round_inputs(w)
+        seqs = [0]
+    _, _, rep = _check(w, W, I, seqs, topk=topk, options=STAGED)
+    assert rep["ids_compared"] >= 1
+
+
 @pytest.mark.parametrize("lm_stream", [1, 0], ids=["streamed", "staged"])
 def test_mid_top1_round(lm_stream):
     """The greedy top-1 round at mid size (3 rows, a vocabulary of 32000 in

@@ -384,6 +384,17 @@ def test_mid_tree_streamed_rows():
     assert rep["ids_compared"] >= 10
 
 
+def test_tiny_tree_staged_rows():
+    """The tree's 12 rows per step (3 sequences x 4 branches) staged in
+    shared memory (tc_stream_rows = 16) instead of streamed: the staged
+    tcgen05 projections and LM head with 16-row operands."""
+    w = synth.WORKLOADS["tiny-bf16-tree"]
+    W = synth.make_weights(w)
+    I = ragged(w, synth.make_round_inputs(w))
+    _, _, rep = run_case(w, W, I, list(range(w.batch)), options={"tc_stream_rows": 16})
+    assert rep["ids_compared"] >= 10
+
+
 @pytest.mark.parametrize("width,n_nodes", [(1, 4), (2, 5), (8, 40)])
 def test_tree_widths(width, n_nodes):
     W = synth.make_weights(MID_TREE)
