@@ -697,6 +697,11 @@ def run_loop(args, w, world, rank, local):
     hid = np.stack([synth.normal(w.seed, f"loop_hidden_{r}", I["hidden"].shape, 1.0, s.dtype) for r in range(R)])
     dr = Drafter.from_shape(s, max_batch=B, max_ctx=mc, max_new=K + 1, topk=1, device=local)
     weights_dev = bind_weights(dr, W, device=dev)
+    options = {}
+    for kv in args.opt:
+        name, value = kv.split("=", 1)
+        options[name] = int(value)
+        dr.set_option(name, int(value))
     t0 = {n: to_device(I[n], dev) for n in ("tokens", "n_new", "kv_len")}
     t = {n: to_device(I[n], dev) for n in ("tokens", "n_new", "kv_len", "k_cache", "v_cache")}
     hd = to_device(hid, dev)
@@ -746,7 +751,7 @@ def run_loop(args, w, world, rank, local):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16" if s.dtype == "bf16" else "f32", "data": "synthetic",
-            "config": dict(config_of(w), loop_rounds=R, max_new=K + 1),
+            "config": dict(config_of(w), loop_rounds=R, max_new=K + 1, options=options),
             "round_latency_us": per_round_ms * 1e3,
             "loop": {"rounds_per_step": R, "mean_accept_len": float(accepted.mean()),
                      "accepted_tokens_per_s": float((accepted + 1).sum()) * args.steps * world / (ms / 1e3)},
